@@ -1,0 +1,490 @@
+#!/usr/bin/env python3
+"""Benchmark of the budgeted, mask-aware merge on GB300.
+
+One step = one pass of the whole hot path over the workload: the catalog pass
+(mp_index_blocks), then for every budget of the sweep the access plan (mp_plan)
+and the budgeted merge (mp_merge).  Inputs are seeded synthetic checkpoint
+families with the published tensor shapes, generated on the device before the
+timed region; every checkpoint is larger than L2, so no flush is needed.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--workload NAME] [--impl native|reference]
+
+Prints one JSON line.  `value` is merged parameters per second over the sweep
+(budgets x params / step time), device-timed with CUDA events; `e2e` is the same
+metric with the inputs copied from pinned host memory and the merged outputs
+copied back inside the timed region.  `--impl reference` times the CPU oracle on
+the host cores on a bounded sample of the same workload.
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import re
+import statistics
+import subprocess
+import sys
+import threading
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "accessed-expert GB/s vs HBM peak; merged params/s per budget (1 GB300)"
+UNIT = "params/s"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def workloads():
+    from paper_2605_29489_gb300 import synth
+
+    return {
+        "qwen2.5-0.5b-ta": dict(make=lambda: synth.qwen25_05b(), op="ta", lam=0.3, budgets=[1.0, 0.5, 0.25, 0.1],
+                                desc="Qwen2.5-0.5B-shaped bf16 family, K=8, task arithmetic lambda=0.3, 64Ki-element blocks"),
+        "qwen2.5-0.5b-ta-2l": dict(make=lambda: synth.qwen25_05b(layers=2), op="ta", lam=0.3,
+                                   budgets=[1.0, 0.5, 0.25, 0.1],
+                                   desc="Qwen2.5-0.5B shapes cut to 2 layers (profiling case), K=8, TA lambda=0.3"),
+        "llama-3-8b-ties": dict(make=lambda: synth.llama3_8b(), op="ties", density=0.2, budgets=[1.0, 0.5, 0.25, 0.1],
+                                desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
+        "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
+                                  desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE p=0.9 then AVG, per-expert active sets"),
+        "tiny-avg": dict(make=lambda: synth.tiny(), op="avg", budgets=[1.0, 0.5, 0.25],
+                         desc="8 fp32 512x512 tensors, K=4, AVG, 4Ki-element blocks"),
+    }
+
+
+DEFAULT_WORKLOAD = "qwen2.5-0.5b-ta"
+
+
+def make_ops(w, K):
+    import oracle
+    import paper_2605_29489_gb300 as mp
+
+    if w["op"] == "ta":
+        a = [w["lam"]] * K
+        return mp.make_op(mp.MP_OP_TA, alpha=a), oracle.Op(oracle.TA, K, alpha=a)
+    if w["op"] == "avg":
+        a = [1.0 / K] * K
+        return mp.make_op(mp.MP_OP_AVG, alpha=a), oracle.Op(oracle.AVG, K, alpha=a)
+    if w["op"] == "ties":
+        return (mp.make_op(mp.MP_OP_TIES, lam=1.0, density=w["density"]),
+                oracle.Op(oracle.TIES, K, lam=1.0, density=w["density"]))
+    if w["op"] == "dare":
+        a = [1.0 / K] * K
+        return (mp.make_op(mp.MP_OP_DARE, alpha=a, drop_p=w["drop_p"], seed=20260),
+                oracle.Op(oracle.DARE, K, alpha=a, drop_p=w["drop_p"], seed=20260))
+    raise ValueError(w["op"])
+
+
+# ---- clocks ---------------------------------------------------------------------------------------
+
+class ClockSampler:
+    """nvidia-smi clock / throttle-reason samples taken during the timed region"""
+
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.lines: list[str] = []
+        self.proc = None
+        self.thread = None
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", f"--id={self.gpu}", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                 "-lms", "100"], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+            return
+        self.thread = threading.Thread(target=self._read, daemon=True)
+        self.thread.start()
+        time.sleep(0.25)
+
+    def _read(self):
+        for line in self.proc.stdout:
+            self.lines.append(line.strip())
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.15)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        if self.thread:
+            self.thread.join(timeout=2)
+        sm, mx, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for ln in self.lines:
+            parts = [p.strip() for p in ln.split(",")]
+            if len(parts) < 9:
+                continue
+            try:
+                sm.append(float(parts[1]))
+                mx.append(float(parts[2]))
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": max(mx), "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+# ---- measured peaks / profiles ------------------------------------------------------------------
+
+def hbm_peak():
+    try:
+        with open(os.path.join(ROOT, "MEASURED_PEAKS.json")) as f:
+            return float(json.load(f)["hbm_gbs"]), "measured"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def merge_source_hash() -> str:
+    h = hashlib.sha256()
+    for name in ("merge.cu", "philox.cuh", "mp_internal.cuh"):
+        with open(os.path.join(ROOT, "paper_2605_29489_gb300", "csrc", name), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str):
+    """dram bytes per merge launch from the committed ncu summary, if it was taken on the
+    current merge kernel source (else None)"""
+    path = os.path.join(ROOT, "profiles", "merge_kernel_traffic.md")
+    if not os.path.exists(path):
+        return None
+    txt = open(path).read()
+    src = re.search(r"source_hash:\s*([0-9a-f]+)", txt)
+    if not src or src.group(1) != merge_source_hash():
+        return None
+    m = re.search(rf"traffic_per_launch\[{re.escape(workload)}\]:\s*([0-9.eE+]+)", txt)
+    return float(m.group(1)) if m else None
+
+
+# ---- CPU oracle sample ----------------------------------------------------------------------------
+
+def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
+    """Time the oracle (index, plan per budget, merge per budget) on a bounded sample of the
+    workload's blocks.  Returns (params_merged_per_s, seconds, sample_description)."""
+    import numpy as np
+    import oracle
+
+    _, oop = make_ops(w, fam.K)
+    bo, bl, bt = fam.block_table()
+    budgets = w["budgets"]
+
+    def run(blocks):
+        data = [fam.block_host(int(b)) for b in blocks]
+        lens = np.array([bl[b] for b in blocks], np.uint32)
+        offs = np.zeros(len(blocks), np.uint64)
+        o = 0
+        for k, b in enumerate(blocks):
+            offs[k] = o
+            o += int(bl[b])
+        base = np.concatenate([d[0] for d in data])
+        experts = [np.concatenate([d[1][i] for d in data]) for i in range(fam.K)]
+        groups = np.zeros(len(blocks), np.uint32)
+        of = oracle.Family(fam.dtype, offs, lens, groups, 1, base, experts)
+        es = fam.elem_size
+        full = fam.K * int(lens.sum()) * es
+        t0 = time.perf_counter()
+        norm, maxabs, nnz = oracle.index(of)
+        tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
+        for f in budgets:
+            pl = oracle.plan(fam.K, lens, groups, 1, es, oop, norm, maxabs, nnz, tau, math.floor(f * full))
+            oracle.merge(of, oop, tau=tau, mask=pl["mask"])
+        dt = time.perf_counter() - t0
+        return dt, int(lens.sum())
+
+    nb = fam.n_blocks
+    dt1, p1 = run([nb // 2])
+    n = max(1, min(nb, int(target_s / max(dt1, 1e-6))))
+    blocks = sorted(set(int(x) for x in np.linspace(0, nb - 1, n)))
+    dt, params = run(blocks)
+    desc = (f"{len(blocks)} of {nb} blocks ({params} params) evenly spaced over the family, regenerated on the "
+            f"host; oracle index + plan and merge at budgets {budgets} (budget relative to the sample)")
+    return len(budgets) * params / dt, dt, desc
+
+
+def cpu_info():
+    model = ""
+    try:
+        out = subprocess.run(["lscpu"], stdout=subprocess.PIPE, text=True).stdout
+        m = re.search(r"Model name:\s*(.+)", out)
+        model = m.group(1).strip() if m else ""
+    except Exception:
+        pass
+    return model, os.cpu_count()
+
+
+# ---- native arm -----------------------------------------------------------------------------------
+
+def native(args, rank, world, local_rank):
+    import numpy as np
+    import torch
+    import paper_2605_29489_gb300 as mp
+
+    torch.cuda.set_device(local_rank)
+    W = workloads()[args.workload]
+    fam = W["make"]()
+    gop, _ = make_ops(W, fam.K)
+    budgets = W["budgets"]
+    base, experts = fam.device_arrays()
+    offs, nums, total = fam.layout()
+    tensors = list(zip(offs.tolist(), nums.tolist()))
+    mf = mp.family(tensors, base, experts, fam.block_elems, fam.dtype, 0)
+    es = fam.elem_size
+    N = fam.n_params
+    free_b, _ = torch.cuda.mem_get_info()
+    shared_out = free_b < (len(budgets) + 2) * total * es
+    outs = [torch.empty_like(base)] if shared_out else [torch.empty_like(base) for _ in budgets]
+    Bs = [mp.mp_budget_from_fraction(mf, f) for f in budgets]
+    stream = torch.cuda.current_stream()
+
+    def step(fam_c, ev=None):
+        hs = []
+        if ev is not None:
+            ev["i0"].record(stream)
+        idx = mp.mp_index_blocks(fam_c, gop, stream)
+        hs.append(idx)
+        if ev is not None:
+            ev["i1"].record(stream)
+        for k, B in enumerate(Bs):
+            if ev is not None:
+                ev["p0"][k].record(stream)
+            plan = mp.mp_plan(idx, gop, B, stream)
+            if ev is not None:
+                ev["p1"][k].record(stream)
+            man = mp.mp_merge(fam_c, idx, plan, outs[0 if shared_out else k], stream)
+            if ev is not None:
+                ev["m1"][k].record(stream)
+            hs += [plan, man]
+        return hs
+
+    def new_events():
+        E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+        return {"i0": E(), "i1": E(), "p0": [E() for _ in Bs], "p1": [E() for _ in Bs], "m1": [E() for _ in Bs]}
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+            dist.barrier()
+
+    for _ in range(args.warmup):
+        hs = step(mf)
+        torch.cuda.synchronize()
+        for h in hs:
+            h.free()
+
+    # ---- timed region (device) ----
+    evs = [new_events() for _ in range(args.steps)]
+    clocks = ClockSampler(local_rank)
+    barrier()
+    torch.cuda.synchronize()
+    clocks.start()
+    launches0 = mp.mp_kernel_launch_count()
+    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    t_start.record(stream)
+    handles = []
+    for s in range(args.steps):
+        handles.append(step(mf, evs[s]))
+    t_end.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    launches = mp.mp_kernel_launch_count() - launches0
+    clk = clocks.stop()
+    elapsed_ms = t_start.elapsed_time(t_end)
+
+    idx_ms = statistics.mean(e["i0"].elapsed_time(e["i1"]) for e in evs)
+    plan_ms = [statistics.mean(e["p0"][k].elapsed_time(e["p1"][k]) for e in evs) for k in range(len(Bs))]
+    merge_ms = [statistics.mean(e["p1"][k].elapsed_time(e["m1"][k]) for e in evs) for k in range(len(Bs))]
+    last = handles[-1]
+    per_budget = []
+    for k, f in enumerate(budgets):
+        pi = mp.mp_plan_info(last[1 + 2 * k], with_arrays=False)
+        mi = mp.mp_manifest_info(last[2 + 2 * k], fam.K)
+        per_budget.append(dict(f=f, budget_bytes=Bs[k], planned_bytes=pi["chat"], realized_bytes=mi["realized_total"],
+                               n_selected=pi["n_sel"], n_candidates=pi["n_cand"], touched_blocks=mi["touched"],
+                               touched_ratio=pi["chat"] / (fam.K * N * es), plan_ms=plan_ms[k], merge_ms=merge_ms[k]))
+    for hs in handles:
+        for h in hs:
+            h.free()
+
+    peak, peak_kind = hbm_peak()
+    alg_bytes = [2 * N * es + pb["planned_bytes"] for pb in per_budget]
+    for pb, ab in zip(per_budget, alg_bytes):
+        s = pb["merge_ms"] / 1e3
+        pb.update(merged_params_per_s=N / s, expert_gbs=pb["planned_bytes"] / s / 1e9, hbm_bytes=ab,
+                  hbm_gbs=ab / s / 1e9, hbm_frac_measured=ab / s / 1e9 / peak,
+                  hbm_frac_nominal=ab / s / 1e9 / NOMINAL_HBM_GBS)
+    merge_total_s = sum(merge_ms) / 1e3
+    achieved = sum(alg_bytes) / merge_total_s / 1e9
+
+    # ---- e2e: pinned host inputs in, merged outputs back, inside the timed region ----
+    e2e = None
+    if not args.no_e2e:
+        base_h = base.cpu().pin_memory()
+        experts_h = [e.cpu().pin_memory() for e in experts]
+        outs_h = [torch.empty(outs[0].shape, dtype=outs[0].dtype, pin_memory=True) for _ in budgets]
+        base_d = torch.empty_like(base)
+        experts_d = [torch.empty_like(e) for e in experts]
+        mf_d = mp.family(tensors, base_d, experts_d, fam.block_elems, fam.dtype, 0)
+        e2e_steps = max(3, min(args.steps, 10))
+
+        def e2e_step():
+            base_d.copy_(base_h, non_blocking=True)
+            for d, h in zip(experts_d, experts_h):
+                d.copy_(h, non_blocking=True)
+            hs = []
+            idx = mp.mp_index_blocks(mf_d, gop, stream)
+            hs.append(idx)
+            for k, B in enumerate(Bs):
+                plan = mp.mp_plan(idx, gop, B, stream)
+                out = outs[0 if shared_out else k]
+                man = mp.mp_merge(mf_d, idx, plan, out, stream)
+                outs_h[k].copy_(out, non_blocking=True)
+                hs += [plan, man]
+            return hs
+
+        hs = e2e_step()
+        torch.cuda.synchronize()
+        for h in hs:
+            h.free()
+        barrier()
+        torch.cuda.synchronize()
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record(stream)
+        hl = []
+        for _ in range(e2e_steps):
+            hl.append(e2e_step())
+        b.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e2e_ms = a.elapsed_time(b) / e2e_steps
+        for hs in hl:
+            for h in hs:
+                h.free()
+        e2e_ms = _max_over_ranks(e2e_ms, world)
+        e2e = {"value": world * len(budgets) * N / (e2e_ms / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": (fam.K + 1) * N * es, "d2h_bytes_per_step": len(budgets) * N * es,
+               "ms_per_step": e2e_ms}
+        del base_h, experts_h, outs_h, base_d, experts_d
+
+    elapsed_ms = _max_over_ranks(elapsed_ms, world)
+    ms_per_step = elapsed_ms / args.steps
+    value = world * len(budgets) * N / (ms_per_step / 1e3)
+
+    line = {
+        "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16" if fam.dtype == 0 else "f32", "data": "synthetic",
+        "config": {"workload": args.workload, "description": W["desc"], "params": N, "K": fam.K,
+                   "blocks": fam.n_blocks, "block_elems": fam.block_elems, "budgets": budgets,
+                   "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (no flush)",
+                   "step": "index + (plan + merge) per budget"},
+        "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
+        "index_ms": idx_ms, "per_budget": per_budget,
+        "roofline": {"bound": "hbm", "kernel": "merge_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
+                     "frac": achieved / peak, "peak_kind": peak_kind,
+                     "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+                     "traffic": profiled_traffic(args.workload),
+                     "algorithmic_bytes": "per merged parameter 2*s + s*(selected experts); summed over the "
+                                          "budget sweep's launches / their summed CUDA-event time"},
+        "gpu_launches": launches,
+        "clocks": clk,
+        "e2e": e2e,
+    }
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        v, dt, desc = oracle_sample_run(W, fam, args.cpu_seconds)
+        model, ncpu = cpu_info()
+        line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
+                                "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
+    return line
+
+
+def _max_over_ranks(x: float, world: int) -> float:
+    if world == 1:
+        return x
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+# ---- reference arm (the CPU oracle) ----------------------------------------------------------------
+
+def reference(args):
+    W = workloads()[args.workload]
+    fam = W["make"]()
+    per_step = max(0.2, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
+    for _ in range(args.warmup):
+        oracle_sample_run(W, fam, per_step)
+    vals, secs, desc = [], [], ""
+    for _ in range(args.steps):
+        v, dt, desc = oracle_sample_run(W, fam, per_step)
+        vals.append(v)
+        secs.append(dt)
+    v = statistics.mean(vals)
+    model, ncpu = cpu_info()
+    return {"impl": "reference", "metric": METRIC, "value": v, "unit": UNIT, "n_gpus": 1, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(secs), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16" if fam.dtype == 0 else "f32", "data": "synthetic",
+            "config": {"workload": args.workload, "description": W["desc"], "budgets": W["budgets"]},
+            "cpu_baseline": {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
+                             "host_cpu": model, "host_cores_available": ncpu},
+            "e2e": {"value": v, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=100)
+    ap.add_argument("--warmup", type=int, default=5)
+    ap.add_argument("--impl", choices=["native", "reference"], default="native")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads().keys()))
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    args = ap.parse_args()
+    if args.warmup < 3:
+        ap.error("--warmup must be >= 3")
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local_rank = int(os.environ.get("LOCAL_RANK", "0"))
+
+    if args.impl == "reference":
+        if rank == 0:
+            print(json.dumps(reference(args)), flush=True)
+        return
+
+    if world > 1:
+        import torch
+        import torch.distributed as dist
+
+        torch.cuda.set_device(local_rank)
+        dist.init_process_group("nccl" if torch.cuda.is_available() else "gloo")
+    line = native(args, rank, world, local_rank)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+        dist.destroy_process_group()
+
+
+if __name__ == "__main__":
+    main()

@@ -1,0 +1,194 @@
+/*
+ * mergepipe.h — C ABI of the GB300 budgeted, mask-aware merge.
+ *
+ * The method (MergePipe, "Access Sets Matter: Budgeting Expert Reads for
+ * Scalable Weight-Space Model Merging") merges a base checkpoint M_0 with K
+ * experts M_1..M_K that share its weight coordinates.  It runs in three calls:
+ *
+ *   mp_index_blocks  per-block statistics of every expert delta (the catalog
+ *                    of Sec. 3; the Analyze reads of Sec. 2), plus the TIES
+ *                    trim thresholds when the operator is TIES;
+ *   mp_plan          a deterministic access plan under an expert-read budget
+ *                    B (Alg. 1 PlanGen; Eq. 2, 3 and 6);
+ *   mp_merge         the induced budgeted operator over only the planned
+ *                    blocks (Eq. 4; Alg. 2 ExecuteMerge) and its manifest.
+ *
+ * Conventions
+ *  - Data pointers are device pointers unless stated (experts may also live in
+ *    pinned host memory, see mp_family.experts_location).  The caller owns
+ *    every data buffer; the library owns the opaque handles (release them with
+ *    mp_free).  No torch or CUDA types appear in this header: a stream is the
+ *    CUDA runtime's cudaStream_t passed as mp_stream (NULL = legacy default).
+ *  - Every call enqueues its GPU work on the given stream and returns without
+ *    waiting for it, except the accessors (mp_*_info, mp_index_stats), which
+ *    wait for the handle's work to finish.  Errors found by a kernel (a
+ *    non-finite delta, a timed-out wait) are reported by the next accessor on
+ *    that handle or on a handle derived from it.
+ *  - On an error return no handle is produced and *out is set to NULL; the
+ *    contents of a merge output buffer are then unspecified.
+ *  - mp_last_error() returns a thread-local message for the last failure.
+ */
+#ifndef MERGEPIPE_H
+#define MERGEPIPE_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef int32_t mp_status;
+#define MP_OK 0
+#define MP_ERR_INVALID_ARG (-1) /* a bad argument; nothing was enqueued */
+#define MP_ERR_CUDA (-2)        /* a CUDA runtime call failed */
+#define MP_ERR_OOM (-3)         /* device or host allocation failed */
+#define MP_ERR_NONFINITE (-4)   /* a delta was NaN or infinite (reported by accessors) */
+#define MP_ERR_BUDGET (-5)      /* realized reads exceeded the plan (Prop. 1 violated) */
+#define MP_ERR_TIMEOUT (-6)     /* a bounded device wait gave up (reported by accessors) */
+#define MP_ERR_UNSUPPORTED (-7) /* valid request this build does not handle */
+#define MP_ERR_MISMATCH (-8)    /* handles that do not belong together */
+
+typedef struct CUstream_st* mp_stream;
+
+typedef enum { MP_BF16 = 0, MP_F32 = 1 } mp_dtype;
+
+/* Merge operators (Sec. 1, App. A.1).  AVG and TA are the fixed-coefficient additive
+   operator sum_i alpha_i A_i Delta_i (Prop. 2); they differ only in how the caller
+   chose alpha (AVG: sum alpha = 1; TA: alpha_i = lambda). */
+typedef enum { MP_OP_AVG = 0, MP_OP_TA = 1, MP_OP_TIES = 2, MP_OP_DARE = 3 } mp_op_kind;
+
+/* One tensor of the tensor set T (Sec. 2), as a span of the flat checkpoint buffers. */
+typedef struct {
+  uint64_t offset_elems; /* start, in elements, in every flat buffer; offset*elem_size % 16 == 0 */
+  uint64_t numel;        /* elements; any value >= 1 */
+} mp_tensor;
+
+/* A checkpoint family: base, K experts and the block partition (Sec. 2: tensor set T,
+   deterministic blocks B_t).  Tensor t is cut into ceil(numel_t / block_elems)
+   contiguous blocks; the last may be partial; blocks never cross tensors.  Blocks are
+   numbered globally in tensor order (b = 0, 1, ...); unit (i, b) is expert i's block b.
+   Tensors must be given in ascending, non-overlapping offset order.  Elements that lie
+   in no tensor are never read and never written. */
+typedef struct {
+  mp_dtype dtype;
+  uint32_t n_tensors;
+  const mp_tensor* tensors;       /* host array of n_tensors, in checkpoint order */
+  uint32_t block_elems;           /* elements per block; multiple of 8, in [256, 2^24] */
+  const void* base;               /* device pointer: M_0 */
+  uint32_t K;                     /* number of experts, 1..32 */
+  const void* const* experts;     /* host array of K pointers: M_1..M_K */
+  uint32_t experts_location;      /* 0 = device memory, 1 = pinned host memory */
+} mp_family;
+
+/* Operator and its parameters theta (Alg. 1 records op and theta with the plan). */
+typedef struct {
+  mp_op_kind kind;
+  const float* alpha;  /* host array of K coefficients; required for AVG, TA, DARE */
+  float lambda;        /* TIES: scale of the merged task vector (1 = standard TIES) */
+  float density;       /* TIES: fraction rho of each trim population kept, in [0, 1] */
+  uint32_t trim_scope; /* TIES: 0 = trim per (expert, tensor), 1 = per expert */
+  double drop_p;       /* DARE: drop probability p in [0, 1] */
+  uint64_t seed;       /* DARE: seed of the fixed random mask omega */
+} mp_op;
+
+typedef struct mp_index_s mp_index;
+typedef struct mp_plan_s mp_plan_t;
+typedef struct mp_manifest_s mp_manifest;
+
+/*
+ * mp_index_blocks — the catalog pass (Sec. 3 "Catalog"; Sec. 2: Analyze reads that build
+ * norms are amortised catalog construction).  For every unit (i, b) with
+ * delta = fp32(M_i) - fp32(M_0) it computes nnz = #{delta != 0}, maxabs = max |delta|
+ * and norm = ||Delta_{i,t,b}||_2 (fp32, one fixed summation order: 256 lanes over
+ * 16-byte vectors, a per-lane fma chain, then a butterfly over lanes).  If op->kind is
+ * MP_OP_TIES it also computes the trim threshold tau of each (expert, trim group): the
+ * k-th largest 15-bit key bits(bf16(|delta|)) & 0x7FFF with k = floor(density * numel)
+ * (k = 0 gives tau = 0x8000, nothing kept).  op may be NULL for non-TIES use.
+ * The family's buffers must stay valid and unchanged until the stream reaches this work.
+ * Errors: MP_ERR_INVALID_ARG (bad family or op), MP_ERR_OOM, MP_ERR_CUDA; a non-finite
+ * delta makes mp_index_stats (and plans built on this index) report MP_ERR_NONFINITE.
+ */
+mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream stream, mp_index** out);
+
+/*
+ * mp_plan — Alg. 1 PlanGen under budget B (bytes of expert reads, Eq. 3; cost of unit
+ * (i,b) = elements(b) * element size, App. A.1).
+ *  candidates: units with nnz > 0 (for TIES also bf16 key of maxabs >= tau); the others
+ *              contribute exactly nothing and are never read;
+ *  score:      |alpha_i| * norm (TIES: |lambda| * norm), fp32 (Prop. 2's utility);
+ *  order:      decreasing score, ties by ascending unit id b*K + i;
+ *  select:     greedy with skip — a candidate is taken iff C_hat + c <= B.
+ * The plan records the access mask (bit i of word b = A_{i,t,b}), C_hat, the number of
+ * selected units, the traversal order and a digest (FNV-1a 64 over op, theta, B, C_hat,
+ * count and the sum of splitmix64(unit) over the selected units).  Budget soundness
+ * (Prop. 1) holds by construction: C_hat <= B.  op must have the same kind and, for
+ * TIES, the same density and trim scope as the op given to mp_index_blocks.
+ * Errors: MP_ERR_INVALID_ARG, MP_ERR_MISMATCH (op differs from the index's), MP_ERR_OOM,
+ * MP_ERR_CUDA.
+ */
+mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes, mp_stream stream,
+                  mp_plan_t** out);
+
+/*
+ * mp_merge — Alg. 2 ExecuteMerge: M_A = M_0 + Psi_op(A, Delta; omega) (Eq. 4) written in
+ * full to out (a device buffer laid out like the base; every tensor element is written,
+ * untouched blocks as copies of the base).  Only planned expert blocks are read;
+ * omitted entries enter as zeros (non-anticipatory, Sec. 2).  Per element, fp32:
+ *  AVG/TA: acc = fma(alpha_i, delta_i, acc) over selected i ascending; out = M_0 + acc
+ *  DARE:   delta_i kept iff a Philox4x32-10 word >= floor(p*65536), then scaled by
+ *          fp32(1/(1-p)); combined as AVG
+ *  TIES:   trimmed by tau, sign elected from the sum, disjoint mean m; out = fma(lambda, m, M_0)
+ * then bf16 round-to-nearest-even for bf16 families.  At B >= the full candidate cost
+ * the result equals the full-read merge (Eq. 5, Prop. 1).  out must not overlap the base
+ * or an expert.  The family must be the one the index was built from (same geometry).
+ * *man receives the manifest: per-expert realized read bytes counted by the kernels,
+ * touched blocks and the plan digest (Sec. 3 "Executor").
+ * Errors: MP_ERR_INVALID_ARG, MP_ERR_MISMATCH, MP_ERR_OOM, MP_ERR_CUDA; MP_ERR_TIMEOUT
+ * from mp_manifest_info if a bounded device wait gave up.
+ */
+mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out,
+                   mp_stream stream, mp_manifest** man);
+
+/* Release an mp_index, mp_plan_t or mp_manifest (waits for its pending work).  NULL is a
+   no-op.  Passing anything else is undefined. */
+void mp_free(void* handle);
+
+/* Host copies of the index statistics, expert-major [K][n_blocks]; tau is [K][n_groups]
+   (n_groups = n_tensors for trim_scope 0, 1 for trim_scope 1).  Any pointer may be NULL.
+   Waits for the index work.  Returns MP_ERR_NONFINITE if a delta was not finite. */
+mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint32_t* nnz, uint32_t* tau);
+
+/* Geometry of an index: number of blocks, units (K * n_blocks) and TIES trim groups. */
+mp_status mp_index_shape(const mp_index* index, uint64_t* n_blocks, uint64_t* n_units, uint32_t* n_groups);
+
+/* Plan summary (waits for the plan work).  mask: n_blocks words; order: the traversal
+   order (unit ids of the n_candidates candidates, decreasing score).  Any pointer may be
+   NULL. */
+mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t* n_selected,
+                       uint64_t* n_candidates, uint64_t* digest, uint32_t* mask, uint32_t* order);
+
+/* Manifest (waits for the merge): realized expert-read bytes per expert (K words),
+   their total, touched blocks (#{b : mask_b != 0}) and the plan digest.  Returns
+   MP_ERR_BUDGET if realized reads exceed the planned bytes. */
+mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_bytes_per_expert,
+                           uint64_t* realized_total, uint64_t* touched_blocks, uint64_t* digest);
+
+/* B = floor(f * C_full) with C_full = K * sum_t numel_t * element size (the full expert
+   read); f in [0, 1] (clamped).  Returns 0 for an invalid family. */
+uint64_t mp_budget_from_fraction(const mp_family* family, double f);
+
+/* Thread-local text of the last error ("" if none). */
+const char* mp_last_error(void);
+
+/* Library version string. */
+const char* mp_version(void);
+
+/* Number of CUDA kernels this library has launched in this process (all devices,
+   all threads).  A diagnostic for counting launches per step; never resets. */
+uint64_t mp_kernel_launch_count(void);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* MERGEPIPE_H */

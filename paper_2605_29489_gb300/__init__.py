@@ -1,1 +1,271 @@
+"""GB300 (sm_103a) budgeted, mask-aware model merge — Python binding of the C ABI.
 
+The three steps of the method (MergePipe: index, plan, merge) run in the CUDA
+library ``_build/libmergepipe.so`` behind ``include/mergepipe.h``.  This module
+only marshals arguments: torch tensors provide device memory and streams, and
+every call goes straight to the C entry point of the same name.  There is no
+CPU fallback: if the library cannot be built or loaded, the calls raise.
+
+    fam   = family(tensors, base, experts, block_elems=65536)
+    op    = make_op(MP_OP_TA, alpha=[0.3] * K)
+    idx   = mp_index_blocks(fam, op)
+    plan  = mp_plan(idx, op, mp_budget_from_fraction(fam, 0.25))
+    man   = mp_merge(fam, idx, plan, out)
+    info  = mp_manifest_info(man)
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+__all__ = [
+    "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MergePipeError",
+    "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_free", "mp_index_stats",
+    "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_budget_from_fraction", "mp_last_error",
+    "mp_version", "mp_kernel_launch_count", "lib", "library_path",
+]
+
+MP_OK = 0
+MP_ERR = {-1: "MP_ERR_INVALID_ARG", -2: "MP_ERR_CUDA", -3: "MP_ERR_OOM", -4: "MP_ERR_NONFINITE",
+          -5: "MP_ERR_BUDGET", -6: "MP_ERR_TIMEOUT", -7: "MP_ERR_UNSUPPORTED", -8: "MP_ERR_MISMATCH"}
+MP_BF16, MP_F32 = 0, 1
+MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE = 0, 1, 2, 3
+
+
+class MergePipeError(RuntimeError):
+    def __init__(self, status: int, msg: str):
+        super().__init__(f"{MP_ERR.get(status, status)}: {msg}")
+        self.status = status
+
+
+class _Tensor(ctypes.Structure):
+    _fields_ = [("offset_elems", ctypes.c_uint64), ("numel", ctypes.c_uint64)]
+
+
+class _Family(ctypes.Structure):
+    _fields_ = [("dtype", ctypes.c_int), ("n_tensors", ctypes.c_uint32), ("tensors", ctypes.POINTER(_Tensor)),
+                ("block_elems", ctypes.c_uint32), ("base", ctypes.c_void_p), ("K", ctypes.c_uint32),
+                ("experts", ctypes.POINTER(ctypes.c_void_p)), ("experts_location", ctypes.c_uint32)]
+
+
+class _Op(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_int), ("alpha", ctypes.POINTER(ctypes.c_float)), ("lambda_", ctypes.c_float),
+                ("density", ctypes.c_float), ("trim_scope", ctypes.c_uint32), ("drop_p", ctypes.c_double),
+                ("seed", ctypes.c_uint64)]
+
+
+_lib = None
+
+
+def library_path() -> str:
+    from . import build as _build
+    return _build.build_mergepipe()
+
+
+def lib():
+    """The loaded CUDA library (built in-tree on first use)."""
+    global _lib
+    if _lib is None:
+        L = ctypes.CDLL(library_path())
+        vp, u64, st = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int32
+        for name, args in [
+            ("mp_index_blocks", [vp, vp, vp, vp]),
+            ("mp_plan", [vp, vp, u64, vp, vp]),
+            ("mp_merge", [vp, vp, vp, vp, vp, vp]),
+            ("mp_index_stats", [vp, vp, vp, vp, vp]),
+            ("mp_index_shape", [vp, vp, vp, vp]),
+            ("mp_plan_info", [vp, vp, vp, vp, vp, vp, vp]),
+            ("mp_manifest_info", [vp, vp, vp, vp, vp]),
+        ]:
+            f = getattr(L, name)
+            f.restype, f.argtypes = st, args
+        L.mp_free.restype, L.mp_free.argtypes = None, [vp]
+        L.mp_budget_from_fraction.restype, L.mp_budget_from_fraction.argtypes = u64, [vp, ctypes.c_double]
+        L.mp_last_error.restype, L.mp_last_error.argtypes = ctypes.c_char_p, []
+        L.mp_version.restype, L.mp_version.argtypes = ctypes.c_char_p, []
+        L.mp_kernel_launch_count.restype, L.mp_kernel_launch_count.argtypes = u64, []
+        _lib = L
+    return _lib
+
+
+def _check(rc: int):
+    if rc != MP_OK:
+        raise MergePipeError(rc, mp_last_error())
+
+
+def _stream_ptr(stream) -> int | None:
+    if stream is None:
+        import torch
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, int):
+        return stream
+    return stream.cuda_stream
+
+
+class Family:
+    """An mp_family plus the Python objects that keep its memory alive."""
+
+    def __init__(self, tensors, base, experts, block_elems, dtype, experts_location):
+        self.tensors = [(int(o), int(n)) for o, n in tensors]
+        self.base, self.experts = base, list(experts)
+        self._tarr = (_Tensor * len(self.tensors))(*[_Tensor(o, n) for o, n in self.tensors])
+        self._earr = (ctypes.c_void_p * len(self.experts))(*[_ptr(e) for e in self.experts])
+        self.c = _Family(dtype, len(self.tensors), self._tarr, block_elems, _ptr(base), len(self.experts),
+                         self._earr, experts_location)
+
+    @property
+    def K(self):
+        return self.c.K
+
+    def ref(self):
+        return ctypes.byref(self.c)
+
+
+def _ptr(t) -> int:
+    if hasattr(t, "data_ptr"):
+        return t.data_ptr()
+    if isinstance(t, np.ndarray):
+        return t.ctypes.data
+    return int(t)
+
+
+def family(tensors, base, experts, block_elems=65536, dtype=None, experts_location=None) -> Family:
+    """tensors: [(offset_elems, numel)] in checkpoint order; base/experts: flat torch tensors"""
+    if dtype is None:
+        import torch
+        dtype = MP_BF16 if base.dtype == torch.bfloat16 else MP_F32
+    if experts_location is None:
+        experts_location = 0 if getattr(experts[0], "is_cuda", True) else 1
+    return Family(tensors, base, experts, block_elems, dtype, experts_location)
+
+
+class Op:
+    def __init__(self, kind, alpha, lam, density, trim_scope, drop_p, seed):
+        self.alpha = None if alpha is None else np.ascontiguousarray(np.asarray(alpha, np.float32))
+        ap = None if self.alpha is None else self.alpha.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+        self.c = _Op(kind, ap, lam, density, trim_scope, drop_p, seed)
+        self.kind = kind
+
+    def ref(self):
+        return ctypes.byref(self.c)
+
+
+def make_op(kind, alpha=None, lam=1.0, density=0.2, trim_scope=0, drop_p=0.0, seed=0) -> Op:
+    return Op(kind, alpha, float(lam), float(density), int(trim_scope), float(drop_p), int(seed))
+
+
+class Handle:
+    """Owns an opaque library handle; released by mp_free (or on garbage collection)."""
+
+    def __init__(self, ptr: int, kind: str, keep=()):
+        self.ptr, self.kind, self._keep = ptr, kind, keep
+
+    def free(self):
+        if self.ptr:
+            lib().mp_free(ctypes.c_void_p(self.ptr))
+            self.ptr = 0
+
+    def __del__(self):
+        try:
+            self.free()
+        except Exception:
+            pass
+
+    def __enter__(self):
+        return self
+
+    def __exit__(self, *a):
+        self.free()
+
+
+def mp_index_blocks(fam: Family, op: Op | None = None, stream=None) -> Handle:
+    out = ctypes.c_void_p()
+    _check(lib().mp_index_blocks(fam.ref(), None if op is None else op.ref(), ctypes.c_void_p(_stream_ptr(stream)),
+                                 ctypes.byref(out)))
+    return Handle(out.value, "index")
+
+
+def mp_plan(index: Handle, op: Op, budget_bytes: int, stream=None) -> Handle:
+    out = ctypes.c_void_p()
+    _check(lib().mp_plan(ctypes.c_void_p(index.ptr), op.ref(), int(budget_bytes),
+                         ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(out)))
+    return Handle(out.value, "plan")
+
+
+def mp_merge(fam: Family, index: Handle, plan: Handle, out, stream=None) -> Handle:
+    man = ctypes.c_void_p()
+    _check(lib().mp_merge(fam.ref(), ctypes.c_void_p(index.ptr), ctypes.c_void_p(plan.ptr), ctypes.c_void_p(_ptr(out)),
+                          ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(man)))
+    return Handle(man.value, "manifest")
+
+
+def mp_free(h: Handle | None):
+    if h is not None:
+        h.free()
+
+
+def mp_index_shape(index: Handle):
+    nb, nu, ng = ctypes.c_uint64(), ctypes.c_uint64(), ctypes.c_uint32()
+    _check(lib().mp_index_shape(ctypes.c_void_p(index.ptr), ctypes.byref(nb), ctypes.byref(nu), ctypes.byref(ng)))
+    return nb.value, nu.value, ng.value
+
+
+def mp_index_stats(index: Handle, check: bool = True):
+    """(norm, maxabs, nnz, tau) as numpy arrays [K, n_blocks] / [K, n_groups]"""
+    nb, nu, ng = mp_index_shape(index)
+    K = nu // nb
+    norm = np.zeros((K, nb), np.float32)
+    maxabs = np.zeros((K, nb), np.float32)
+    nnz = np.zeros((K, nb), np.uint32)
+    tau = np.zeros((K, ng), np.uint32)
+    rc = lib().mp_index_stats(ctypes.c_void_p(index.ptr), norm.ctypes.data, maxabs.ctypes.data, nnz.ctypes.data,
+                              tau.ctypes.data)
+    if check:
+        _check(rc)
+    return norm, maxabs, nnz, tau
+
+
+def mp_plan_info(plan: Handle, index: Handle | None = None, with_arrays: bool = True, check: bool = True):
+    """dict(chat, n_sel, n_cand, digest[, mask, order])"""
+    v = [ctypes.c_uint64() for _ in range(4)]
+    rc = lib().mp_plan_info(ctypes.c_void_p(plan.ptr), *[ctypes.byref(x) for x in v], None, None)
+    if check:
+        _check(rc)
+    d = dict(chat=v[0].value, n_sel=v[1].value, n_cand=v[2].value, digest=v[3].value, status=rc)
+    if with_arrays and index is not None:
+        nb, nu, _ = mp_index_shape(index)
+        mask = np.zeros(nb, np.uint32)
+        order = np.zeros(max(d["n_cand"], 1), np.uint32)
+        rc2 = lib().mp_plan_info(ctypes.c_void_p(plan.ptr), None, None, None, None, mask.ctypes.data, order.ctypes.data)
+        if check:
+            _check(rc2)
+        d["mask"], d["order"] = mask, order[: d["n_cand"]]
+    return d
+
+
+def mp_manifest_info(man: Handle, K: int, check: bool = True):
+    per = np.zeros(K, np.uint64)
+    tot, touched, dig = ctypes.c_uint64(), ctypes.c_uint64(), ctypes.c_uint64()
+    rc = lib().mp_manifest_info(ctypes.c_void_p(man.ptr), per.ctypes.data, ctypes.byref(tot), ctypes.byref(touched),
+                                ctypes.byref(dig))
+    if check:
+        _check(rc)
+    return dict(realized=per, realized_total=tot.value, touched=touched.value, digest=dig.value, status=rc)
+
+
+def mp_budget_from_fraction(fam: Family, f: float) -> int:
+    return int(lib().mp_budget_from_fraction(fam.ref(), float(f)))
+
+
+def mp_last_error() -> str:
+    return lib().mp_last_error().decode()
+
+
+def mp_version() -> str:
+    return lib().mp_version().decode()
+
+
+def mp_kernel_launch_count() -> int:
+    return int(lib().mp_kernel_launch_count())

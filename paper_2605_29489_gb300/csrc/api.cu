@@ -1,0 +1,674 @@
+// Host side of the C ABI: argument validation, handle lifetime, block tables and the
+// launch sequence of index, plan and merge.  Every device step runs in the kernels of
+// index.cu, plan.cu and merge.cu; this file only marshals arguments and memory.
+#include <math.h>
+#include <string.h>
+
+#include <atomic>
+#include <mutex>
+#include <string>
+#include <vector>
+
+#include "mp_internal.cuh"
+
+namespace mp {
+
+namespace {
+thread_local std::string g_last_error;
+std::atomic<uint64_t> g_next_id{1};
+std::atomic<uint64_t> g_launches{0};
+
+// pinned host slots for the small results copied back per handle, in two size classes
+// (256 bytes: plan summaries; 32 KiB: manifest counters), recycled through free lists
+std::mutex g_pin_mu;
+std::vector<void*> g_pin_free[2];
+constexpr size_t kPinSlot[2] = {256, 32768};
+constexpr size_t kPinChunk = 1 << 20;
+
+int pin_class(size_t bytes) { return bytes <= kPinSlot[0] ? 0 : (bytes <= kPinSlot[1] ? 1 : -1); }
+
+void* pin_get(size_t bytes) {
+  int c = pin_class(bytes);
+  if (c < 0) return nullptr;
+  std::lock_guard<std::mutex> lk(g_pin_mu);
+  if (g_pin_free[c].empty()) {
+    void* chunk = nullptr;
+    if (cudaHostAlloc(&chunk, kPinChunk, cudaHostAllocDefault) != cudaSuccess) return nullptr;
+    for (size_t k = 0; k < kPinChunk / kPinSlot[c]; ++k) g_pin_free[c].push_back(static_cast<char*>(chunk) + kPinSlot[c] * k);
+  }
+  void* p = g_pin_free[c].back();
+  g_pin_free[c].pop_back();
+  return p;
+}
+
+void pin_put(void* p, size_t bytes) {
+  int c = pin_class(bytes);
+  if (!p || c < 0) return;
+  std::lock_guard<std::mutex> lk(g_pin_mu);
+  g_pin_free[c].push_back(p);
+}
+
+size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
+
+mp_status fail(mp_status st, const std::string& msg) {
+  g_last_error = msg;
+  return st;
+}
+
+mp_status dev_alloc(Alloc& a, size_t bytes, cudaStream_t st) {
+  a.bytes = bytes;
+  a.stream = st;
+  cudaError_t e = cudaMallocAsync(&a.ptr, bytes ? bytes : 256, st);
+  if (e != cudaSuccess) {
+    a.ptr = nullptr;
+    return cuda_fail(e, "cudaMallocAsync");
+  }
+  return MP_OK;
+}
+
+void dev_free(Alloc& a) {
+  if (a.ptr) cudaFree(a.ptr);  // synchronising free: no pending work can still use it
+  a.ptr = nullptr;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return at.type == cudaMemoryTypeDevice || at.type == cudaMemoryTypeManaged;
+}
+
+const void* pinned_device_view(const void* p) {
+  cudaPointerAttributes at;
+  if (cudaPointerGetAttributes(&at, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  if (at.type != cudaMemoryTypeHost) return nullptr;
+  return at.devicePointer;
+}
+
+mp_status build_geometry(const mp_family* f, Geometry& g) {
+  if (!f) return fail(MP_ERR_INVALID_ARG, "family is NULL");
+  if (f->dtype != MP_BF16 && f->dtype != MP_F32) return fail(MP_ERR_INVALID_ARG, "dtype must be MP_BF16 or MP_F32");
+  if (f->K < 1 || f->K > (uint32_t)kMaxK) return fail(MP_ERR_INVALID_ARG, "K must be in 1..32");
+  if (f->n_tensors < 1 || !f->tensors) return fail(MP_ERR_INVALID_ARG, "family has no tensors");
+  if (f->block_elems < 256 || f->block_elems > (1u << 24) || f->block_elems % 8 != 0)
+    return fail(MP_ERR_INVALID_ARG, "block_elems must be a multiple of 8 in [256, 2^24]");
+  if (!f->base || !f->experts) return fail(MP_ERR_INVALID_ARG, "base or experts is NULL");
+  if (f->experts_location > 1) return fail(MP_ERR_INVALID_ARG, "experts_location must be 0 or 1");
+  g.dtype = f->dtype;
+  g.elem_size = f->dtype == MP_BF16 ? 2u : 4u;
+  g.K = f->K;
+  g.block_elems = f->block_elems;
+  g.n_tensors = f->n_tensors;
+  g.t_off.resize(f->n_tensors);
+  g.t_numel.resize(f->n_tensors);
+  g.t_first_block.resize(f->n_tensors);
+  uint64_t nb = 0, np = 0, end = 0;
+  uint32_t maxlen = 0;
+  for (uint32_t t = 0; t < f->n_tensors; ++t) {
+    const mp_tensor& ts = f->tensors[t];
+    if (ts.numel == 0) return fail(MP_ERR_INVALID_ARG, "tensor " + std::to_string(t) + " has numel 0");
+    if ((ts.offset_elems * g.elem_size) % 16 != 0)
+      return fail(MP_ERR_INVALID_ARG, "tensor " + std::to_string(t) + " does not start on a 16-byte boundary");
+    if (ts.offset_elems < end)
+      return fail(MP_ERR_INVALID_ARG, "tensors must be in ascending, non-overlapping offset order");
+    g.t_off[t] = ts.offset_elems;
+    g.t_numel[t] = ts.numel;
+    g.t_first_block[t] = nb;
+    uint64_t tb = (ts.numel + f->block_elems - 1) / f->block_elems;
+    nb += tb;
+    np += ts.numel;
+    end = ts.offset_elems + ts.numel;
+    uint32_t l = (uint32_t)(ts.numel < f->block_elems ? ts.numel : f->block_elems);
+    if (l > maxlen) maxlen = l;
+  }
+  if (nb * (uint64_t)f->K > 0xFFFFFFFFull) return fail(MP_ERR_INVALID_ARG, "too many units (K * blocks >= 2^32)");
+  g.n_blocks = nb;
+  g.n_params = np;
+  g.span_elems = end;
+  g.max_blk_len = maxlen;
+  if (reinterpret_cast<uintptr_t>(f->base) % 16 != 0) return fail(MP_ERR_INVALID_ARG, "base is not 16-byte aligned");
+  for (uint32_t i = 0; i < f->K; ++i) {
+    if (!f->experts[i]) return fail(MP_ERR_INVALID_ARG, "expert " + std::to_string(i) + " is NULL");
+    if (reinterpret_cast<uintptr_t>(f->experts[i]) % 16 != 0)
+      return fail(MP_ERR_INVALID_ARG, "expert " + std::to_string(i) + " is not 16-byte aligned");
+  }
+  return MP_OK;
+}
+
+mp_status resolve_pointers(const mp_family* f, const void*& base, ExpertPtrs& ex) {
+  if (!is_device_ptr(f->base)) return fail(MP_ERR_INVALID_ARG, "base must be device memory");
+  base = f->base;
+  memset(&ex, 0, sizeof(ex));
+  for (uint32_t i = 0; i < f->K; ++i) {
+    if (f->experts_location == 0) {
+      if (!is_device_ptr(f->experts[i]))
+        return fail(MP_ERR_INVALID_ARG, "expert " + std::to_string(i) + " must be device memory");
+      ex.p[i] = f->experts[i];
+    } else {
+      const void* d = pinned_device_view(f->experts[i]);
+      if (!d) return fail(MP_ERR_INVALID_ARG, "expert " + std::to_string(i) + " must be pinned host memory");
+      ex.p[i] = d;
+    }
+  }
+  return MP_OK;
+}
+
+mp_status check_op(const mp_op* op, uint32_t K) {
+  if (!op) return fail(MP_ERR_INVALID_ARG, "op is NULL");
+  if (op->kind < MP_OP_AVG || op->kind > MP_OP_DARE) return fail(MP_ERR_INVALID_ARG, "unknown operator kind");
+  if (op->kind != MP_OP_TIES) {
+    if (!op->alpha) return fail(MP_ERR_INVALID_ARG, "alpha is required for AVG, TA and DARE");
+    for (uint32_t i = 0; i < K; ++i)
+      if (!isfinite(op->alpha[i])) return fail(MP_ERR_INVALID_ARG, "alpha must be finite");
+  } else {
+    if (!(op->density >= 0.0f && op->density <= 1.0f)) return fail(MP_ERR_INVALID_ARG, "density must be in [0, 1]");
+    if (!isfinite(op->lambda)) return fail(MP_ERR_INVALID_ARG, "lambda must be finite");
+    if (op->trim_scope > 1) return fail(MP_ERR_INVALID_ARG, "trim_scope must be 0 or 1");
+  }
+  if (op->kind == MP_OP_DARE && !(op->drop_p >= 0.0 && op->drop_p <= 1.0))
+    return fail(MP_ERR_INVALID_ARG, "drop_p must be in [0, 1]");
+  return MP_OK;
+}
+
+mp_status check_handle(const void* h, uint32_t magic, const char* what) {
+  if (!h || *static_cast<const uint32_t*>(h) != magic) return fail(MP_ERR_INVALID_ARG, std::string(what) + " handle is invalid");
+  return MP_OK;
+}
+
+void put_u32(std::vector<uint8_t>& v, uint32_t x) {
+  for (int k = 0; k < 4; ++k) v.push_back((uint8_t)(x >> (8 * k)));
+}
+void put_u64(std::vector<uint8_t>& v, uint64_t x) {
+  for (int k = 0; k < 8; ++k) v.push_back((uint8_t)(x >> (8 * k)));
+}
+uint32_t fbits(float f) {
+  uint32_t u;
+  memcpy(&u, &f, 4);
+  return u;
+}
+
+}  // namespace
+
+void set_error(const std::string& msg) { g_last_error = msg; }
+
+void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+mp_status cuda_fail(cudaError_t e, const char* what) {
+  cudaGetLastError();
+  g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
+  return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
+}
+
+}  // namespace mp
+
+using namespace mp;
+
+extern "C" {
+
+const char* mp_last_error(void) { return g_last_error.c_str(); }
+
+const char* mp_version(void) { return "mergepipe-gb300 0.1 (sm_103a)"; }
+
+uint64_t mp_kernel_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
+
+uint64_t mp_budget_from_fraction(const mp_family* family, double f) {
+  Geometry g;
+  if (build_geometry(family, g) != MP_OK) return 0;
+  if (!(f > 0.0)) return 0;
+  if (f > 1.0) f = 1.0;
+  const uint64_t full = (uint64_t)g.K * g.n_params * g.elem_size;
+  return (uint64_t)floor(f * (double)full);
+}
+
+mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream stream, mp_index** out) {
+  if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  Geometry g;
+  mp_status st = build_geometry(family, g);
+  if (st != MP_OK) return st;
+  const bool ties = op && op->kind == MP_OP_TIES;
+  if (op && (st = check_op(op, g.K)) != MP_OK) return st;
+  const void* base;
+  ExpertPtrs ex;
+  if ((st = resolve_pointers(family, base, ex)) != MP_OK) return st;
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+
+  const uint32_t scope = ties ? op->trim_scope : 0u;
+  const uint32_t n_groups = scope == 0 ? g.n_tensors : 1u;
+  const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
+
+  std::vector<uint64_t> h_off(nb);
+  std::vector<uint32_t> h_len(nb), h_grp(nb);
+  std::vector<unsigned long long> h_kth(n_groups, 0);
+  std::vector<uint64_t> gnumel(n_groups, 0);
+  for (uint32_t t = 0; t < g.n_tensors; ++t) {
+    uint64_t b0 = g.t_first_block[t];
+    uint64_t tb = (g.t_numel[t] + g.block_elems - 1) / g.block_elems;
+    for (uint64_t k = 0; k < tb; ++k) {
+      h_off[b0 + k] = g.t_off[t] + k * g.block_elems;
+      uint64_t rem = g.t_numel[t] - k * g.block_elems;
+      h_len[b0 + k] = (uint32_t)(rem < g.block_elems ? rem : g.block_elems);
+      h_grp[b0 + k] = scope == 0 ? t : 0u;
+    }
+    gnumel[scope == 0 ? t : 0] += g.t_numel[t];
+  }
+  if (ties)
+    for (uint32_t q = 0; q < n_groups; ++q)
+      h_kth[q] = (unsigned long long)floor((double)op->density * (double)gnumel[q]);
+
+  size_t o = 0;
+  auto slot = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
+  const size_t o_off = slot(nb * 8), o_len = slot(nb * 4), o_grp = slot(nb * 4);
+  const size_t o_norm = slot(U * 4), o_max = slot(U * 4), o_nnz = slot(U * 4), o_tau = slot(KG * 4);
+  const size_t o_err = slot(16);
+  size_t o_coarse = 0, o_fine = 0, o_kth = 0, o_est = 0, o_rank = 0;
+  if (ties) {
+    o_coarse = slot(KG * 256 * 8);
+    o_fine = slot(KG * 128 * 8);
+    o_kth = slot(n_groups * 8);
+    o_est = slot(KG * 4);
+    o_rank = slot(KG * 8);
+  }
+  mp_index_s* ix = new (std::nothrow) mp_index_s();
+  if (!ix) return fail(MP_ERR_OOM, "host allocation failed");
+  ix->magic = kMagicIndex;
+  ix->id = g_next_id++;
+  cudaGetDevice(&ix->device);
+  ix->g = g;
+  ix->op_kind = op ? (int)op->kind : -1;
+  ix->density = ties ? op->density : 0.0f;
+  ix->trim_scope = scope;
+  ix->n_groups = n_groups;
+  ix->done = nullptr;
+  if ((st = dev_alloc(ix->mem, o, cs)) != MP_OK) {
+    delete ix;
+    return st;
+  }
+  char* m = static_cast<char*>(ix->mem.ptr);
+  ix->d_blk_off = (uint64_t*)(m + o_off);
+  ix->d_blk_len = (uint32_t*)(m + o_len);
+  ix->d_blk_group = (uint32_t*)(m + o_grp);
+  ix->d_norm = (float*)(m + o_norm);
+  ix->d_maxabs = (float*)(m + o_max);
+  ix->d_nnz = (uint32_t*)(m + o_nnz);
+  ix->d_tau = (uint32_t*)(m + o_tau);
+  ix->d_err = (uint32_t*)(m + o_err);
+
+  cudaError_t e;
+  auto bail = [&](cudaError_t err, const char* what) {
+    mp_status r = cuda_fail(err, what);
+    cudaStreamSynchronize(cs);
+    dev_free(ix->mem);
+    if (ix->done) cudaEventDestroy(ix->done);
+    delete ix;
+    return r;
+  };
+  if ((e = cudaMemcpyAsync(ix->d_blk_off, h_off.data(), nb * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "block table copy");
+  if ((e = cudaMemcpyAsync(ix->d_blk_len, h_len.data(), nb * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "block table copy");
+  if ((e = cudaMemcpyAsync(ix->d_blk_group, h_grp.data(), nb * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "block table copy");
+  if ((e = cudaMemsetAsync(ix->d_err, 0, 16, cs)) != cudaSuccess) return bail(e, "memset");
+  if ((e = cudaMemsetAsync(ix->d_tau, 0, KG * 4, cs)) != cudaSuccess) return bail(e, "memset");
+
+  IndexLaunch p;
+  memset(&p, 0, sizeof(p));
+  p.dtype = g.dtype;
+  p.K = g.K;
+  p.n_blocks = nb;
+  p.n_groups = n_groups;
+  p.base = base;
+  p.experts = ex;
+  p.blk_off = ix->d_blk_off;
+  p.blk_len = ix->d_blk_len;
+  p.blk_group = ix->d_blk_group;
+  p.norm = ix->d_norm;
+  p.maxabs = ix->d_maxabs;
+  p.nnz = ix->d_nnz;
+  p.err = ix->d_err;
+  if (ties) {
+    p.coarse = (unsigned long long*)(m + o_coarse);
+    p.fine = (unsigned long long*)(m + o_fine);
+    p.kth = (const unsigned long long*)(m + o_kth);
+    p.estar = (uint32_t*)(m + o_est);
+    p.rank = (unsigned long long*)(m + o_rank);
+    p.tau = ix->d_tau;
+    if ((e = cudaMemsetAsync(p.coarse, 0, KG * 256 * 8, cs)) != cudaSuccess) return bail(e, "memset");
+    if ((e = cudaMemsetAsync(p.fine, 0, KG * 128 * 8, cs)) != cudaSuccess) return bail(e, "memset");
+    if ((e = cudaMemcpyAsync((void*)p.kth, h_kth.data(), n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+      return bail(e, "k copy");
+  }
+  if ((e = launch_index(p, cs)) != cudaSuccess) return bail(e, "index kernels");
+  if ((e = cudaEventCreateWithFlags(&ix->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
+  if ((e = cudaEventRecord(ix->done, cs)) != cudaSuccess) return bail(e, "event record");
+  *out = ix;
+  return MP_OK;
+}
+
+mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes, mp_stream stream, mp_plan_t** out) {
+  if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  const Geometry& g = index->g;
+  if ((st = check_op(op, g.K)) != MP_OK) return st;
+  if (op->kind == MP_OP_TIES &&
+      (index->op_kind != MP_OP_TIES || index->density != op->density || index->trim_scope != op->trim_scope))
+    return fail(MP_ERR_MISMATCH, "a TIES plan needs an index built with the same TIES density and trim scope");
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  const uint64_t nb = g.n_blocks, U = nb * g.K;
+
+  mp_plan_s* pl = new (std::nothrow) mp_plan_s();
+  if (!pl) return fail(MP_ERR_OOM, "host allocation failed");
+  pl->magic = kMagicPlan;
+  pl->id = g_next_id++;
+  pl->index_id = index->id;
+  pl->device = index->device;
+  pl->g = g;
+  pl->op_kind = op->kind;
+  for (uint32_t i = 0; i < kMaxK; ++i) pl->alpha[i] = (op->alpha && i < g.K) ? op->alpha[i] : 0.0f;
+  pl->lambda = op->lambda;
+  pl->density = op->density;
+  pl->trim_scope = op->trim_scope;
+  pl->drop_p = op->drop_p;
+  pl->seed = op->seed;
+  pl->budget = budget_bytes;
+  pl->n_groups = index->n_groups;
+  pl->done = nullptr;
+  pl->h_summary = static_cast<uint64_t*>(pin_get(64));
+  if (!pl->h_summary) {
+    delete pl;
+    return fail(MP_ERR_OOM, "pinned host allocation failed");
+  }
+  size_t o = 0;
+  auto slot = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
+  const size_t o_mask = slot(nb * 4), o_order = slot(U * 4), o_sum = slot(8 * 8);
+  if ((st = dev_alloc(pl->mem, o, cs)) != MP_OK) {
+    pin_put(pl->h_summary, 64);
+    delete pl;
+    return st;
+  }
+  char* m = static_cast<char*>(pl->mem.ptr);
+  pl->d_mask = (uint32_t*)(m + o_mask);
+  pl->d_order = (uint32_t*)(m + o_order);
+  pl->d_summary = (uint64_t*)(m + o_sum);
+
+  Alloc scratch;
+  auto bail = [&](cudaError_t err, const char* what) {
+    mp_status r = cuda_fail(err, what);
+    cudaStreamSynchronize(cs);
+    if (scratch.ptr) cudaFree(scratch.ptr);
+    dev_free(pl->mem);
+    pin_put(pl->h_summary, 64);
+    if (pl->done) cudaEventDestroy(pl->done);
+    delete pl;
+    return r;
+  };
+  cudaError_t e;
+  if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = cudaMallocAsync(&scratch.ptr, plan_scratch_bytes(U), cs)) != cudaSuccess) {
+    scratch.ptr = nullptr;
+    return bail(e, "plan scratch");
+  }
+
+  PlanLaunch p;
+  memset(&p, 0, sizeof(p));
+  p.K = g.K;
+  p.n_blocks = nb;
+  p.n_groups = index->n_groups;
+  p.elem_size = g.elem_size;
+  p.op_kind = op->kind;
+  for (uint32_t i = 0; i < g.K; ++i) p.coef[i] = fabsf(op->kind == MP_OP_TIES ? op->lambda : op->alpha[i]);
+  p.blk_len = index->d_blk_len;
+  p.blk_group = index->d_blk_group;
+  p.norm = index->d_norm;
+  p.maxabs = index->d_maxabs;
+  p.nnz = index->d_nnz;
+  p.tau = index->d_tau;
+  p.index_err = index->d_err;
+  p.budget = budget_bytes;
+  p.mask = pl->d_mask;
+  p.order = pl->d_order;
+  p.summary = pl->d_summary;
+  std::vector<uint8_t> hdr;
+  put_u32(hdr, (uint32_t)op->kind);
+  put_u32(hdr, g.K);
+  for (uint32_t i = 0; i < g.K; ++i) put_u32(hdr, op->alpha ? fbits(op->alpha[i]) : 0u);
+  put_u32(hdr, fbits(op->lambda));
+  put_u32(hdr, fbits(op->density));
+  put_u32(hdr, op->trim_scope);
+  uint64_t pb;
+  memcpy(&pb, &op->drop_p, 8);
+  put_u64(hdr, pb);
+  put_u64(hdr, op->seed);
+  put_u64(hdr, budget_bytes);
+  memcpy(p.hdr_prefix, hdr.data(), hdr.size());
+  p.hdr_prefix_len = (uint32_t)hdr.size();
+
+  if ((e = launch_plan(p, scratch.ptr, cs)) != cudaSuccess) return bail(e, "plan kernels");
+  if ((e = cudaFreeAsync(scratch.ptr, cs)) != cudaSuccess) return bail(e, "free scratch");
+  scratch.ptr = nullptr;
+  if ((e = cudaMemcpyAsync(pl->h_summary, pl->d_summary, 64, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)
+    return bail(e, "summary copy");
+  if ((e = cudaEventCreateWithFlags(&pl->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
+  if ((e = cudaEventRecord(pl->done, cs)) != cudaSuccess) return bail(e, "event record");
+  *out = pl;
+  return MP_OK;
+}
+
+mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
+                   mp_stream stream, mp_manifest** man_out) {
+  if (!man_out) return fail(MP_ERR_INVALID_ARG, "manifest out is NULL");
+  *man_out = nullptr;
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  if ((st = check_handle(plan, kMagicPlan, "plan")) != MP_OK) return st;
+  if (plan->index_id != index->id) return fail(MP_ERR_MISMATCH, "plan was built from a different index");
+  Geometry g;
+  if ((st = build_geometry(family, g)) != MP_OK) return st;
+  if (!g.same_as(index->g)) return fail(MP_ERR_MISMATCH, "family geometry differs from the index's");
+  if (!out_buf || reinterpret_cast<uintptr_t>(out_buf) % 16 != 0)
+    return fail(MP_ERR_INVALID_ARG, "out must be a 16-byte aligned device buffer");
+  if (!is_device_ptr(out_buf)) return fail(MP_ERR_INVALID_ARG, "out must be device memory");
+  const void* base;
+  ExpertPtrs ex;
+  if ((st = resolve_pointers(family, base, ex)) != MP_OK) return st;
+  {
+    const char* o0 = static_cast<const char*>(out_buf);
+    const char* o1 = o0 + g.span_elems * g.elem_size;
+    auto overlaps = [&](const void* q) {
+      const char* a = static_cast<const char*>(q);
+      return a < o1 && o0 < a + g.span_elems * g.elem_size;
+    };
+    if (overlaps(base)) return fail(MP_ERR_INVALID_ARG, "out overlaps the base");
+    for (uint32_t i = 0; i < g.K; ++i)
+      if (family->experts_location == 0 && overlaps(ex.p[i]))
+        return fail(MP_ERR_INVALID_ARG, "out overlaps an expert");
+  }
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+
+  mp_manifest_s* mf = new (std::nothrow) mp_manifest_s();
+  if (!mf) return fail(MP_ERR_OOM, "host allocation failed");
+  mf->magic = kMagicManifest;
+  mf->plan_id = plan->id;
+  mf->device = plan->device;
+  mf->K = g.K;
+  mf->done = nullptr;
+  const size_t counters_bytes = (size_t)kCounterSlots * g.K * 8;
+  // the counters (64 slots x K), the plan summary and the error word come back in one copy
+  const size_t back_bytes = counters_bytes + 64 + 16;
+  mf->h_realized = static_cast<unsigned long long*>(pin_get(back_bytes));
+  if (!mf->h_realized) {
+    delete mf;
+    return fail(MP_ERR_OOM, "pinned host allocation failed");
+  }
+  auto release_pinned = [&]() { pin_put(mf->h_realized, back_bytes); };
+  if ((st = dev_alloc(mf->mem, back_bytes, cs)) != MP_OK) {
+    release_pinned();
+    delete mf;
+    return st;
+  }
+  mf->d_realized = static_cast<unsigned long long*>(mf->mem.ptr);
+  uint64_t* d_sum_copy = reinterpret_cast<uint64_t*>(static_cast<char*>(mf->mem.ptr) + counters_bytes);
+  mf->d_err = reinterpret_cast<uint32_t*>(static_cast<char*>(mf->mem.ptr) + counters_bytes + 64);
+  auto bail = [&](cudaError_t err, const char* what) {
+    mp_status r = cuda_fail(err, what);
+    cudaStreamSynchronize(cs);
+    dev_free(mf->mem);
+    release_pinned();
+    if (mf->done) cudaEventDestroy(mf->done);
+    delete mf;
+    return r;
+  };
+  cudaError_t e;
+  if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = cudaStreamWaitEvent(cs, plan->done, 0)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = cudaMemsetAsync(mf->mem.ptr, 0, back_bytes, cs)) != cudaSuccess) return bail(e, "memset");
+
+  MergeLaunch p;
+  memset(&p, 0, sizeof(p));
+  p.dtype = g.dtype;
+  p.op_kind = plan->op_kind;
+  p.K = g.K;
+  p.n_blocks = g.n_blocks;
+  p.block_elems = g.block_elems;
+  p.n_groups = plan->n_groups;
+  p.base = base;
+  p.experts = ex;
+  p.out = out_buf;
+  p.blk_off = index->d_blk_off;
+  p.blk_len = index->d_blk_len;
+  p.blk_group = index->d_blk_group;
+  p.mask = plan->d_mask;
+  p.tau = index->d_tau;
+  for (uint32_t i = 0; i < kMaxK; ++i) p.alpha[i] = plan->alpha[i];
+  p.lambda = plan->lambda;
+  p.sigma = plan->drop_p < 1.0 ? (float)(1.0 / (1.0 - plan->drop_p)) : 0.0f;
+  {
+    double t = floor(plan->drop_p * 65536.0);
+    p.dare_T = !(t > 0.0) ? 0u : (t > 65536.0 ? 65536u : (uint32_t)t);
+  }
+  p.seed = plan->seed;
+  p.realized = mf->d_realized;
+  p.err = mf->d_err;
+  if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
+  if ((e = cudaMemcpyAsync(d_sum_copy, plan->d_summary, 64, cudaMemcpyDeviceToDevice, cs)) != cudaSuccess)
+    return bail(e, "summary copy");
+  if ((e = cudaMemcpyAsync(mf->h_realized, mf->mem.ptr, back_bytes, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)
+    return bail(e, "manifest copy");
+  if ((e = cudaEventCreateWithFlags(&mf->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
+  if ((e = cudaEventRecord(mf->done, cs)) != cudaSuccess) return bail(e, "event record");
+  *man_out = mf;
+  return MP_OK;
+}
+
+void mp_free(void* handle) {
+  if (!handle) return;
+  uint32_t magic = *static_cast<uint32_t*>(handle);
+  if (magic == kMagicIndex) {
+    mp_index_s* ix = static_cast<mp_index_s*>(handle);
+    if (ix->done) cudaEventSynchronize(ix->done), cudaEventDestroy(ix->done);
+    dev_free(ix->mem);
+    ix->magic = 0;
+    delete ix;
+  } else if (magic == kMagicPlan) {
+    mp_plan_s* pl = static_cast<mp_plan_s*>(handle);
+    if (pl->done) cudaEventSynchronize(pl->done), cudaEventDestroy(pl->done);
+    dev_free(pl->mem);
+    pin_put(pl->h_summary, 64);
+    pl->magic = 0;
+    delete pl;
+  } else if (magic == kMagicManifest) {
+    mp_manifest_s* mf = static_cast<mp_manifest_s*>(handle);
+    if (mf->done) cudaEventSynchronize(mf->done), cudaEventDestroy(mf->done);
+    dev_free(mf->mem);
+    pin_put(mf->h_realized, (size_t)kCounterSlots * mf->K * 8 + 64 + 16);
+    mf->magic = 0;
+    delete mf;
+  }
+}
+
+mp_status mp_index_shape(const mp_index* index, uint64_t* n_blocks, uint64_t* n_units, uint32_t* n_groups) {
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  if (n_blocks) *n_blocks = index->g.n_blocks;
+  if (n_units) *n_units = index->g.n_blocks * index->g.K;
+  if (n_groups) *n_groups = index->n_groups;
+  return MP_OK;
+}
+
+mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint32_t* nnz, uint32_t* tau) {
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(index->done)) != cudaSuccess) return cuda_fail(e, "index work");
+  const uint64_t U = index->g.n_blocks * index->g.K;
+  if (norm && (e = cudaMemcpy(norm, index->d_norm, U * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (maxabs && (e = cudaMemcpy(maxabs, index->d_maxabs, U * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (nnz && (e = cudaMemcpy(nnz, index->d_nnz, U * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (tau && (e = cudaMemcpy(tau, index->d_tau, (size_t)index->g.K * index->n_groups * 4,
+                             cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  uint32_t err = 0;
+  if ((e = cudaMemcpy(&err, index->d_err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
+  if (err & kErrNonfinite) return fail(MP_ERR_NONFINITE, "a delta in the family is NaN or infinite");
+  if (err) return fail(MP_ERR_TIMEOUT, "index kernels reported an error");
+  return MP_OK;
+}
+
+mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t* n_selected, uint64_t* n_candidates,
+                       uint64_t* digest, uint32_t* mask, uint32_t* order) {
+  mp_status st;
+  if ((st = check_handle(plan, kMagicPlan, "plan")) != MP_OK) return st;
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(plan->done)) != cudaSuccess) return cuda_fail(e, "plan work");
+  const uint64_t* s = plan->h_summary;
+  if (planned_bytes) *planned_bytes = s[0];
+  if (n_selected) *n_selected = s[1];
+  if (n_candidates) *n_candidates = s[2];
+  if (digest) *digest = s[4];
+  if (mask && (e = cudaMemcpy(mask, plan->d_mask, plan->g.n_blocks * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (order && s[2] && (e = cudaMemcpy(order, plan->d_order, s[2] * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (s[6] & kErrNonfinite) return fail(MP_ERR_NONFINITE, "the index saw a NaN or infinite delta");
+  if (s[6]) return fail(MP_ERR_TIMEOUT, "index kernels reported an error");
+  if (s[0] > plan->budget) return fail(MP_ERR_BUDGET, "planned bytes exceed the budget");
+  return MP_OK;
+}
+
+mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_per_expert, uint64_t* realized_total,
+                           uint64_t* touched_blocks, uint64_t* digest) {
+  mp_status st;
+  if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(man->done)) != cudaSuccess) return cuda_fail(e, "merge work");
+  const unsigned long long* c = man->h_realized;
+  const uint64_t* s = reinterpret_cast<const uint64_t*>(c + (size_t)kCounterSlots * man->K);
+  const uint32_t err = *reinterpret_cast<const uint32_t*>(s + 8);
+  uint64_t tot = 0;
+  for (uint32_t i = 0; i < man->K; ++i) {
+    uint64_t r = 0;
+    for (int k = 0; k < kCounterSlots; ++k) r += c[(size_t)k * man->K + i];
+    if (realized_per_expert) realized_per_expert[i] = r;
+    tot += r;
+  }
+  if (realized_total) *realized_total = tot;
+  if (touched_blocks) *touched_blocks = s[5];
+  if (digest) *digest = s[4];
+  if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the merge gave up");
+  if (err) return fail(MP_ERR_CUDA, "merge kernels reported an error");
+  if (tot > s[0]) return fail(MP_ERR_BUDGET, "realized expert reads exceed the planned bytes");
+  return MP_OK;
+}
+
+}  // extern "C"

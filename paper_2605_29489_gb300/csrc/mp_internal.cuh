@@ -1,0 +1,201 @@
+// Internal declarations of the merge library: handle layouts, kernel parameter blocks
+// and the launch functions each translation unit provides to api.cu.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include <string>
+#include <vector>
+
+#include "mergepipe.h"
+
+namespace mp {
+
+constexpr uint32_t kMagicIndex = 0x58495043u;  // handle tags
+constexpr uint32_t kMagicPlan = 0x4C505043u;
+constexpr uint32_t kMagicManifest = 0x464D5043u;
+
+constexpr uint32_t kTauNone = 0x8000u;  // TIES threshold meaning "keep nothing"
+constexpr int kLanes = 256;             // lanes of the canonical norm order (one CTA)
+constexpr int kMaxK = 32;
+constexpr int kCounterSlots = 64;  // realized-byte counters are spread over slots
+
+// device error word bits
+enum : uint32_t { kErrNonfinite = 1u, kErrTimeout = 2u, kErrInternal = 4u };
+
+struct ExpertPtrs {
+  const void* p[kMaxK];
+};
+
+// geometry shared by every handle built from one family
+struct Geometry {
+  mp_dtype dtype = MP_BF16;
+  uint32_t elem_size = 2;
+  uint32_t K = 0;
+  uint32_t block_elems = 0;
+  uint32_t n_tensors = 0;
+  uint64_t n_blocks = 0;
+  uint64_t n_params = 0;      // sum of numel
+  uint64_t span_elems = 0;    // max(offset + numel)
+  uint32_t max_blk_len = 0;
+  std::vector<uint64_t> t_off, t_numel, t_first_block;
+  bool same_as(const Geometry& o) const {
+    return dtype == o.dtype && K == o.K && block_elems == o.block_elems && t_off == o.t_off &&
+           t_numel == o.t_numel;
+  }
+};
+
+struct Alloc {
+  void* ptr = nullptr;
+  size_t bytes = 0;
+  cudaStream_t stream = nullptr;
+};
+
+}  // namespace mp
+
+struct mp_index_s {
+  uint32_t magic;
+  uint64_t id;
+  int device;
+  mp::Geometry g;
+  int op_kind;
+  float density;
+  uint32_t trim_scope;
+  uint32_t n_groups;
+  mp::Alloc mem;
+  uint64_t* d_blk_off;     // [n_blocks] element offset of each block
+  uint32_t* d_blk_len;     // [n_blocks] elements of each block
+  uint32_t* d_blk_group;   // [n_blocks] TIES trim group of each block
+  float* d_norm;           // [K][n_blocks]
+  float* d_maxabs;         // [K][n_blocks]
+  uint32_t* d_nnz;         // [K][n_blocks]
+  uint32_t* d_tau;         // [K][n_groups] (TIES only)
+  uint32_t* d_err;         // error word
+  cudaEvent_t done;
+};
+
+struct mp_plan_s {
+  uint32_t magic;
+  uint64_t id;
+  uint64_t index_id;
+  int device;
+  mp::Geometry g;
+  int op_kind;
+  float alpha[mp::kMaxK];
+  float lambda, density;
+  uint32_t trim_scope;
+  double drop_p;
+  uint64_t seed;
+  uint64_t budget;
+  uint32_t n_groups;
+  mp::Alloc mem;
+  uint32_t* d_mask;        // [n_blocks] access mask
+  uint32_t* d_order;       // [K*n_blocks] traversal order (first n_cand valid)
+  uint64_t* d_summary;     // [8] chat, n_sel, n_cand, set_hash, digest, touched, err, pad
+  uint64_t* h_summary;     // pinned host copy of d_summary
+  cudaEvent_t done;
+};
+
+struct mp_manifest_s {
+  uint32_t magic;
+  uint64_t plan_id;
+  int device;
+  uint32_t K;
+  mp::Alloc mem;
+  unsigned long long* d_realized;  // [kCounterSlots][K]
+  uint32_t* d_err;
+  unsigned long long* h_realized;  // pinned host copy (slots summed on host)
+  uint32_t* h_err;
+  uint64_t planned, touched, digest;
+  cudaEvent_t done;
+};
+
+namespace mp {
+
+// ---- launch accounting (api.cu) ------------------------------------------------------------
+void count_launches(uint64_t n);
+
+// ---- error reporting (api.cu) -----------------------------------------------------------
+void set_error(const std::string& msg);
+mp_status cuda_fail(cudaError_t e, const char* what);
+
+// ---- index (index.cu) -------------------------------------------------------------------
+struct IndexLaunch {
+  mp_dtype dtype;
+  uint32_t K;
+  uint64_t n_blocks;
+  uint32_t n_groups;
+  const void* base;
+  ExpertPtrs experts;
+  const uint64_t* blk_off;
+  const uint32_t* blk_len;
+  const uint32_t* blk_group;
+  float* norm;
+  float* maxabs;
+  uint32_t* nnz;
+  uint32_t* err;
+  // TIES (null when not TIES)
+  unsigned long long* coarse;  // [K][n_groups][256]
+  unsigned long long* fine;    // [K][n_groups][128]
+  const unsigned long long* kth;  // [n_groups] k = floor(density * numel_g)
+  uint32_t* estar;             // [K][n_groups] coarse bin of tau (or 0xFFFFFFFF)
+  unsigned long long* rank;    // [K][n_groups] rank of tau inside that bin
+  uint32_t* tau;               // [K][n_groups]
+};
+cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
+
+// ---- plan (plan.cu) ---------------------------------------------------------------------
+struct PlanLaunch {
+  uint32_t K;
+  uint64_t n_blocks;
+  uint32_t n_groups;
+  uint32_t elem_size;
+  int op_kind;
+  float coef[kMaxK];   // |alpha_i| or |lambda|
+  const uint32_t* blk_len;
+  const uint32_t* blk_group;
+  const float* norm;
+  const float* maxabs;
+  const uint32_t* nnz;
+  const uint32_t* tau;
+  const uint32_t* index_err;
+  uint64_t budget;
+  uint32_t* mask;
+  uint32_t* order;
+  uint64_t* summary;
+  // digest header fields (host-built, hashed on the device after C_hat is known)
+  uint8_t hdr_prefix[256];
+  uint32_t hdr_prefix_len;
+};
+// scratch bytes plan_run needs for n_units units
+size_t plan_scratch_bytes(uint64_t n_units);
+cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st);
+
+// ---- merge (merge.cu) -------------------------------------------------------------------
+struct MergeLaunch {
+  mp_dtype dtype;
+  int op_kind;
+  uint32_t K;
+  uint64_t n_blocks;
+  uint32_t block_elems;
+  uint32_t n_groups;
+  const void* base;
+  ExpertPtrs experts;
+  void* out;
+  const uint64_t* blk_off;
+  const uint32_t* blk_len;
+  const uint32_t* blk_group;
+  const uint32_t* mask;
+  const uint32_t* tau;  // TIES
+  float alpha[kMaxK];
+  float lambda;
+  float sigma;          // DARE rescale
+  uint32_t dare_T;      // DARE keep threshold on 16-bit words
+  uint64_t seed;
+  unsigned long long* realized;  // [kCounterSlots][K]
+  uint32_t* err;
+};
+cudaError_t launch_merge(const MergeLaunch& p, cudaStream_t st);
+
+}  // namespace mp

@@ -266,9 +266,10 @@ def tiny(seed: int = 0) -> Family:
                   active_frac=0.3, log_mu=math.log(1e-3), log_sigma=1.0, seed=seed)
 
 
-def qwen25_05b(seed: int = 0, K: int = 8) -> Family:
+def qwen25_05b(seed: int = 0, K: int = 8, layers: int = 24) -> Family:
     """Qwen2.5-0.5B shapes (hidden 896, 24 layers, 14/2 heads, inter 4864, vocab 151936 tied), bf16"""
-    return Family("qwen2.5-0.5b", BF16, _qwen2_tensors(896, 24, 14, 2, 4864, 151936), 65536, K,
+    name = "qwen2.5-0.5b" if layers == 24 else f"qwen2.5-0.5b-{layers}l"
+    return Family(name, BF16, _qwen2_tensors(896, layers, 14, 2, 4864, 151936), 65536, K,
                   active_frac=0.3, log_mu=math.log(1e-3), log_sigma=1.0, seed=seed)
 
 

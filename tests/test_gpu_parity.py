@@ -1,0 +1,282 @@
+"""Parity of the CUDA path (through the C ABI) with the CPU oracle on seeded inputs.
+
+Bars: bit-exact for statistics' integer fields, norm/maxabs bits, TIES thresholds,
+plans (mask, C_hat, counts, traversal order, digest) and manifests; merged bf16
+within one bf16 ulp (fp32 checkpoints within 1e-6 relative) — the kernels follow
+the same fp32 operation order as the oracle, so the merge is also expected to be
+identical and the test reports any difference.
+"""
+import math
+
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from conftest import oracle_family
+
+pytestmark = pytest.mark.gpu
+
+import paper_2605_29489_gb300 as mp  # noqa: E402
+from paper_2605_29489_gb300 import synth  # noqa: E402
+
+
+# ---- helpers ------------------------------------------------------------------------------------
+
+def dev(fam, a):
+    if fam.dtype == synth.BF16:
+        return torch.from_numpy(a.view(np.int16)).cuda().view(torch.bfloat16)
+    return torch.from_numpy(a).cuda()
+
+
+def host(fam, t):
+    if fam.dtype == synth.BF16:
+        return t.view(torch.int16).cpu().numpy().view(np.uint16)
+    return t.cpu().numpy()
+
+
+def upload(fam, base, experts):
+    b = dev(fam, base)
+    ex = [dev(fam, e) for e in experts]
+    offs, nums, _ = fam.layout()
+    mf = mp.family(list(zip(offs.tolist(), nums.tolist())), b, ex, fam.block_elems, fam.dtype, 0)
+    return mf, b, ex
+
+
+def ordered(bits):
+    b = bits.astype(np.int64)
+    return np.where(b & 0x8000, -(b & 0x7FFF), b)
+
+
+def assert_merge_close(fam, got, want, what=""):
+    if fam.dtype == synth.BF16:
+        d = np.abs(ordered(got) - ordered(want))
+        assert d.max(initial=0) <= 1, f"{what}: max ulp diff {d.max()}"
+        n_diff = int((d != 0).sum())
+    else:
+        g, w = got.astype(np.float64), want.astype(np.float64)
+        rel = np.abs(g - w) / np.maximum(np.abs(w), 1e-30)
+        assert np.all((rel <= 1e-6) | (g == w)), f"{what}: max rel {rel.max()}"
+        n_diff = int((got.view(np.uint32) != want.view(np.uint32)).sum())
+    assert n_diff == 0, f"{what}: {n_diff} elements differ from the oracle (within tolerance, but not identical)"
+
+
+def tensor_mask(fam):
+    """bool mask of elements covered by tensors (gap elements are never written)"""
+    offs, nums, total = fam.layout()
+    m = np.zeros(total, bool)
+    for o, n in zip(offs.tolist(), nums.tolist()):
+        m[o:o + n] = True
+    return m
+
+
+def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
+    out = []
+    for k in kinds:
+        if k == "avg":
+            out.append(("avg", mp.make_op(mp.MP_OP_AVG, alpha=[1.0 / K] * K),
+                        oracle.Op(oracle.AVG, K, alpha=[1.0 / K] * K)))
+        elif k == "ta":
+            out.append(("ta", mp.make_op(mp.MP_OP_TA, alpha=[0.3] * K), oracle.Op(oracle.TA, K, alpha=[0.3] * K)))
+        elif k == "ties":
+            out.append(("ties", mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, trim_scope=0),
+                        oracle.Op(oracle.TIES, K, lam=1.0, density=0.2, trim_scope=0)))
+        elif k == "ties1":
+            out.append(("ties1", mp.make_op(mp.MP_OP_TIES, lam=0.7, density=0.35, trim_scope=1),
+                        oracle.Op(oracle.TIES, K, lam=0.7, density=0.35, trim_scope=1)))
+        elif k == "dare":
+            alpha = [1.0 / K] * K
+            out.append(("dare", mp.make_op(mp.MP_OP_DARE, alpha=alpha, drop_p=0.9, seed=1234567),
+                        oracle.Op(oracle.DARE, K, alpha=alpha, drop_p=0.9, seed=1234567)))
+    return out
+
+
+def run_case(fam, base, experts, kinds, fracs, check_merge=True):
+    mf, b, ex = upload(fam, base, experts)
+    covered = tensor_mask(fam)
+    bo, bl, bt = fam.block_table()
+    es = fam.elem_size
+    C_full = fam.K * fam.n_params * es
+    for name, gop, oop in ops_for(fam.K, kinds):
+        scope = oop.trim_scope if oop.kind == oracle.TIES else 0
+        of = oracle_family(fam, base, experts, trim_scope=scope)
+        idx = mp.mp_index_blocks(mf, gop)
+        norm, maxabs, nnz, tau = mp.mp_index_stats(idx)
+        o_norm, o_max, o_nnz = oracle.index(of)
+        assert np.array_equal(nnz, o_nnz), name
+        assert np.array_equal(maxabs.view(np.uint32), o_max.view(np.uint32)), name
+        assert np.array_equal(norm.view(np.uint32), o_norm.view(np.uint32)), name
+        o_tau = None
+        if oop.kind == oracle.TIES:
+            o_tau = oracle.ties_thresholds(of, oop.density)
+            assert np.array_equal(tau, o_tau), name
+        for f in fracs:
+            B = mp.mp_budget_from_fraction(mf, f) if f <= 1.0 else C_full + int(f)
+            assert B == (math.floor(f * C_full) if f <= 1.0 else B)
+            plan = mp.mp_plan(idx, gop, B)
+            pi = mp.mp_plan_info(plan, idx)
+            ng = of.n_groups
+            opl = oracle.plan(fam.K, bl, of.blk_group, ng, es, oop, o_norm, o_max, o_nnz, o_tau, B)
+            what = f"{fam.name}/{name}/f={f}"
+            assert pi["chat"] == opl["chat"] <= B, what
+            assert pi["n_sel"] == opl["n_sel"], what
+            assert pi["n_cand"] == opl["n_cand"], what
+            assert np.array_equal(pi["mask"], opl["mask"]), what
+            assert np.array_equal(pi["order"], opl["order"]), what
+            assert pi["digest"] == opl["digest"], what
+            if not check_merge:
+                plan.free()
+                continue
+            out = torch.full_like(b, float("nan"))
+            man = mp.mp_merge(mf, idx, plan, out)
+            mi = mp.mp_manifest_info(man, fam.K)
+            assert mi["realized_total"] == opl["chat"], what          # Prop. 1, realized = planned
+            assert mi["touched"] == int((opl["mask"] != 0).sum()), what
+            assert mi["digest"] == opl["digest"], what
+            want = oracle.merge(of, oop, tau=o_tau, mask=opl["mask"])
+            got = host(fam, out)
+            assert_merge_close(fam, got[covered], want[covered], what)
+            if f >= 1.0:   # Eq. 5: full budget reproduces the unmasked operator
+                phi = oracle.merge(of, oop, tau=o_tau, mask=None)
+                assert_merge_close(fam, got[covered], phi[covered], what + " vs Phi")
+            man.free()
+            plan.free()
+        idx.free()
+
+
+# ---- families -------------------------------------------------------------------------------------
+
+def fam_ragged_bf16():
+    return synth.custom([5000, 70001, 65536, 8, 131072 + 17, 300, 4096], dtype=synth.BF16, block_elems=4096, K=3,
+                        active_frac=0.5, name="ragged-bf16")
+
+
+def fam_ragged_f32():
+    return synth.custom([4096 * 3 + 5, 1000, 77, 2048], dtype=synth.F32, block_elems=1024, K=5, active_frac=0.4,
+                        name="ragged-f32", log_mu=math.log(1e-3))
+
+
+def fam_k9():
+    return synth.custom([30000, 12345, 65536 * 2 + 100], dtype=synth.BF16, block_elems=8192, K=9, active_frac=0.5,
+                        per_expert_active=True, name="k9")
+
+
+def fam_k17():
+    return synth.custom([20000, 7777, 40000], dtype=synth.BF16, block_elems=2048, K=17, active_frac=0.3,
+                        per_expert_active=True, name="k17")
+
+
+FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
+
+
+@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17], ids=lambda f: f.__name__)
+def test_parity_small_families(make):
+    fam = make()
+    base, experts = fam.host_arrays()
+    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare"), FRACS)
+
+
+def test_parity_tiny_config():
+    """8 fp32 512x512 tensors, K=4: AVG, TIES rho=0.2, DARE p=0.9 at budgets 1.0/0.5/0.25"""
+    fam = synth.tiny()
+    base, experts = fam.host_arrays()
+    run_case(fam, base, experts, ("avg", "ties", "dare"), [1.0, 0.5, 0.25])
+
+
+def test_device_fill_matches_host_fill():
+    fam = fam_k9()
+    base, experts = fam.host_arrays()
+    db, dex = fam.device_arrays()
+    assert np.array_equal(host(fam, db), base)
+    for e, d in zip(experts, dex):
+        assert np.array_equal(host(fam, d), e)
+
+
+# ---- semantics on the GPU -------------------------------------------------------------------------
+
+def test_non_anticipation_unselected_blocks_never_read():
+    """Sec. 2: omitted entries enter only through the mask.  Poison every unselected
+    expert block with NaN after planning: the merged output must not change."""
+    fam = fam_ragged_bf16()
+    base, experts = fam.host_arrays()
+    mf, b, ex = upload(fam, base, experts)
+    bo, bl, _ = fam.block_table()
+    for name, gop, _ in ops_for(fam.K, ("ta", "ties", "dare")):
+        idx = mp.mp_index_blocks(mf, gop)
+        plan = mp.mp_plan(idx, gop, mp.mp_budget_from_fraction(mf, 0.3))
+        mask = mp.mp_plan_info(plan, idx)["mask"]
+        out1 = torch.empty_like(b)
+        mp.mp_merge(mf, idx, plan, out1).free()
+        poisoned = [e.clone() for e in ex]
+        for bb in range(fam.n_blocks):
+            for i in range(fam.K):
+                if not (mask[bb] >> i) & 1:
+                    poisoned[i][int(bo[bb]):int(bo[bb] + bl[bb])] = float("nan")
+        offs, nums, _ = fam.layout()
+        mf2 = mp.family(list(zip(offs.tolist(), nums.tolist())), b, poisoned, fam.block_elems, fam.dtype, 0)
+        out2 = torch.empty_like(b)
+        mp.mp_merge(mf2, idx, plan, out2).free()
+        cov = torch.from_numpy(tensor_mask(fam)).cuda()
+        assert torch.equal(out1.view(torch.int16)[cov], out2.view(torch.int16)[cov]), name
+        assert not torch.isnan(out2[cov].float()).any(), name
+        plan.free()
+        idx.free()
+
+
+def test_nonfinite_delta_reported():
+    fam = synth.custom([9000], dtype=synth.BF16, block_elems=2048, K=2)
+    base, experts = fam.host_arrays()
+    experts[1] = experts[1].copy()
+    experts[1][4321] = 0x7FC0  # NaN
+    mf, b, ex = upload(fam, base, experts)
+    op = mp.make_op(mp.MP_OP_AVG, alpha=[0.5, 0.5])
+    idx = mp.mp_index_blocks(mf, op)
+    with pytest.raises(mp.MergePipeError) as ei:
+        mp.mp_index_stats(idx)
+    assert ei.value.status == -4
+    plan = mp.mp_plan(idx, op, 10 ** 9)
+    with pytest.raises(mp.MergePipeError) as ei:
+        mp.mp_plan_info(plan)
+    assert ei.value.status == -4
+
+
+def test_invalid_arguments_rejected():
+    fam = synth.custom([4096], dtype=synth.BF16, block_elems=1024, K=2)
+    base, experts = fam.host_arrays()
+    mf, b, ex = upload(fam, base, experts)
+    op = mp.make_op(mp.MP_OP_AVG, alpha=[0.5, 0.5])
+    bad = mp.family([(0, 4096)], b, ex, 1004, mp.MP_BF16, 0)       # block size not a multiple of 8
+    with pytest.raises(mp.MergePipeError) as ei:
+        mp.mp_index_blocks(bad, op)
+    assert ei.value.status == -1
+    bad = mp.family([(3, 4000)], b, ex, 1024, mp.MP_BF16, 0)       # tensor not 16-byte aligned
+    with pytest.raises(mp.MergePipeError):
+        mp.mp_index_blocks(bad, op)
+    with pytest.raises(mp.MergePipeError):                          # alpha missing
+        mp.mp_index_blocks(mf, mp.make_op(mp.MP_OP_AVG))
+    idx = mp.mp_index_blocks(mf, op)
+    with pytest.raises(mp.MergePipeError) as ei:                    # TIES plan on a non-TIES index
+        mp.mp_plan(idx, mp.make_op(mp.MP_OP_TIES, density=0.2), 100)
+    assert ei.value.status == -8
+    plan = mp.mp_plan(idx, op, 10 ** 6)
+    with pytest.raises(mp.MergePipeError):                          # out aliases the base
+        mp.mp_merge(mf, idx, plan, b)
+    host_base = torch.zeros_like(b, device="cpu")
+    with pytest.raises(mp.MergePipeError):                          # out on the host
+        mp.mp_merge(mf, idx, plan, host_base)
+
+
+def test_replay_is_bit_identical():
+    """A manifest's plan replayed gives the same bytes (replayable manifests, Sec. 3)."""
+    fam = fam_k9()
+    base, experts = fam.host_arrays()
+    mf, b, ex = upload(fam, base, experts)
+    _, gop, _ = ops_for(fam.K, ("dare",))[0]
+    idx = mp.mp_index_blocks(mf, gop)
+    plan = mp.mp_plan(idx, gop, mp.mp_budget_from_fraction(mf, 0.4))
+    o1, o2 = torch.empty_like(b), torch.empty_like(b)
+    m1 = mp.mp_merge(mf, idx, plan, o1)
+    m2 = mp.mp_merge(mf, idx, plan, o2)
+    cov = torch.from_numpy(tensor_mask(fam)).cuda()   # padding between tensors is never written
+    assert torch.equal(o1.view(torch.int16)[cov], o2.view(torch.int16)[cov])
+    assert mp.mp_manifest_info(m1, fam.K)["digest"] == mp.mp_manifest_info(m2, fam.K)["digest"]
