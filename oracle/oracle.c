@@ -230,17 +230,17 @@ uint64_t orc_splitmix64(uint64_t state) {
 
 /* ---------------------------------------------------------------------------------------
  * Alg. 1 PlanGen (Sec. 3), cost model Eq. 3 and App. A.1.
- *  1. Candidates Q: units (i, b) whose delta can change the output.  Reading: a unit
- *     with nnz = 0 contributes exactly nothing to any operator, and under TIES a unit
- *     whose largest key is below tau is trimmed entirely; both are left out (exact).
- *  2. Score s(i,t,b) = |coef_i| * ||Delta_{i,t,b}||_2 in fp32 (the utility u of Prop. 2);
- *     coef_i = alpha_i (AVG, TA, DARE) or lambda (TIES).
- *  3. Sort by decreasing score; ties by ascending unit id = b*K + i (block order is
- *     tensor/block order, then expert).  The key is unique, so the order is total.
- *  4-9. Greedy fill: take a candidate if C_hat + c <= B, otherwise skip it and go on.
- *     c_{i,t,b} = elements(b) * bytes per element (App. A.1: stored byte length).
- * 10. Record: mask (bit i of word b = A_{i,t,b}), C_hat, number selected, the selected-
- *     block digest and the traversal order.  Reading of the digest: FNV-1a 64 over the
+ *  - Candidates Q: units (i, b) whose delta can change the output.  Reading: a unit
+ *    with nnz = 0 contributes exactly nothing to any operator, and under TIES a unit
+ *    whose largest key is below tau is trimmed entirely; both are left out (exact).
+ *  - Score s(i,t,b) = |coef_i| * ||Delta_{i,t,b}||_2 in fp32 (the utility u of Prop. 2);
+ *    coef_i = alpha_i (AVG, TA, DARE) or lambda (TIES).
+ *  - Sort by decreasing score; ties by ascending unit id = b*K + i (block order is
+ *    tensor/block order, then expert).  The key is unique, so the order is total.
+ *  - Greedy fill: take a candidate if C_hat + c <= B, otherwise skip it and go on.
+ *    c_{i,t,b} = elements(b) * bytes per element (App. A.1: stored byte length).
+ *  - Record: mask (bit i of word b = A_{i,t,b}), C_hat, number selected, the selected-
+ *    block digest and the traversal order.  Reading of the digest: FNV-1a 64 over the
  *     little-endian bytes of (kind, K, alpha[0..K-1] bits, lambda bits, density bits,
  *     trim_scope, drop_p bits, seed, B, C_hat, n_sel, set_hash), where set_hash is the
  *     wrapping sum over selected units u of splitmix64(u).
