@@ -150,6 +150,36 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
 mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out,
                    mp_stream stream, mp_manifest** man);
 
+/*
+ * mp_plan_noalloc — the same access plan as mp_plan, for callers that cannot allocate.
+ * The paper has no counterpart: this is a deployment variant.  Some callers may not call
+ * cudaMalloc or any allocator — code whose device memory must all come from another
+ * framework's arena, latency-critical loops that cannot afford an allocation or the
+ * synchronisation of a free, code running where CUDA allocation calls are not allowed.
+ * This call allocates nothing: every input and output is a caller buffer, and the
+ * planner's scratch is one file-scope device array of 16 MiB that every GPU loading the
+ * library holds until the process exits.
+ *  inputs (device): blk_len[n_blocks], blk_group[n_blocks] (TIES trim group of each
+ *    block; may be NULL unless TIES), norm/maxabs/nnz [K][n_blocks] expert-major as
+ *    mp_index_stats returns them, tau[K][n_groups] (TIES only, else NULL), index_err (one
+ *    uint32 error word of whatever produced the statistics; 0 = fine);
+ *  outputs (device): mask[n_blocks], order[K*n_blocks] (first n_candidates valid),
+ *    summary[8] uint64 = {planned bytes, selected, candidates, selected-unit set hash,
+ *    digest, touched blocks, error word, 0}.  The results equal mp_plan's bit for bit.
+ * Limit: K * n_blocks <= 524288 units; larger requests return MP_ERR_INVALID_ARG and
+ * launch nothing.  The first call on a device looks up the array's device address
+ * (cudaGetSymbolAddress, with that device current); make that first call before any
+ * stream capture.  Every call shares the one array and leaves its contents behind (the
+ * planner clears what must start at zero), so calls whose GPU work overlaps — on
+ * different streams, or from different threads — race and must be serialised by the
+ * caller.  Errors are reported without allocating (mp_last_error returns a literal).
+ */
+mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_groups, mp_dtype dtype,
+                          const uint32_t* blk_len, const uint32_t* blk_group, const float* norm,
+                          const float* maxabs, const uint32_t* nnz, const uint32_t* tau,
+                          const uint32_t* index_err, const mp_op* op, uint64_t budget_bytes,
+                          uint32_t* mask, uint32_t* order, uint64_t* summary, mp_stream stream);
+
 /* Release an mp_index, mp_plan_t or mp_manifest (waits for its pending work).  NULL is a
    no-op.  Passing anything else is undefined. */
 void mp_free(void* handle);

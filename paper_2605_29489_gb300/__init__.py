@@ -24,7 +24,7 @@ __all__ = [
     "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_budget_from_fraction", "mp_last_error",
-    "mp_version", "mp_kernel_launch_count", "lib", "library_path",
+    "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "lib", "library_path",
 ]
 
 MP_OK = 0
@@ -269,3 +269,21 @@ def mp_version() -> str:
 
 def mp_kernel_launch_count() -> int:
     return int(lib().mp_kernel_launch_count())
+
+
+def mp_plan_noalloc(K, n_blocks, n_groups, dtype, blk_len, blk_group, norm, maxabs, nnz, tau, index_err, op: Op,
+                    budget_bytes, mask, order, summary, stream=None):
+    """The plan without any allocation: every argument is a caller device buffer (torch
+    tensors or raw pointers; blk_group and tau may be None).  For callers that must not
+    allocate; the planner's scratch is a fixed 16 MiB device array inside the library."""
+    L = lib()
+    if not getattr(L, "_noalloc_typed", False):
+        vp = ctypes.c_void_p
+        L.mp_plan_noalloc.restype = ctypes.c_int32
+        L.mp_plan_noalloc.argtypes = [ctypes.c_uint32, ctypes.c_uint64, ctypes.c_uint32, ctypes.c_int, vp, vp, vp,
+                                      vp, vp, vp, vp, vp, ctypes.c_uint64, vp, vp, vp, vp]
+        L._noalloc_typed = True
+    opt = lambda t: None if t is None else ctypes.c_void_p(_ptr(t))  # noqa: E731
+    _check(L.mp_plan_noalloc(K, n_blocks, n_groups, dtype, opt(blk_len), opt(blk_group), opt(norm), opt(maxabs),
+                             opt(nnz), opt(tau), opt(index_err), op.ref(), int(budget_bytes), opt(mask), opt(order),
+                             opt(summary), ctypes.c_void_p(_stream_ptr(stream))))

@@ -15,6 +15,7 @@ namespace mp {
 
 namespace {
 thread_local std::string g_last_error;
+thread_local const char* g_static_error = nullptr;  // set instead of g_last_error by allocation-free paths
 std::atomic<uint64_t> g_next_id{1};
 std::atomic<uint64_t> g_launches{0};
 
@@ -51,6 +52,7 @@ void pin_put(void* p, size_t bytes) {
 size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
 
 mp_status fail(mp_status st, const std::string& msg) {
+  g_static_error = nullptr;
   g_last_error = msg;
   return st;
 }
@@ -194,12 +196,18 @@ uint32_t fbits(float f) {
 
 }  // namespace
 
-void set_error(const std::string& msg) { g_last_error = msg; }
+void set_error(const std::string& msg) {
+  g_static_error = nullptr;
+  g_last_error = msg;
+}
+
+void set_static_error(const char* msg) { g_static_error = msg; }
 
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
 
 mp_status cuda_fail(cudaError_t e, const char* what) {
   cudaGetLastError();
+  g_static_error = nullptr;
   g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
   return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
 }
@@ -210,7 +218,7 @@ using namespace mp;
 
 extern "C" {
 
-const char* mp_last_error(void) { return g_last_error.c_str(); }
+const char* mp_last_error(void) { return g_static_error ? g_static_error : g_last_error.c_str(); }
 
 const char* mp_version(void) { return "mergepipe-gb300 0.1 (sm_103a)"; }
 

@@ -118,6 +118,8 @@ void count_launches(uint64_t n);
 
 // ---- error reporting (api.cu) -----------------------------------------------------------
 void set_error(const std::string& msg);
+// records a string literal as the last error without allocating
+void set_static_error(const char* msg);
 mp_status cuda_fail(cudaError_t e, const char* what);
 
 // ---- index (index.cu) -------------------------------------------------------------------
