@@ -47,6 +47,9 @@ def workloads():
         "qwen2.5-0.5b-ta-2l": dict(make=lambda: synth.qwen25_05b(layers=2), op="ta", lam=0.3,
                                    budgets=[1.0, 0.5, 0.25, 0.1],
                                    desc="Qwen2.5-0.5B shapes cut to 2 layers (profiling case), K=8, TA lambda=0.3"),
+        "qwen2.5-0.5b-ties-2l": dict(make=lambda: synth.qwen25_05b(layers=2, K=4), op="ties", density=0.2,
+                                     budgets=[1.0, 0.5, 0.25, 0.1],
+                                     desc="Qwen2.5-0.5B shapes cut to 2 layers (profiling case), K=4, TIES density 0.2"),
         "llama-3-8b-ties": dict(make=lambda: synth.llama3_8b(), op="ties", density=0.2, budgets=[1.0, 0.5, 0.25, 0.1],
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
         "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
@@ -153,7 +156,7 @@ def hbm_peak():
 
 def merge_source_hash() -> str:
     h = hashlib.sha256()
-    for name in ("merge.cu", "philox.cuh", "mp_internal.cuh"):
+    for name in ("merge.cu", "philox.cuh", "tma.cuh"):
         with open(os.path.join(ROOT, "paper_2605_29489_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]

@@ -274,6 +274,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   const size_t o_off = slot(nb * 8), o_len = slot(nb * 4), o_grp = slot(nb * 4);
   const size_t o_norm = slot(U * 4), o_max = slot(U * 4), o_nnz = slot(U * 4), o_tau = slot(KG * 4);
   const size_t o_err = slot(16);
+  const size_t o_work = slot(16);  // the index kernel's work counter
   size_t o_coarse = 0, o_fine = 0, o_kth = 0, o_est = 0, o_rank = 0;
   if (ties) {
     o_coarse = slot(KG * 256 * 8);
@@ -340,6 +341,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   p.maxabs = ix->d_maxabs;
   p.nnz = ix->d_nnz;
   p.err = ix->d_err;
+  p.work = (unsigned long long*)(m + o_work);
   if (ties) {
     p.coarse = (unsigned long long*)(m + o_coarse);
     p.fine = (unsigned long long*)(m + o_fine);
@@ -517,7 +519,8 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
     return fail(MP_ERR_OOM, "pinned host allocation failed");
   }
   auto release_pinned = [&]() { pin_put(mf->h_realized, back_bytes); };
-  if ((st = dev_alloc(mf->mem, back_bytes, cs)) != MP_OK) {
+  // device side: what comes back, then the merge kernel's work counter
+  if ((st = dev_alloc(mf->mem, back_bytes + 16, cs)) != MP_OK) {
     release_pinned();
     delete mf;
     return st;
@@ -564,6 +567,7 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
   }
   p.seed = plan->seed;
   p.realized = mf->d_realized;
+  p.work = reinterpret_cast<unsigned long long*>(static_cast<char*>(mf->mem.ptr) + back_bytes);
   p.err = mf->d_err;
   if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
   if ((e = cudaMemcpyAsync(d_sum_copy, plan->d_summary, 64, cudaMemcpyDeviceToDevice, cs)) != cudaSuccess)

@@ -16,6 +16,7 @@
 #include <cuda_bf16.h>
 
 #include "mp_internal.cuh"
+#include "tma.cuh"
 
 namespace mp {
 namespace {
@@ -68,28 +69,138 @@ __device__ __forceinline__ uint32_t ties_key(float d) {
   return (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(fabsf(d))) & 0x7FFFu;
 }
 
+// ---- the catalog pass: TMA producer / consumer pipeline ---------------------------------
+//
+// Work item = (block, group of up to KG experts); items are handed out through a global
+// counter.  The producer thread streams every 8 KiB chunk of the item's block — the base
+// chunk, then each expert's chunk — into a ring of shared-memory slots (cp.async.bulk,
+// completion on the slot's "full" mbarrier).  Consumer thread l (0..255) is lane l of the
+// fixed summation order: chunk c holds vectors 512c .. 512c+511, and thread l takes
+// vectors 512c+l and 512c+256+l, i.e. exactly its own vectors l, l+256, ... in increasing
+// order.  At the end of the block the 256 lane sums are combined by the xor butterfly.
+constexpr int kIxConsumers = 256;
+constexpr int kIxThreads = kIxConsumers + 32;
+constexpr uint32_t kIxSlotBytes = 8192;
+constexpr int kIxSlots = 12;
+constexpr uint32_t kIxEnd = 0xFFFFFFFFu;
+
+struct IxMeta {
+  uint64_t off;    // element offset of the chunk
+  uint32_t item;   // work item, or kIxEnd
+  uint32_t n;      // elements in the chunk
+  uint32_t last;   // 1 on the block's last chunk
+  uint32_t pad;
+};
+
+template <int KG>
+struct __align__(128) IxSmem {
+  uint8_t slot[kIxSlots][kIxSlotBytes];
+  IxMeta meta[kIxSlots];
+  uint64_t full[kIxSlots];
+  uint64_t empty[kIxSlots];
+  uint32_t hist[KG][256];
+  float red_ss[KG][8];
+  float red_mx[KG][8];
+  uint32_t red_nz[KG][8];
+  uint32_t nnz_tot[KG];
+  uint64_t cbar;  // consumer-only barrier (one arrival per consumer warp)
+  int abort;
+};
+
+template <bool BF16>
+__device__ __forceinline__ void ix_read_vec(const uint8_t* slot, const void* gsrc, uint64_t off, uint32_t k0,
+                                            uint32_t n, uint32_t n_tma, float (&x)[BF16 ? 8 : 4]) {
+  constexpr uint32_t V = BF16 ? 8u : 4u;
+  if (k0 + V <= n_tma) {
+    unpack<BF16>(*reinterpret_cast<const uint4*>(slot + k0 * (BF16 ? 2u : 4u)), x);
+    return;
+  }
+#pragma unroll
+  for (uint32_t e = 0; e < V; ++e) {
+    float v = 0.0f;
+    if (k0 + e < n) {
+      if constexpr (BF16) v = __uint_as_float((uint32_t)(static_cast<const uint16_t*>(gsrc)[off + k0 + e]) << 16);
+      else v = static_cast<const float*>(gsrc)[off + k0 + e];
+    }
+    x[e] = v;
+  }
+}
+
 template <bool BF16, int KG, bool TIES>
-__global__ void __launch_bounds__(256) index_kernel(const IndexLaunch p) {
+__global__ void __launch_bounds__(kIxThreads, 2)
+    index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
+  constexpr uint32_t ES = BF16 ? 2u : 4u;
+  constexpr uint32_t CH = kIxSlotBytes / ES;
   constexpr int V = BF16 ? 8 : 4;
-  __shared__ uint32_t s_hist[TIES ? KG : 1][TIES ? 256 : 1];
-  __shared__ float s_ss[KG][8];
-  __shared__ float s_mx[KG][8];
-  __shared__ uint32_t s_nz[KG][8];
+  constexpr int VPT = (int)(CH / (kIxConsumers * V));
+  static_assert(VPT == 2, "chunk geometry");
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  IxSmem<KG>& S = *reinterpret_cast<IxSmem<KG>*>(smem_raw);
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
+  volatile int* abort_flag = &S.abort;
 
-  const uint32_t G = (p.K + KG - 1) / KG;
-  const uint64_t b = blockIdx.x / G;
-  const uint32_t i0 = (blockIdx.x % G) * KG;
-  const uint32_t kc = min((uint32_t)KG, p.K - i0);
-  const uint64_t off = p.blk_off[b];
-  const uint32_t len = p.blk_len[b];
-  const uint32_t nvec = (len + V - 1) / V;
-  const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
+  if (tid == 0) {
+    for (int s = 0; s < kIxSlots; ++s) {
+      mbar_init(&S.full[s], 1);
+      mbar_init(&S.empty[s], kIxConsumers / 32);
+    }
+    mbar_init(&S.cbar, kIxConsumers / 32);
+    S.abort = 0;
+    mbar_fence_init();
+  }
+  for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += blockDim.x) (&S.hist[0][0])[x] = 0u;
+  __syncthreads();
 
-  if constexpr (TIES) {
-    for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += 256u) (&s_hist[0][0])[x] = 0u;
-    __syncthreads();
+  if (warp == kIxConsumers / 32) {
+    // ---------------- producer ----------------
+    if (lane == 0) {
+      uint32_t fill = 0;
+      bool ok = true;
+      auto produce = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, const void* src,
+                         uint32_t bytes) -> bool {
+        const uint32_t s = fill % kIxSlots, r = fill / kIxSlots;
+        if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+        S.meta[s].off = off;
+        S.meta[s].item = item;
+        S.meta[s].n = n;
+        S.meta[s].last = last;
+        mbar_arrive_expect_tx(&S.full[s], bytes);
+        if (bytes) tma_load_1d(S.slot[s], static_cast<const char*>(src) + off * ES, bytes, &S.full[s]);
+        ++fill;
+        return true;
+      };
+      while (ok) {
+        const unsigned long long it = atomicAdd(work, 1ull);
+        if (it >= n_items) break;
+        const uint64_t b = it / G;
+        const uint32_t i0 = (uint32_t)(it % G) * KG;
+        const uint32_t kc = min((uint32_t)KG, p.K - i0);
+        const uint32_t len = p.blk_len[b];
+        const uint64_t off0 = p.blk_off[b];
+        const uint32_t nch = (len + CH - 1) / CH;
+        for (uint32_t c = 0; c < nch && ok; ++c) {
+          const uint32_t n = min(CH, len - c * CH);
+          const uint64_t off = off0 + (uint64_t)c * CH;
+          const uint32_t bytes = (n * ES) & ~15u;
+          const uint32_t last = c + 1 == nch ? 1u : 0u;
+          ok = produce((uint32_t)it, off, n, last, p.base, bytes);
+          for (uint32_t k = 0; k < kc && ok; ++k) ok = produce((uint32_t)it, off, n, last, p.experts.p[i0 + k], bytes);
+        }
+      }
+      if (ok) ok = produce(kIxEnd, 0, 0, 0, nullptr, 0);
+      if (!ok) {
+        atomicOr(p.err, kErrTimeout);
+        S.abort = 1;
+      }
+      for (uint32_t s = 0; s < (uint32_t)kIxSlots && s < fill; ++s) {
+        const uint32_t lastf = fill - 1 - ((fill - 1 + kIxSlots - s) % kIxSlots);
+        mbar_wait_drain(&S.full[s], (lastf / kIxSlots) & 1u);
+      }
+    }
+    return;
   }
 
+  // ---------------- consumers (lane l of the summation order) ----------------
   float ss[KG], mx[KG];
   uint32_t nz[KG];
 #pragma unroll
@@ -98,91 +209,135 @@ __global__ void __launch_bounds__(256) index_kernel(const IndexLaunch p) {
     mx[k] = 0.0f;
     nz[k] = 0u;
   }
-  uint32_t bad = 0u;
-
-  for (uint32_t v0 = tid; v0 < nvec; v0 += 2u * kLanes) {
-    uint4 rb[2], re[2][KG];
+  uint32_t fill = 0, cphase = 0;
+  bool alive = true;
+  auto wait_full = [&](uint32_t f) -> bool {
+    if (!warp_wait(&S.full[f % kIxSlots], (f / kIxSlots) & 1u, abort_flag)) {
+      atomicOr(p.err, kErrTimeout);
+      S.abort = 1;
+      return false;
+    }
+    return true;
+  };
+  auto release = [&](uint32_t f) {
+    __syncwarp();
+    if (lane == 0) mbar_arrive(&S.empty[f % kIxSlots]);
+  };
+  while (alive) {
+    if (!wait_full(fill)) break;
+    const IxMeta mt = S.meta[fill % kIxSlots];
+    if (mt.item == kIxEnd) break;
+    const uint64_t b = mt.item / G;
+    const uint32_t i0 = (mt.item % G) * KG;
+    const uint32_t kc = min((uint32_t)KG, p.K - i0);
+    const uint32_t n = mt.n, n_tma = ((n * ES) & ~15u) / ES;
+    const uint64_t off = mt.off;
+    float xb[VPT][V];
+    {
+      const uint8_t* slot = S.slot[fill % kIxSlots];
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      uint32_t v = v0 + (uint32_t)u * kLanes;
-      if (v < nvec) {
-        rb[u] = load_vec_raw(p.base, BF16, off, v, len);
-#pragma unroll
-        for (int k = 0; k < KG; ++k)
-          if ((uint32_t)k < kc) re[u][k] = load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len);
-      }
+      for (int u = 0; u < VPT; ++u)
+        ix_read_vec<BF16>(slot, p.base, off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma, xb[u]);
+      release(fill);
+      ++fill;
     }
 #pragma unroll
-    for (int u = 0; u < 2; ++u) {
-      uint32_t v = v0 + (uint32_t)u * kLanes;
-      if (v >= nvec) break;
-      float xb[V];
-      unpack<BF16>(rb[u], xb);
+    for (int k = 0; k < KG; ++k) {
+      if ((uint32_t)k >= kc) break;
+      if (!wait_full(fill)) {
+        alive = false;
+        break;
+      }
+      const uint8_t* slot = S.slot[fill % kIxSlots];
 #pragma unroll
-      for (int k = 0; k < KG; ++k) {
-        if ((uint32_t)k >= kc) continue;
+      for (int u = 0; u < VPT; ++u) {
         float xe[V];
-        unpack<BF16>(re[u][k], xe);
+        ix_read_vec<BF16>(slot, p.experts.p[i0 + k], off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma, xe);
 #pragma unroll
         for (int e = 0; e < V; ++e) {
-          float d = __fsub_rn(xe[e], xb[e]);
+          const float d = __fsub_rn(xe[e], xb[u][e]);
           ss[k] = __fmaf_rn(d, d, ss[k]);
           mx[k] = fmaxf(mx[k], fabsf(d));
           nz[k] += d != 0.0f ? 1u : 0u;
-          bad |= ((__float_as_uint(d) & 0x7F800000u) == 0x7F800000u) ? 1u : 0u;
           if constexpr (TIES) {
-            if (d != 0.0f) atomicAdd(&s_hist[k][ties_key(d) >> 7], 1u);
+            if (d != 0.0f) atomicAdd(&S.hist[k][ties_key(d) >> 7], 1u);
           }
         }
       }
+      release(fill);
+      ++fill;
     }
-  }
+    if (!alive || !mt.last) continue;
 
-  // canonical combine: xor butterfly within each warp, then over the 8 warp sums
-#pragma unroll
-  for (int k = 0; k < KG; ++k) {
-#pragma unroll
-    for (int s = 16; s >= 1; s >>= 1) {
-      ss[k] = __fadd_rn(ss[k], __shfl_xor_sync(0xFFFFFFFFu, ss[k], s));
-      mx[k] = fmaxf(mx[k], __shfl_xor_sync(0xFFFFFFFFu, mx[k], s));
-      nz[k] += __shfl_xor_sync(0xFFFFFFFFu, nz[k], s);
-    }
-    if (lane == 0) {
-      s_ss[k][warp] = ss[k];
-      s_mx[k][warp] = mx[k];
-      s_nz[k][warp] = nz[k];
-    }
-  }
-  if (__syncthreads_or(bad) && tid == 0) atomicOr(p.err, kErrNonfinite);
-  if (warp == 0) {
+    // end of the block: the canonical combine, then the statistics (and TIES bins)
 #pragma unroll
     for (int k = 0; k < KG; ++k) {
-      float a = lane < 8 ? s_ss[k][lane] : 0.0f;
-      float m = lane < 8 ? s_mx[k][lane] : 0.0f;
-      uint32_t c = lane < 8 ? s_nz[k][lane] : 0u;
 #pragma unroll
-      for (int s = 4; s >= 1; s >>= 1) {
-        a = __fadd_rn(a, __shfl_xor_sync(0xFFFFFFFFu, a, s));
-        m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, s));
-        c += __shfl_xor_sync(0xFFFFFFFFu, c, s);
+      for (int s = 16; s >= 1; s >>= 1) {
+        ss[k] = __fadd_rn(ss[k], __shfl_xor_sync(0xFFFFFFFFu, ss[k], s));
+        mx[k] = fmaxf(mx[k], __shfl_xor_sync(0xFFFFFFFFu, mx[k], s));
+        nz[k] += __shfl_xor_sync(0xFFFFFFFFu, nz[k], s);
       }
-      if (lane == 0 && (uint32_t)k < kc) {
-        uint64_t u = (uint64_t)(i0 + k) * p.n_blocks + b;
-        p.norm[u] = __fsqrt_rn(a);
-        p.maxabs[u] = m;
-        p.nnz[u] = c;
-        s_nz[k][0] = c;
+      if (lane == 0) {
+        S.red_ss[k][warp] = ss[k];
+        S.red_mx[k][warp] = mx[k];
+        S.red_nz[k][warp] = nz[k];
+      }
+      ss[k] = 0.0f;
+      mx[k] = 0.0f;
+      nz[k] = 0u;
+    }
+    if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+      atomicOr(p.err, kErrTimeout);
+      S.abort = 1;
+      break;
+    }
+    if (warp == 0) {
+      uint32_t bad = 0u;
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        float a = lane < 8 ? S.red_ss[k][lane] : 0.0f;
+        float m = lane < 8 ? S.red_mx[k][lane] : 0.0f;
+        uint32_t c = lane < 8 ? S.red_nz[k][lane] : 0u;
+#pragma unroll
+        for (int s = 4; s >= 1; s >>= 1) {
+          a = __fadd_rn(a, __shfl_xor_sync(0xFFFFFFFFu, a, s));
+          m = fmaxf(m, __shfl_xor_sync(0xFFFFFFFFu, m, s));
+          c += __shfl_xor_sync(0xFFFFFFFFu, c, s);
+        }
+        if (lane == 0 && (uint32_t)k < kc) {
+          const uint64_t u = (uint64_t)(i0 + k) * p.n_blocks + b;
+          p.norm[u] = __fsqrt_rn(a);
+          p.maxabs[u] = m;
+          p.nnz[u] = c;
+          S.nnz_tot[k] = c;
+          // a NaN delta makes the sum of squares NaN; an infinite one makes max |delta| infinite
+          if (isnan(a) || isinf(m)) bad = 1u;
+        }
+      }
+      if (lane == 0 && bad) atomicOr(p.err, kErrNonfinite);
+    }
+    if constexpr (TIES) {
+      if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+      atomicOr(p.err, kErrTimeout);
+      S.abort = 1;
+      break;
+    }
+      const uint32_t grp = p.blk_group[b];
+      const uint32_t len = p.blk_len[b];
+      for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += kIxConsumers) {
+        const uint32_t k = x >> 8, e = x & 255u;
+        unsigned long long c = S.hist[k][e];
+        S.hist[k][e] = 0u;
+        if (k >= kc) continue;
+        if (e == 0) c += len - S.nnz_tot[k];  // zero deltas have key 0
+        if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + e], c);
       }
     }
-  }
-  if constexpr (TIES) {
-    __syncthreads();
-    const uint32_t grp = p.blk_group[b];
-    for (uint32_t x = tid; x < kc * 256u; x += 256u) {
-      uint32_t k = x >> 8, e = x & 255u;
-      unsigned long long c = s_hist[k][e];
-      if (e == 0) c += len - s_nz[k][0];  // zero deltas have key 0
-      if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + e], c);
+    if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+      atomicOr(p.err, kErrTimeout);
+      S.abort = 1;
+      break;
     }
   }
 }
@@ -295,19 +450,35 @@ __global__ void ties_fine_select(const IndexLaunch p) {
 template <bool BF16, int KG>
 cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   const uint32_t G = (p.K + KG - 1) / KG;
-  const uint64_t grid = p.n_blocks * G;
-  if (grid == 0) return cudaSuccess;
-  if (grid > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+  const uint64_t n_items = p.n_blocks * G;
+  if (n_items == 0) return cudaSuccess;
+  if (n_items > 0x7FFFFFFFull) return cudaErrorInvalidValue;
   const bool ties = p.coarse != nullptr;
-  if (ties) index_kernel<BF16, KG, true><<<(unsigned)grid, 256, 0, st>>>(p);
-  else index_kernel<BF16, KG, false><<<(unsigned)grid, 256, 0, st>>>(p);
+  int dev = 0, sms = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const size_t smem = sizeof(IxSmem<KG>);
+  uint64_t grid = (uint64_t)sms * 2;
+  if (grid > n_items) grid = n_items;
+  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if (ties) {
+    auto k = index_tma_kernel<BF16, KG, true>;
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
+    k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);
+  } else {
+    auto k = index_tma_kernel<BF16, KG, false>;
+    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
+    k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);
+  }
   count_launches(1);
-  cudaError_t e = cudaGetLastError();
+  e = cudaGetLastError();
   if (e != cudaSuccess || !ties) return e;
   const uint64_t nsel = (uint64_t)p.K * p.n_groups;
   const unsigned sgrid = (unsigned)((nsel + 127) / 128);
+  const uint64_t fgrid = p.n_blocks * G;
   ties_coarse_select<<<sgrid, 128, 0, st>>>(p);
-  ties_fine_kernel<BF16, KG><<<(unsigned)grid, 256, 0, st>>>(p);
+  ties_fine_kernel<BF16, KG><<<(unsigned)fgrid, 256, 0, st>>>(p);
   ties_fine_select<<<sgrid, 128, 0, st>>>(p);
   count_launches(3);
   return cudaGetLastError();

@@ -144,6 +144,7 @@ struct IndexLaunch {
   uint32_t* estar;             // [K][n_groups] coarse bin of tau (or 0xFFFFFFFF)
   unsigned long long* rank;    // [K][n_groups] rank of tau inside that bin
   uint32_t* tau;               // [K][n_groups]
+  unsigned long long* work;    // item counter of the dynamic scheduler (zeroed per launch)
 };
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
 
@@ -196,6 +197,7 @@ struct MergeLaunch {
   uint32_t dare_T;      // DARE keep threshold on 16-bit words
   uint64_t seed;
   unsigned long long* realized;  // [kCounterSlots][K]
+  unsigned long long* work;      // chunk counter of the dynamic scheduler (zeroed per launch)
   uint32_t* err;
 };
 cudaError_t launch_merge(const MergeLaunch& p, cudaStream_t st);

@@ -1,0 +1,79 @@
+// Inline-PTX helpers for the bulk-copy pipelines: mbarriers with bounded waits and the
+// 1-D TMA bulk copy global -> shared (cp.async.bulk, completion counted in bytes on an
+// mbarrier).  Every wait here has an iteration limit so that no kernel can hang.
+#pragma once
+
+#include <stdint.h>
+
+namespace mp {
+
+constexpr uint32_t kWaitLimit = 1u << 22;  // try_wait rounds before a wait gives up
+
+__device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
+
+__device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(su32(bar)), "r"(count) : "memory");
+}
+
+__device__ __forceinline__ void mbar_fence_init() {
+  asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(su32(bar)), "r"(bytes) : "memory");
+}
+
+__device__ __forceinline__ void mbar_arrive(uint64_t* bar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(su32(bar)) : "memory");
+}
+
+__device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity)
+      : "memory");
+  return ok != 0;
+}
+
+// bounded wait for the phase with the given parity; false on expiry or when *abort is set
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  for (uint32_t k = 0; k < kWaitLimit; ++k) {
+    if (mbar_try_wait(bar, parity)) return true;
+    if ((k & 255u) == 255u && *abort) return false;
+  }
+  return false;
+}
+
+// bounded wait that ignores the abort flag (drains copies still in flight before exit)
+__device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity) {
+  for (uint32_t k = 0; k < kWaitLimit; ++k)
+    if (mbar_try_wait(bar, parity)) return;
+}
+
+__device__ __forceinline__ void tma_load_1d(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(su32(dst)),
+      "l"(src), "r"(bytes), "r"(su32(bar))
+      : "memory");
+}
+
+// every lane of the warp waits (each acquires the barrier); the outcome is made uniform
+// across the warp so that a give-up never splits a warp
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
+  const bool ok = mbar_wait(bar, parity, abort);
+  return __all_sync(0xFFFFFFFFu, ok);
+}
+
+// barrier over the consumer warps only (bar counts one arrival per warp), with a bounded
+// wait: a warp that has given up cannot leave the others blocked; phase counts the uses
+__device__ __forceinline__ bool consumer_barrier(uint64_t* bar, uint32_t& phase, volatile int* abort) {
+  __syncwarp();
+  if ((threadIdx.x & 31u) == 0) mbar_arrive(bar);
+  const bool ok = warp_wait(bar, phase & 1u, abort);
+  ++phase;
+  return ok;
+}
+
+}  // namespace mp
