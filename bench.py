@@ -54,6 +54,14 @@ def workloads():
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
         "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
                                   desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE p=0.9 then AVG, per-expert active sets"),
+        "llama-3-8b-hostpool-avg": dict(make=lambda: synth.llama3_8b(K=8), op="avg", budgets=[1.0, 0.25, 0.1],
+                                        host_pool=True,
+                                        desc="Llama-3-8B-shaped bf16 base in HBM, K=8 experts (128 GB) in pinned host "
+                                             "memory, AVG, planned blocks gathered over NVLink-C2C"),
+        "llama-3-8b-hostpool-ties": dict(make=lambda: synth.llama3_8b(K=8), op="ties", density=0.2,
+                                         budgets=[1.0, 0.25, 0.1], host_pool=True,
+                                         desc="Llama-3-8B-shaped bf16 base in HBM, K=8 experts (128 GB) in pinned host "
+                                              "memory, TIES density 0.2"),
         "tiny-avg": dict(make=lambda: synth.tiny(), op="avg", budgets=[1.0, 0.5, 0.25],
                          desc="8 fp32 512x512 tensors, K=4, AVG, 4Ki-element blocks"),
     }
@@ -245,9 +253,22 @@ def native(args, rank, world, local_rank):
     gop, _ = make_ops(W, fam.K)
     budgets = W["budgets"]
     base, experts = fam.device_arrays()
+    host_pool = bool(W.get("host_pool"))
+    link = None
+    if host_pool:
+        # the experts live in pinned host memory; only the base (and the output) stay in HBM
+        experts_h = []
+        for e in experts:
+            h = torch.empty(e.shape, dtype=e.dtype, pin_memory=True)
+            h.copy_(e)
+            experts_h.append(h)
+        del e
+        experts = experts_h
+        torch.cuda.empty_cache()
+        link = measure_h2d(experts[0])
     offs, nums, total = fam.layout()
     tensors = list(zip(offs.tolist(), nums.tolist()))
-    mf = mp.family(tensors, base, experts, fam.block_elems, fam.dtype, 0)
+    mf = mp.family(tensors, base, experts, fam.block_elems, fam.dtype, 1 if host_pool else 0)
     es = fam.elem_size
     N = fam.n_params
     free_b, _ = torch.cuda.mem_get_info()
@@ -337,7 +358,7 @@ def native(args, rank, world, local_rank):
 
     # ---- e2e: pinned host inputs in, merged outputs back, inside the timed region ----
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not host_pool:
         base_h = base.cpu().pin_memory()
         experts_h = [e.cpu().pin_memory() for e in experts]
         outs_h = [torch.empty(outs[0].shape, dtype=outs[0].dtype, pin_memory=True) for _ in budgets]
@@ -406,6 +427,11 @@ def native(args, rank, world, local_rank):
                      "algorithmic_bytes": "per merged parameter 2*s + s*(selected experts); summed over the "
                                           "budget sweep's launches / their summed CUDA-event time"},
         "gpu_launches": launches,
+        "host_link": None if link is None else dict(
+            h2d_gbs_measured=link, gathered_bytes=[pb["planned_bytes"] for pb in per_budget],
+            gathered_gbs=[pb["planned_bytes"] / (pb["merge_ms"] / 1e3) / 1e9 for pb in per_budget],
+            frac_of_link=[pb["planned_bytes"] / (pb["merge_ms"] / 1e3) / 1e9 / link for pb in per_budget],
+            index_reads_gbs=fam.K * N * es / (idx_ms / 1e3) / 1e9),
         "clocks": clk,
         "e2e": e2e,
     }
@@ -415,6 +441,24 @@ def native(args, rank, world, local_rank):
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
                                 "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
     return line
+
+
+def measure_h2d(pinned_src) -> float:
+    """host -> device copy bandwidth (GB/s) from the pinned pool: 256 MiB copies, best of 10"""
+    import torch
+
+    n = min(pinned_src.numel(), (256 << 20) // pinned_src.element_size())
+    src = pinned_src[:n]
+    dst = torch.empty(n, dtype=pinned_src.dtype, device="cuda")
+    best = 0.0
+    for _ in range(10):
+        a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a.record()
+        dst.copy_(src, non_blocking=True)
+        b.record()
+        b.synchronize()
+        best = max(best, n * pinned_src.element_size() / (a.elapsed_time(b) / 1e3) / 1e9)
+    return best
 
 
 def _max_over_ranks(x: float, world: int) -> float:

@@ -212,6 +212,194 @@ mp_status cuda_fail(cudaError_t e, const char* what) {
   return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
 }
 
+// ---- experts in pinned host memory: segment pipeline -------------------------------------
+//
+// The family is walked in segments of consecutive blocks (about kSegmentElems elements
+// each).  Two HBM staging buffers alternate: while the kernels of the caller's stream
+// work on segment s, segment s+1 is brought in on a side stream by a gather kernel that
+// reads the host experts over the host mapping — every expert block for the index pass,
+// only the planned (block, expert) pairs for the merge.  The planned blocks are scattered
+// (one copy call per run of consecutive blocks would mean ~10^5 calls per merge), and the
+// kernel reads them at the host link's rate.
+
+namespace {
+
+constexpr uint64_t kSegmentElems = 32ull << 20;
+constexpr int kSide = 2;
+
+struct Segment {
+  uint64_t b0, b1, e0, e1;  // blocks [b0, b1), elements [e0, e1)
+};
+
+std::vector<Segment> make_segments(const std::vector<uint64_t>& off, const std::vector<uint32_t>& len,
+                                   uint64_t& max_span) {
+  std::vector<Segment> segs;
+  max_span = 0;
+  const uint64_t nb = off.size();
+  uint64_t b0 = 0;
+  while (b0 < nb) {
+    uint64_t b1 = b0, acc = 0;
+    while (b1 < nb && (b1 == b0 || acc + len[b1] <= kSegmentElems)) acc += len[b1++];
+    const uint64_t e0 = off[b0], e1 = off[b1 - 1] + len[b1 - 1];
+    segs.push_back({b0, b1, e0, e1});
+    if (e1 - e0 > max_span) max_span = e1 - e0;
+    b0 = b1;
+  }
+  return segs;
+}
+
+struct HostPipe {
+  cudaStream_t main = nullptr;
+  cudaStream_t side[kSide] = {};
+  cudaEvent_t ready[2][kSide] = {};
+  cudaEvent_t freed[2] = {};
+  void* staging = nullptr;
+  size_t per_expert = 0;
+  uint32_t K = 0;
+
+  cudaError_t init(cudaStream_t m, uint32_t k, uint64_t span_elems, uint32_t es) {
+    main = m;
+    K = k;
+    per_expert = align_up(span_elems * es);
+    cudaError_t e;
+    for (int q = 0; q < kSide; ++q)
+      if ((e = cudaStreamCreateWithFlags(&side[q], cudaStreamNonBlocking)) != cudaSuccess) return e;
+    for (int b = 0; b < 2; ++b) {
+      for (int q = 0; q < kSide; ++q)
+        if ((e = cudaEventCreateWithFlags(&ready[b][q], cudaEventDisableTiming)) != cudaSuccess) return e;
+      if ((e = cudaEventCreateWithFlags(&freed[b], cudaEventDisableTiming)) != cudaSuccess) return e;
+    }
+    if ((e = cudaMallocAsync(&staging, 2 * (size_t)K * per_expert, main)) != cudaSuccess) {
+      staging = nullptr;
+      return e;
+    }
+    for (int b = 0; b < 2; ++b)
+      if ((e = cudaEventRecord(freed[b], main)) != cudaSuccess) return e;
+    return cudaSuccess;
+  }
+
+  void* buf(int b, uint32_t i) const { return static_cast<char*>(staging) + ((size_t)b * K + i) * per_expert; }
+
+  // side streams may fill buffer b once the caller's stream has finished with it
+  cudaError_t side_acquire(int b) {
+    cudaError_t e;
+    for (int q = 0; q < kSide; ++q)
+      if ((e = cudaStreamWaitEvent(side[q], freed[b], 0)) != cudaSuccess) return e;
+    return cudaSuccess;
+  }
+
+  // the caller's stream may use buffer b once the side streams have filled it
+  cudaError_t main_acquire(int b) {
+    cudaError_t e;
+    for (int q = 0; q < kSide; ++q) {
+      if ((e = cudaEventRecord(ready[b][q], side[q])) != cudaSuccess) return e;
+      if ((e = cudaStreamWaitEvent(main, ready[b][q], 0)) != cudaSuccess) return e;
+    }
+    return cudaSuccess;
+  }
+
+  cudaError_t main_release(int b) { return cudaEventRecord(freed[b], main); }
+
+  // everything the side streams did precedes the caller stream's last wait, so the
+  // staging memory can be returned in the caller's stream order
+  void finish() {
+    if (staging) cudaFreeAsync(staging, main);
+    staging = nullptr;
+    for (int b = 0; b < 2; ++b) {
+      for (int q = 0; q < kSide; ++q)
+        if (ready[b][q]) cudaEventDestroy(ready[b][q]);
+      if (freed[b]) cudaEventDestroy(freed[b]);
+    }
+    for (int q = 0; q < kSide; ++q)
+      if (side[q]) cudaStreamDestroy(side[q]);
+  }
+};
+
+}  // namespace
+
+cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs) {
+  uint64_t span = 0;
+  const std::vector<Segment> segs = make_segments(ix->h_blk_off, ix->h_blk_len, span);
+  const uint32_t es = ix->g.elem_size;
+  HostPipe hp;
+  cudaError_t e = hp.init(cs, p.K, span, es);
+  for (size_t s = 0; s < segs.size() && e == cudaSuccess; ++s) {
+    const int b = (int)(s & 1);
+    const Segment& g = segs[s];
+    if ((e = hp.side_acquire(b)) != cudaSuccess) break;
+    // every expert block of the segment, read over the host mapping by a copy kernel: on
+    // GB300 this reaches the host link's rate where 64 MiB cudaMemcpyAsync copies on two
+    // side streams reached about 60 % of it
+    GatherLaunch gl;
+    memset(&gl, 0, sizeof(gl));
+    gl.K = p.K;
+    gl.elem_size = es;
+    gl.b_begin = g.b0;
+    gl.b_end = g.b1;
+    gl.origin = g.e0;
+    gl.blk_off = p.blk_off;
+    gl.blk_len = p.blk_len;
+    gl.mask = nullptr;
+    gl.src = p.experts;
+    for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
+    if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
+    if ((e = hp.main_acquire(b)) != cudaSuccess) break;
+    IndexLaunch ps = p;
+    ps.b_begin = g.b0;
+    ps.b_end = g.b1;
+    ps.expert_origin = g.e0;
+    ps.defer_ties_select = 1;
+    for (uint32_t i = 0; i < p.K; ++i) ps.experts.p[i] = hp.buf(b, i);
+    if ((e = launch_index(ps, cs)) != cudaSuccess) break;
+    e = hp.main_release(b);
+  }
+  if (e == cudaSuccess && p.coarse) {
+    // the second level of the TIES select reads the host experts directly (fewer blocks)
+    p.b_begin = 0;
+    p.b_end = p.n_blocks;
+    p.expert_origin = 0;
+    e = launch_ties_finish(p, cs);
+  }
+  hp.finish();
+  return e;
+}
+
+cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs) {
+  uint64_t span = 0;
+  const std::vector<Segment> segs = make_segments(ix->h_blk_off, ix->h_blk_len, span);
+  const uint32_t es = ix->g.elem_size;
+  HostPipe hp;
+  cudaError_t e = hp.init(cs, p.K, span, es);
+  for (size_t s = 0; s < segs.size() && e == cudaSuccess; ++s) {
+    const int b = (int)(s & 1);
+    const Segment& g = segs[s];
+    if ((e = hp.side_acquire(b)) != cudaSuccess) break;
+    GatherLaunch gl;
+    memset(&gl, 0, sizeof(gl));
+    gl.K = p.K;
+    gl.elem_size = es;
+    gl.b_begin = g.b0;
+    gl.b_end = g.b1;
+    gl.origin = g.e0;
+    gl.blk_off = p.blk_off;
+    gl.blk_len = p.blk_len;
+    gl.mask = p.mask;
+    gl.src = p.experts;
+    for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
+    if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
+    if ((e = hp.main_acquire(b)) != cudaSuccess) break;
+    MergeLaunch ps = p;
+    ps.b_begin = g.b0;
+    ps.b_end = g.b1;
+    ps.expert_origin = g.e0;
+    ps.experts = gl.dst;
+    if ((e = launch_merge(ps, cs)) != cudaSuccess) break;
+    e = hp.main_release(b);
+  }
+  hp.finish();
+  return e;
+}
+
 }  // namespace mp
 
 using namespace mp;
@@ -354,7 +542,16 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     if ((e = cudaMemcpyAsync((void*)p.kth, h_kth.data(), n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
       return bail(e, "k copy");
   }
-  if ((e = launch_index(p, cs)) != cudaSuccess) return bail(e, "index kernels");
+  p.b_begin = 0;
+  p.b_end = nb;
+  p.expert_origin = 0;
+  if (family->experts_location == 0) {
+    if ((e = launch_index(p, cs)) != cudaSuccess) return bail(e, "index kernels");
+  } else {
+    ix->h_blk_off = h_off;
+    ix->h_blk_len = h_len;
+    if ((e = index_host_pool(p, ix, cs)) != cudaSuccess) return bail(e, "index (host pool)");
+  }
   if ((e = cudaEventCreateWithFlags(&ix->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
   if ((e = cudaEventRecord(ix->done, cs)) != cudaSuccess) return bail(e, "event record");
   *out = ix;
@@ -569,7 +766,16 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
   p.realized = mf->d_realized;
   p.work = reinterpret_cast<unsigned long long*>(static_cast<char*>(mf->mem.ptr) + back_bytes);
   p.err = mf->d_err;
-  if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
+  p.b_begin = 0;
+  p.b_end = g.n_blocks;
+  p.expert_origin = 0;
+  if (family->experts_location == 0) {
+    if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
+  } else {
+    if (index->h_blk_off.size() != g.n_blocks)
+      return bail(cudaErrorInvalidValue, "an index of a host-resident pool is needed for a host-pool merge");
+    if ((e = merge_host_pool(p, index, cs)) != cudaSuccess) return bail(e, "merge (host pool)");
+  }
   if ((e = cudaMemcpyAsync(d_sum_copy, plan->d_summary, 64, cudaMemcpyDeviceToDevice, cs)) != cudaSuccess)
     return bail(e, "summary copy");
   if ((e = cudaMemcpyAsync(mf->h_realized, mf->mem.ptr, back_bytes, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)

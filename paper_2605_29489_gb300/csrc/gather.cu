@@ -1,0 +1,60 @@
+// Host-resident expert pool: the gather stage of Alg. 2 (DeltaIterator materialising only
+// the selected deltas, Sec. 3 "Executor").  For a range of blocks it copies exactly the
+// planned (block, expert) pairs (or, with no mask, every expert block: the index pass) — read from the experts' pinned host memory through the
+// host mapping, i.e. over NVLink-C2C on GB300 — into HBM staging buffers laid out like the
+// flat checkpoint from element `origin` on.  The mask is read on the device, so the gather
+// needs no host synchronisation; unselected expert blocks are never touched (the realized
+// reads stay within the plan, Prop. 1).  One CTA per block; four 16-byte loads in flight
+// per thread.
+#include "mp_internal.cuh"
+
+namespace mp {
+namespace {
+
+constexpr int kThreads = 256;
+constexpr int kUnroll = 4;
+
+__global__ void __launch_bounds__(kThreads) gather_kernel(const GatherLaunch g) {
+  const uint64_t b = g.b_begin + blockIdx.x;
+  if (b >= g.b_end) return;
+  const uint32_t all = g.K >= 32 ? 0xFFFFFFFFu : ((1u << g.K) - 1u);
+  const uint32_t m = g.mask ? g.mask[b] : all;
+  if (m == 0u) return;
+  const uint64_t off = g.blk_off[b];
+  const uint64_t bytes = (uint64_t)g.blk_len[b] * g.elem_size;
+  const uint64_t nvec = bytes / 16u;
+  const uint32_t tail = (uint32_t)(bytes % 16u);
+  unsigned long long copied = 0;
+  for (uint32_t mm = m; mm; mm &= mm - 1u) {
+    const uint32_t i = __ffs(mm) - 1u;
+    const char* src = static_cast<const char*>(g.src.p[i]) + off * g.elem_size;
+    char* dst = static_cast<char*>(const_cast<void*>(g.dst.p[i])) + (off - g.origin) * g.elem_size;
+    const uint4* s4 = reinterpret_cast<const uint4*>(src);
+    uint4* d4 = reinterpret_cast<uint4*>(dst);
+    for (uint64_t v = threadIdx.x; v < nvec; v += (uint64_t)kUnroll * kThreads) {
+      uint4 r[kUnroll];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u)
+        if (v + (uint64_t)u * kThreads < nvec) r[u] = s4[v + (uint64_t)u * kThreads];
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u)
+        if (v + (uint64_t)u * kThreads < nvec) d4[v + (uint64_t)u * kThreads] = r[u];
+    }
+    if (threadIdx.x < tail) dst[nvec * 16u + threadIdx.x] = src[nvec * 16u + threadIdx.x];
+    copied += bytes;
+  }
+  if (threadIdx.x == 0 && g.gathered) atomicAdd(g.gathered, copied);
+}
+
+}  // namespace
+
+cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st) {
+  const uint64_t nb = g.b_end - g.b_begin;
+  if (nb == 0) return cudaSuccess;
+  if (nb > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+  gather_kernel<<<(unsigned)nb, kThreads, 0, st>>>(g);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+}  // namespace mp

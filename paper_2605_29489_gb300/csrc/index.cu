@@ -156,7 +156,7 @@ __global__ void __launch_bounds__(kIxThreads, 2)
     if (lane == 0) {
       uint32_t fill = 0;
       bool ok = true;
-      auto produce = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, const void* src,
+      auto produce = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, const char* src_row,
                          uint32_t bytes) -> bool {
         const uint32_t s = fill % kIxSlots, r = fill / kIxSlots;
         if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
@@ -165,14 +165,14 @@ __global__ void __launch_bounds__(kIxThreads, 2)
         S.meta[s].n = n;
         S.meta[s].last = last;
         mbar_arrive_expect_tx(&S.full[s], bytes);
-        if (bytes) tma_load_1d(S.slot[s], static_cast<const char*>(src) + off * ES, bytes, &S.full[s]);
+        if (bytes) tma_load_1d(S.slot[s], src_row, bytes, &S.full[s]);
         ++fill;
         return true;
       };
       while (ok) {
         const unsigned long long it = atomicAdd(work, 1ull);
         if (it >= n_items) break;
-        const uint64_t b = it / G;
+        const uint64_t b = p.b_begin + it / G;
         const uint32_t i0 = (uint32_t)(it % G) * KG;
         const uint32_t kc = min((uint32_t)KG, p.K - i0);
         const uint32_t len = p.blk_len[b];
@@ -183,8 +183,10 @@ __global__ void __launch_bounds__(kIxThreads, 2)
           const uint64_t off = off0 + (uint64_t)c * CH;
           const uint32_t bytes = (n * ES) & ~15u;
           const uint32_t last = c + 1 == nch ? 1u : 0u;
-          ok = produce((uint32_t)it, off, n, last, p.base, bytes);
-          for (uint32_t k = 0; k < kc && ok; ++k) ok = produce((uint32_t)it, off, n, last, p.experts.p[i0 + k], bytes);
+          ok = produce((uint32_t)it, off, n, last, static_cast<const char*>(p.base) + off * ES, bytes);
+          for (uint32_t k = 0; k < kc && ok; ++k)
+            ok = produce((uint32_t)it, off, n, last,
+                         static_cast<const char*>(p.experts.p[i0 + k]) + (off - p.expert_origin) * ES, bytes);
         }
       }
       if (ok) ok = produce(kIxEnd, 0, 0, 0, nullptr, 0);
@@ -227,7 +229,7 @@ __global__ void __launch_bounds__(kIxThreads, 2)
     if (!wait_full(fill)) break;
     const IxMeta mt = S.meta[fill % kIxSlots];
     if (mt.item == kIxEnd) break;
-    const uint64_t b = mt.item / G;
+    const uint64_t b = p.b_begin + mt.item / G;
     const uint32_t i0 = (mt.item % G) * KG;
     const uint32_t kc = min((uint32_t)KG, p.K - i0);
     const uint32_t n = mt.n, n_tma = ((n * ES) & ~15u) / ES;
@@ -252,7 +254,8 @@ __global__ void __launch_bounds__(kIxThreads, 2)
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
         float xe[V];
-        ix_read_vec<BF16>(slot, p.experts.p[i0 + k], off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma, xe);
+        ix_read_vec<BF16>(slot, p.experts.p[i0 + k], off - p.expert_origin, (tid + (uint32_t)u * kIxConsumers) * V, n,
+                          n_tma, xe);
 #pragma unroll
         for (int e = 0; e < V; ++e) {
           const float d = __fsub_rn(xe[e], xb[u][e]);
@@ -447,10 +450,26 @@ __global__ void ties_fine_select(const IndexLaunch p) {
   p.tau[x] = es << 7;
 }
 
+// the TIES threshold from the coarse bins of the whole family: select the bin, count
+// the lower key bits inside it (a second pass over the blocks that can reach it; experts
+// addressed with origin 0), select the threshold
+template <bool BF16, int KG>
+cudaError_t ties_finish_t(const IndexLaunch& p, cudaStream_t st) {
+  const uint32_t G = (p.K + KG - 1) / KG;
+  const uint64_t nsel = (uint64_t)p.K * p.n_groups;
+  const unsigned sgrid = (unsigned)((nsel + 127) / 128);
+  const uint64_t fgrid = p.n_blocks * G;
+  ties_coarse_select<<<sgrid, 128, 0, st>>>(p);
+  ties_fine_kernel<BF16, KG><<<(unsigned)fgrid, 256, 0, st>>>(p);
+  ties_fine_select<<<sgrid, 128, 0, st>>>(p);
+  count_launches(3);
+  return cudaGetLastError();
+}
+
 template <bool BF16, int KG>
 cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   const uint32_t G = (p.K + KG - 1) / KG;
-  const uint64_t n_items = p.n_blocks * G;
+  const uint64_t n_items = (p.b_end - p.b_begin) * G;
   if (n_items == 0) return cudaSuccess;
   if (n_items > 0x7FFFFFFFull) return cudaErrorInvalidValue;
   const bool ties = p.coarse != nullptr;
@@ -473,15 +492,8 @@ cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   }
   count_launches(1);
   e = cudaGetLastError();
-  if (e != cudaSuccess || !ties) return e;
-  const uint64_t nsel = (uint64_t)p.K * p.n_groups;
-  const unsigned sgrid = (unsigned)((nsel + 127) / 128);
-  const uint64_t fgrid = p.n_blocks * G;
-  ties_coarse_select<<<sgrid, 128, 0, st>>>(p);
-  ties_fine_kernel<BF16, KG><<<(unsigned)fgrid, 256, 0, st>>>(p);
-  ties_fine_select<<<sgrid, 128, 0, st>>>(p);
-  count_launches(3);
-  return cudaGetLastError();
+  if (e != cudaSuccess || !ties || p.defer_ties_select) return e;
+  return ties_finish_t<BF16, KG>(p, st);
 }
 
 template <bool BF16>
@@ -496,6 +508,14 @@ cudaError_t launch_dtype(const IndexLaunch& p, cudaStream_t st) {
 
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st) {
   return p.dtype == MP_BF16 ? launch_dtype<true>(p, st) : launch_dtype<false>(p, st);
+}
+
+cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st) {
+  const bool bf = p.dtype == MP_BF16;
+  if (p.K <= 1) return bf ? ties_finish_t<true, 1>(p, st) : ties_finish_t<false, 1>(p, st);
+  if (p.K <= 2) return bf ? ties_finish_t<true, 2>(p, st) : ties_finish_t<false, 2>(p, st);
+  if (p.K <= 4) return bf ? ties_finish_t<true, 4>(p, st) : ties_finish_t<false, 4>(p, st);
+  return bf ? ties_finish_t<true, 8>(p, st) : ties_finish_t<false, 8>(p, st);
 }
 
 }  // namespace mp

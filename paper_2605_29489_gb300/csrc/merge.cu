@@ -162,7 +162,7 @@ __global__ void __launch_bounds__(kThreads, 2)
       uint32_t fill = 0;
       bool ok = true;
       auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t grp,
-                         const void* src, uint32_t bytes) -> bool {
+                         const char* src_row, uint32_t bytes) -> bool {
         const uint32_t s = fill % kSlots, r = fill / kSlots;
         if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
         S.meta[s].off = off;
@@ -173,7 +173,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         S.meta[s].grp = grp;
         S.meta[s].tau = (OPC == OP_TIES && which > 0) ? p.tau[(uint64_t)(which - 1) * p.n_groups + grp] : 0u;
         mbar_arrive_expect_tx(&S.full[s], bytes);
-        if (bytes) tma_load_1d(S.slot[s], static_cast<const char*>(src) + off * ES, bytes, &S.full[s]);
+        if (bytes) tma_load_1d(S.slot[s], src_row, bytes, &S.full[s]);
         ++fill;
         return true;
       };
@@ -182,7 +182,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         if (q0 >= n_chunks) break;
         const unsigned long long q1 = min(q0 + kGrab, (unsigned long long)n_chunks);
         for (unsigned long long q = q0; q < q1 && ok; ++q) {
-          const uint64_t b = q / cpb;
+          const uint64_t b = p.b_begin + q / cpb;
           const uint32_t start = (uint32_t)(q % cpb) * CH;
           const uint32_t len = p.blk_len[b];
           if (start >= len) continue;
@@ -191,10 +191,11 @@ __global__ void __launch_bounds__(kThreads, 2)
           const uint32_t m = p.mask[b];
           const uint32_t grp = OPC == OP_TIES ? p.blk_group[b] : 0u;
           const uint32_t bytes = (n * ES) & ~15u;
-          ok = produce((uint32_t)q, 0, off, n, m, grp, p.base, bytes);
+          ok = produce((uint32_t)q, 0, off, n, m, grp, static_cast<const char*>(p.base) + off * ES, bytes);
           for (uint32_t mm = m; ok && mm; mm &= mm - 1) {
             const uint32_t i = __ffs(mm) - 1;
-            ok = produce((uint32_t)q, 1 + i, off, n, m, grp, p.experts.p[i], bytes);
+            ok = produce((uint32_t)q, 1 + i, off, n, m, grp,
+                         static_cast<const char*>(p.experts.p[i]) + (off - p.expert_origin) * ES, bytes);
             S.realized[i] += (unsigned long long)n * ES;
           }
         }
@@ -258,7 +259,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
-          read_vec<BF16>(slot, src, off, k0, n, n_tma, xe);
+          read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
 #pragma unroll
           for (int e = 0; e < V; ++e) {
             const float d = __fsub_rn(xe[e], x0[u][e]);
@@ -278,7 +279,7 @@ __global__ void __launch_bounds__(kThreads, 2)
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
-          read_vec<BF16>(slot, src, off, k0, n, n_tma, xe);
+          read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
           uint32_t keep = 0xFFu;
           if constexpr (OPC == OP_DARE) {
             const uint64_t j0 = off + k0;
@@ -325,7 +326,7 @@ template <bool BF16, int OPC>
 cudaError_t launch_op(const MergeLaunch& p, cudaStream_t st) {
   const uint32_t chunk = Geo<OPC>::kSlotBytes / (BF16 ? 2u : 4u);
   const uint32_t cpb = (p.block_elems + chunk - 1) / chunk;
-  const uint64_t n_chunks = p.n_blocks * cpb;
+  const uint64_t n_chunks = (p.b_end - p.b_begin) * cpb;
   if (n_chunks == 0) return cudaSuccess;
   if (n_chunks >= 0xFFFFFFFFull) return cudaErrorInvalidValue;
   int dev = 0, sms = 0;

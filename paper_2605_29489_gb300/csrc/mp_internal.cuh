@@ -73,6 +73,8 @@ struct mp_index_s {
   uint32_t* d_tau;         // [K][n_groups] (TIES only)
   uint32_t* d_err;         // error word
   cudaEvent_t done;
+  std::vector<uint64_t> h_blk_off;  // host copy of the block table (segments of a host pool)
+  std::vector<uint32_t> h_blk_len;
 };
 
 struct mp_plan_s {
@@ -145,8 +147,14 @@ struct IndexLaunch {
   unsigned long long* rank;    // [K][n_groups] rank of tau inside that bin
   uint32_t* tau;               // [K][n_groups]
   unsigned long long* work;    // item counter of the dynamic scheduler (zeroed per launch)
+  // the launch covers blocks [b_begin, b_end); expert pointers address element
+  // expert_origin of the flat layout (0 for resident experts, a segment start when they
+  // point into a staging buffer)
+  uint64_t b_begin, b_end, expert_origin;
+  int defer_ties_select;  // 1: leave the TIES selection to launch_ties_finish
 };
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
+cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st);
 
 // ---- plan (plan.cu) ---------------------------------------------------------------------
 struct PlanLaunch {
@@ -199,7 +207,25 @@ struct MergeLaunch {
   unsigned long long* realized;  // [kCounterSlots][K]
   unsigned long long* work;      // chunk counter of the dynamic scheduler (zeroed per launch)
   uint32_t* err;
+  uint64_t b_begin, b_end, expert_origin;  // as in IndexLaunch
 };
 cudaError_t launch_merge(const MergeLaunch& p, cudaStream_t st);
+
+// ---- host-pool gather (gather.cu) ---------------------------------------------------------
+// copies the planned (block, expert) pairs of blocks [b_begin, b_end) from the experts'
+// pinned host memory into staging buffers laid out like the flat checkpoint from element
+// `origin` on
+struct GatherLaunch {
+  uint32_t K;
+  uint32_t elem_size;
+  uint64_t b_begin, b_end, origin;
+  const uint64_t* blk_off;
+  const uint32_t* blk_len;
+  const uint32_t* mask;   // the access mask of the plan; NULL copies every expert block
+  ExpertPtrs src;         // device views of the host experts
+  ExpertPtrs dst;         // staging buffers
+  unsigned long long* gathered;  // bytes copied, accumulated (may be NULL)
+};
+cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st);
 
 }  // namespace mp

@@ -35,11 +35,18 @@ def host(fam, t):
     return t.cpu().numpy()
 
 
-def upload(fam, base, experts):
+def pinned(fam, a):
+    t = torch.from_numpy(a.view(np.int16) if fam.dtype == synth.BF16 else a).pin_memory()
+    return t.view(torch.bfloat16) if fam.dtype == synth.BF16 else t
+
+
+def upload(fam, base, experts, host_experts=False):
+    """base on the GPU; experts on the GPU, or in pinned host memory (a host-resident pool)"""
     b = dev(fam, base)
-    ex = [dev(fam, e) for e in experts]
+    ex = [pinned(fam, e) if host_experts else dev(fam, e) for e in experts]
     offs, nums, _ = fam.layout()
-    mf = mp.family(list(zip(offs.tolist(), nums.tolist())), b, ex, fam.block_elems, fam.dtype, 0)
+    mf = mp.family(list(zip(offs.tolist(), nums.tolist())), b, ex, fam.block_elems, fam.dtype,
+                   1 if host_experts else 0)
     return mf, b, ex
 
 
@@ -91,8 +98,8 @@ def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
     return out
 
 
-def run_case(fam, base, experts, kinds, fracs, check_merge=True):
-    mf, b, ex = upload(fam, base, experts)
+def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=False):
+    mf, b, ex = upload(fam, base, experts, host_experts)
     covered = tensor_mask(fam)
     bo, bl, bt = fam.block_table()
     es = fam.elem_size
