@@ -1,83 +1,78 @@
-// Alg. 1 PlanGen on the device.
+// Alg. 1 PlanGen on the device, as one cooperative persistent kernel.
 //
-//  1. score: unit u = b*K + i is a candidate iff nnz > 0 (TIES: and key(maxabs) >= tau);
-//     score = |coef_i| * norm (fp32), sort key = ~bits(score) so ascending key order is
-//     decreasing score;
-//  2. stable compaction of the candidates in unit order (so equal scores stay in
-//     ascending unit order);
-//  3. stable LSD radix sort of (key, unit) pairs, four 8-bit digits; stability plus the
-//     unit-ordered input gives the total order (score desc, unit asc);
-//  4. inclusive prefix sum of the costs in that order; every position before the first
-//     prefix > B is selected (the greedy takes them all);
-//  5. after that first overflow only candidates with cost <= the remaining budget R0 can
-//     ever be taken (R only shrinks): they are compacted and one warp runs the greedy
-//     with skip over them in order;
-//  6. the mask, the set hash and the count are scattered from the selected positions,
-//     then the last CTA computes the touched-block count and the digest.
+// The grid's CTAs all stay resident (cooperative launch) and move through the phases
+// below together, separated by grid barriers whose waits are bounded.  Every phase
+// gives CTA c a contiguous slice of the data, so order is preserved wherever it matters.
+//
+//  A  score: unit u = b*K + i is a candidate iff nnz > 0 (TIES: and key(maxabs) >= tau);
+//     score = |coef_i| * norm (fp32); sort key = ~bits(score), so ascending key order is
+//     decreasing score.  Each CTA counts the candidates of its unit slice.
+//  B  stable compaction of the candidates in unit order (so equal scores stay in
+//     ascending unit order).
+//  C  stable LSD radix sort of (key, unit) pairs, four 8-bit digits; a digit that is the
+//     same for every key is skipped.  Stability plus the unit-ordered input gives the
+//     total order (score desc, unit asc).
+//  D  costs in that order: every position before the first prefix sum > B is selected.
+//  E  after that first overflow only candidates with cost <= the remaining budget R0 can
+//     ever be taken (R only shrinks): they are compacted, then one warp of CTA 0 runs the
+//     greedy with skip over them in order, from shared memory.
+//  F  the mask, the set hash and the count are scattered from the selected positions;
+//     the last CTA counts touched blocks and computes the digest.
 #include "mp_internal.cuh"
 
 namespace mp {
 namespace {
 
-constexpr int kThreads = 256;
-constexpr int kItems = 8;
-constexpr uint32_t kTile = kThreads * kItems;  // 2048
-constexpr uint32_t kNone = 0xFFFFFFFFu;
+constexpr int kPT = 256;            // threads per CTA
+constexpr uint32_t kMaxGrid = 1024;  // upper bound of the cooperative grid (scratch sizing)
+constexpr uint32_t kTailChunk = 4096;
+constexpr uint32_t kBarrierLimit = 1u << 24;
 
-// summary words (plan handle) and scratch scalars
+// summary words (plan handle)
 enum { S_CHAT = 0, S_NSEL = 1, S_NCAND = 2, S_SETHASH = 3, S_DIGEST = 4, S_TOUCHED = 5, S_ERR = 6 };
-enum { X_Q = 0, X_P = 1, X_L = 2, X_R0 = 3, X_PREFIX_BEFORE_P = 4, X_TAILSUM = 5, X_DONE = 6, X_COUNT = 8 };
+// scratch scalars
+enum { X_BAR_COUNT = 0, X_BAR_GEN = 1, X_P = 2, X_PBP = 3, X_TAILSUM = 4, X_DONE = 5, X_TOTAL = 6, X_COUNT = 8 };
+
+constexpr unsigned long long kNoP = ~0ull;
 
 struct Scratch {
-  uint8_t* flag;        // [U] candidate flag in unit order
-  uint32_t* key;        // [U] sort key in unit order
-  uint32_t* keys_a;     // [U]
-  uint32_t* keys_b;     // [U]
-  uint32_t* vals_b;     // [U]
-  uint32_t* tile_a;     // [n_tiles]
-  uint32_t* thist;      // [256 * n_tiles]
-  unsigned long long* prefix;   // [U]
-  unsigned long long* tile64;   // [n_tiles]
-  uint32_t* tail;       // [U]
-  uint8_t* tailsel;     // [U]
+  uint32_t* keys_a;             // [U]
+  uint32_t* keys_b;             // [U]
+  uint32_t* vals_b;             // [U]
+  uint32_t* tail_pos;           // [U]
+  uint8_t* tailsel;             // [U]
+  uint32_t* hist;               // [256][kMaxGrid]
+  uint32_t* tot;                // [256]
+  unsigned long long* cta_a;    // [kMaxGrid]
+  unsigned long long* cta_b;    // [kMaxGrid]
   unsigned long long* x;        // [X_COUNT]
 };
 
 inline size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
 
-Scratch carve(void* base, uint64_t U) {
-  const uint64_t nt = (U + kTile - 1) / kTile;
+size_t carve(void* base, uint64_t U, Scratch* s) {
   char* p = static_cast<char*>(base);
-  Scratch s;
   size_t o = 0;
   auto take = [&](size_t bytes) { char* r = p + o; o += align_up(bytes); return r; };
-  s.flag = (uint8_t*)take(U);
-  s.key = (uint32_t*)take(U * 4);
-  s.keys_a = (uint32_t*)take(U * 4);
-  s.keys_b = (uint32_t*)take(U * 4);
-  s.vals_b = (uint32_t*)take(U * 4);
-  s.tile_a = (uint32_t*)take(nt * 4);
-  s.thist = (uint32_t*)take(nt * 256 * 4);
-  s.prefix = (unsigned long long*)take(U * 8);
-  s.tile64 = (unsigned long long*)take(nt * 8);
-  s.tail = (uint32_t*)take(U * 4);
-  s.tailsel = (uint8_t*)take(U);
-  s.x = (unsigned long long*)take(X_COUNT * 8);
-  return s;
-}
-
-size_t carve_bytes(uint64_t U) {
-  const uint64_t nt = (U + kTile - 1) / kTile;
-  return align_up(U) + 4 * align_up(U * 4) + align_up(nt * 4) + align_up(nt * 256 * 4) + align_up(U * 8) +
-         align_up(nt * 8) + align_up(U * 4) + align_up(U) + align_up(X_COUNT * 8);
+  Scratch t;
+  t.keys_a = (uint32_t*)take(U * 4);
+  t.keys_b = (uint32_t*)take(U * 4);
+  t.vals_b = (uint32_t*)take(U * 4);
+  t.tail_pos = (uint32_t*)take(U * 4);
+  t.tailsel = (uint8_t*)take(U);
+  t.hist = (uint32_t*)take((size_t)256 * kMaxGrid * 4);
+  t.tot = (uint32_t*)take(256 * 4);
+  t.cta_a = (unsigned long long*)take(kMaxGrid * 8);
+  t.cta_b = (unsigned long long*)take(kMaxGrid * 8);
+  t.x = (unsigned long long*)take(X_COUNT * 8);
+  if (s) *s = t;
+  return o;
 }
 
 __device__ __forceinline__ uint32_t ties_key(float d) {
-  // bits(bf16_rne(|d|)) & 0x7FFF, written with integer rounding so it does not depend on
-  // a conversion intrinsic: |d| is finite and non-negative here
+  // bits(bf16_rne(|d|)) & 0x7FFF by integer rounding; |d| is finite and non-negative here
   uint32_t u = __float_as_uint(fabsf(d));
-  uint32_t r = (u + 0x7FFFu + ((u >> 16) & 1u)) >> 16;
-  return r & 0x7FFFu;
+  return ((u + 0x7FFFu + ((u >> 16) & 1u)) >> 16) & 0x7FFFu;
 }
 
 __device__ __forceinline__ uint64_t splitmix64(uint64_t state) {
@@ -87,11 +82,48 @@ __device__ __forceinline__ uint64_t splitmix64(uint64_t state) {
   return z ^ (z >> 31);
 }
 
-// block-wide exclusive scan of one value per thread (256 threads); returns the exclusive
-// prefix and the block total
+__device__ __forceinline__ unsigned ld_acquire(const unsigned long long* p) {
+  unsigned long long v;
+  asm volatile("ld.acquire.gpu.global.u64 %0, [%1];" : "=l"(v) : "l"(p) : "memory");
+  return (unsigned)v;
+}
+
+// grid barrier: the last CTA to arrive bumps the generation; the others wait for it with
+// a bounded number of polls.  Returns false (uniformly inside the CTA) if the wait expired.
+__device__ __forceinline__ bool grid_sync(unsigned long long* x, unsigned& gen, uint64_t* summary) {
+  __shared__ int s_ok;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    int ok = 1;
+    const unsigned target = gen + 1;
+    __threadfence();
+    if (atomicAdd(&x[X_BAR_COUNT], 1ull) == (unsigned long long)(gridDim.x - 1)) {
+      x[X_BAR_COUNT] = 0;
+      __threadfence();
+      atomicExch(&x[X_BAR_GEN], (unsigned long long)target);
+    } else {
+      uint32_t k = 0;
+      while (ld_acquire(&x[X_BAR_GEN]) != target) {
+        if (++k > kBarrierLimit) {
+          ok = 0;
+          atomicOr((unsigned long long*)&summary[S_ERR], (unsigned long long)kErrTimeout);
+          break;
+        }
+        __nanosleep(32);
+      }
+    }
+    __threadfence();
+    gen = target;
+    s_ok = ok;
+  }
+  __syncthreads();
+  return s_ok != 0;
+}
+
+// block-wide exclusive scan (256 threads) with total
 template <typename T>
-__device__ __forceinline__ T block_exclusive_scan(T v, T& total) {
-  __shared__ T s_warp[kThreads / 32];
+__device__ __forceinline__ T block_scan(T v, T& total) {
+  __shared__ T s_w[kPT / 32];
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5;
   T x = v;
 #pragma unroll
@@ -99,393 +131,354 @@ __device__ __forceinline__ T block_exclusive_scan(T v, T& total) {
     T y = __shfl_up_sync(0xFFFFFFFFu, x, s);
     if (lane >= s) x += y;
   }
-  if (lane == 31) s_warp[warp] = x;
+  if (lane == 31) s_w[warp] = x;
   __syncthreads();
   if (warp == 0) {
-    T t = lane < kThreads / 32 ? s_warp[lane] : T(0);
+    T t = lane < kPT / 32 ? s_w[lane] : T(0);
 #pragma unroll
-    for (int s = 1; s < kThreads / 32; s <<= 1) {
+    for (int s = 1; s < kPT / 32; s <<= 1) {
       T y = __shfl_up_sync(0xFFFFFFFFu, t, s);
       if (lane >= s) t += y;
     }
-    if (lane < kThreads / 32) s_warp[lane] = t;
+    if (lane < kPT / 32) s_w[lane] = t;
   }
   __syncthreads();
-  T before = warp > 0 ? s_warp[warp - 1] : T(0);
-  total = s_warp[kThreads / 32 - 1];
-  __syncthreads();  // s_warp reusable by the next call
+  const T before = warp > 0 ? s_w[warp - 1] : T(0);
+  total = s_w[kPT / 32 - 1];
+  __syncthreads();
   return before + x - v;
 }
 
 template <typename T>
 __device__ __forceinline__ T block_sum(T v) {
-  T total;
-  block_exclusive_scan<T>(v, total);
-  return total;
+  T t;
+  block_scan<T>(v, t);
+  return t;
 }
 
-// ---- 1. score + per-tile candidate counts ---------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_score(const PlanLaunch p, Scratch s, uint64_t U) {
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  uint32_t cnt = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    uint64_t u = t0 + k;
-    if (u >= U) break;
-    uint64_t b = u / p.K;
-    uint32_t i = (uint32_t)(u % p.K);
-    uint64_t st = (uint64_t)i * p.n_blocks + b;
-    bool cand = p.nnz[st] != 0u;
-    if (cand && p.op_kind == MP_OP_TIES)
-      cand = ties_key(p.maxabs[st]) >= p.tau[(uint64_t)i * p.n_groups + p.blk_group[b]];
-    float score = __fmul_rn(p.coef[i], p.norm[st]);
-    s.flag[u] = cand ? 1 : 0;
-    s.key[u] = ~__float_as_uint(score);
-    cnt += cand ? 1u : 0u;
-  }
-  uint32_t tot = block_sum<uint32_t>(cnt);
-  if (threadIdx.x == 0) s.tile_a[blockIdx.x] = tot;
+// sum of a[0..n) (n <= kMaxGrid), computed by the whole CTA
+__device__ __forceinline__ unsigned long long block_sum_prefix(const unsigned long long* a, uint32_t n) {
+  unsigned long long s = 0;
+  for (uint32_t k = threadIdx.x; k < n; k += kPT) s += a[k];
+  return block_sum<unsigned long long>(s);
 }
 
-// single-CTA exclusive scan of n values in place; total to *total_out
-template <typename T>
-__global__ void __launch_bounds__(1024) k_scan_single(T* data, uint64_t n, unsigned long long* total_out) {
-  __shared__ T s_part[1024];
-  __shared__ T s_w[32];
-  const uint32_t tid = threadIdx.x;
-  const uint64_t per = (n + 1023) / 1024;
-  const uint64_t a = (uint64_t)tid * per, e = min(n, a + per);
-  T sum = 0;
-  for (uint64_t j = a; j < e; ++j) sum += data[j];
-  // block scan over 1024 thread sums
-  const int lane = tid & 31, warp = tid >> 5;
-  T x = sum;
-  for (int s = 1; s < 32; s <<= 1) {
-    T y = __shfl_up_sync(0xFFFFFFFFu, x, s);
-    if (lane >= s) x += y;
-  }
-  if (lane == 31) s_w[warp] = x;
-  __syncthreads();
-  if (warp == 0) {
-    T t = s_w[lane];
-    for (int s = 1; s < 32; s <<= 1) {
-      T y = __shfl_up_sync(0xFFFFFFFFu, t, s);
-      if (lane >= s) t += y;
-    }
-    s_w[lane] = t;
-  }
-  __syncthreads();
-  T run = (warp > 0 ? s_w[warp - 1] : T(0)) + x - sum;
-  for (uint64_t j = a; j < e; ++j) {
-    T v = data[j];
-    data[j] = run;
-    run += v;
-  }
-  if (tid == 1023 && total_out) *total_out = (unsigned long long)(s_w[31]);
-  (void)s_part;
+struct Unit {
+  bool cand;
+  uint32_t key;
+};
+
+__device__ __forceinline__ Unit score_unit(const PlanLaunch& p, uint64_t u) {
+  const uint64_t b = u / p.K;
+  const uint32_t i = (uint32_t)(u % p.K);
+  const uint64_t st = (uint64_t)i * p.n_blocks + b;
+  bool cand = p.nnz[st] != 0u;
+  if (cand && p.op_kind == MP_OP_TIES)
+    cand = ties_key(p.maxabs[st]) >= p.tau[(uint64_t)i * p.n_groups + p.blk_group[b]];
+  const float score = __fmul_rn(p.coef[i], p.norm[st]);
+  return Unit{cand, ~__float_as_uint(score)};
 }
 
-// ---- 2. stable compaction of candidates -----------------------------------------------
-__global__ void __launch_bounds__(kThreads) k_compact(Scratch s, uint32_t* vals_a, uint64_t U) {
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  uint32_t cnt = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k)
-    if (t0 + k < U) cnt += s.flag[t0 + k];
-  uint32_t tot;
-  uint32_t pos = s.tile_a[blockIdx.x] + block_exclusive_scan<uint32_t>(cnt, tot);
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    uint64_t u = t0 + k;
-    if (u < U && s.flag[u]) {
-      s.keys_a[pos] = s.key[u];
-      vals_a[pos] = (uint32_t)u;
-      ++pos;
-    }
-  }
-}
-
-// ---- 3. stable LSD radix sort, one 8-bit digit per pass --------------------------------
-__global__ void __launch_bounds__(kThreads) k_sort_hist(const uint32_t* keys, const unsigned long long* x,
-                                                        uint32_t* thist, uint32_t shift, uint32_t n_tiles) {
-  __shared__ uint32_t h[256];
-  h[threadIdx.x] = 0;
-  __syncthreads();
-  const uint64_t Q = x[X_Q];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile;
-  for (int r = 0; r < kItems; ++r) {
-    uint64_t j = t0 + (uint64_t)r * kThreads + threadIdx.x;
-    if (j < Q) atomicAdd(&h[(keys[j] >> shift) & 255u], 1u);
-  }
-  __syncthreads();
-  thist[(uint64_t)threadIdx.x * n_tiles + blockIdx.x] = h[threadIdx.x];
-}
-
-__global__ void __launch_bounds__(kThreads) k_sort_scatter(const uint32_t* keys_in, const uint32_t* vals_in,
-                                                           uint32_t* keys_out, uint32_t* vals_out,
-                                                           const unsigned long long* x, const uint32_t* thist,
-                                                           uint32_t shift, uint32_t n_tiles) {
-  __shared__ uint32_t run[256];
-  __shared__ uint32_t wcnt[kThreads / 32][256];
-  const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
-  const uint64_t Q = x[X_Q];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile;
-  if (t0 >= Q) return;
-  run[tid] = thist[(uint64_t)tid * n_tiles + blockIdx.x];  // global start of digit tid in this tile
-  const uint32_t lt = (1u << lane) - 1u;
-  for (int r = 0; r < kItems; ++r) {
-    for (int w = 0; w < kThreads / 32; ++w) wcnt[w][tid] = 0;
-    __syncthreads();
-    uint64_t j = t0 + (uint64_t)r * kThreads + tid;
-    bool valid = j < Q;
-    uint32_t key = valid ? keys_in[j] : 0u;
-    uint32_t val = valid ? vals_in[j] : 0u;
-    uint32_t d = valid ? ((key >> shift) & 255u) : 256u;
-    uint32_t peers = __match_any_sync(0xFFFFFFFFu, d);
-    uint32_t rank = __popc(peers & lt);
-    if (valid && rank == 0) wcnt[warp][d] = __popc(peers);
-    __syncthreads();
-    {
-      uint32_t acc = run[tid];
-      for (int w = 0; w < kThreads / 32; ++w) {
-        uint32_t c = wcnt[w][tid];
-        wcnt[w][tid] = acc;
-        acc += c;
-      }
-      run[tid] = acc;
-    }
-    __syncthreads();
-    if (valid) {
-      uint32_t pos = wcnt[warp][d] + rank;
-      keys_out[pos] = key;
-      vals_out[pos] = val;
-    }
-    __syncthreads();
-  }
-}
-
-// ---- 4. costs in sorted order: tile sums, then prefix and the first overflow ------------
 __device__ __forceinline__ unsigned long long unit_cost(const PlanLaunch& p, uint32_t u) {
   return (unsigned long long)p.blk_len[u / p.K] * p.elem_size;
 }
 
-__global__ void __launch_bounds__(kThreads) k_cost_tiles(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint64_t Q = s.x[X_Q];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  unsigned long long c = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k)
-    if (t0 + k < Q) c += unit_cost(p, order[t0 + k]);
-  unsigned long long tot = block_sum<unsigned long long>(c);
-  if (threadIdx.x == 0) s.tile64[blockIdx.x] = tot;
+__device__ __forceinline__ void slice(uint64_t n, uint64_t& a, uint64_t& b) {
+  a = n * blockIdx.x / gridDim.x;
+  b = n * (blockIdx.x + 1) / gridDim.x;
 }
 
-__global__ void __launch_bounds__(kThreads) k_cost_prefix(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint64_t Q = s.x[X_Q];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  unsigned long long c[kItems];
-  unsigned long long sum = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    c[k] = t0 + k < Q ? unit_cost(p, order[t0 + k]) : 0ull;
-    sum += c[k];
+__global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s) {
+  __shared__ uint32_t s_run[256];
+  __shared__ uint32_t s_wcnt[kPT / 32][256];
+  __shared__ uint32_t s_cost[kTailChunk];
+  __shared__ unsigned long long s_bcast[1];
+  const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
+  const uint32_t G = gridDim.x, c = blockIdx.x;
+  const uint64_t U = (uint64_t)p.K * p.n_blocks;
+  unsigned gen = 0;
+
+  // ---- zero the outputs; A: count the candidates of this CTA's unit slice ----
+  for (uint64_t k = (uint64_t)c * kPT + tid; k < p.n_blocks; k += (uint64_t)G * kPT) p.mask[k] = 0u;
+  for (uint64_t k = (uint64_t)c * kPT + tid; k < U; k += (uint64_t)G * kPT) s.tailsel[k] = 0;
+  if (c == 0 && tid < 8) p.summary[tid] = 0;
+  if (c == 0 && tid == 0) s.x[X_P] = kNoP;
+  uint64_t u0, u1;
+  slice(U, u0, u1);
+  {
+    unsigned long long cnt = 0;
+    for (uint64_t u = u0 + tid; u < u1; u += kPT) cnt += score_unit(p, u).cand ? 1ull : 0ull;
+    cnt = block_sum<unsigned long long>(cnt);
+    if (tid == 0) s.cta_a[c] = cnt;
   }
-  unsigned long long tot;
-  unsigned long long run = s.tile64[blockIdx.x] + block_exclusive_scan<unsigned long long>(sum, tot);
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    uint64_t j = t0 + k;
-    if (j >= Q) break;
-    unsigned long long before = run;
-    run += c[k];
-    s.prefix[j] = run;
-    if (run > p.budget && before <= p.budget) {  // unique: the prefix is non-decreasing
-      s.x[X_P] = j;
-      s.x[X_PREFIX_BEFORE_P] = before;
+  if (!grid_sync(s.x, gen, p.summary)) return;
+
+  // ---- B: stable compaction into (keys_a, order) ----
+  uint64_t Q;
+  {
+    const unsigned long long before = block_sum_prefix(s.cta_a, c);
+    Q = block_sum_prefix(s.cta_a, G);
+    unsigned long long run = before;
+    for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
+      const uint64_t u = t0 + tid;
+      Unit x = u < u1 ? score_unit(p, u) : Unit{false, 0u};
+      uint32_t tot;
+      const uint32_t pos = block_scan<uint32_t>(x.cand ? 1u : 0u, tot);
+      if (x.cand) {
+        s.keys_a[run + pos] = x.key;
+        p.order[run + pos] = (uint32_t)u;
+      }
+      run += tot;
     }
   }
-}
+  if (!grid_sync(s.x, gen, p.summary)) return;
 
-// ---- 5. the tail after the first overflow ------------------------------------------------
-__device__ __forceinline__ bool tail_candidate(const PlanLaunch& p, const Scratch& s, const uint32_t* order,
-                                               uint64_t j, uint64_t Q, uint64_t P, unsigned long long R0) {
-  return j < Q && j > P && unit_cost(p, order[j]) <= R0;
-}
-
-__global__ void __launch_bounds__(kThreads) k_tail_count(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint64_t Q = s.x[X_Q], P = s.x[X_P];
-  if (P == kNone || P == 0xFFFFFFFFFFFFFFFFull) {
-    if (threadIdx.x == 0) s.tile_a[blockIdx.x] = 0;
-    return;
-  }
-  const unsigned long long R0 = p.budget - s.x[X_PREFIX_BEFORE_P];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  uint32_t cnt = 0;
+  // ---- C: stable LSD radix sort, 8-bit digits ----
+  uint32_t *kin = s.keys_a, *vin = p.order, *kout = s.keys_b, *vout = s.vals_b;
+  uint64_t q0, q1;
+  slice(Q, q0, q1);
+  for (uint32_t pass = 0; pass < 4; ++pass) {
+    const uint32_t shift = 8u * pass;
+    // C1: digit histogram of this CTA's slice
+    s_run[tid] = 0;
+    __syncthreads();
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) atomicAdd(&s_run[(kin[j] >> shift) & 255u], 1u);
+    __syncthreads();
+    s.hist[(uint64_t)tid * G + c] = s_run[tid];
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    // C2: per digit, exclusive prefix over the CTAs (one warp per digit) and the total
+    for (uint32_t d = c + warp * G; d < 256u; d += (kPT / 32) * G) {
+      uint32_t* h = s.hist + (uint64_t)d * G;
+      uint32_t carry = 0;
+      for (uint32_t k0 = 0; k0 < G; k0 += 32) {
+        const uint32_t v = k0 + lane < G ? h[k0 + lane] : 0u;
+        uint32_t x = v;
 #pragma unroll
-  for (int k = 0; k < kItems; ++k) cnt += tail_candidate(p, s, order, t0 + k, Q, P, R0) ? 1u : 0u;
-  uint32_t tot = block_sum<uint32_t>(cnt);
-  if (threadIdx.x == 0) s.tile_a[blockIdx.x] = tot;
-}
-
-__global__ void __launch_bounds__(kThreads) k_tail_compact(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint64_t Q = s.x[X_Q], P = s.x[X_P];
-  if (P == 0xFFFFFFFFFFFFFFFFull) return;
-  const unsigned long long R0 = p.budget - s.x[X_PREFIX_BEFORE_P];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  uint32_t cnt = 0;
-  bool f[kItems];
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    f[k] = tail_candidate(p, s, order, t0 + k, Q, P, R0);
-    cnt += f[k] ? 1u : 0u;
+        for (int sh = 1; sh < 32; sh <<= 1) {
+          const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, sh);
+          if ((int)lane >= sh) x += y;
+        }
+        if (k0 + lane < G) h[k0 + lane] = carry + x - v;
+        carry += __shfl_sync(0xFFFFFFFFu, x, 31);
+      }
+      if (lane == 0) s.tot[d] = carry;
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    // C3: digit starts; skip the pass if one digit holds every key; stable scatter
+    uint32_t total;
+    const uint32_t t_d = s.tot[tid];
+    const uint32_t start = block_scan<uint32_t>(t_d, total);
+    const bool skip = __syncthreads_or(t_d == (uint32_t)Q && Q > 0) != 0 || Q == 0;
+    if (skip) continue;  // uniform over the grid: every CTA reads the same totals
+    s_run[tid] = start + s.hist[(uint64_t)tid * G + c];
+    const uint32_t lt = (1u << lane) - 1u;
+    for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
+      for (int w = 0; w < kPT / 32; ++w) s_wcnt[w][tid] = 0;
+      __syncthreads();
+      const uint64_t j = t0 + tid;
+      const bool valid = j < q1;
+      const uint32_t key = valid ? kin[j] : 0u;
+      const uint32_t val = valid ? vin[j] : 0u;
+      const uint32_t d = valid ? ((key >> shift) & 255u) : 256u;
+      const uint32_t peers = __match_any_sync(0xFFFFFFFFu, d);
+      const uint32_t rank = __popc(peers & lt);
+      if (valid && rank == 0) s_wcnt[warp][d] = __popc(peers);
+      __syncthreads();
+      {
+        uint32_t acc = s_run[tid];
+        for (int w = 0; w < kPT / 32; ++w) {
+          const uint32_t cw = s_wcnt[w][tid];
+          s_wcnt[w][tid] = acc;
+          acc += cw;
+        }
+        s_run[tid] = acc;
+      }
+      __syncthreads();
+      if (valid) {
+        const uint32_t pos = s_wcnt[warp][d] + rank;
+        kout[pos] = key;
+        vout[pos] = val;
+      }
+      __syncthreads();  // every warp has read its offsets before the next tile clears them
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    uint32_t* t;
+    t = kin, kin = kout, kout = t;
+    t = vin, vin = vout, vout = t;
   }
-  uint32_t tot;
-  uint32_t pos = s.tile_a[blockIdx.x] + block_exclusive_scan<uint32_t>(cnt, tot);
-#pragma unroll
-  for (int k = 0; k < kItems; ++k)
-    if (f[k]) s.tail[pos++] = (uint32_t)(t0 + k);
-}
-
-// one warp: greedy with skip over the compacted tail, in order
-__global__ void k_tail_greedy(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint32_t lane = threadIdx.x;
-  const uint64_t P = s.x[X_P];
-  if (P == 0xFFFFFFFFFFFFFFFFull) {
-    if (lane == 0) s.x[X_TAILSUM] = 0;
-    return;
+  // the sorted units end in p.order, or in vals_b if an odd number of passes ran (a
+  // uniform fact: every CTA made the same skip decisions)
+  if (vin != p.order) {
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) p.order[j] = vin[j];
+    if (!grid_sync(s.x, gen, p.summary)) return;
   }
-  const uint64_t L = s.x[X_L];
-  const unsigned long long R0 = p.budget - s.x[X_PREFIX_BEFORE_P];
-  unsigned long long R = R0;
-  for (uint64_t c0 = 0; c0 < L; c0 += 32) {
-    uint64_t j = c0 + lane;
-    uint32_t pos = j < L ? s.tail[j] : 0u;
-    unsigned long long c = j < L ? unit_cost(p, order[pos]) : ~0ull;
-    uint32_t done = 0u;
-    for (;;) {
-      uint32_t m = __ballot_sync(0xFFFFFFFFu, c <= R) & ~done;
-      if (m == 0u) break;
-      int f = __ffs(m) - 1;
-      unsigned long long cf = __shfl_sync(0xFFFFFFFFu, c, f);
-      if ((int)lane == f) s.tailsel[pos] = 1;
-      R -= cf;
-      done = f == 31 ? 0xFFFFFFFFu : ((2u << f) - 1u);
+  const uint32_t* order = p.order;
+
+  // ---- D: cost prefix in sorted order; the first position where it exceeds B ----
+  {
+    unsigned long long sum = 0;
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) sum += unit_cost(p, order[j]);
+    sum = block_sum<unsigned long long>(sum);
+    if (tid == 0) s.cta_b[c] = sum;
+  }
+  if (!grid_sync(s.x, gen, p.summary)) return;
+  {
+    unsigned long long run = block_sum_prefix(s.cta_b, c);
+    const unsigned long long total_cost = block_sum_prefix(s.cta_b, G);
+    if (c == 0 && tid == 0) s.x[X_TOTAL] = total_cost;
+    for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
+      const uint64_t j = t0 + tid;
+      const unsigned long long cj = j < q1 ? unit_cost(p, order[j]) : 0ull;
+      unsigned long long tot;
+      const unsigned long long before = run + block_scan<unsigned long long>(cj, tot);
+      if (j < q1 && before + cj > p.budget && before <= p.budget) {  // unique: prefixes only grow
+        s.x[X_P] = j;
+        s.x[X_PBP] = before;
+      }
+      run += tot;
     }
   }
-  if (lane == 0) s.x[X_TAILSUM] = R0 - R;
-}
+  if (!grid_sync(s.x, gen, p.summary)) return;
+  const unsigned long long P = s.x[X_P];
+  const unsigned long long R0 = P == kNoP ? 0ull : p.budget - s.x[X_PBP];
 
-// ---- 6. mask, set hash, count; then touched blocks and digest (last CTA) ----------------
-__global__ void __launch_bounds__(kThreads) k_mask(const PlanLaunch p, Scratch s, const uint32_t* order) {
-  const uint64_t Q = s.x[X_Q], P = s.x[X_P];
-  const uint64_t t0 = (uint64_t)blockIdx.x * kTile + (uint64_t)threadIdx.x * kItems;
-  unsigned long long h = 0, n = 0;
-#pragma unroll
-  for (int k = 0; k < kItems; ++k) {
-    uint64_t j = t0 + k;
-    if (j >= Q) break;
-    if (j < P || s.tailsel[j]) {
-      uint32_t u = order[j];
-      atomicOr(&p.mask[u / p.K], 1u << (u % p.K));
-      h += splitmix64(u);
-      ++n;
+  // ---- E: the tail after the first overflow ----
+  if (P != kNoP) {
+    {
+      unsigned long long cnt = 0;
+      for (uint64_t j = q0 + tid; j < q1; j += kPT) cnt += (j > P && unit_cost(p, order[j]) <= R0) ? 1ull : 0ull;
+      cnt = block_sum<unsigned long long>(cnt);
+      if (tid == 0) s.cta_a[c] = cnt;
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    const unsigned long long L = block_sum_prefix(s.cta_a, G);
+    {
+      unsigned long long run = block_sum_prefix(s.cta_a, c);
+      for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
+        const uint64_t j = t0 + tid;
+        const bool f = j < q1 && j > P && unit_cost(p, order[j]) <= R0;
+        uint32_t tot;
+        const uint32_t pos = block_scan<uint32_t>(f ? 1u : 0u, tot);
+        if (f) s.tail_pos[run + pos] = (uint32_t)j;
+        run += tot;
+      }
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    if (c == 0) {
+      // greedy with skip over the compacted tail, in order, from shared memory
+      unsigned long long R = R0;
+      for (unsigned long long k0 = 0; k0 < L; k0 += kTailChunk) {
+        const uint32_t n = (uint32_t)min((unsigned long long)kTailChunk, L - k0);
+        for (uint32_t k = tid; k < n; k += kPT) s_cost[k] = (uint32_t)unit_cost(p, order[s.tail_pos[k0 + k]]);
+        __syncthreads();
+        if (warp == 0) {
+          for (uint32_t b0 = 0; b0 < n; b0 += 32) {
+            const uint32_t k = b0 + lane;
+            const unsigned long long ck = k < n ? s_cost[k] : ~0ull;
+            uint32_t done = 0u;
+            for (;;) {
+              const uint32_t m = __ballot_sync(0xFFFFFFFFu, ck <= R) & ~done;
+              if (m == 0u) break;
+              const int f = __ffs(m) - 1;
+              if ((int)lane == f) s.tailsel[s.tail_pos[k0 + k]] = 1;
+              R -= __shfl_sync(0xFFFFFFFFu, ck, f);
+              done = f == 31 ? 0xFFFFFFFFu : ((2u << f) - 1u);
+            }
+          }
+          if (lane == 0) s_bcast[0] = R;
+        }
+        __syncthreads();
+        R = s_bcast[0];
+      }
+      if (tid == 0) s.x[X_TAILSUM] = R0 - R;
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+  }
+
+  // ---- F: mask, set hash, count; then touched blocks and the digest (last CTA) ----
+  {
+    unsigned long long h = 0, n = 0;
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) {
+      if ((P == kNoP || j < P) || s.tailsel[j]) {
+        const uint32_t u = order[j];
+        atomicOr(&p.mask[u / p.K], 1u << (u % p.K));
+        h += splitmix64(u);
+        ++n;
+      }
+    }
+    h = block_sum<unsigned long long>(h);
+    n = block_sum<unsigned long long>(n);
+    if (tid == 0 && n) {
+      atomicAdd((unsigned long long*)&p.summary[S_SETHASH], h);
+      atomicAdd((unsigned long long*)&p.summary[S_NSEL], n);
     }
   }
-  h = block_sum<unsigned long long>(h);
-  n = block_sum<unsigned long long>(n);
-  if (threadIdx.x == 0 && n) {
-    atomicAdd((unsigned long long*)&p.summary[S_SETHASH], h);
-    atomicAdd((unsigned long long*)&p.summary[S_NSEL], n);
+  if (!grid_sync(s.x, gen, p.summary)) return;
+  {
+    uint64_t b0, b1;
+    slice(p.n_blocks, b0, b1);
+    unsigned long long t = 0;
+    for (uint64_t b = b0 + tid; b < b1; b += kPT) t += p.mask[b] != 0u ? 1ull : 0ull;
+    t = block_sum<unsigned long long>(t);
+    __shared__ bool last;
+    if (tid == 0) {
+      if (t) atomicAdd((unsigned long long*)&p.summary[S_TOUCHED], t);
+      __threadfence();
+      last = atomicAdd(&s.x[X_DONE], 1ull) == (unsigned long long)(G - 1);
+    }
+    __syncthreads();
+    if (!last || tid != 0) return;
   }
-}
-
-__device__ __forceinline__ uint64_t fnv_u64(uint64_t h, uint64_t v) {
-  for (int k = 0; k < 8; ++k) {
-    h ^= (v >> (8 * k)) & 0xFFu;
-    h *= 1099511628211ull;
-  }
-  return h;
-}
-
-__global__ void __launch_bounds__(kThreads) k_touched_finalize(const PlanLaunch p, Scratch s) {
-  __shared__ bool last;
-  unsigned long long cnt = 0;
-  for (uint64_t b = (uint64_t)blockIdx.x * kThreads + threadIdx.x; b < p.n_blocks;
-       b += (uint64_t)gridDim.x * kThreads)
-    cnt += p.mask[b] != 0u ? 1ull : 0ull;
-  cnt = block_sum<unsigned long long>(cnt);
-  if (threadIdx.x == 0) {
-    if (cnt) atomicAdd((unsigned long long*)&p.summary[S_TOUCHED], cnt);
-    __threadfence();
-    unsigned long long prev = atomicAdd(&s.x[X_DONE], 1ull);
-    last = prev == gridDim.x - 1;
-  }
-  __syncthreads();
-  if (!last || threadIdx.x != 0) return;
+  // the digest: FNV-1a 64 over the host-built prefix and C_hat, n_sel, set_hash
   __threadfence();
-  const uint64_t P = s.x[X_P], Q = s.x[X_Q];
-  unsigned long long chat =
-      P == 0xFFFFFFFFFFFFFFFFull ? (Q ? s.prefix[Q - 1] : 0ull) : s.x[X_PREFIX_BEFORE_P] + s.x[X_TAILSUM];
   volatile unsigned long long* sum = (volatile unsigned long long*)p.summary;
-  unsigned long long nsel = sum[S_NSEL], sh = sum[S_SETHASH];
+  const unsigned long long chat = P == kNoP ? s.x[X_TOTAL] : s.x[X_PBP] + s.x[X_TAILSUM];
+  const unsigned long long nsel = sum[S_NSEL], sh = sum[S_SETHASH];
   uint64_t h = 14695981039346656037ull;
   for (uint32_t k = 0; k < p.hdr_prefix_len; ++k) {
     h ^= p.hdr_prefix[k];
     h *= 1099511628211ull;
   }
-  h = fnv_u64(h, chat);
-  h = fnv_u64(h, nsel);
-  h = fnv_u64(h, sh);
+  const unsigned long long tail[3] = {chat, nsel, sh};
+  for (int w = 0; w < 3; ++w)
+    for (int k = 0; k < 8; ++k) {
+      h ^= (tail[w] >> (8 * k)) & 0xFFu;
+      h *= 1099511628211ull;
+    }
   sum[S_CHAT] = chat;
   sum[S_NCAND] = Q;
   sum[S_DIGEST] = h;
-  sum[S_ERR] = *p.index_err;
+  sum[S_ERR] = sum[S_ERR] | (unsigned long long)*p.index_err;
 }
 
 }  // namespace
 
-size_t plan_scratch_bytes(uint64_t n_units) { return carve_bytes(n_units); }
+size_t plan_scratch_bytes(uint64_t n_units) { return carve(nullptr, n_units, nullptr); }
 
 cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st) {
   const uint64_t U = (uint64_t)p.K * p.n_blocks;
-  const uint64_t nt64 = (U + kTile - 1) / kTile;
-  if (nt64 > 0x7FFFFFFFull || U > 0xFFFFFFFFull) return cudaErrorInvalidValue;
-  const uint32_t nt = (uint32_t)nt64;
-  Scratch s = carve(scratch, U);
+  if (U > 0xFFFFFFFFull) return cudaErrorInvalidValue;
+  Scratch s;
+  carve(scratch, U, &s);
+  int dev = 0, sms = 0, per_sm = 0;
   cudaError_t e;
-  if ((e = cudaMemsetAsync(p.summary, 0, 8 * sizeof(uint64_t), st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(p.mask, 0, p.n_blocks * sizeof(uint32_t), st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(s.tailsel, 0, U, st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(s.x, 0, X_COUNT * 8, st)) != cudaSuccess) return e;
-  if ((e = cudaMemsetAsync(&s.x[X_P], 0xFF, 8, st)) != cudaSuccess) return e;
-
-  uint32_t* vals_a = p.order;
-  k_score<<<nt, kThreads, 0, st>>>(p, s, U);
-  k_scan_single<uint32_t><<<1, 1024, 0, st>>>(s.tile_a, nt, &s.x[X_Q]);
-  k_compact<<<nt, kThreads, 0, st>>>(s, vals_a, U);
-  // four passes: a -> b -> a -> b -> a, final order in vals_a (= the plan's order array)
-  uint32_t *kin = s.keys_a, *vin = vals_a, *kout = s.keys_b, *vout = s.vals_b;
-  for (uint32_t pass = 0; pass < 4; ++pass) {
-    k_sort_hist<<<nt, kThreads, 0, st>>>(kin, s.x, s.thist, 8u * pass, nt);
-    k_scan_single<uint32_t><<<1, 1024, 0, st>>>(s.thist, (uint64_t)nt * 256u, nullptr);
-    k_sort_scatter<<<nt, kThreads, 0, st>>>(kin, vin, kout, vout, s.x, s.thist, 8u * pass, nt);
-    uint32_t* t;
-    t = kin, kin = kout, kout = t;
-    t = vin, vin = vout, vout = t;
-  }
-  const uint32_t* order = vals_a;
-  k_cost_tiles<<<nt, kThreads, 0, st>>>(p, s, order);
-  k_scan_single<unsigned long long><<<1, 1024, 0, st>>>(s.tile64, nt, nullptr);
-  k_cost_prefix<<<nt, kThreads, 0, st>>>(p, s, order);
-  k_tail_count<<<nt, kThreads, 0, st>>>(p, s, order);
-  k_scan_single<uint32_t><<<1, 1024, 0, st>>>(s.tile_a, nt, &s.x[X_L]);
-  k_tail_compact<<<nt, kThreads, 0, st>>>(p, s, order);
-  k_tail_greedy<<<1, 32, 0, st>>>(p, s, order);
-  k_mask<<<nt, kThreads, 0, st>>>(p, s, order);
-  uint64_t tb = (p.n_blocks + kThreads - 1) / kThreads;
-  unsigned tgrid = (unsigned)(tb < 1024 ? (tb ? tb : 1) : 1024);
-  k_touched_finalize<<<tgrid, kThreads, 0, st>>>(p, s);
-  count_launches(3 + 4 * 3 + 9);
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, plan_kernel, kPT, 0)) != cudaSuccess) return e;
+  // about 512 units per CTA (two tiles), at most one CTA per SM, all co-resident
+  if (per_sm < 1) return cudaErrorInvalidConfiguration;
+  uint64_t grid = (U + 511) / 512;
+  const uint64_t cap = (uint64_t)sms;
+  if (grid > cap) grid = cap;
+  if (grid > kMaxGrid) grid = kMaxGrid;
+  if (grid < 1) grid = 1;
+  if ((e = cudaMemsetAsync(s.x, 0, X_COUNT * sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  PlanLaunch pc = p;
+  void* args[] = {&pc, &s};
+  if ((e = cudaLaunchCooperativeKernel((const void*)plan_kernel, dim3((unsigned)grid), dim3(kPT), args, 0, st)) !=
+      cudaSuccess)
+    return e;
+  count_launches(1);
   return cudaGetLastError();
 }
 
