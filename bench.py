@@ -164,7 +164,7 @@ def hbm_peak():
 
 def merge_source_hash() -> str:
     h = hashlib.sha256()
-    for name in ("merge.cu", "philox.cuh", "tma.cuh"):
+    for name in ("merge.cu", "philox.cuh", "small_div.cuh", "tma.cuh"):
         with open(os.path.join(ROOT, "paper_2605_29489_gb300", "csrc", name), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]

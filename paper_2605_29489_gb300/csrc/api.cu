@@ -763,6 +763,10 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
     p.dare_T = !(t > 0.0) ? 0u : (t > 65536.0 ? 65536u : (uint32_t)t);
   }
   p.seed = plan->seed;
+  for (int r = 0; r < 10; ++r) {
+    p.dare_rk[r][0] = (uint32_t)plan->seed + (uint32_t)r * 0x9E3779B9u;
+    p.dare_rk[r][1] = (uint32_t)(plan->seed >> 32) + (uint32_t)r * 0xBB67AE85u;
+  }
   p.realized = mf->d_realized;
   p.work = reinterpret_cast<unsigned long long*>(static_cast<char*>(mf->mem.ptr) + back_bytes);
   p.err = mf->d_err;

@@ -107,23 +107,55 @@ struct __align__(128) IxSmem {
   int abort;
 };
 
+// raw 16-byte vector at element k0 of a fill: from the slot when inside the bulk-copied
+// bytes, else (the ragged tail of a tensor) from global memory, zero past the chunk
 template <bool BF16>
-__device__ __forceinline__ void ix_read_vec(const uint8_t* slot, const void* gsrc, uint64_t off, uint32_t k0,
-                                            uint32_t n, uint32_t n_tma, float (&x)[BF16 ? 8 : 4]) {
+__device__ __forceinline__ uint4 ix_read_raw(const uint8_t* slot, const void* gsrc, uint64_t off, uint32_t k0,
+                                             uint32_t n, uint32_t n_tma) {
   constexpr uint32_t V = BF16 ? 8u : 4u;
-  if (k0 + V <= n_tma) {
-    unpack<BF16>(*reinterpret_cast<const uint4*>(slot + k0 * (BF16 ? 2u : 4u)), x);
-    return;
-  }
+  if (k0 + V <= n_tma) return *reinterpret_cast<const uint4*>(slot + k0 * (BF16 ? 2u : 4u));
+  uint32_t w[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
   for (uint32_t e = 0; e < V; ++e) {
-    float v = 0.0f;
     if (k0 + e < n) {
-      if constexpr (BF16) v = __uint_as_float((uint32_t)(static_cast<const uint16_t*>(gsrc)[off + k0 + e]) << 16);
-      else v = static_cast<const float*>(gsrc)[off + k0 + e];
+      if constexpr (BF16) w[e >> 1] |= (uint32_t)(static_cast<const uint16_t*>(gsrc)[off + k0 + e]) << (16u * (e & 1u));
+      else w[e] = static_cast<const uint32_t*>(gsrc)[off + k0 + e];
     }
-    x[e] = v;
   }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+__device__ __forceinline__ bool same_vec(const uint4 a, const uint4 b) {
+  return a.x == b.x && a.y == b.y && a.z == b.z && a.w == b.w;
+}
+
+// TIES coarse bins of two deltas: bin = upper 8 bits of the 15-bit key bits(bf16(|d|)),
+// i.e. bits 7..14 of the round-to-nearest-even bf16 of d (the sign bit 15 is masked off);
+// both are converted by one packed cvt.  A nonzero delta adds 1 to its bin of the
+// shared histogram at hist (byte address in the shared window) and 1 to nz; a zero delta
+// adds nothing.  Predicated, so that no branch is taken per element.
+__device__ __forceinline__ void ties_bin2(float d0, float d1, uint32_t hist, uint32_t& nz) {
+  asm volatile(
+      "{\n"
+      " .reg .pred p0, p1;\n"
+      " .reg .b32 w, a0, a1;\n"
+      " cvt.rn.bf16x2.f32 w, %3, %2;\n"
+      " setp.ne.f32 p0, %2, 0f00000000;\n"
+      " setp.ne.f32 p1, %3, 0f00000000;\n"
+      " shr.b32 a0, w, 5;\n"
+      " and.b32 a0, a0, 1020;\n"
+      " add.u32 a0, a0, %1;\n"
+      " shr.b32 a1, w, 21;\n"
+      " and.b32 a1, a1, 1020;\n"
+      " add.u32 a1, a1, %1;\n"
+      " @p0 red.shared.add.u32 [a0], 1;\n"
+      " @p1 red.shared.add.u32 [a1], 1;\n"
+      " @p0 add.u32 %0, %0, 1;\n"
+      " @p1 add.u32 %0, %0, 1;\n"
+      "}\n"
+      : "+r"(nz)
+      : "r"(hist), "f"(d0), "f"(d1)
+      : "memory");
 }
 
 template <bool BF16, int KG, bool TIES>
@@ -160,6 +192,7 @@ __global__ void __launch_bounds__(kIxThreads, 2)
                          uint32_t bytes) -> bool {
         const uint32_t s = fill % kIxSlots, r = fill / kIxSlots;
         if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+        if (r > 0) fence_proxy_async_smem();
         S.meta[s].off = off;
         S.meta[s].item = item;
         S.meta[s].n = n;
@@ -235,11 +268,17 @@ __global__ void __launch_bounds__(kIxThreads, 2)
     const uint32_t n = mt.n, n_tma = ((n * ES) & ~15u) / ES;
     const uint64_t off = mt.off;
     float xb[VPT][V];
+    uint4 rb[VPT];     // the base vectors as read, for the equality test
+    bool bfin = true;  // every base element finite (Inf - Inf and NaN - NaN are not zero)
     {
       const uint8_t* slot = S.slot[fill % kIxSlots];
 #pragma unroll
-      for (int u = 0; u < VPT; ++u)
-        ix_read_vec<BF16>(slot, p.base, off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma, xb[u]);
+      for (int u = 0; u < VPT; ++u) {
+        rb[u] = ix_read_raw<BF16>(slot, p.base, off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma);
+        unpack<BF16>(rb[u], xb[u]);
+#pragma unroll
+        for (int e = 0; e < V; ++e) bfin = bfin && fabsf(xb[u][e]) < __int_as_float(0x7F800000);
+      }
       release(fill);
       ++fill;
     }
@@ -251,19 +290,37 @@ __global__ void __launch_bounds__(kIxThreads, 2)
         break;
       }
       const uint8_t* slot = S.slot[fill % kIxSlots];
+      uint4 re[VPT];
+      bool same = bfin;
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
-        float xe[V];
-        ix_read_vec<BF16>(slot, p.experts.p[i0 + k], off - p.expert_origin, (tid + (uint32_t)u * kIxConsumers) * V, n,
-                          n_tma, xe);
+        re[u] = ix_read_raw<BF16>(slot, p.experts.p[i0 + k], off - p.expert_origin,
+                                  (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma);
+        same = same && same_vec(re[u], rb[u]);
+      }
+      // a finite vector equal bit for bit to the base gives deltas of exactly +0, which
+      // change neither the sum of squares (>= +0), the max (>= +0), the count nor the bins:
+      // a warp whose vectors all match skips them (warp-uniform, so the summation order is
+      // untouched)
+      if (!__all_sync(0xFFFFFFFFu, same)) {
 #pragma unroll
-        for (int e = 0; e < V; ++e) {
-          const float d = __fsub_rn(xe[e], xb[u][e]);
-          ss[k] = __fmaf_rn(d, d, ss[k]);
-          mx[k] = fmaxf(mx[k], fabsf(d));
-          nz[k] += d != 0.0f ? 1u : 0u;
-          if constexpr (TIES) {
-            if (d != 0.0f) atomicAdd(&S.hist[k][ties_key(d) >> 7], 1u);
+        for (int u = 0; u < VPT; ++u) {
+          float xe[V];
+          unpack<BF16>(re[u], xe);
+#pragma unroll
+          for (int e = 0; e < V; e += 2) {
+            const float d0 = __fsub_rn(xe[e], xb[u][e]);
+            const float d1 = __fsub_rn(xe[e + 1], xb[u][e + 1]);
+            ss[k] = __fmaf_rn(d0, d0, ss[k]);
+            ss[k] = __fmaf_rn(d1, d1, ss[k]);
+            mx[k] = fmaxf(mx[k], fabsf(d0));
+            mx[k] = fmaxf(mx[k], fabsf(d1));
+            if constexpr (TIES) {
+              ties_bin2(d0, d1, su32(&S.hist[k][0]), nz[k]);
+            } else {
+              nz[k] += d0 != 0.0f ? 1u : 0u;
+              nz[k] += d1 != 0.0f ? 1u : 0u;
+            }
           }
         }
       }

@@ -1,32 +1,38 @@
 // Alg. 2 ExecuteMerge on the device: M_A[t,b] = M_0[t,b] + Psi_op(A_{.,t,b}, Delta_{.,t,b})
 // (Eq. 4) for every block, reading only the experts the access mask selects.
 //
-// Pipeline (one persistent CTA pair per SM, 256 consumer threads + 1 producer warp):
-//  * work unit = one chunk of 8 KiB of a block (4096 bf16 / 2048 fp32 elements); chunks
-//    are handed out dynamically through a global counter, GRAB at a time;
-//  * the producer thread walks each chunk's fills — the base chunk, then every selected
-//    expert's chunk in ascending expert order — and streams each fill into the next slot
-//    of a ring of NS shared-memory slots with one cp.async.bulk (TMA 1-D bulk copy),
-//    completing on the slot's "full" mbarrier; it writes the slot's metadata (chunk,
-//    which checkpoint, offset, length, mask) before arming the barrier;
+// Pipeline (persistent CTAs, 2 or 3 per SM, 256 consumer threads + 1 producer warp):
+//  * work unit = one chunk of a block (8 KiB for AVG/TA, 4 KiB for TIES/DARE); chunks are
+//    handed out dynamically through a global counter, GRAB at a time;
+//  * the producer warp takes a grab: its lanes load the chunks' block metadata (and, for
+//    TIES, every expert's trim threshold) in parallel into shared memory, and the counter
+//    value of the next grab is requested before this one is issued, so that no fill waits
+//    on a global-memory round trip;
+//  * lane 0 then walks each chunk's fills — the base chunk, then every selected expert's
+//    chunk in ascending expert order — and streams each fill into the next slot of a ring
+//    of NS shared-memory slots with one cp.async.bulk (TMA 1-D bulk copy), completing on
+//    the slot's "full" mbarrier; it writes the slot's metadata (chunk, which checkpoint,
+//    offset, length, mask, threshold) before arming the barrier;
 //  * consumers take the slots in the same order: the base fill loads M_0 into registers,
 //    each expert fill folds Delta_i into fp32 accumulators, the last fill of a chunk
 //    writes the output with 16-byte streaming stores; each warp releases a slot on its
 //    "empty" mbarrier as soon as it has read it;
-//  * the bytes in flight are the ring (NS x 8 KiB per CTA), independent of registers and
-//    of how many experts a block selects.
+//  * the bytes in flight are the ring (NS slots per CTA), independent of registers and of
+//    how many experts a block selects.
 // Per element, in the fixed ascending expert order:
 //   AVG/TA: acc = fma(alpha_i, delta_i, acc)                          out = M_0 + acc
 //   DARE:   delta_i kept by a Philox word >= T, scaled by sigma; then as AVG
 //   TIES:   trimmed by tau_i; S, P, N, counts;  m = P/c+ | N/c- | 0;   out = fma(lambda, m, M_0)
 // An omitted expert contributes exactly zero to every accumulator, so skipping it equals
-// reading a zero-completed tuple (App. A.1) and it is never dereferenced.
+// reading a zero-completed tuple (App. A.1) and it is never dereferenced; a chunk that
+// selects no expert is M_0 plus the zero the operator adds.
 // Every mbarrier wait is bounded: on expiry the CTA records kErrTimeout, stops, waits
 // (bounded) for its own copies in flight and returns.
 #include <cuda_bf16.h>
 
 #include "mp_internal.cuh"
 #include "philox.cuh"
+#include "small_div.cuh"
 #include "tma.cuh"
 
 namespace mp {
@@ -34,18 +40,21 @@ namespace {
 
 constexpr int kConsumers = 256;
 constexpr int kThreads = kConsumers + 32;  // + one producer warp
-constexpr uint32_t kRingBytes = 98304;     // slot ring per CTA (96 KiB; two CTAs per SM)
-constexpr uint32_t kGrab = 4;              // chunks taken per counter increment
 constexpr uint32_t kEnd = 0xFFFFFFFFu;
 
 enum { OP_ADD = 0, OP_TIES = 1, OP_DARE = 2 };
 
-// slot geometry per operator: TIES keeps five fp32 values per element in flight, so its
-// chunks are half as long (one 16-byte vector per consumer thread, no register spills)
+// slot geometry per operator.  The additive merge is bound by HBM: two CTAs per SM with a
+// 96 KiB ring each.  TIES and DARE spend more arithmetic per byte: three CTAs per SM (more
+// warps to hide it) with a 64 KiB ring each, and chunks half as long (one 16-byte vector per
+// consumer thread) so that their per-element state fits the register budget.
 template <int OPC>
 struct Geo {
-  static constexpr uint32_t kSlotBytes = OPC == OP_TIES ? 4096u : 8192u;  // one chunk of one checkpoint
+  static constexpr int kCtasPerSm = OPC == OP_ADD ? 2 : 3;
+  static constexpr uint32_t kRingBytes = OPC == OP_ADD ? 98304u : 65536u;
+  static constexpr uint32_t kSlotBytes = OPC == OP_ADD ? 8192u : 4096u;  // one chunk of one checkpoint
   static constexpr int kSlots = (int)(kRingBytes / kSlotBytes);
+  static constexpr uint32_t kGrab = 8;  // chunks taken per counter increment (<= 32)
 };
 
 struct SlotMeta {
@@ -54,19 +63,85 @@ struct SlotMeta {
   uint32_t which; // 0 = base, 1 + i = expert i
   uint32_t n;     // elements in the chunk
   uint32_t m;     // the block's access mask
-  uint32_t grp;   // the block's trim group
-  uint32_t tau;   // TIES threshold of this (expert, trim group)
+  uint32_t tau;   // TIES: bits threshold of this (expert, trim group)
 };
 
-template <int NS, uint32_t SB>
+// block metadata of one chunk of a grab, staged by the producer warp
+struct ChunkMeta {
+  uint64_t off;  // element offset of the chunk
+  uint32_t n;    // elements (0: nothing to do)
+  uint32_t m;    // access mask
+};
+
+template <int NS, uint32_t SB, uint32_t G>
 struct __align__(128) Smem {
   uint8_t slot[NS][SB];
   SlotMeta meta[NS];
+  ChunkMeta chunk[G];
+  uint32_t thr[G][kMaxK];  // TIES: bits threshold of (chunk, expert)
   uint64_t full[NS];
   uint64_t empty[NS];
   unsigned long long realized[kMaxK];
+  float2 ctab[kMaxK + 1];  // TIES: {c, RN(1/c)} for the counts c = 0..kMaxK (entry 0: {1, 1})
   int abort;
 };
+
+// packed fp32x2 arithmetic (two independent IEEE round-to-nearest operations per
+// instruction): (d0, d1) = (a0 op b0, a1 op b1)
+__device__ __forceinline__ void f2_sub(float a0, float a1, float b0, float b1, float& d0, float& d1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n sub.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+__device__ __forceinline__ void f2_mul(float a0, float a1, float b0, float b1, float& d0, float& d1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mul.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
+// (d0, d1) = (a0 * b0 + c0, a1 * b1 + c1), each a single fused rounding
+__device__ __forceinline__ void f2_fma(float a0, float a1, float b0, float b1, float c0, float c1, float& d0,
+                                       float& d1) {
+  asm("{\n .reg .b64 ra, rb, rc, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n mov.b64 rc, {%6, %7};\n"
+      " fma.rn.f32x2 rd, ra, rb, rc;\n mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1), "f"(c0), "f"(c1));
+}
+
+// The TIES trim compares the 15-bit key bits(bf16_rne(|d|)) & 0x7FFF with tau.  For
+// |d| >= 0 the key reaches tau >= 1 exactly when bits(|d|) >= (tau << 16) - 0x8000 +
+// (tau & 1): the halfway point below tau rounds up to tau only when tau is even.  tau = 0
+// keeps everything; tau = 0x8000 ("keep nothing") gives 0x7FFF8000, a NaN pattern, so a
+// float compare against it is never true.
+__host__ __device__ __forceinline__ uint32_t ties_bits_threshold(uint32_t tau) {
+  return tau == 0u ? 0u : (tau << 16) - 0x8000u + (tau & 1u);
+}
+
+// One expert's contribution to an element's TIES tally, with predicated adds: the delta d
+// is kept when |d| >= thr; a kept d goes into S, and into P (with count +1) when positive
+// or into N (count + 0x10000) otherwise.  thr is at least the smallest subnormal, so a kept
+// d is never zero and "not positive" means negative; one compare with two destination
+// predicates splits the kept entries by sign.  A skipped add is the same as adding the +0
+// of a trimmed entry: S, P and N are never -0, so +0 leaves them unchanged.
+__device__ __forceinline__ void ties_tally(float d, float thr, float& S, float& P, float& N, uint32_t& cnt) {
+  asm("{\n"
+      " .reg .pred pk, pp, pn;\n"
+      " .reg .f32 ad;\n"
+      " abs.f32 ad, %4;\n"
+      " setp.ge.f32 pk, ad, %5;\n"
+      " setp.gt.and.f32 pp|pn, %4, 0f00000000, pk;\n"
+      " @pk add.rn.f32 %0, %0, %4;\n"
+      " @pp add.rn.f32 %1, %1, %4;\n"
+      " @pn add.rn.f32 %2, %2, %4;\n"
+      " @pp add.u32 %3, %3, 1;\n"
+      " @pn add.u32 %3, %3, 65536;\n"
+      "}\n"
+      : "+f"(S), "+f"(P), "+f"(N), "+r"(cnt)
+      : "f"(d), "f"(thr));
+}
 
 template <bool BF16>
 __device__ __forceinline__ void unpack(const uint4 r, float* x) {
@@ -108,6 +183,8 @@ __device__ __forceinline__ void read_vec(const uint8_t* slot, const void* gsrc, 
   }
 }
 
+// the tail loops are unrolled over the vector with a predicate, so that h and y stay in
+// registers (a loop bounded by navail would index them at run time, through local memory)
 template <bool BF16>
 __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t navail, const float* y) {
   constexpr uint32_t V = BF16 ? 8u : 4u;
@@ -119,29 +196,34 @@ __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t nav
       uint4 w = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
       __stcs(reinterpret_cast<uint4*>(static_cast<char*>(ptr) + elem * 2u), w);
     } else {
-      for (uint32_t e = 0; e < navail; ++e) static_cast<uint16_t*>(ptr)[elem + e] = (uint16_t)h[e];
+#pragma unroll
+      for (uint32_t e = 0; e < V; ++e)
+        if (e < navail) static_cast<uint16_t*>(ptr)[elem + e] = (uint16_t)h[e];
     }
   } else {
     if (navail >= V) {
       __stcs(reinterpret_cast<float4*>(static_cast<char*>(ptr) + elem * 4u), make_float4(y[0], y[1], y[2], y[3]));
     } else {
-      for (uint32_t e = 0; e < navail; ++e) static_cast<float*>(ptr)[elem + e] = y[e];
+#pragma unroll
+      for (uint32_t e = 0; e < V; ++e)
+        if (e < navail) static_cast<float*>(ptr)[elem + e] = y[e];
     }
   }
 }
 
 template <bool BF16, int OPC>
-__global__ void __launch_bounds__(kThreads, 2)
+__global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     merge_tma_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t SB = Geo<OPC>::kSlotBytes;
   constexpr int kSlots = Geo<OPC>::kSlots;
+  constexpr uint32_t G = Geo<OPC>::kGrab;
   constexpr uint32_t CH = SB / ES;  // elements per chunk
   constexpr int V = BF16 ? 8 : 4;
   constexpr int VPT = (int)(CH / (kConsumers * V));  // vectors per consumer thread per chunk
   static_assert(CH == (uint32_t)(kConsumers * VPT * V), "chunk geometry");
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  Smem<kSlots, SB>& S = *reinterpret_cast<Smem<kSlots, SB>*>(smem_raw);
+  Smem<kSlots, SB, G>& S = *reinterpret_cast<Smem<kSlots, SB, G>*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   volatile int* abort_flag = &S.abort;
 
@@ -154,53 +236,86 @@ __global__ void __launch_bounds__(kThreads, 2)
     mbar_fence_init();
   }
   if (tid < (uint32_t)kMaxK) S.realized[tid] = 0;
+  if (tid <= (uint32_t)kMaxK) {
+    const float c = tid == 0 ? 1.0f : (float)tid;
+    S.ctab[tid] = make_float2(c, __fdiv_rn(1.0f, c));
+  }
   __syncthreads();
 
   if (warp == kConsumers / 32) {
     // ---------------- producer ----------------
-    if (lane == 0) {
-      uint32_t fill = 0;
-      bool ok = true;
-      auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t grp,
-                         const char* src_row, uint32_t bytes) -> bool {
-        const uint32_t s = fill % kSlots, r = fill / kSlots;
-        if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
-        S.meta[s].off = off;
-        S.meta[s].q = q;
-        S.meta[s].which = which;
-        S.meta[s].n = n;
-        S.meta[s].m = m;
-        S.meta[s].grp = grp;
-        S.meta[s].tau = (OPC == OP_TIES && which > 0) ? p.tau[(uint64_t)(which - 1) * p.n_groups + grp] : 0u;
-        mbar_arrive_expect_tx(&S.full[s], bytes);
-        if (bytes) tma_load_1d(S.slot[s], src_row, bytes, &S.full[s]);
-        ++fill;
-        return true;
-      };
-      while (ok) {
-        const unsigned long long q0 = atomicAdd(work, (unsigned long long)kGrab);
-        if (q0 >= n_chunks) break;
-        const unsigned long long q1 = min(q0 + kGrab, (unsigned long long)n_chunks);
-        for (unsigned long long q = q0; q < q1 && ok; ++q) {
+    uint32_t fill = 0;
+    bool ok = true;
+    // lane 0 arms slot `fill` with the given chunk data and starts its bulk copy
+    auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t thr,
+                       const char* src_row, uint32_t bytes) -> bool {
+      const uint32_t s = fill % kSlots, r = fill / kSlots;
+      if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+      if (r > 0) fence_proxy_async_smem();
+      S.meta[s].off = off;
+      S.meta[s].q = q;
+      S.meta[s].which = which;
+      S.meta[s].n = n;
+      S.meta[s].m = m;
+      S.meta[s].tau = thr;
+      mbar_arrive_expect_tx(&S.full[s], bytes);
+      if (bytes) tma_load_1d(S.slot[s], src_row, bytes, &S.full[s]);
+      ++fill;
+      return true;
+    };
+    unsigned long long q_next = 0;
+    if (lane == 0) q_next = atomicAdd(work, (unsigned long long)G);
+    for (;;) {
+      const unsigned long long q0 = __shfl_sync(0xFFFFFFFFu, q_next, 0);
+      if (q0 >= n_chunks || !ok) break;
+      if (lane == 0) q_next = atomicAdd(work, (unsigned long long)G);  // used by the next grab
+      // lanes c < G: metadata of chunk q0 + c
+      uint32_t grp = 0;
+      if (lane < G) {
+        const unsigned long long q = q0 + lane;
+        ChunkMeta cm{0, 0, 0};
+        if (q < n_chunks) {
           const uint64_t b = p.b_begin + q / cpb;
           const uint32_t start = (uint32_t)(q % cpb) * CH;
           const uint32_t len = p.blk_len[b];
-          if (start >= len) continue;
-          const uint32_t n = min(CH, len - start);
-          const uint64_t off = p.blk_off[b] + start;
-          const uint32_t m = p.mask[b];
-          const uint32_t grp = OPC == OP_TIES ? p.blk_group[b] : 0u;
-          const uint32_t bytes = (n * ES) & ~15u;
-          ok = produce((uint32_t)q, 0, off, n, m, grp, static_cast<const char*>(p.base) + off * ES, bytes);
-          for (uint32_t mm = m; ok && mm; mm &= mm - 1) {
+          cm.off = p.blk_off[b] + start;
+          cm.m = p.mask[b];
+          cm.n = start < len ? min(CH, len - start) : 0u;
+          if constexpr (OPC == OP_TIES) grp = p.blk_group[b];
+        }
+        S.chunk[lane] = cm;
+      }
+      if constexpr (OPC == OP_TIES) {
+        // lane i < K: the trim thresholds of expert i for every chunk of the grab, at least
+        // the smallest subnormal (a zero delta is never kept: it would add nothing)
+#pragma unroll
+        for (uint32_t c = 0; c < G; ++c) {
+          const uint32_t g = __shfl_sync(0xFFFFFFFFu, grp, c);
+          if (lane < p.K) S.thr[c][lane] = max(ties_bits_threshold(p.tau[(uint64_t)lane * p.n_groups + g]), 1u);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) {
+        const uint32_t nq = (uint32_t)min((unsigned long long)G, n_chunks - q0);
+        for (uint32_t c = 0; c < nq && ok; ++c) {
+          const ChunkMeta cm = S.chunk[c];
+          if (cm.n == 0) continue;
+          const uint32_t q = (uint32_t)(q0 + c);
+          const uint32_t bytes = (cm.n * ES) & ~15u;
+          ok = produce(q, 0, cm.off, cm.n, cm.m, 0u, static_cast<const char*>(p.base) + cm.off * ES, bytes);
+          for (uint32_t mm = cm.m; ok && mm; mm &= mm - 1) {
             const uint32_t i = __ffs(mm) - 1;
-            ok = produce((uint32_t)q, 1 + i, off, n, m, grp,
-                         static_cast<const char*>(p.experts.p[i]) + (off - p.expert_origin) * ES, bytes);
-            S.realized[i] += (unsigned long long)n * ES;
+            ok = produce(q, 1 + i, cm.off, cm.n, cm.m, OPC == OP_TIES ? S.thr[c][i] : 0u,
+                         static_cast<const char*>(p.experts.p[i]) + (cm.off - p.expert_origin) * ES, bytes);
+            S.realized[i] += (unsigned long long)cm.n * ES;
           }
         }
       }
-      if (ok) ok = produce(kEnd, 0, 0, 0, 0, 0, nullptr, 0);
+      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+      __syncwarp();
+    }
+    if (lane == 0) {
+      if (ok) ok = produce(kEnd, 0, 0, 0, 0, 0u, nullptr, 0);
       if (!ok) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
@@ -241,36 +356,36 @@ __global__ void __launch_bounds__(kThreads, 2)
       for (int u = 0; u < VPT; ++u) {
         const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
         read_vec<BF16>(slot, p.base, off, k0, n, n_tma, x0[u]);
+        if (remaining) {
 #pragma unroll
-        for (int e = 0; e < V; ++e) {
-          acc[u][e] = 0.0f;
-          Sg[u][e] = 0.0f;
-          Pp[u][e] = 0.0f;
-          Nn[u][e] = 0.0f;
-          cnt[u][e] = 0u;
+          for (int e = 0; e < V; ++e) {
+            acc[u][e] = 0.0f;
+            Sg[u][e] = 0.0f;
+            Pp[u][e] = 0.0f;
+            Nn[u][e] = 0.0f;
+            cnt[u][e] = 0u;
+          }
         }
       }
     } else {
       const uint32_t i = mt.which - 1;
       const void* src = p.experts.p[i];
       if constexpr (OPC == OP_TIES) {
-        const uint32_t tau = mt.tau;
+        // trim test on the magnitude's bits: key(|d|) >= tau exactly when bits(|d|) >= the
+        // producer's threshold (a NaN pattern, never true, when nothing is kept)
+        const float thr = __uint_as_float(mt.tau);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
           read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
 #pragma unroll
-          for (int e = 0; e < V; ++e) {
-            const float d = __fsub_rn(xe[e], x0[u][e]);
-            const uint32_t key = (uint32_t)__bfloat16_as_ushort(__float2bfloat16_rn(fabsf(d))) & 0x7FFFu;
-            const float dh = key >= tau ? d : 0.0f;
-            // branch-free tally: S, P and N are never -0, so adding +0 leaves them unchanged
-            const bool pos = dh > 0.0f, neg = dh < 0.0f;
-            Sg[u][e] = __fadd_rn(Sg[u][e], dh);
-            Pp[u][e] = __fadd_rn(Pp[u][e], pos ? dh : 0.0f);
-            Nn[u][e] = __fadd_rn(Nn[u][e], neg ? dh : 0.0f);
-            cnt[u][e] += (pos ? 1u : 0u) + (neg ? 0x10000u : 0u);
+          for (int e = 0; e < V; e += 2) {
+            // the deltas of an element pair in one packed fp32x2 subtract
+            float d0, d1;
+            f2_sub(xe[e], xe[e + 1], x0[u][e], x0[u][e + 1], d0, d1);
+            ties_tally(d0, thr, Sg[u][e], Pp[u][e], Nn[u][e], cnt[u][e]);
+            ties_tally(d1, thr, Sg[u][e + 1], Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
           }
         }
       } else {
@@ -283,13 +398,19 @@ __global__ void __launch_bounds__(kThreads, 2)
           uint32_t keep = 0xFFu;
           if constexpr (OPC == OP_DARE) {
             const uint64_t j0 = off + k0;
-            keep = dare_keep8(p.seed, i, j0 >> 3, p.dare_T) >> (uint32_t)(j0 & 7u);
+            keep = dare_keep8_rk(p.dare_rk, i, j0 >> 3, p.dare_T) >> (uint32_t)(j0 & 7u);
           }
 #pragma unroll
-          for (int e = 0; e < V; ++e) {
-            float d = __fsub_rn(xe[e], x0[u][e]);
-            if constexpr (OPC == OP_DARE) d = ((keep >> e) & 1u) ? __fmul_rn(d, p.sigma) : 0.0f;
-            acc[u][e] = __fmaf_rn(a, d, acc[u][e]);
+          for (int e = 0; e < V; e += 2) {
+            float d0, d1;
+            f2_sub(xe[e], xe[e + 1], x0[u][e], x0[u][e + 1], d0, d1);
+            if constexpr (OPC == OP_DARE) {
+              float s0, s1;
+              f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
+              d0 = ((keep >> e) & 1u) ? s0 : 0.0f;
+              d1 = ((keep >> (e + 1)) & 1u) ? s1 : 0.0f;
+            }
+            f2_fma(a, a, d0, d1, acc[u][e], acc[u][e + 1], acc[u][e], acc[u][e + 1]);
           }
         }
       }
@@ -303,14 +424,25 @@ __global__ void __launch_bounds__(kThreads, 2)
         const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
         if (k0 >= n) continue;
         float y[V];
+        if (mt.m == 0) {
+          // no expert selected: every accumulator is +0, so the output is M_0 plus the
+          // zero the operator adds (lambda * +0 for TIES, +0 otherwise)
+          const float z = OPC == OP_TIES ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
+#pragma unroll
+          for (int e = 0; e < V; ++e) y[e] = __fadd_rn(x0[u][e], z);
+          store_vec<BF16>(p.out, off + k0, n - k0, y);
+          continue;
+        }
 #pragma unroll
         for (int e = 0; e < V; ++e) {
           if constexpr (OPC == OP_TIES) {
             // one division per element: the mean of the entries whose sign was elected
-            const bool pos = Sg[u][e] > 0.0f;
-            const float num = pos ? Pp[u][e] : Nn[u][e];
-            const uint32_t c = pos ? (cnt[u][e] & 0xFFFFu) : (cnt[u][e] >> 16);
-            const float mm = Sg[u][e] != 0.0f ? __fdiv_rn(num, __uint2float_rn(c)) : 0.0f;
+            // (S != 0 implies at least one of them, so c >= 1; otherwise +0 / 1 = +0)
+            const bool pos = Sg[u][e] > 0.0f, any = Sg[u][e] != 0.0f;
+            const float num = any ? (pos ? Pp[u][e] : Nn[u][e]) : 0.0f;
+            const uint32_t c = any ? (pos ? (cnt[u][e] & 0xFFFFu) : (cnt[u][e] >> 16)) : 0u;
+            const float2 cy = S.ctab[c];
+            const float mm = div_small(num, cy.x, cy.y);
             y[e] = __fmaf_rn(p.lambda, mm, x0[u][e]);
           } else {
             y[e] = __fadd_rn(x0[u][e], acc[u][e]);
@@ -333,11 +465,11 @@ cudaError_t launch_op(const MergeLaunch& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  const size_t smem = sizeof(Smem<Geo<OPC>::kSlots, Geo<OPC>::kSlotBytes>);
+  const size_t smem = sizeof(Smem<Geo<OPC>::kSlots, Geo<OPC>::kSlotBytes, Geo<OPC>::kGrab>);
   if ((e = cudaFuncSetAttribute(merge_tma_kernel<BF16, OPC>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) !=
       cudaSuccess)
     return e;
-  uint64_t grid = (uint64_t)sms * 2;
+  uint64_t grid = (uint64_t)sms * Geo<OPC>::kCtasPerSm;
   if (grid > n_chunks) grid = n_chunks;
   if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
   merge_tma_kernel<BF16, OPC><<<(unsigned)grid, kThreads, smem, st>>>(p, cpb, n_chunks, p.work);

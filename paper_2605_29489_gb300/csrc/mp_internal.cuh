@@ -203,6 +203,7 @@ struct MergeLaunch {
   float lambda;
   float sigma;          // DARE rescale
   uint32_t dare_T;      // DARE keep threshold on 16-bit words
+  uint32_t dare_rk[10][2];  // DARE: Philox round keys of the seed (precomputed on the host)
   uint64_t seed;
   unsigned long long* realized;  // [kCounterSlots][K]
   unsigned long long* work;      // chunk counter of the dynamic scheduler (zeroed per launch)

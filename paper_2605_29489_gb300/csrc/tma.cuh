@@ -52,6 +52,15 @@ __device__ __forceinline__ void mbar_wait_drain(uint64_t* bar, uint32_t parity) 
     if (mbar_try_wait(bar, parity)) return;
 }
 
+// Orders the shared-memory accesses this thread has observed before the async-proxy writes
+// of a bulk copy it issues next.  The producer calls it after acquiring a slot's "empty"
+// mbarrier and before refilling the slot: the consumers' reads of the old contents are
+// generic-proxy accesses, the refill an async-proxy write, and only a proxy fence orders
+// the two (without it a refill can land before a consumer's read has been performed).
+__device__ __forceinline__ void fence_proxy_async_smem() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
 __device__ __forceinline__ void tma_load_1d(void* dst, const void* src, uint32_t bytes, uint64_t* bar) {
   asm volatile(
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(su32(dst)),
