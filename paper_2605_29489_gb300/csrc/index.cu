@@ -72,17 +72,27 @@ __device__ __forceinline__ uint32_t ties_key(float d) {
 // ---- the catalog pass: TMA producer / consumer pipeline ---------------------------------
 //
 // Work item = (block, group of up to KG experts); items are handed out through a global
-// counter.  The producer thread streams every 8 KiB chunk of the item's block — the base
-// chunk, then each expert's chunk — into a ring of shared-memory slots (cp.async.bulk,
-// completion on the slot's "full" mbarrier).  Consumer thread l (0..255) is lane l of the
-// fixed summation order: chunk c holds vectors 512c .. 512c+511, and thread l takes
-// vectors 512c+l and 512c+256+l, i.e. exactly its own vectors l, l+256, ... in increasing
-// order.  At the end of the block the 256 lane sums are combined by the xor butterfly.
+// counter.  The producer thread streams every chunk of the item's block — the base chunk,
+// then each expert's chunk — into a ring of shared-memory slots (cp.async.bulk, completion
+// on the slot's "full" mbarrier).  Consumer thread l (0..255) is lane l of the fixed
+// summation order: a chunk of VPT * 256 vectors starts at vector VPT * 256 * c, and thread
+// l takes its vectors VPT * 256 * c + 256 u + l (u < VPT), i.e. exactly its own vectors l,
+// l + 256, ... in increasing order.  At the end of the block the 256 lane sums are
+// combined by the xor butterfly.
 constexpr int kIxConsumers = 256;
 constexpr int kIxThreads = kIxConsumers + 32;
-constexpr uint32_t kIxSlotBytes = 8192;
-constexpr int kIxSlots = 12;
 constexpr uint32_t kIxEnd = 0xFFFFFFFFu;
+
+// ring geometry.  The plain catalog is bound by HBM: two CTAs per SM with twelve 8 KiB
+// slots.  The TIES catalog also bins every delta, which makes it bound by instruction
+// latency: three CTAs per SM (more warps to hide it) with sixteen 4 KiB slots (one vector
+// per consumer thread and fill, so that the state fits the smaller register budget).
+template <bool TIES>
+struct IxGeo {
+  static constexpr int kCtasPerSm = TIES ? 3 : 2;
+  static constexpr uint32_t kSlotBytes = TIES ? 4096u : 8192u;
+  static constexpr int kSlots = TIES ? 16 : 12;
+};
 
 struct IxMeta {
   uint64_t off;    // element offset of the chunk
@@ -92,12 +102,12 @@ struct IxMeta {
   uint32_t pad;
 };
 
-template <int KG>
+template <int KG, int NS, uint32_t SB>
 struct __align__(128) IxSmem {
-  uint8_t slot[kIxSlots][kIxSlotBytes];
-  IxMeta meta[kIxSlots];
-  uint64_t full[kIxSlots];
-  uint64_t empty[kIxSlots];
+  uint8_t slot[NS][SB];
+  IxMeta meta[NS];
+  uint64_t full[NS];
+  uint64_t empty[NS];
   uint32_t hist[KG][256];
   float red_ss[KG][8];
   float red_mx[KG][8];
@@ -158,16 +168,49 @@ __device__ __forceinline__ void ties_bin2(float d0, float d1, uint32_t hist, uin
       : "memory");
 }
 
+// TIES fine bins of two deltas: a nonzero delta whose coarse bin (key bits 7..14) is es
+// adds 1 to fine bin (key & 127) of the shared histogram at hist; predicated, no branch
+__device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint32_t hist) {
+  asm volatile(
+      "{\n"
+      " .reg .pred p0, p1;\n"
+      " .reg .b32 w, k0, k1, e0, e1, a0, a1;\n"
+      " cvt.rn.bf16x2.f32 w, %2, %1;\n"
+      " and.b32 k0, w, 32767;\n"
+      " shr.b32 k1, w, 16;\n"
+      " and.b32 k1, k1, 32767;\n"
+      " shr.b32 e0, k0, 7;\n"
+      " shr.b32 e1, k1, 7;\n"
+      " setp.ne.f32 p0, %1, 0f00000000;\n"
+      " setp.ne.f32 p1, %2, 0f00000000;\n"
+      " setp.eq.and.u32 p0, e0, %3, p0;\n"
+      " setp.eq.and.u32 p1, e1, %3, p1;\n"
+      " and.b32 a0, k0, 127;\n"
+      " and.b32 a1, k1, 127;\n"
+      " shl.b32 a0, a0, 2;\n"
+      " shl.b32 a1, a1, 2;\n"
+      " add.u32 a0, a0, %0;\n"
+      " add.u32 a1, a1, %0;\n"
+      " @p0 red.shared.add.u32 [a0], 1;\n"
+      " @p1 red.shared.add.u32 [a1], 1;\n"
+      "}\n" ::"r"(hist),
+      "f"(d0), "f"(d1), "r"(es)
+      : "memory");
+}
+
 template <bool BF16, int KG, bool TIES>
-__global__ void __launch_bounds__(kIxThreads, 2)
+__global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
+  constexpr int kIxSlots = IxGeo<TIES>::kSlots;
+  constexpr uint32_t kIxSlotBytes = IxGeo<TIES>::kSlotBytes;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t CH = kIxSlotBytes / ES;
   constexpr int V = BF16 ? 8 : 4;
   constexpr int VPT = (int)(CH / (kIxConsumers * V));
-  static_assert(VPT == 2, "chunk geometry");
+  static_assert(VPT >= 1 && CH == (uint32_t)(VPT * kIxConsumers * V), "chunk geometry");
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  IxSmem<KG>& S = *reinterpret_cast<IxSmem<KG>*>(smem_raw);
+  using Sm = IxSmem<KG, kIxSlots, kIxSlotBytes>;
+  Sm& S = *reinterpret_cast<Sm*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   volatile int* abort_flag = &S.abort;
 
@@ -291,7 +334,9 @@ __global__ void __launch_bounds__(kIxThreads, 2)
       }
       const uint8_t* slot = S.slot[fill % kIxSlots];
       uint4 re[VPT];
-      bool same = bfin;
+      // the equality test pays off only for TIES, whose per-element binning it skips; for
+      // the other operators the comparison and vote cost more than the arithmetic they save
+      bool same = TIES && bfin;
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
         re[u] = ix_read_raw<BF16>(slot, p.experts.p[i0 + k], off - p.expert_origin,
@@ -307,19 +352,28 @@ __global__ void __launch_bounds__(kIxThreads, 2)
         for (int u = 0; u < VPT; ++u) {
           float xe[V];
           unpack<BF16>(re[u], xe);
+          float d[V];
+#pragma unroll
+          for (int e = 0; e < V; ++e) d[e] = __fsub_rn(xe[e], xb[u][e]);
+          // the sum of squares is one fma chain in element order (the canonical order);
+          // max |d| and the counts are exact in any order, so they take a tree
+#pragma unroll
+          for (int e = 0; e < V; ++e) ss[k] = __fmaf_rn(d[e], d[e], ss[k]);
+          float m[V / 2];
+#pragma unroll
+          for (int e = 0; e < V / 2; ++e) m[e] = fmaxf(fabsf(d[2 * e]), fabsf(d[2 * e + 1]));
+#pragma unroll
+          for (int w = V / 4; w >= 1; w >>= 1)
+#pragma unroll
+            for (int e = 0; e < w; ++e) m[e] = fmaxf(m[e], m[e + w]);
+          mx[k] = fmaxf(mx[k], m[0]);
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
-            const float d0 = __fsub_rn(xe[e], xb[u][e]);
-            const float d1 = __fsub_rn(xe[e + 1], xb[u][e + 1]);
-            ss[k] = __fmaf_rn(d0, d0, ss[k]);
-            ss[k] = __fmaf_rn(d1, d1, ss[k]);
-            mx[k] = fmaxf(mx[k], fabsf(d0));
-            mx[k] = fmaxf(mx[k], fabsf(d1));
             if constexpr (TIES) {
-              ties_bin2(d0, d1, su32(&S.hist[k][0]), nz[k]);
+              ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]), nz[k]);
             } else {
-              nz[k] += d0 != 0.0f ? 1u : 0u;
-              nz[k] += d1 != 0.0f ? 1u : 0u;
+              nz[k] += d[e] != 0.0f ? 1u : 0u;
+              nz[k] += d[e + 1] != 0.0f ? 1u : 0u;
             }
           }
         }
@@ -470,11 +524,8 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
       float xe[V];
       unpack<BF16>(load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len), xe);
 #pragma unroll
-      for (int e = 0; e < V; ++e) {
-        float d = __fsub_rn(xe[e], xb[e]);
-        uint32_t key = ties_key(d);
-        if (d != 0.0f && (key >> 7) == estar[k]) atomicAdd(&s_fine[k][key & 127u], 1u);
-      }
+      for (int e = 0; e < V; e += 2)
+        ties_fine2(__fsub_rn(xe[e], xb[e]), __fsub_rn(xe[e + 1], xb[e + 1]), estar[k], su32(&s_fine[k][0]));
     }
   }
   __syncthreads();
@@ -534,8 +585,10 @@ cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  const size_t smem = sizeof(IxSmem<KG>);
-  uint64_t grid = (uint64_t)sms * 2;
+  const int per_sm = ties ? IxGeo<true>::kCtasPerSm : IxGeo<false>::kCtasPerSm;
+  const size_t smem = ties ? sizeof(IxSmem<KG, IxGeo<true>::kSlots, IxGeo<true>::kSlotBytes>)
+                           : sizeof(IxSmem<KG, IxGeo<false>::kSlots, IxGeo<false>::kSlotBytes>);
+  uint64_t grid = (uint64_t)sms * per_sm;
   if (grid > n_items) grid = n_items;
   if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
   if (ties) {
