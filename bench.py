@@ -54,6 +54,8 @@ def workloads():
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
         "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
                                   desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE p=0.9 then AVG, per-expert active sets"),
+        "qwen2.5-1.5b-dare-2l": dict(make=lambda: synth.qwen25_15b(layers=2), op="dare", drop_p=0.9, budgets=[0.25],
+                                     desc="Qwen2.5-1.5B shapes cut to 2 layers (profiling case), K=16, DARE p=0.9"),
         "llama-3-8b-hostpool-avg": dict(make=lambda: synth.llama3_8b(K=8), op="avg", budgets=[1.0, 0.25, 0.1],
                                         host_pool=True,
                                         desc="Llama-3-8B-shaped bf16 base in HBM, K=8 experts (128 GB) in pinned host "
@@ -62,6 +64,10 @@ def workloads():
                                          budgets=[1.0, 0.25, 0.1], host_pool=True,
                                          desc="Llama-3-8B-shaped bf16 base in HBM, K=8 experts (128 GB) in pinned host "
                                               "memory, TIES density 0.2"),
+        "qwen2.5-0.5b-ta-touched": dict(make=lambda: synth.qwen25_05b(), op="ta", lam=0.3,
+                                        budgets=[1.0, 0.5, 0.25, 0.1], touched=True,
+                                        desc="as qwen2.5-0.5b-ta, merged with mp_merge_touched: only touched blocks "
+                                             "are read and written (Alg. 2 WriteBlockOrReference)"),
         "tiny-avg": dict(make=lambda: synth.tiny(), op="avg", budgets=[1.0, 0.5, 0.25],
                          desc="8 fp32 512x512 tensors, K=4, AVG, 4Ki-element blocks"),
     }
@@ -276,6 +282,8 @@ def native(args, rank, world, local_rank):
     outs = [torch.empty_like(base)] if shared_out else [torch.empty_like(base) for _ in budgets]
     Bs = [mp.mp_budget_from_fraction(mf, f) for f in budgets]
     stream = torch.cuda.current_stream()
+    touched_mode = bool(W.get("touched"))
+    merge_fn = mp.mp_merge_touched if touched_mode else mp.mp_merge
 
     def step(fam_c, ev=None):
         hs = []
@@ -291,7 +299,7 @@ def native(args, rank, world, local_rank):
             plan = mp.mp_plan(idx, gop, B, stream)
             if ev is not None:
                 ev["p1"][k].record(stream)
-            man = mp.mp_merge(fam_c, idx, plan, outs[0 if shared_out else k], stream)
+            man = merge_fn(fam_c, idx, plan, outs[0 if shared_out else k], stream)
             if ev is not None:
                 ev["m1"][k].record(stream)
             hs += [plan, man]
@@ -336,18 +344,22 @@ def native(args, rank, world, local_rank):
     merge_ms = [statistics.mean(e["p1"][k].elapsed_time(e["m1"][k]) for e in evs) for k in range(len(Bs))]
     last = handles[-1]
     per_budget = []
+    blk_len = fam.block_table()[1]
     for k, f in enumerate(budgets):
-        pi = mp.mp_plan_info(last[1 + 2 * k], with_arrays=False)
+        pi = mp.mp_plan_info(last[1 + 2 * k], last[0] if touched_mode else None, with_arrays=touched_mode)
         mi = mp.mp_manifest_info(last[2 + 2 * k], fam.K)
         per_budget.append(dict(f=f, budget_bytes=Bs[k], planned_bytes=pi["chat"], realized_bytes=mi["realized_total"],
                                n_selected=pi["n_sel"], n_candidates=pi["n_cand"], touched_blocks=mi["touched"],
                                touched_ratio=pi["chat"] / (fam.K * N * es), plan_ms=plan_ms[k], merge_ms=merge_ms[k]))
+        if touched_mode:
+            per_budget[-1]["touched_elements"] = int(np.asarray(blk_len)[np.asarray(pi["mask"]) != 0].sum())
     for hs in handles:
         for h in hs:
             h.free()
 
     peak, peak_kind = hbm_peak()
-    alg_bytes = [2 * N * es + pb["planned_bytes"] for pb in per_budget]
+    # base read + output write of every materialised element, plus the planned expert reads
+    alg_bytes = [2 * (pb["touched_elements"] if touched_mode else N) * es + pb["planned_bytes"] for pb in per_budget]
     for pb, ab in zip(per_budget, alg_bytes):
         s = pb["merge_ms"] / 1e3
         pb.update(merged_params_per_s=N / s, expert_gbs=pb["planned_bytes"] / s / 1e9, hbm_bytes=ab,
@@ -420,11 +432,12 @@ def native(args, rank, world, local_rank):
                    "step": "index + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
         "index_ms": idx_ms, "per_budget": per_budget,
-        "roofline": {"bound": "hbm", "kernel": "merge_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
+        "roofline": {"bound": "hbm", "kernel": "merge_tma_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
                      "traffic": profiled_traffic(args.workload),
-                     "algorithmic_bytes": "per merged parameter 2*s + s*(selected experts); summed over the "
+                     "algorithmic_bytes": ("per materialised (touched) parameter" if touched_mode else
+                                           "per merged parameter") + " 2*s + s*(selected experts); summed over the "
                                           "budget sweep's launches / their summed CUDA-event time"},
         "gpu_launches": launches,
         "host_link": None if link is None else dict(
@@ -472,6 +485,87 @@ def _max_over_ranks(x: float, world: int) -> float:
     return float(t.item())
 
 
+# ---- K-scaling at a fixed absolute budget (Cor. 1) --------------------------------------------------
+
+def k_sweep(args):
+    """Cor. 1: with the expert-read budget B fixed in bytes, the bytes a merge reads from the
+    experts stay at most B however many experts the family has, while a full read grows as K.
+    For Qwen2.5-0.5B-shaped families with K = 4 ... 32 and the operators of Tab. 1 (AVG, TIES,
+    DARE), time the catalog, then plan + merge at the full budget (the naive full read) and at
+    the fixed budget, all with CUDA events on the launching stream."""
+    import torch
+    import paper_2605_29489_gb300 as mp
+    from paper_2605_29489_gb300 import synth
+
+    torch.cuda.set_device(0)
+    stream = torch.cuda.current_stream()
+    ks = [int(k) for k in args.k_list.split(",")]
+    rows = []
+    launches0 = mp.mp_kernel_launch_count()
+    clocks = ClockSampler(0)
+    clocks.start()
+    for K in ks:
+        fam = synth.qwen25_05b(K=K)
+        base, experts = fam.device_arrays()
+        offs, nums, total = fam.layout()
+        mf = mp.family(list(zip(offs.tolist(), nums.tolist())), base, experts, fam.block_elems, fam.dtype, 0)
+        N, es = fam.n_params, fam.elem_size
+        B_fixed = int(args.k_budget_experts * N * es)
+        out = torch.empty_like(base)
+        for opn in ("avg", "ties", "dare"):
+            W = {"op": opn, "density": 0.2, "drop_p": 0.9}
+            gop, _ = make_ops(W, K)
+            t = {"index": [], "plan_full": [], "merge_full": [], "plan_fixed": [], "merge_fixed": []}
+            info = {}
+            for it in range(args.warmup + args.steps):
+                ev = [torch.cuda.Event(enable_timing=True) for _ in range(6)]
+                ev[0].record(stream)
+                idx = mp.mp_index_blocks(mf, gop, stream)
+                ev[1].record(stream)
+                hs = [idx]
+                for j, B in enumerate((mp.mp_budget_from_fraction(mf, 1.0), B_fixed)):
+                    plan = mp.mp_plan(idx, gop, B, stream)
+                    ev[2 + 2 * j].record(stream)
+                    man = mp.mp_merge(mf, idx, plan, out, stream)
+                    ev[3 + 2 * j].record(stream)
+                    hs += [plan, man]
+                torch.cuda.synchronize()
+                if it >= args.warmup:
+                    t["index"].append(ev[0].elapsed_time(ev[1]))
+                    t["plan_full"].append(ev[1].elapsed_time(ev[2]))
+                    t["merge_full"].append(ev[2].elapsed_time(ev[3]))
+                    t["plan_fixed"].append(ev[3].elapsed_time(ev[4]))
+                    t["merge_fixed"].append(ev[4].elapsed_time(ev[5]))
+                if it == args.warmup + args.steps - 1:
+                    for name, (pl, mn) in (("full", (hs[1], hs[2])), ("fixed", (hs[3], hs[4]))):
+                        pi = mp.mp_plan_info(pl, with_arrays=False)
+                        mi = mp.mp_manifest_info(mn, K)
+                        info[name] = dict(planned_bytes=pi["chat"], realized_bytes=mi["realized_total"],
+                                          touched_blocks=mi["touched"], n_selected=pi["n_sel"])
+                for h in hs:
+                    h.free()
+            med = {k: statistics.median(v) for k, v in t.items()}
+            rows.append(dict(K=K, op=opn, budget_fixed_bytes=B_fixed, c_full_bytes=K * N * es,
+                             index_ms=med["index"],
+                             full=dict(plan_ms=med["plan_full"], merge_ms=med["merge_full"], **info["full"]),
+                             fixed=dict(plan_ms=med["plan_fixed"], merge_ms=med["merge_fixed"], **info["fixed"]),
+                             io_reduction=1.0 - info["fixed"]["realized_bytes"] / max(1, info["full"]["realized_bytes"]),
+                             merge_speedup=med["merge_full"] / med["merge_fixed"]))
+        del base, experts, out, mf
+        torch.cuda.empty_cache()
+    clk = clocks.stop()
+    launches = mp.mp_kernel_launch_count() - launches0
+    fixed_ms = sum(r["fixed"]["merge_ms"] + r["fixed"]["plan_ms"] for r in rows)
+    return {"metric": "merge time and expert-read bytes vs K at a fixed absolute budget (Cor. 1)",
+            "value": statistics.mean(r["merge_speedup"] for r in rows), "unit": "x (full-read merge / fixed-budget merge)",
+            "n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "ms_per_step": fixed_ms / len(rows),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": "k-sweep", "family": "Qwen2.5-0.5B shapes", "K": ks,
+                       "budget_fixed": f"{args.k_budget_experts} x one expert's bytes",
+                       "ops": ["avg", "ties rho=0.2", "dare p=0.9"], "l2": "inputs larger than L2 (no flush)"},
+            "rows": rows, "gpu_launches": launches, "clocks": clk}
+
+
 # ---- reference arm (the CPU oracle) ----------------------------------------------------------------
 
 def reference(args):
@@ -506,6 +600,11 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--k-sweep", action="store_true",
+                    help="K-scaling at a fixed absolute budget (Cor. 1) instead of the workload sweep")
+    ap.add_argument("--k-list", default="4,8,16,32")
+    ap.add_argument("--k-budget-experts", type=float, default=0.25,
+                    help="the fixed budget of --k-sweep, in units of one expert checkpoint's bytes")
     args = ap.parse_args()
     if args.warmup < 3:
         ap.error("--warmup must be >= 3")
@@ -517,6 +616,10 @@ def main():
     if args.impl == "reference":
         if rank == 0:
             print(json.dumps(reference(args)), flush=True)
+        return
+    if args.k_sweep:
+        if rank == 0:
+            print(json.dumps(k_sweep(args)), flush=True)
         return
 
     if world > 1:

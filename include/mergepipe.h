@@ -11,7 +11,9 @@
  *   mp_plan          a deterministic access plan under an expert-read budget
  *                    B (Alg. 1 PlanGen; Eq. 2, 3 and 6);
  *   mp_merge         the induced budgeted operator over only the planned
- *                    blocks (Eq. 4; Alg. 2 ExecuteMerge) and its manifest.
+ *                    blocks (Eq. 4; Alg. 2 ExecuteMerge) and its manifest;
+ *                    mp_merge_touched writes only the touched blocks and leaves
+ *                    the rest as references to the base (WriteBlockOrReference).
  *
  * Conventions
  *  - Data pointers are device pointers unless stated (experts may also live in
@@ -90,6 +92,9 @@ typedef struct {
   uint32_t trim_scope; /* TIES: 0 = trim per (expert, tensor), 1 = per expert */
   double drop_p;       /* DARE: drop probability p in [0, 1] */
   uint64_t seed;       /* DARE: seed of the fixed random mask omega */
+  uint32_t score_mode; /* planning score (Sec. 3, Eq. 6 and the heuristics that follow it):
+                          0 = u = |coef_i| * ||Delta||_2 (Prop. 2's utility);
+                          1 = score per byte, u / c in fp32 (c = the block's bytes) */
 } mp_op;
 
 typedef struct mp_index_s mp_index;
@@ -149,6 +154,21 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
  */
 mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out,
                    mp_stream stream, mp_manifest** man);
+
+/*
+ * mp_merge_touched — Alg. 2 with WriteBlockOrReference: only the touched blocks (at least
+ * one selected expert) are materialised; every other block of the merged checkpoint is a
+ * reference to the base block and is neither read nor written.  For a touched block, out
+ * receives exactly what mp_merge writes there; out keeps its previous contents everywhere
+ * else.  out may therefore be the base itself (an in-place merge: each chunk is read before
+ * its output is written and chunks are disjoint) or any buffer the caller has filled, e.g.
+ * a copy of the base; it must not overlap an expert, nor overlap the base without being the
+ * base.  The bytes moved drop from 2 N s + C_hat to 2 (touched elements) s + C_hat.  Untouched
+ * blocks keep the base's bits exactly, where mp_merge writes M_0 + 0 (which turns a -0
+ * into +0).  Other arguments, the manifest and errors as mp_merge.
+ */
+mp_status mp_merge_touched(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out,
+                           mp_stream stream, mp_manifest** man);
 
 /*
  * mp_plan_noalloc — the same access plan as mp_plan, for callers that cannot allocate.

@@ -27,7 +27,7 @@ _lib = None
 class _Op(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("K", ctypes.c_uint32), ("alpha", ctypes.c_void_p),
                 ("lambda_", ctypes.c_float), ("density", ctypes.c_float), ("trim_scope", ctypes.c_uint32),
-                ("drop_p", ctypes.c_double), ("seed", ctypes.c_uint64)]
+                ("drop_p", ctypes.c_double), ("seed", ctypes.c_uint64), ("score_mode", ctypes.c_uint32)]
 
 
 class _Family(ctypes.Structure):
@@ -88,15 +88,15 @@ class OracleError(RuntimeError):
 class Op:
     """Merge operator and parameters (mirrors the oracle's orc_op)."""
 
-    def __init__(self, kind, K, alpha=None, lam=1.0, density=0.2, trim_scope=0, drop_p=0.0, seed=0):
+    def __init__(self, kind, K, alpha=None, lam=1.0, density=0.2, trim_scope=0, drop_p=0.0, seed=0, score_mode=0):
         self.kind, self.K = kind, K
         self.alpha = None if alpha is None else np.ascontiguousarray(np.asarray(alpha, np.float32))
         self.lam, self.density, self.trim_scope = float(lam), float(density), int(trim_scope)
-        self.drop_p, self.seed = float(drop_p), int(seed)
+        self.drop_p, self.seed, self.score_mode = float(drop_p), int(seed), int(score_mode)
 
     def c(self):
         return _Op(self.kind, self.K, None if self.alpha is None else self.alpha.ctypes.data,
-                   self.lam, self.density, self.trim_scope, self.drop_p, self.seed)
+                   self.lam, self.density, self.trim_scope, self.drop_p, self.seed, self.score_mode)
 
 
 class Family:

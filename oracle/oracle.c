@@ -234,7 +234,9 @@ uint64_t orc_splitmix64(uint64_t state) {
  *    with nnz = 0 contributes exactly nothing to any operator, and under TIES a unit
  *    whose largest key is below tau is trimmed entirely; both are left out (exact).
  *  - Score s(i,t,b) = |coef_i| * ||Delta_{i,t,b}||_2 in fp32 (the utility u of Prop. 2);
- *    coef_i = alpha_i (AVG, TA, DARE) or lambda (TIES).
+ *    coef_i = alpha_i (AVG, TA, DARE) or lambda (TIES).  In the score-per-byte mode (the
+ *    second heuristic Sec. 3 names for the objective of Eq. 6) s is divided by the unit's
+ *    byte cost c, one fp32 division.
  *  - Sort by decreasing score; ties by ascending unit id = b*K + i (block order is
  *    tensor/block order, then expert).  The key is unique, so the order is total.
  *  - Greedy fill: take a candidate if C_hat + c <= B, otherwise skip it and go on.
@@ -242,7 +244,7 @@ uint64_t orc_splitmix64(uint64_t state) {
  *  - Record: mask (bit i of word b = A_{i,t,b}), C_hat, number selected, the selected-
  *    block digest and the traversal order.  Reading of the digest: FNV-1a 64 over the
  *     little-endian bytes of (kind, K, alpha[0..K-1] bits, lambda bits, density bits,
- *     trim_scope, drop_p bits, seed, B, C_hat, n_sel, set_hash), where set_hash is the
+ *     trim_scope, drop_p bits, seed, score_mode, B, C_hat, n_sel, set_hash), where set_hash is the
  *     wrapping sum over selected units u of splitmix64(u).
  * Pins: brute force over all subsets on tiny inputs; the cardinality-knapsack optimum
  * when all costs are equal; Prop. 1 (C_hat <= B); full budget selects every candidate.
@@ -293,6 +295,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
       q[nq].score = fabsf(coef) * norm[s];
       q[nq].unit = (uint32_t)(b * K + i);
       q[nq].cost = blk_len[b] * elem_size;
+      if (op->score_mode) q[nq].score = q[nq].score / (float)q[nq].cost;
       ++nq;
     }
   }
@@ -311,7 +314,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
   }
   free(q);
 
-  uint8_t hdr[4 + 4 + 4 * 32 + 4 + 4 + 4 + 8 + 8 + 8 + 8 + 8 + 8];
+  uint8_t hdr[4 + 4 + 4 * 32 + 4 + 4 + 4 + 8 + 8 + 4 + 8 + 8 + 8 + 8];
   size_t o = 0;
   o += put_u32(hdr + o, (uint32_t)op->kind);
   o += put_u32(hdr + o, K);
@@ -323,6 +326,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
   memcpy(&pbits, &op->drop_p, 8);
   o += put_u64(hdr + o, pbits);
   o += put_u64(hdr + o, op->seed);
+  o += put_u32(hdr + o, op->score_mode);
   o += put_u64(hdr + o, budget);
   o += put_u64(hdr + o, chat);
   o += put_u64(hdr + o, nsel);

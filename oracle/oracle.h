@@ -38,6 +38,7 @@ typedef struct {
   uint32_t trim_scope; /* TIES: 0 = per (expert, tensor), 1 = per expert */
   double drop_p;       /* DARE: drop probability p */
   uint64_t seed;       /* DARE: seed of the fixed random mask omega */
+  uint32_t score_mode; /* planning score: 0 = |coef_i| * norm; 1 = that per byte of the block */
 } orc_op;
 
 /* block geometry plus data: blocks are disjoint spans of the flat checkpoints (Sec. 2) */

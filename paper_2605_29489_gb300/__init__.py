@@ -22,7 +22,7 @@ import numpy as np
 
 __all__ = [
     "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MergePipeError",
-    "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_free", "mp_index_stats",
+    "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_budget_from_fraction", "mp_last_error",
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "lib", "library_path",
 ]
@@ -53,7 +53,7 @@ class _Family(ctypes.Structure):
 class _Op(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("alpha", ctypes.POINTER(ctypes.c_float)), ("lambda_", ctypes.c_float),
                 ("density", ctypes.c_float), ("trim_scope", ctypes.c_uint32), ("drop_p", ctypes.c_double),
-                ("seed", ctypes.c_uint64)]
+                ("seed", ctypes.c_uint64), ("score_mode", ctypes.c_uint32)]
 
 
 _lib = None
@@ -74,6 +74,7 @@ def lib():
             ("mp_index_blocks", [vp, vp, vp, vp]),
             ("mp_plan", [vp, vp, u64, vp, vp]),
             ("mp_merge", [vp, vp, vp, vp, vp, vp]),
+            ("mp_merge_touched", [vp, vp, vp, vp, vp, vp]),
             ("mp_index_stats", [vp, vp, vp, vp, vp]),
             ("mp_index_shape", [vp, vp, vp, vp]),
             ("mp_plan_info", [vp, vp, vp, vp, vp, vp, vp]),
@@ -142,18 +143,18 @@ def family(tensors, base, experts, block_elems=65536, dtype=None, experts_locati
 
 
 class Op:
-    def __init__(self, kind, alpha, lam, density, trim_scope, drop_p, seed):
+    def __init__(self, kind, alpha, lam, density, trim_scope, drop_p, seed, score_mode=0):
         self.alpha = None if alpha is None else np.ascontiguousarray(np.asarray(alpha, np.float32))
         ap = None if self.alpha is None else self.alpha.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
-        self.c = _Op(kind, ap, lam, density, trim_scope, drop_p, seed)
+        self.c = _Op(kind, ap, lam, density, trim_scope, drop_p, seed, score_mode)
         self.kind = kind
 
     def ref(self):
         return ctypes.byref(self.c)
 
 
-def make_op(kind, alpha=None, lam=1.0, density=0.2, trim_scope=0, drop_p=0.0, seed=0) -> Op:
-    return Op(kind, alpha, float(lam), float(density), int(trim_scope), float(drop_p), int(seed))
+def make_op(kind, alpha=None, lam=1.0, density=0.2, trim_scope=0, drop_p=0.0, seed=0, score_mode=0) -> Op:
+    return Op(kind, alpha, float(lam), float(density), int(trim_scope), float(drop_p), int(seed), int(score_mode))
 
 
 class Handle:
@@ -198,6 +199,13 @@ def mp_merge(fam: Family, index: Handle, plan: Handle, out, stream=None) -> Hand
     man = ctypes.c_void_p()
     _check(lib().mp_merge(fam.ref(), ctypes.c_void_p(index.ptr), ctypes.c_void_p(plan.ptr), ctypes.c_void_p(_ptr(out)),
                           ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(man)))
+    return Handle(man.value, "manifest")
+
+
+def mp_merge_touched(fam: Family, index: Handle, plan: Handle, out, stream=None) -> Handle:
+    man = ctypes.c_void_p()
+    _check(lib().mp_merge_touched(fam.ref(), ctypes.c_void_p(index.ptr), ctypes.c_void_p(plan.ptr),
+                                  ctypes.c_void_p(_ptr(out)), ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(man)))
     return Handle(man.value, "manifest")
 
 

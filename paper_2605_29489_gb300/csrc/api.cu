@@ -174,6 +174,7 @@ mp_status check_op(const mp_op* op, uint32_t K) {
   }
   if (op->kind == MP_OP_DARE && !(op->drop_p >= 0.0 && op->drop_p <= 1.0))
     return fail(MP_ERR_INVALID_ARG, "drop_p must be in [0, 1]");
+  if (op->score_mode > 1) return fail(MP_ERR_INVALID_ARG, "score_mode must be 0 or 1");
   return MP_OK;
 }
 
@@ -631,6 +632,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   p.n_groups = index->n_groups;
   p.elem_size = g.elem_size;
   p.op_kind = op->kind;
+  p.score_mode = op->score_mode;
   for (uint32_t i = 0; i < g.K; ++i) p.coef[i] = fabsf(op->kind == MP_OP_TIES ? op->lambda : op->alpha[i]);
   p.blk_len = index->d_blk_len;
   p.blk_group = index->d_blk_group;
@@ -654,6 +656,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   memcpy(&pb, &op->drop_p, 8);
   put_u64(hdr, pb);
   put_u64(hdr, op->seed);
+  put_u32(hdr, op->score_mode);
   put_u64(hdr, budget_bytes);
   memcpy(p.hdr_prefix, hdr.data(), hdr.size());
   p.hdr_prefix_len = (uint32_t)hdr.size();
@@ -669,8 +672,14 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   return MP_OK;
 }
 
-mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
-                   mp_stream stream, mp_manifest** man_out) {
+}  // extern "C"
+
+namespace {
+
+// mp_merge and mp_merge_touched: touched_only leaves every block whose mask is empty
+// unwritten (and then out may be the base itself)
+mp_status merge_common(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
+                       mp_stream stream, mp_manifest** man_out, bool touched_only) {
   if (!man_out) return fail(MP_ERR_INVALID_ARG, "manifest out is NULL");
   *man_out = nullptr;
   mp_status st;
@@ -693,7 +702,9 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
       const char* a = static_cast<const char*>(q);
       return a < o1 && o0 < a + g.span_elems * g.elem_size;
     };
-    if (overlaps(base)) return fail(MP_ERR_INVALID_ARG, "out overlaps the base");
+    if (overlaps(base) && !(touched_only && static_cast<const void*>(out_buf) == base))
+      return fail(MP_ERR_INVALID_ARG, touched_only ? "out overlaps the base without being the base"
+                                                   : "out overlaps the base");
     for (uint32_t i = 0; i < g.K; ++i)
       if (family->experts_location == 0 && overlaps(ex.p[i]))
         return fail(MP_ERR_INVALID_ARG, "out overlaps an expert");
@@ -773,6 +784,7 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
   p.b_begin = 0;
   p.b_end = g.n_blocks;
   p.expert_origin = 0;
+  p.touched_only = touched_only ? 1u : 0u;
   if (family->experts_location == 0) {
     if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
   } else {
@@ -788,6 +800,20 @@ mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan
   if ((e = cudaEventRecord(mf->done, cs)) != cudaSuccess) return bail(e, "event record");
   *man_out = mf;
   return MP_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
+                   mp_stream stream, mp_manifest** man_out) {
+  return merge_common(family, index, plan, out_buf, stream, man_out, false);
+}
+
+mp_status mp_merge_touched(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
+                           mp_stream stream, mp_manifest** man_out) {
+  return merge_common(family, index, plan, out_buf, stream, man_out, true);
 }
 
 void mp_free(void* handle) {

@@ -25,7 +25,8 @@
 //   TIES:   trimmed by tau_i; S, P, N, counts;  m = P/c+ | N/c- | 0;   out = fma(lambda, m, M_0)
 // An omitted expert contributes exactly zero to every accumulator, so skipping it equals
 // reading a zero-completed tuple (App. A.1) and it is never dereferenced; a chunk that
-// selects no expert is M_0 plus the zero the operator adds.
+// selects no expert is M_0 plus the zero the operator adds, or, in the touched-only mode
+// (Alg. 2 WriteBlockOrReference), not produced at all: the output keeps its contents there.
 // Every mbarrier wait is bounded: on expiry the CTA records kErrTimeout, stops, waits
 // (bounded) for its own copies in flight and returns.
 #include <cuda_bf16.h>
@@ -281,6 +282,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
           cm.off = p.blk_off[b] + start;
           cm.m = p.mask[b];
           cm.n = start < len ? min(CH, len - start) : 0u;
+          if (p.touched_only && cm.m == 0u) cm.n = 0u;  // left as it is: a reference to M_0
           if constexpr (OPC == OP_TIES) grp = p.blk_group[b];
         }
         S.chunk[lane] = cm;
@@ -395,10 +397,21 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
           read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
-          uint32_t keep = 0xFFu;
+          // DARE keep decisions of the vector's elements: element j keeps its delta iff 16-bit
+          // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is
+          // exactly the 8 words of one call (chunk and tensor offsets are multiples of 8
+          // elements); an fp32 vector is half of one.
+          bool kept[V];
           if constexpr (OPC == OP_DARE) {
             const uint64_t j0 = off + k0;
-            keep = dare_keep8_rk(p.dare_rk, i, j0 >> 3, p.dare_T) >> (uint32_t)(j0 & 7u);
+            const uint64_t g = j0 >> 3;
+            const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
+            const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+              const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
+              kept[e] = ((e & 1) ? (wd >> 16) : (wd & 0xFFFFu)) >= p.dare_T;
+            }
           }
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
@@ -407,8 +420,8 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
             if constexpr (OPC == OP_DARE) {
               float s0, s1;
               f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
-              d0 = ((keep >> e) & 1u) ? s0 : 0.0f;
-              d1 = ((keep >> (e + 1)) & 1u) ? s1 : 0.0f;
+              d0 = kept[e] ? s0 : 0.0f;
+              d1 = kept[e + 1] ? s1 : 0.0f;
             }
             f2_fma(a, a, d0, d1, acc[u][e], acc[u][e + 1], acc[u][e], acc[u][e + 1]);
           }

@@ -163,6 +163,7 @@ struct PlanLaunch {
   uint32_t n_groups;
   uint32_t elem_size;
   int op_kind;
+  uint32_t score_mode;  // 0: |coef_i| * norm; 1: that per byte of the block
   float coef[kMaxK];   // |alpha_i| or |lambda|
   const uint32_t* blk_len;
   const uint32_t* blk_group;
@@ -209,6 +210,7 @@ struct MergeLaunch {
   unsigned long long* work;      // chunk counter of the dynamic scheduler (zeroed per launch)
   uint32_t* err;
   uint64_t b_begin, b_end, expert_origin;  // as in IndexLaunch
+  uint32_t touched_only;  // 1: blocks with an empty mask are neither read nor written
 };
 cudaError_t launch_merge(const MergeLaunch& p, cudaStream_t st);
 

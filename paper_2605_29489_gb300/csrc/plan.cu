@@ -5,7 +5,8 @@
 // gives CTA c a contiguous slice of the data, so order is preserved wherever it matters.
 //
 //  A  score: unit u = b*K + i is a candidate iff nnz > 0 (TIES: and key(maxabs) >= tau);
-//     score = |coef_i| * norm (fp32); sort key = ~bits(score), so ascending key order is
+//     score = |coef_i| * norm (fp32), divided by the block's bytes in the score-per-byte
+//     mode; sort key = ~bits(score), so ascending key order is
 //     decreasing score.  Each CTA counts the candidates of its unit slice.
 //  B  stable compaction of the candidates in unit order (so equal scores stay in
 //     ascending unit order).
@@ -175,7 +176,9 @@ __device__ __forceinline__ Unit score_unit(const PlanLaunch& p, uint64_t u) {
   bool cand = p.nnz[st] != 0u;
   if (cand && p.op_kind == MP_OP_TIES)
     cand = ties_key(p.maxabs[st]) >= p.tau[(uint64_t)i * p.n_groups + p.blk_group[b]];
-  const float score = __fmul_rn(p.coef[i], p.norm[st]);
+  float score = __fmul_rn(p.coef[i], p.norm[st]);
+  // score per byte: one IEEE division by the block's byte cost (exact in fp32, <= 2^20)
+  if (p.score_mode) score = __fdiv_rn(score, (float)(p.blk_len[b] * p.elem_size));
   return Unit{cand, ~__float_as_uint(score)};
 }
 

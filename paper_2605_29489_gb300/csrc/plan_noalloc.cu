@@ -85,6 +85,7 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: bad op");
   if (op->kind != MP_OP_TIES && !op->alpha)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA and DARE");
+  if (op->score_mode > 1) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: score_mode must be 0 or 1");
   if (op->kind == MP_OP_TIES && (!tau || !blk_group))
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: TIES needs tau and blk_group");
   if (!blk_len || !norm || !maxabs || !nnz || !index_err || !mask || !order || !summary)
@@ -101,6 +102,7 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   p.n_groups = n_groups;
   p.elem_size = dtype == MP_BF16 ? 2u : 4u;
   p.op_kind = op->kind;
+  p.score_mode = op->score_mode;
   for (uint32_t i = 0; i < K; ++i) {
     float c = op->kind == MP_OP_TIES ? op->lambda : op->alpha[i];
     p.coef[i] = c < 0.0f ? -c : c;
@@ -127,6 +129,7 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   memcpy(&pb, &op->drop_p, 8);
   put_u64(p.hdr_prefix, o, pb);
   put_u64(p.hdr_prefix, o, op->seed);
+  put_u32(p.hdr_prefix, o, op->score_mode);
   put_u64(p.hdr_prefix, o, budget_bytes);
   p.hdr_prefix_len = o;
 

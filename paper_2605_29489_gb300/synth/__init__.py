@@ -279,10 +279,11 @@ def llama3_8b(seed: int = 0, K: int = 4) -> Family:
                   active_frac=0.4, log_mu=math.log(2e-4), log_sigma=1.2, seed=seed)
 
 
-def qwen25_15b(seed: int = 0, K: int = 16) -> Family:
+def qwen25_15b(seed: int = 0, K: int = 16, layers: int = 28) -> Family:
     """Qwen2.5-1.5B shapes (hidden 1536, 28 layers, 12/2 heads, inter 8960, vocab 151936 tied), bf16,
     per-expert active subsets of 25% of blocks"""
-    return Family("qwen2.5-1.5b", BF16, _qwen2_tensors(1536, 28, 12, 2, 8960, 151936), 65536, K,
+    name = "qwen2.5-1.5b" if layers == 28 else f"qwen2.5-1.5b-{layers}l"
+    return Family(name, BF16, _qwen2_tensors(1536, layers, 12, 2, 8960, 151936), 65536, K,
                   active_frac=0.25, log_mu=math.log(1e-3), log_sigma=1.0, per_expert_active=True, seed=seed)
 
 

@@ -95,6 +95,13 @@ def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
             alpha = [1.0 / K] * K
             out.append(("dare", mp.make_op(mp.MP_OP_DARE, alpha=alpha, drop_p=0.9, seed=1234567),
                         oracle.Op(oracle.DARE, K, alpha=alpha, drop_p=0.9, seed=1234567)))
+        elif k == "ta_pb":   # score per byte (ragged blocks have different costs)
+            alpha = [0.3 + 0.1 * i for i in range(K)]
+            out.append(("ta_pb", mp.make_op(mp.MP_OP_TA, alpha=alpha, score_mode=1),
+                        oracle.Op(oracle.TA, K, alpha=alpha, score_mode=1)))
+        elif k == "ties_pb":
+            out.append(("ties_pb", mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, score_mode=1),
+                        oracle.Op(oracle.TIES, K, lam=1.0, density=0.2, score_mode=1)))
     return out
 
 
@@ -173,14 +180,21 @@ def fam_k17():
                         per_expert_active=True, name="k17")
 
 
+def fam_k32():
+    # K = 32, the largest family: the access mask uses its top bit
+    return synth.custom([9000, 4099, 16384], dtype=synth.BF16, block_elems=2048, K=32, active_frac=0.3,
+                        per_expert_active=True, name="k32")
+
+
 FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 
 
-@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17], ids=lambda f: f.__name__)
+@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17, fam_k32],
+                         ids=lambda f: f.__name__)
 def test_parity_small_families(make):
     fam = make()
     base, experts = fam.host_arrays()
-    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare"), FRACS)
+    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb"), FRACS)
 
 
 def test_parity_tiny_config():

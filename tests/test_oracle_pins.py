@@ -479,3 +479,40 @@ def test_digest_tracks_selection():
     assert p1["digest"] != p3["digest"]
     sel = [b * K + i for b in range(nb) for i in range(K) if (p1["mask"][b] >> i) & 1]
     assert p1["set_hash"] == sum(oracle.splitmix64(u) for u in sel) % 2 ** 64
+
+
+def test_plan_score_per_byte_worked_example():
+    """Hand-worked: one expert, three blocks of 50, 25 and 25 bf16 elements (costs 100, 50 and
+    50 bytes) with norms 10, 6 and 6, budget 100 bytes.  By score the order is block 0, 1, 2:
+    block 0 fills the budget and the others are skipped (utility 10).  By score per byte the
+    densities are 0.10, 0.12 and 0.12: blocks 1 and 2 come first and both fit (utility 12)."""
+    blk_len = [50, 25, 25]
+    norm = np.array([[10.0, 6.0, 6.0]], np.float32)
+    maxabs = np.ones((1, 3), np.float32)
+    nnz = np.ones((1, 3), np.uint32)
+    args = (1, blk_len, [0, 0, 0], 1, 2)
+    by_score = oracle.plan(*args, oracle.Op(oracle.AVG, 1, alpha=[1.0]), norm, maxabs, nnz, None, 100)
+    per_byte = oracle.plan(*args, oracle.Op(oracle.AVG, 1, alpha=[1.0], score_mode=1), norm, maxabs, nnz, None, 100)
+    assert by_score["mask"].tolist() == [1, 0, 0] and by_score["chat"] == 100 and by_score["order"].tolist() == [0, 1, 2]
+    assert per_byte["mask"].tolist() == [0, 1, 1] and per_byte["chat"] == 100 and per_byte["order"].tolist() == [1, 2, 0]
+    assert by_score["digest"] != per_byte["digest"]   # the mode is part of the plan's identity
+
+
+def test_plan_score_per_byte_equal_power_of_two_costs_same_selection():
+    """with every block of the same power-of-two byte cost, dividing by it is an exact scaling
+    of every score, so the order and the selection equal those of the plain score"""
+    rng = np.random.default_rng(11)
+    K, nb = 3, 40
+    blk_len = [4096] * nb
+    norm = rng.lognormal(size=(K, nb)).astype(np.float32)
+    norm[0, :5] = norm[1, :5]          # ties are broken the same way
+    maxabs = np.ones((K, nb), np.float32)
+    nnz = np.ones((K, nb), np.uint32)
+    nnz[2, ::7] = 0
+    for budget in (0, 8192 * 10, 8192 * 33, 8192 * K * nb):
+        a = oracle.plan(K, blk_len, [0] * nb, 1, 2, oracle.Op(oracle.TA, K, alpha=[0.3, -0.7, 1.1]), norm, maxabs, nnz,
+                        None, budget)
+        b = oracle.plan(K, blk_len, [0] * nb, 1, 2, oracle.Op(oracle.TA, K, alpha=[0.3, -0.7, 1.1], score_mode=1), norm,
+                        maxabs, nnz, None, budget)
+        assert np.array_equal(a["mask"], b["mask"]) and np.array_equal(a["order"], b["order"])
+        assert a["chat"] == b["chat"] and a["n_sel"] == b["n_sel"]

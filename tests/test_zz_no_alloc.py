@@ -72,6 +72,7 @@ def test_noalloc_plan_matches_mp_plan_additive_and_dare():
     fam = synth.custom([5000, 70001, 65536, 8, 131089, 300], dtype=synth.BF16, block_elems=4096, K=3,
                        active_frac=0.5)
     _run(fam, mp.make_op(mp.MP_OP_TA, alpha=[0.3] * 3), 0, [0.1, 0.5, 1.0])
+    _run(fam, mp.make_op(mp.MP_OP_TA, alpha=[0.3, 0.5, 0.9], score_mode=1), 0, [0.1, 0.5])
     fam9 = synth.custom([30000, 12345, 131172], dtype=synth.BF16, block_elems=8192, K=9, active_frac=0.5,
                         per_expert_active=True)
     _run(fam9, mp.make_op(mp.MP_OP_DARE, alpha=[1 / 9] * 9, drop_p=0.9, seed=5), 0, [0.25, 0.7])
