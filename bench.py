@@ -54,6 +54,12 @@ def workloads():
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
         "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
                                   desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE p=0.9 then AVG, per-expert active sets"),
+        "qwen2.5-0.5b-avg-renorm": dict(make=lambda: synth.qwen25_05b(), op="avg_renorm", budgets=[1.0, 0.5, 0.25, 0.1],
+                                        desc="Qwen2.5-0.5B-shaped bf16 family, K=8, AVG renormalised over the selected "
+                                             "experts (App. A.1)"),
+        "qwen2.5-1.5b-dare-ties": dict(make=lambda: synth.qwen25_15b(), op="dare_ties", drop_p=0.9, budgets=[0.25],
+                                       desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE-TIES p=0.9 lambda=1, "
+                                            "per-expert active sets"),
         "qwen2.5-1.5b-dare-2l": dict(make=lambda: synth.qwen25_15b(layers=2), op="dare", drop_p=0.9, budgets=[0.25],
                                      desc="Qwen2.5-1.5B shapes cut to 2 layers (profiling case), K=16, DARE p=0.9"),
         "llama-3-8b-hostpool-avg": dict(make=lambda: synth.llama3_8b(K=8), op="avg", budgets=[1.0, 0.25, 0.1],
@@ -93,6 +99,12 @@ def make_ops(w, K):
         a = [1.0 / K] * K
         return (mp.make_op(mp.MP_OP_DARE, alpha=a, drop_p=w["drop_p"], seed=20260),
                 oracle.Op(oracle.DARE, K, alpha=a, drop_p=w["drop_p"], seed=20260))
+    if w["op"] == "avg_renorm":
+        a = [1.0 / K] * K
+        return mp.make_op(mp.MP_OP_AVG_RENORM, alpha=a), oracle.Op(oracle.AVG_RENORM, K, alpha=a)
+    if w["op"] == "dare_ties":
+        return (mp.make_op(mp.MP_OP_DARE_TIES, lam=1.0, drop_p=w["drop_p"], seed=20260),
+                oracle.Op(oracle.DARE_TIES, K, lam=1.0, drop_p=w["drop_p"], seed=20260))
     raise ValueError(w["op"])
 
 
@@ -226,8 +238,10 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
         return dt, int(lens.sum())
 
     nb = fam.n_blocks
-    dt1, p1 = run([nb // 2])
-    n = max(1, min(nb, int(target_s / max(dt1, 1e-6))))
+    # per-block cost from an evenly spaced probe (active and inactive blocks differ in cost)
+    probe = sorted(set(int(x) for x in np.linspace(0, nb - 1, min(nb, 8))))
+    dt1, p1 = run(probe)
+    n = max(1, min(nb, int(target_s / max(dt1 / len(probe), 1e-6))))
     blocks = sorted(set(int(x) for x in np.linspace(0, nb - 1, n)))
     dt, params = run(blocks)
     desc = (f"{len(blocks)} of {nb} blocks ({params} params) evenly spaced over the family, regenerated on the "

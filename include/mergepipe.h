@@ -57,8 +57,20 @@ typedef enum { MP_BF16 = 0, MP_F32 = 1 } mp_dtype;
 
 /* Merge operators (Sec. 1, App. A.1).  AVG and TA are the fixed-coefficient additive
    operator sum_i alpha_i A_i Delta_i (Prop. 2); they differ only in how the caller
-   chose alpha (AVG: sum alpha = 1; TA: alpha_i = lambda). */
-typedef enum { MP_OP_AVG = 0, MP_OP_TA = 1, MP_OP_TIES = 2, MP_OP_DARE = 3 } mp_op_kind;
+   chose alpha (AVG: sum alpha = 1; TA: alpha_i = lambda).  AVG_RENORM is App. A.1's
+   selected-only average: per block, beta_i = alpha_i / (sum of alpha over the selected
+   experts), 0 for an omitted expert (the coefficient-drift bound of App. A.1 applies, not
+   Prop. 2); every alpha_i must be > 0.  DARE_TIES drops and rescales like DARE (same
+   mask omega), then elects signs and takes the disjoint mean like TIES, without the
+   magnitude trim (lambda, drop_p and seed are used; no tau). */
+typedef enum {
+  MP_OP_AVG = 0,
+  MP_OP_TA = 1,
+  MP_OP_TIES = 2,
+  MP_OP_DARE = 3,
+  MP_OP_AVG_RENORM = 4,
+  MP_OP_DARE_TIES = 5
+} mp_op_kind;
 
 /* One tensor of the tensor set T (Sec. 2), as a span of the flat checkpoint buffers. */
 typedef struct {
@@ -86,12 +98,12 @@ typedef struct {
 /* Operator and its parameters theta (Alg. 1 records op and theta with the plan). */
 typedef struct {
   mp_op_kind kind;
-  const float* alpha;  /* host array of K coefficients; required for AVG, TA, DARE */
-  float lambda;        /* TIES: scale of the merged task vector (1 = standard TIES) */
+  const float* alpha;  /* host array of K coefficients; required for AVG, TA, DARE, AVG_RENORM */
+  float lambda;        /* TIES, DARE_TIES: scale of the merged task vector (1 = standard) */
   float density;       /* TIES: fraction rho of each trim population kept, in [0, 1] */
   uint32_t trim_scope; /* TIES: 0 = trim per (expert, tensor), 1 = per expert */
-  double drop_p;       /* DARE: drop probability p in [0, 1] */
-  uint64_t seed;       /* DARE: seed of the fixed random mask omega */
+  double drop_p;       /* DARE, DARE_TIES: drop probability p in [0, 1] */
+  uint64_t seed;       /* DARE, DARE_TIES: seed of the fixed random mask omega */
   uint32_t score_mode; /* planning score (Sec. 3, Eq. 6 and the heuristics that follow it):
                           0 = u = |coef_i| * ||Delta||_2 (Prop. 2's utility);
                           1 = score per byte, u / c in fp32 (c = the block's bytes) */

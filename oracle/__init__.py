@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 BF16, F32 = 0, 1
-AVG, TA, TIES, DARE = 0, 1, 2, 3
+AVG, TA, TIES, DARE, AVG_RENORM, DARE_TIES = 0, 1, 2, 3, 4, 5
 OK, EINVAL, EOOM, ENONFINITE = 0, -1, -3, -4
 TAU_NONE = 0x8000
 
@@ -54,7 +54,7 @@ def lib():
         L.orc_tau_from_hist.argtypes = [vp, u64, ctypes.c_float]
         L.orc_ties_thresholds.argtypes = [vp, ctypes.c_float, vp]
         L.orc_plan.argtypes = [u32, u64, vp, vp, u32, u32, vp, vp, vp, vp, vp, u64, vp, vp, vp, vp, vp, vp, vp]
-        L.orc_merge_block.argtypes = [ctypes.c_int, u64, u64, vp, vp, u32, vp, vp, vp]
+        L.orc_merge_block.argtypes = [ctypes.c_int, u64, u64, vp, vp, u32, u32, vp, vp, vp]
         L.orc_merge.argtypes = [vp, vp, vp, vp, vp]
         L.orc_philox4x32_10.argtypes = [vp, vp, vp]
         L.orc_dare_keep.argtypes = [u64, u32, u64, ctypes.c_double]
@@ -204,8 +204,9 @@ def plan(K, blk_len, blk_group, n_groups, elem_size, op: Op, norm, maxabs, nnz, 
 
 # ---- merge ------------------------------------------------------------------------------------
 
-def merge_block(dtype, j0, base, experts, mask, op: Op, tau_k=None):
-    """Psi_op on one block: experts is a list of K arrays (entries for unselected experts may be None)"""
+def merge_block(dtype, j0, base, experts, mask, op: Op, tau_k=None, known_zero=0):
+    """Psi_op on one block: experts is a list of K arrays (entries for unselected experts may be None);
+    known_zero: bits of the experts whose delta block is exactly zero (renormalised AVG only)"""
     npd = _np_dtype(dtype)
     base = np.ascontiguousarray(base, npd)
     keep = [None if e is None else np.ascontiguousarray(e, npd) for e in experts]
@@ -213,7 +214,8 @@ def merge_block(dtype, j0, base, experts, mask, op: Op, tau_k=None):
     out = np.empty_like(base)
     tk = None if tau_k is None else np.ascontiguousarray(tau_k, np.uint32)
     oc = op.c()
-    _check(lib().orc_merge_block(dtype, base.shape[0], int(j0), _p(base), ptrs, int(mask), ctypes.byref(oc),
+    _check(lib().orc_merge_block(dtype, base.shape[0], int(j0), _p(base), ptrs, int(mask), int(known_zero),
+                                 ctypes.byref(oc),
                                  _p(tk), _p(out)))
     return out
 

@@ -234,7 +234,8 @@ uint64_t orc_splitmix64(uint64_t state) {
  *    with nnz = 0 contributes exactly nothing to any operator, and under TIES a unit
  *    whose largest key is below tau is trimmed entirely; both are left out (exact).
  *  - Score s(i,t,b) = |coef_i| * ||Delta_{i,t,b}||_2 in fp32 (the utility u of Prop. 2);
- *    coef_i = alpha_i (AVG, TA, DARE) or lambda (TIES).  In the score-per-byte mode (the
+ *    coef_i = alpha_i (AVG, TA, DARE, renormalised AVG) or lambda (TIES, DARE-TIES).  In the
+ *    score-per-byte mode (the
  *    second heuristic Sec. 3 names for the objective of Eq. 6) s is divided by the unit's
  *    byte cost c, one fp32 division.
  *  - Sort by decreasing score; ties by ascending unit id = b*K + i (block order is
@@ -279,7 +280,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
              uint64_t* set_hash_out, uint64_t* digest_out, uint32_t* order) {
   if (!op || K == 0 || K > 32 || op->K != K || !norm || !maxabs || !nnz || !mask) return ORC_EINVAL;
   if (op->kind == ORC_TIES && (!tau || !blk_group)) return ORC_EINVAL;
-  if (op->kind != ORC_TIES && !op->alpha) return ORC_EINVAL;
+  if (op->kind != ORC_TIES && op->kind != ORC_DARE_TIES && !op->alpha) return ORC_EINVAL;
   if (n_blocks * K > 0xFFFFFFFFull) return ORC_EINVAL;
 
   orc_cand* q = (orc_cand*)malloc(sizeof(orc_cand) * (size_t)(n_blocks * K + 1));
@@ -291,7 +292,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
       if (nnz[s] == 0) continue;
       if (op->kind == ORC_TIES && orc_ties_key(maxabs[s]) < tau[(size_t)i * n_groups + blk_group[b]])
         continue;
-      float coef = op->kind == ORC_TIES ? op->lambda : op->alpha[i];
+      float coef = (op->kind == ORC_TIES || op->kind == ORC_DARE_TIES) ? op->lambda : op->alpha[i];
       q[nq].score = fabsf(coef) * norm[s];
       q[nq].unit = (uint32_t)(b * K + i);
       q[nq].cost = blk_len[b] * elem_size;
@@ -405,32 +406,58 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  *  TIES: d^_i = A_i delta_i if key(delta_i) >= tau_i else 0;  S = sum_i d^_i;
  *        gamma = sign(S);  m = (sum of d^_i with sign gamma) / (their count), 0 if S = 0;
  *        out = round(fma(lambda, m, M_0))
+ *  AVG, renormalised over the selected experts (App. A.1, the selected-only variant with
+ *        coefficients beta_i(A) = 0 when A_i = 0): s = sum of alpha_j over the experts j that
+ *        are selected or whose delta block is exactly zero (ascending fp32 adds from +0);
+ *        beta_i = alpha_i / s;
+ *        acc = sum_i fma(beta_i, A_i delta_i, acc); out = round(M_0 + acc)
+ *  DARE-TIES: DARE's drop and rescale with the same mask omega, then TIES's election and
+ *        disjoint mean without magnitude trimming: d^_i = A_i (keep_i ? delta_i * sigma : 0),
+ *        then S, gamma, m and out as TIES
  * round = bf16 round-to-nearest-even, or none for fp32 checkpoints.
- * Pins: hand-computed TIES and AVG examples; Eq. 5 against an fp64 restatement of the
- * unmasked operator (within one bf16 ulp); Prop. 2 bound; DARE at p = 0 equals AVG and
- * the DARE mean over seeds tends to AVG.
+ * Pins: hand-computed TIES, AVG and renormalised-AVG examples; Eq. 5 against an fp64
+ * restatement of the unmasked operator (within one bf16 ulp); Prop. 2 bound and the
+ * coefficient-drift bound of App. A.1; DARE at p = 0 equals AVG and the DARE mean over
+ * seeds tends to AVG; DARE-TIES at p = 0 equals TIES at density 1.
  * ------------------------------------------------------------------------------------- */
 int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const void* const* experts,
-                    uint32_t mask, const orc_op* op, const uint32_t* tau_k, void* out) {
+                    uint32_t mask, uint32_t known_zero, const orc_op* op, const uint32_t* tau_k, void* out) {
   if (!op || op->K == 0 || op->K > 32 || (n > 0 && (!base || !out))) return ORC_EINVAL;
   const uint32_t K = op->K;
   for (uint32_t i = 0; i < K; ++i)
     if (((mask >> i) & 1u) && !experts[i]) return ORC_EINVAL;
+  const int ties_like = op->kind == ORC_TIES || op->kind == ORC_DARE_TIES;
   if (op->kind == ORC_TIES && !tau_k) return ORC_EINVAL;
-  if (op->kind != ORC_TIES && !op->alpha) return ORC_EINVAL;
+  if (!ties_like && !op->alpha) return ORC_EINVAL;
   float sigma = op->drop_p < 1.0 ? (float)(1.0 / (1.0 - op->drop_p)) : 0.0f;
+  /* renormalised AVG: the sum, ascending, of the coefficients of the experts that take part:
+     the selected ones and those whose delta block is exactly zero (known from the catalog
+     without a read; counting them is what makes the full budget equal the full-read
+     average, Eq. 5) */
+  float s_sel = 0.0f;
+  if (op->kind == ORC_AVG_RENORM) {
+    for (uint32_t i = 0; i < K; ++i)
+      if (((mask | known_zero) >> i) & 1u) {
+        if (!(op->alpha[i] > 0.0f)) return ORC_EINVAL;
+        s_sel = s_sel + op->alpha[i];
+      }
+  }
 
   for (uint64_t k = 0; k < n; ++k) {
     float x0 = load_elem(dtype, base, k);
     float res;
-    if (op->kind == ORC_TIES) {
+    if (ties_like) {
       float S = 0.0f, P = 0.0f, Nn = 0.0f;
       uint32_t cp = 0, cn = 0;
       for (uint32_t i = 0; i < K; ++i) {
         float dh = 0.0f;
         if ((mask >> i) & 1u) {
           float d = load_elem(dtype, experts[i], k) - x0;
-          if (orc_ties_key(d) >= tau_k[i]) dh = d;
+          if (op->kind == ORC_TIES) {
+            if (orc_ties_key(d) >= tau_k[i]) dh = d;
+          } else if (orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) {
+            dh = d * sigma;
+          }
         }
         S = S + dh;
         if (dh > 0.0f) {
@@ -451,7 +478,8 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
         if (!((mask >> i) & 1u)) continue; /* omitted: zero entry, never read */
         float d = load_elem(dtype, experts[i], k) - x0;
         if (op->kind == ORC_DARE) d = orc_dare_keep(op->seed, i, j0 + k, op->drop_p) ? d * sigma : 0.0f;
-        acc = fmaf(op->alpha[i], d, acc);
+        const float coef = op->kind == ORC_AVG_RENORM ? op->alpha[i] / s_sel : op->alpha[i];
+        acc = fmaf(coef, d, acc);
       }
       res = x0 + acc;
     }
@@ -475,8 +503,17 @@ int orc_merge(const orc_family* f, const orc_op* op, const uint32_t* tau, const 
       ex[i] = elem_ptr(f->dtype, f->experts[i], off);
       if (op->kind == ORC_TIES) tau_k[i] = tau[(size_t)i * f->n_groups + f->blk_group[b]];
     }
+    uint32_t known_zero = 0;
+    if (op->kind == ORC_AVG_RENORM) {
+      const void* b0 = elem_ptr(f->dtype, f->base, off);
+      for (uint32_t i = 0; i < f->K; ++i) {
+        uint64_t k = 0;
+        while (k < f->blk_len[b] && load_elem(f->dtype, ex[i], k) - load_elem(f->dtype, b0, k) == 0.0f) ++k;
+        if (k == f->blk_len[b]) known_zero |= 1u << i;
+      }
+    }
     int rc = orc_merge_block(f->dtype, f->blk_len[b], off, elem_ptr(f->dtype, f->base, off), ex,
-                             mask ? mask[b] : all, op, tau_k,
+                             mask ? mask[b] : all, known_zero, op, tau_k,
                              (char*)out + off * (f->dtype == ORC_BF16 ? 2u : 4u));
     if (rc != ORC_OK) return rc;
   }

@@ -21,7 +21,7 @@ import os
 import numpy as np
 
 __all__ = [
-    "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MergePipeError",
+    "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_budget_from_fraction", "mp_last_error",
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "lib", "library_path",
@@ -31,7 +31,7 @@ MP_OK = 0
 MP_ERR = {-1: "MP_ERR_INVALID_ARG", -2: "MP_ERR_CUDA", -3: "MP_ERR_OOM", -4: "MP_ERR_NONFINITE",
           -5: "MP_ERR_BUDGET", -6: "MP_ERR_TIMEOUT", -7: "MP_ERR_UNSUPPORTED", -8: "MP_ERR_MISMATCH"}
 MP_BF16, MP_F32 = 0, 1
-MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE = 0, 1, 2, 3
+MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES = 0, 1, 2, 3, 4, 5
 
 
 class MergePipeError(RuntimeError):

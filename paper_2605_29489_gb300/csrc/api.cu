@@ -162,17 +162,22 @@ mp_status resolve_pointers(const mp_family* f, const void*& base, ExpertPtrs& ex
 
 mp_status check_op(const mp_op* op, uint32_t K) {
   if (!op) return fail(MP_ERR_INVALID_ARG, "op is NULL");
-  if (op->kind < MP_OP_AVG || op->kind > MP_OP_DARE) return fail(MP_ERR_INVALID_ARG, "unknown operator kind");
-  if (op->kind != MP_OP_TIES) {
-    if (!op->alpha) return fail(MP_ERR_INVALID_ARG, "alpha is required for AVG, TA and DARE");
+  if (op->kind < MP_OP_AVG || op->kind > MP_OP_DARE_TIES) return fail(MP_ERR_INVALID_ARG, "unknown operator kind");
+  if (op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES) {
+    if (!isfinite(op->lambda)) return fail(MP_ERR_INVALID_ARG, "lambda must be finite");
+  } else {
+    if (!op->alpha) return fail(MP_ERR_INVALID_ARG, "alpha is required for AVG, TA, DARE and AVG_RENORM");
     for (uint32_t i = 0; i < K; ++i)
       if (!isfinite(op->alpha[i])) return fail(MP_ERR_INVALID_ARG, "alpha must be finite");
-  } else {
+    if (op->kind == MP_OP_AVG_RENORM)
+      for (uint32_t i = 0; i < K; ++i)
+        if (!(op->alpha[i] > 0.0f)) return fail(MP_ERR_INVALID_ARG, "AVG_RENORM needs every alpha > 0");
+  }
+  if (op->kind == MP_OP_TIES) {
     if (!(op->density >= 0.0f && op->density <= 1.0f)) return fail(MP_ERR_INVALID_ARG, "density must be in [0, 1]");
-    if (!isfinite(op->lambda)) return fail(MP_ERR_INVALID_ARG, "lambda must be finite");
     if (op->trim_scope > 1) return fail(MP_ERR_INVALID_ARG, "trim_scope must be 0 or 1");
   }
-  if (op->kind == MP_OP_DARE && !(op->drop_p >= 0.0 && op->drop_p <= 1.0))
+  if ((op->kind == MP_OP_DARE || op->kind == MP_OP_DARE_TIES) && !(op->drop_p >= 0.0 && op->drop_p <= 1.0))
     return fail(MP_ERR_INVALID_ARG, "drop_p must be in [0, 1]");
   if (op->score_mode > 1) return fail(MP_ERR_INVALID_ARG, "score_mode must be 0 or 1");
   return MP_OK;
@@ -633,7 +638,8 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   p.elem_size = g.elem_size;
   p.op_kind = op->kind;
   p.score_mode = op->score_mode;
-  for (uint32_t i = 0; i < g.K; ++i) p.coef[i] = fabsf(op->kind == MP_OP_TIES ? op->lambda : op->alpha[i]);
+  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES;
+  for (uint32_t i = 0; i < g.K; ++i) p.coef[i] = fabsf(by_lambda ? op->lambda : op->alpha[i]);
   p.blk_len = index->d_blk_len;
   p.blk_group = index->d_blk_group;
   p.norm = index->d_norm;
@@ -766,6 +772,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   p.blk_group = index->d_blk_group;
   p.mask = plan->d_mask;
   p.tau = index->d_tau;
+  p.nnz = index->d_nnz;
   for (uint32_t i = 0; i < kMaxK; ++i) p.alpha[i] = plan->alpha[i];
   p.lambda = plan->lambda;
   p.sigma = plan->drop_p < 1.0 ? (float)(1.0 / (1.0 - plan->drop_p)) : 0.0f;

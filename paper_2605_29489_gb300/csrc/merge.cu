@@ -23,6 +23,9 @@
 //   AVG/TA: acc = fma(alpha_i, delta_i, acc)                          out = M_0 + acc
 //   DARE:   delta_i kept by a Philox word >= T, scaled by sigma; then as AVG
 //   TIES:   trimmed by tau_i; S, P, N, counts;  m = P/c+ | N/c- | 0;   out = fma(lambda, m, M_0)
+//   renormalised AVG (App. A.1): as AVG with alpha_i / (sum of alpha over the experts that are
+//           selected or have an exactly zero delta block, known from the catalog)
+//   DARE-TIES: DARE's keep and rescale, then TIES's election and mean without trimming
 // An omitted expert contributes exactly zero to every accumulator, so skipping it equals
 // reading a zero-completed tuple (App. A.1) and it is never dereferenced; a chunk that
 // selects no expert is M_0 plus the zero the operator adds, or, in the touched-only mode
@@ -43,17 +46,24 @@ constexpr int kConsumers = 256;
 constexpr int kThreads = kConsumers + 32;  // + one producer warp
 constexpr uint32_t kEnd = 0xFFFFFFFFu;
 
-enum { OP_ADD = 0, OP_TIES = 1, OP_DARE = 2 };
+enum { OP_ADD = 0, OP_TIES = 1, OP_DARE = 2, OP_RENORM = 3, OP_DTIES = 4 };
 
-// slot geometry per operator.  The additive merge is bound by HBM: two CTAs per SM with a
-// 96 KiB ring each.  TIES and DARE spend more arithmetic per byte: three CTAs per SM (more
+// TIES and DARE-TIES share the sign election and disjoint mean (DARE and DARE-TIES share
+// the random keep mask); AVG/TA and the renormalised AVG share the additive geometry
+template <int OPC>
+constexpr bool kTiesLike = OPC == OP_TIES || OPC == OP_DTIES;
+template <int OPC>
+constexpr bool kAddGeo = OPC == OP_ADD || OPC == OP_RENORM;
+
+// slot geometry per operator.  The additive merges are bound by HBM: two CTAs per SM with a
+// 96 KiB ring each.  TIES, DARE and DARE-TIES spend more arithmetic per byte: three CTAs per SM (more
 // warps to hide it) with a 64 KiB ring each, and chunks half as long (one 16-byte vector per
 // consumer thread) so that their per-element state fits the register budget.
 template <int OPC>
 struct Geo {
-  static constexpr int kCtasPerSm = OPC == OP_ADD ? 2 : 3;
-  static constexpr uint32_t kRingBytes = OPC == OP_ADD ? 98304u : 65536u;
-  static constexpr uint32_t kSlotBytes = OPC == OP_ADD ? 8192u : 4096u;  // one chunk of one checkpoint
+  static constexpr int kCtasPerSm = kAddGeo<OPC> ? 2 : 3;
+  static constexpr uint32_t kRingBytes = kAddGeo<OPC> ? 98304u : 65536u;
+  static constexpr uint32_t kSlotBytes = kAddGeo<OPC> ? 8192u : 4096u;  // one chunk of one checkpoint
   static constexpr int kSlots = (int)(kRingBytes / kSlotBytes);
   static constexpr uint32_t kGrab = 8;  // chunks taken per counter increment (<= 32)
 };
@@ -64,7 +74,8 @@ struct SlotMeta {
   uint32_t which; // 0 = base, 1 + i = expert i
   uint32_t n;     // elements in the chunk
   uint32_t m;     // the block's access mask
-  uint32_t tau;   // TIES: bits threshold of this (expert, trim group)
+  uint32_t aux;   // TIES: bits threshold of this (expert, trim group); renormalised AVG: the
+                  // experts counted in the normaliser (selected or with a zero delta block)
 };
 
 // block metadata of one chunk of a grab, staged by the producer warp
@@ -80,6 +91,7 @@ struct __align__(128) Smem {
   SlotMeta meta[NS];
   ChunkMeta chunk[G];
   uint32_t thr[G][kMaxK];  // TIES: bits threshold of (chunk, expert)
+  uint32_t zmask[G];       // renormalised AVG: experts whose delta block is exactly zero
   uint64_t full[NS];
   uint64_t empty[NS];
   unsigned long long realized[kMaxK];
@@ -248,7 +260,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     uint32_t fill = 0;
     bool ok = true;
     // lane 0 arms slot `fill` with the given chunk data and starts its bulk copy
-    auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t thr,
+    auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t aux,
                        const char* src_row, uint32_t bytes) -> bool {
       const uint32_t s = fill % kSlots, r = fill / kSlots;
       if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
@@ -258,7 +270,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
       S.meta[s].which = which;
       S.meta[s].n = n;
       S.meta[s].m = m;
-      S.meta[s].tau = thr;
+      S.meta[s].aux = aux;
       mbar_arrive_expect_tx(&S.full[s], bytes);
       if (bytes) tma_load_1d(S.slot[s], src_row, bytes, &S.full[s]);
       ++fill;
@@ -272,11 +284,13 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
       if (lane == 0) q_next = atomicAdd(work, (unsigned long long)G);  // used by the next grab
       // lanes c < G: metadata of chunk q0 + c
       uint32_t grp = 0;
+      uint64_t bq = 0;  // block of chunk q0 + lane
       if (lane < G) {
         const unsigned long long q = q0 + lane;
         ChunkMeta cm{0, 0, 0};
         if (q < n_chunks) {
           const uint64_t b = p.b_begin + q / cpb;
+          bq = b;
           const uint32_t start = (uint32_t)(q % cpb) * CH;
           const uint32_t len = p.blk_len[b];
           cm.off = p.blk_off[b] + start;
@@ -296,6 +310,17 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
           if (lane < p.K) S.thr[c][lane] = max(ties_bits_threshold(p.tau[(uint64_t)lane * p.n_groups + g]), 1u);
         }
       }
+      if constexpr (OPC == OP_RENORM) {
+        // lane i < K: is expert i's delta block exactly zero (catalog nnz = 0)?  Such an
+        // expert is counted in the normaliser without being read.
+#pragma unroll
+        for (uint32_t c = 0; c < G; ++c) {
+          const uint64_t b = __shfl_sync(0xFFFFFFFFu, bq, c);
+          const bool z = lane < p.K && p.nnz[(uint64_t)lane * p.n_blocks + b] == 0u;
+          const uint32_t zb = __ballot_sync(0xFFFFFFFFu, z);
+          if (lane == 0) S.zmask[c] = zb;
+        }
+      }
       __syncwarp();
       if (lane == 0) {
         const uint32_t nq = (uint32_t)min((unsigned long long)G, n_chunks - q0);
@@ -304,10 +329,12 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
           if (cm.n == 0) continue;
           const uint32_t q = (uint32_t)(q0 + c);
           const uint32_t bytes = (cm.n * ES) & ~15u;
-          ok = produce(q, 0, cm.off, cm.n, cm.m, 0u, static_cast<const char*>(p.base) + cm.off * ES, bytes);
+          const uint32_t aux0 = OPC == OP_RENORM ? (cm.m | S.zmask[c]) : 0u;
+          ok = produce(q, 0, cm.off, cm.n, cm.m, aux0, static_cast<const char*>(p.base) + cm.off * ES, bytes);
           for (uint32_t mm = cm.m; ok && mm; mm &= mm - 1) {
             const uint32_t i = __ffs(mm) - 1;
-            ok = produce(q, 1 + i, cm.off, cm.n, cm.m, OPC == OP_TIES ? S.thr[c][i] : 0u,
+            // DARE-TIES keeps every nonzero rescaled delta: threshold = the smallest subnormal
+            ok = produce(q, 1 + i, cm.off, cm.n, cm.m, OPC == OP_TIES ? S.thr[c][i] : 1u,
                          static_cast<const char*>(p.experts.p[i]) + (cm.off - p.expert_origin) * ES, bytes);
             S.realized[i] += (unsigned long long)cm.n * ES;
           }
@@ -339,6 +366,21 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
   uint32_t cnt[VPT][V];  // TIES: positive count | negative count << 16
   uint64_t off = 0;
   uint32_t n = 0, n_tma = 0, remaining = 0;
+  float s_sel = 0.0f;  // renormalised AVG: sum of the counted experts' alpha (ascending)
+  // DARE keep decisions of the vector's elements: element j keeps its delta iff 16-bit
+  // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is exactly
+  // the 8 words of one call (chunk and tensor offsets are multiples of 8 elements); an
+  // fp32 vector is half of one.
+  auto dare_kept = [&](uint32_t i, uint64_t j0, bool (&kept)[V]) {
+    const uint64_t g = j0 >> 3;
+    const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
+    const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
+#pragma unroll
+    for (int e = 0; e < V; ++e) {
+      const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
+      kept[e] = ((e & 1) ? (wd >> 16) : (wd & 0xFFFFu)) >= p.dare_T;
+    }
+  };
   for (uint32_t fill = 0;; ++fill) {
     const uint32_t s = fill % kSlots, r = fill / kSlots;
     if (!warp_wait(&S.full[s], r & 1u, abort_flag)) {
@@ -354,6 +396,10 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
       n = mt.n;
       n_tma = ((n * ES) & ~15u) / ES;
       remaining = __popc(mt.m);
+      if constexpr (OPC == OP_RENORM) {
+        s_sel = 0.0f;
+        for (uint32_t mm = mt.aux; mm; mm &= mm - 1) s_sel = __fadd_rn(s_sel, p.alpha[__ffs(mm) - 1]);
+      }
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
         const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
@@ -372,47 +418,44 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     } else {
       const uint32_t i = mt.which - 1;
       const void* src = p.experts.p[i];
-      if constexpr (OPC == OP_TIES) {
-        // trim test on the magnitude's bits: key(|d|) >= tau exactly when bits(|d|) >= the
-        // producer's threshold (a NaN pattern, never true, when nothing is kept)
-        const float thr = __uint_as_float(mt.tau);
+      if constexpr (kTiesLike<OPC>) {
+        // TIES: trim test on the magnitude's bits: key(|d|) >= tau exactly when bits(|d|) >=
+        // the producer's threshold (a NaN pattern, never true, when nothing is kept).
+        // DARE-TIES: the delta is first dropped or rescaled by the keep mask, and every
+        // nonzero result is kept (threshold = the smallest subnormal).
+        const float thr = __uint_as_float(mt.aux);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
           read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
+          bool kept[V];
+          if constexpr (OPC == OP_DTIES) dare_kept(i, off + k0, kept);
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
             // the deltas of an element pair in one packed fp32x2 subtract
             float d0, d1;
             f2_sub(xe[e], xe[e + 1], x0[u][e], x0[u][e + 1], d0, d1);
+            if constexpr (OPC == OP_DTIES) {
+              float s0, s1;
+              f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
+              d0 = kept[e] ? s0 : 0.0f;
+              d1 = kept[e + 1] ? s1 : 0.0f;
+            }
             ties_tally(d0, thr, Sg[u][e], Pp[u][e], Nn[u][e], cnt[u][e]);
             ties_tally(d1, thr, Sg[u][e + 1], Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
           }
         }
       } else {
-        const float a = p.alpha[i];
+        // renormalised AVG: beta_i = alpha_i / (sum of the selected alpha), one IEEE division
+        const float a = OPC == OP_RENORM ? __fdiv_rn(p.alpha[i], s_sel) : p.alpha[i];
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
           read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
-          // DARE keep decisions of the vector's elements: element j keeps its delta iff 16-bit
-          // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is
-          // exactly the 8 words of one call (chunk and tensor offsets are multiples of 8
-          // elements); an fp32 vector is half of one.
           bool kept[V];
-          if constexpr (OPC == OP_DARE) {
-            const uint64_t j0 = off + k0;
-            const uint64_t g = j0 >> 3;
-            const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
-            const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
-#pragma unroll
-            for (int e = 0; e < V; ++e) {
-              const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
-              kept[e] = ((e & 1) ? (wd >> 16) : (wd & 0xFFFFu)) >= p.dare_T;
-            }
-          }
+          if constexpr (OPC == OP_DARE) dare_kept(i, off + k0, kept);
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
             float d0, d1;
@@ -440,7 +483,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
         if (mt.m == 0) {
           // no expert selected: every accumulator is +0, so the output is M_0 plus the
           // zero the operator adds (lambda * +0 for TIES, +0 otherwise)
-          const float z = OPC == OP_TIES ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
+          const float z = kTiesLike<OPC> ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
 #pragma unroll
           for (int e = 0; e < V; ++e) y[e] = __fadd_rn(x0[u][e], z);
           store_vec<BF16>(p.out, off + k0, n - k0, y);
@@ -448,7 +491,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
         }
 #pragma unroll
         for (int e = 0; e < V; ++e) {
-          if constexpr (OPC == OP_TIES) {
+          if constexpr (kTiesLike<OPC>) {
             // one division per element: the mean of the entries whose sign was elected
             // (S != 0 implies at least one of them, so c >= 1; otherwise +0 / 1 = +0)
             const bool pos = Sg[u][e] > 0.0f, any = Sg[u][e] != 0.0f;
@@ -497,6 +540,8 @@ cudaError_t launch_dtype(const MergeLaunch& p, cudaStream_t st) {
     case MP_OP_TA: return launch_op<BF16, OP_ADD>(p, st);
     case MP_OP_TIES: return launch_op<BF16, OP_TIES>(p, st);
     case MP_OP_DARE: return launch_op<BF16, OP_DARE>(p, st);
+    case MP_OP_AVG_RENORM: return launch_op<BF16, OP_RENORM>(p, st);
+    case MP_OP_DARE_TIES: return launch_op<BF16, OP_DTIES>(p, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -200,6 +200,7 @@ struct MergeLaunch {
   const uint32_t* blk_group;
   const uint32_t* mask;
   const uint32_t* tau;  // TIES
+  const uint32_t* nnz;  // renormalised AVG: catalog nonzero counts [K][n_blocks]
   float alpha[kMaxK];
   float lambda;
   float sigma;          // DARE rescale

@@ -81,10 +81,11 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   if (U > kNoAllocMaxUnits || mp::plan_scratch_bytes(U) > kNoAllocScratchBytes)
     return fail_static(MP_ERR_INVALID_ARG,
                        "mp_plan_noalloc: K * n_blocks exceeds the static scratch limit of 524288 units");
-  if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_DARE)
+  if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_DARE_TIES)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: bad op");
-  if (op->kind != MP_OP_TIES && !op->alpha)
-    return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA and DARE");
+  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES;
+  if (!by_lambda && !op->alpha)
+    return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA, DARE and AVG_RENORM");
   if (op->score_mode > 1) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: score_mode must be 0 or 1");
   if (op->kind == MP_OP_TIES && (!tau || !blk_group))
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: TIES needs tau and blk_group");
@@ -104,7 +105,7 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   p.op_kind = op->kind;
   p.score_mode = op->score_mode;
   for (uint32_t i = 0; i < K; ++i) {
-    float c = op->kind == MP_OP_TIES ? op->lambda : op->alpha[i];
+    float c = by_lambda ? op->lambda : op->alpha[i];
     p.coef[i] = c < 0.0f ? -c : c;
   }
   p.blk_len = blk_len;

@@ -99,6 +99,13 @@ def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
             alpha = [0.3 + 0.1 * i for i in range(K)]
             out.append(("ta_pb", mp.make_op(mp.MP_OP_TA, alpha=alpha, score_mode=1),
                         oracle.Op(oracle.TA, K, alpha=alpha, score_mode=1)))
+        elif k == "avg_renorm":   # App. A.1's selected-only average
+            alpha = [(i + 1) / (K * (K + 1) / 2) for i in range(K)]
+            out.append(("avg_renorm", mp.make_op(mp.MP_OP_AVG_RENORM, alpha=alpha),
+                        oracle.Op(oracle.AVG_RENORM, K, alpha=alpha)))
+        elif k == "dare_ties":
+            out.append(("dare_ties", mp.make_op(mp.MP_OP_DARE_TIES, lam=0.8, drop_p=0.7, seed=424242),
+                        oracle.Op(oracle.DARE_TIES, K, lam=0.8, drop_p=0.7, seed=424242)))
         elif k == "ties_pb":
             out.append(("ties_pb", mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, score_mode=1),
                         oracle.Op(oracle.TIES, K, lam=1.0, density=0.2, score_mode=1)))
@@ -194,7 +201,8 @@ FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 def test_parity_small_families(make):
     fam = make()
     base, experts = fam.host_arrays()
-    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb"), FRACS)
+    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb", "avg_renorm", "dare_ties"),
+             FRACS)
 
 
 def test_parity_tiny_config():

@@ -85,7 +85,7 @@ def dev_copy(t):
 
 @pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k32], ids=lambda f: f.__name__)
 def test_touched_only_matches_oracle_on_touched_blocks(make):
-    check_family(make(), ("avg", "ta", "ties", "dare"), [0.1, 0.5, 1.0])
+    check_family(make(), ("avg", "ta", "ties", "dare", "avg_renorm", "dare_ties"), [0.1, 0.5, 1.0])
 
 
 def test_touched_only_zero_budget_writes_nothing():

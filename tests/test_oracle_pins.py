@@ -516,3 +516,111 @@ def test_plan_score_per_byte_equal_power_of_two_costs_same_selection():
                         maxabs, nnz, None, budget)
         assert np.array_equal(a["mask"], b["mask"]) and np.array_equal(a["order"], b["order"])
         assert a["chat"] == b["chat"] and a["n_sel"] == b["n_sel"]
+
+
+# ---- operator variants (App. A.1): renormalised AVG, DARE-TIES ----------------------------------------
+
+def test_avg_renorm_worked_example():
+    """Hand-worked, fp32 (every value dyadic, every step exact): alpha = (0.5, 0.25, 0.25).
+    Experts 1 and 2 selected: s = 0.5, beta = (0, 0.5, 0.5), so out = base + (D1 + D2) / 2.
+    All three selected: s = 1, beta = alpha (the plain average)."""
+    base = np.array([1.0, -2.0, 0.5, 0.0], np.float32)
+    e0 = np.array([9.0, 9.0, 9.0, 9.0], np.float32)      # omitted below: must not matter
+    e1 = np.array([2.0, -1.0, 0.5, 1.0], np.float32)     # D1 = ( 1,  1, 0,  1)
+    e2 = np.array([1.0, -3.0, 1.5, -1.0], np.float32)    # D2 = ( 0, -1, 1, -1)
+    op = oracle.Op(oracle.AVG_RENORM, 3, alpha=[0.5, 0.25, 0.25])
+    out = oracle.merge_block(oracle.F32, 0, base, [e0, e1, e2], 0b110, op)
+    assert out.tolist() == [1.5, -2.0, 1.0, 0.0]
+    out_all = oracle.merge_block(oracle.F32, 0, base, [e0, e1, e2], 0b111, op)
+    # base + 0.5*(8,11,8.5,9) + 0.25*(1,1,0,1) + 0.25*(0,-1,1,-1)
+    assert out_all.tolist() == [5.25, 3.5, 5.0, 4.5]
+    out_none = oracle.merge_block(oracle.F32, 0, base, [e0, e1, e2], 0, op)
+    assert out_none.tolist() == base.tolist()
+
+
+def test_avg_renorm_full_budget_equals_avg(tiny_family):
+    """with sum alpha = 1 exactly (0.25 x 4), the full-read renormalised average divides by 1"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    a = [0.25] * fam.K
+    r = oracle.merge(of, oracle.Op(oracle.AVG_RENORM, fam.K, alpha=a))
+    m = oracle.merge(of, oracle.Op(oracle.AVG, fam.K, alpha=a))
+    assert np.array_equal(r.view(np.uint32), m.view(np.uint32))
+
+
+def test_avg_renorm_coefficient_drift_bound(tiny_family):
+    """App. A.1: ||M_full - M_A||_2 <= sqrt(sum_b r_b^2), r_b = sum_i |alpha_i - beta_i(A)| ||Delta_i,b||_2,
+    checked in fp64 on plans at several budgets (slack for the fp32 arithmetic)"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    norm, maxabs, nnz = oracle.index(of)
+    bo, bl, bt = fam.block_table()
+    alpha = np.array([0.4, 0.3, 0.2, 0.1], np.float32)[: fam.K]
+    alpha = alpha / alpha.sum()
+    op = oracle.Op(oracle.AVG_RENORM, fam.K, alpha=alpha)
+    full = oracle.merge(of, op).astype(np.float64)
+    x0 = base.astype(np.float64)
+    exact_norm = np.zeros((fam.K, fam.n_blocks))
+    for i in range(fam.K):
+        d = experts[i].astype(np.float64) - x0
+        for b in range(fam.n_blocks):
+            s = slice(int(bo[b]), int(bo[b] + bl[b]))
+            exact_norm[i, b] = np.sqrt((d[s] ** 2).sum())
+    C_full = fam.K * fam.total_elems * 4
+    checked_drift = False
+    for f in (1.0, 0.6, 0.3, 0.1):
+        B = int(math.floor(f * C_full))
+        pl = oracle.plan(fam.K, bl, bt, len(fam.tensors), 4, op, norm, maxabs, nnz, None, B)
+        out = oracle.merge(of, op, mask=pl["mask"]).astype(np.float64)
+        A = ((pl["mask"][None, :] >> np.arange(fam.K)[:, None]) & 1).astype(np.float64)
+        ssel = (A * alpha.astype(np.float64)[:, None]).sum(0)
+        beta = np.where(ssel > 0, A * alpha.astype(np.float64)[:, None] / np.where(ssel > 0, ssel, 1.0), 0.0)
+        r = (np.abs(alpha.astype(np.float64)[:, None] - beta) * exact_norm).sum(0)
+        lhs = np.sqrt(((full - out) ** 2).sum())
+        slack = 8 * 2.0 ** -24 * np.sqrt((full ** 2).sum())
+        assert lhs <= np.sqrt((r ** 2).sum()) + slack, f
+        checked_drift |= lhs > slack
+    assert checked_drift   # some budget actually moved the result
+
+
+def test_dare_ties_p0_equals_ties_density_one():
+    """p = 0 keeps every delta with sigma = 1, and TIES at density 1 trims nothing: the two
+    are the same operator (election, disjoint mean, lambda)"""
+    rng = np.random.default_rng(21)
+    n, K = 1500, 5
+    base = to_bf16(rng.standard_normal(n) * 0.02)
+    ex = [to_bf16(bf16_to_f32(base) + (rng.standard_normal(n) * 1e-2 * (k + 1)).astype(np.float32)) for k in range(K)]
+    for k in range(K):
+        z = rng.random(n) < 0.3
+        ex[k][z] = base[z]   # some exact zero deltas
+    taus = [oracle.tau_from_hist(oracle.key_hist(oracle.BF16, base, e), n, 1.0) for e in ex]
+    for mask in (0b11111, 0b10110, 0b00001):
+        t = oracle.merge_block(oracle.BF16, 0, base, ex, mask, oracle.Op(oracle.TIES, K, lam=0.7, density=1.0), taus)
+        d = oracle.merge_block(oracle.BF16, 0, base, ex, mask,
+                               oracle.Op(oracle.DARE_TIES, K, lam=0.7, drop_p=0.0, seed=5))
+        assert np.array_equal(t, d), mask
+
+
+def test_dare_ties_uses_the_dare_mask():
+    """an element whose every selected delta is dropped by the (cuRAND-pinned) keep mask
+    stays at the base; an element with exactly one kept nonzero delta gets
+    fma(lambda, delta * sigma, base), the mean of a single entry"""
+    rng = np.random.default_rng(22)
+    n, K, p, seed, j0 = 4096, 3, 0.6, 77, 8 * 1000
+    base = to_bf16(rng.standard_normal(n) * 0.02)
+    ex = [to_bf16(bf16_to_f32(base) + (rng.standard_normal(n) * 1e-2).astype(np.float32)) for _ in range(K)]
+    op = oracle.Op(oracle.DARE_TIES, K, lam=0.9, drop_p=p, seed=seed)
+    out = bf16_to_f32(oracle.merge_block(oracle.BF16, j0, base, ex, 0b111, op))
+    keep = np.array([[oracle.dare_keep(seed, i, j0 + k, p) for k in range(n)] for i in range(K)])
+    x0 = bf16_to_f32(base)
+    d = np.stack([bf16_to_f32(e) - x0 for e in ex])
+    sigma = np.float32(1.0 / (1.0 - p))
+    none = ~keep.any(0)
+    assert none.any() and np.array_equal(out[none], x0[none])
+    one = (keep & (d != 0)).sum(0) == 1
+    assert one.any()
+    for k in np.nonzero(one)[0][:200]:
+        i = int(np.nonzero(keep[:, k] & (d[:, k] != 0))[0][0])
+        v = np.float32(d[i, k] * sigma)
+        want = np.float32(np.float64(np.float32(0.9)) * np.float64(v) + np.float64(x0[k]))  # one rounding (fma)
+        assert out[k] == bf16_to_f32(to_bf16(np.array([want], np.float32)))[0], k
