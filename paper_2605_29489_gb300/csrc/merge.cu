@@ -263,7 +263,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t aux,
                        const char* src_row, uint32_t bytes) -> bool {
       const uint32_t s = fill % kSlots, r = fill / kSlots;
-      if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+      if (r > 0 && !mbar_wait<true>(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
       if (r > 0) fence_proxy_async_smem();
       S.meta[s].off = off;
       S.meta[s].q = q;
@@ -383,7 +383,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
   };
   for (uint32_t fill = 0;; ++fill) {
     const uint32_t s = fill % kSlots, r = fill / kSlots;
-    if (!warp_wait(&S.full[s], r & 1u, abort_flag)) {
+    if (!warp_wait<true>(&S.full[s], r & 1u, abort_flag)) {
       atomicOr(p.err, kErrTimeout);
       S.abort = 1;
       break;

@@ -7,7 +7,13 @@
 
 namespace mp {
 
-constexpr uint32_t kWaitLimit = 1u << 22;  // try_wait rounds before a wait gives up
+// A sleeping wait suspends the thread for up to kSuspendHintNs per try_wait round (it resumes
+// as soon as the phase completes), so waiting warps do not spin on the issue slots that working
+// warps need; a polling wait returns after each round.  Which one a kernel uses is a measured
+// choice (the merge kernel sleeps, the catalog kernel polls).  kWaitLimit rounds bound every
+// wait to a few seconds.
+constexpr uint32_t kSuspendHintNs = 2000;
+constexpr uint32_t kWaitLimit = 1u << 21;  // try_wait rounds before a wait gives up
 
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
@@ -37,11 +43,23 @@ __device__ __forceinline__ bool mbar_try_wait(uint64_t* bar, uint32_t parity) {
   return ok != 0;
 }
 
+// try_wait that may suspend the thread for up to kSuspendHintNs
+__device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n selp.u32 %0, 1, 0, p;\n}\n"
+      : "=r"(ok)
+      : "r"(su32(bar)), "r"(parity), "r"(kSuspendHintNs)
+      : "memory");
+  return ok != 0;
+}
+
 // bounded wait for the phase with the given parity; false on expiry or when *abort is set
+template <bool SLEEP = false>
 __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
   for (uint32_t k = 0; k < kWaitLimit; ++k) {
-    if (mbar_try_wait(bar, parity)) return true;
-    if ((k & 255u) == 255u && *abort) return false;
+    if (SLEEP ? mbar_try_wait_sleep(bar, parity) : mbar_try_wait(bar, parity)) return true;
+    if ((k & 15u) == 15u && *abort) return false;
   }
   return false;
 }
@@ -70,8 +88,9 @@ __device__ __forceinline__ void tma_load_1d(void* dst, const void* src, uint32_t
 
 // every lane of the warp waits (each acquires the barrier); the outcome is made uniform
 // across the warp so that a give-up never splits a warp
+template <bool SLEEP = false>
 __device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const bool ok = mbar_wait(bar, parity, abort);
+  const bool ok = mbar_wait<SLEEP>(bar, parity, abort);
   return __all_sync(0xFFFFFFFFu, ok);
 }
 
