@@ -11,8 +11,8 @@
 //  * lane 0 then walks each chunk's fills — the base chunk, then every selected expert's
 //    chunk in ascending expert order — and streams each fill into the next slot of a ring
 //    of NS shared-memory slots with one cp.async.bulk (TMA 1-D bulk copy), completing on
-//    the slot's "full" mbarrier; it writes the slot's metadata (chunk, which checkpoint,
-//    offset, length, mask, threshold) before arming the barrier;
+//    the slot's "full" mbarrier; it writes the slot's metadata (chunk, offset, length,
+//    mask, TIES threshold) before arming the barrier;
 //  * consumers take the slots in the same order: the base fill loads M_0 into registers,
 //    each expert fill folds Delta_i into fp32 accumulators, the last fill of a chunk
 //    writes the output with 16-byte streaming stores; each warp releases a slot on its
@@ -42,8 +42,6 @@
 namespace mp {
 namespace {
 
-constexpr int kConsumers = 256;
-constexpr int kThreads = kConsumers + 32;  // + one producer warp
 constexpr uint32_t kEnd = 0xFFFFFFFFu;
 
 enum { OP_ADD = 0, OP_TIES = 1, OP_DARE = 2, OP_RENORM = 3, OP_DTIES = 4 };
@@ -56,11 +54,14 @@ template <int OPC>
 constexpr bool kAddGeo = OPC == OP_ADD || OPC == OP_RENORM;
 
 // slot geometry per operator.  The additive merges are bound by HBM: two CTAs per SM with a
-// 96 KiB ring each.  TIES, DARE and DARE-TIES spend more arithmetic per byte: three CTAs per SM (more
-// warps to hide it) with a 64 KiB ring each, and chunks half as long (one 16-byte vector per
-// consumer thread) so that their per-element state fits the register budget.
+// 96 KiB ring each (two 16-byte vectors per consumer thread and fill).  TIES, DARE and
+// DARE-TIES spend more arithmetic per byte: three CTAs per SM (more warps to hide it; measured
+// better than fewer consumer threads with more work each) with a 64 KiB ring of 4 KiB slots
+// (one vector per consumer thread and fill, so that their state fits the register budget).
 template <int OPC>
 struct Geo {
+  static constexpr int kConsumers = 256;
+  static constexpr int kThreads = kConsumers + 32;  // + one producer warp
   static constexpr int kCtasPerSm = kAddGeo<OPC> ? 2 : 3;
   static constexpr uint32_t kRingBytes = kAddGeo<OPC> ? 98304u : 65536u;
   static constexpr uint32_t kSlotBytes = kAddGeo<OPC> ? 8192u : 4096u;  // one chunk of one checkpoint
@@ -71,7 +72,6 @@ struct Geo {
 struct SlotMeta {
   uint64_t off;   // element offset of the chunk in the flat buffers
   uint32_t q;     // chunk id, or kEnd
-  uint32_t which; // 0 = base, 1 + i = expert i
   uint32_t n;     // elements in the chunk
   uint32_t m;     // the block's access mask
   uint32_t aux;   // TIES: bits threshold of this (expert, trim group); renormalised AVG: the
@@ -225,8 +225,9 @@ __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t nav
 }
 
 template <bool BF16, int OPC>
-__global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
+__global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
     merge_tma_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
+  constexpr int kConsumers = Geo<OPC>::kConsumers;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t SB = Geo<OPC>::kSlotBytes;
   constexpr int kSlots = Geo<OPC>::kSlots;
@@ -260,14 +261,13 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     uint32_t fill = 0;
     bool ok = true;
     // lane 0 arms slot `fill` with the given chunk data and starts its bulk copy
-    auto produce = [&](uint32_t q, uint32_t which, uint64_t off, uint32_t n, uint32_t m, uint32_t aux,
+    auto produce = [&](uint32_t q, uint64_t off, uint32_t n, uint32_t m, uint32_t aux,
                        const char* src_row, uint32_t bytes) -> bool {
       const uint32_t s = fill % kSlots, r = fill / kSlots;
       if (r > 0 && !mbar_wait<true>(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
       if (r > 0) fence_proxy_async_smem();
       S.meta[s].off = off;
       S.meta[s].q = q;
-      S.meta[s].which = which;
       S.meta[s].n = n;
       S.meta[s].m = m;
       S.meta[s].aux = aux;
@@ -330,11 +330,11 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
           const uint32_t q = (uint32_t)(q0 + c);
           const uint32_t bytes = (cm.n * ES) & ~15u;
           const uint32_t aux0 = OPC == OP_RENORM ? (cm.m | S.zmask[c]) : 0u;
-          ok = produce(q, 0, cm.off, cm.n, cm.m, aux0, static_cast<const char*>(p.base) + cm.off * ES, bytes);
+          ok = produce(q, cm.off, cm.n, cm.m, aux0, static_cast<const char*>(p.base) + cm.off * ES, bytes);
           for (uint32_t mm = cm.m; ok && mm; mm &= mm - 1) {
             const uint32_t i = __ffs(mm) - 1;
             // DARE-TIES keeps every nonzero rescaled delta: threshold = the smallest subnormal
-            ok = produce(q, 1 + i, cm.off, cm.n, cm.m, OPC == OP_TIES ? S.thr[c][i] : 1u,
+            ok = produce(q, cm.off, cm.n, cm.m, OPC == OP_TIES ? S.thr[c][i] : 1u,
                          static_cast<const char*>(p.experts.p[i]) + (cm.off - p.expert_origin) * ES, bytes);
             S.realized[i] += (unsigned long long)cm.n * ES;
           }
@@ -344,7 +344,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
       __syncwarp();
     }
     if (lane == 0) {
-      if (ok) ok = produce(kEnd, 0, 0, 0, 0, 0u, nullptr, 0);
+      if (ok) ok = produce(kEnd, 0, 0, 0, 0u, nullptr, 0);
       if (!ok) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
@@ -366,6 +366,7 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
   uint32_t cnt[VPT][V];  // TIES: positive count | negative count << 16
   uint64_t off = 0;
   uint32_t n = 0, n_tma = 0, remaining = 0;
+  uint32_t m_chunk = 0, m_rest = 0;  // the chunk's access mask; its experts still to come
   float s_sel = 0.0f;  // renormalised AVG: sum of the counted experts' alpha (ascending)
   // DARE keep decisions of the vector's elements: element j keeps its delta iff 16-bit
   // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is exactly
@@ -388,13 +389,16 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
       S.abort = 1;
       break;
     }
-    const SlotMeta mt = S.meta[s];
-    if (mt.q == kEnd) break;
     const uint8_t* slot = S.slot[s];
-    if (mt.which == 0) {
+    // fills come as the base chunk, then its selected experts in ascending order: only a
+    // base fill needs the slot's metadata; an expert fill's expert is the next set bit
+    if (remaining == 0) {
+      const SlotMeta mt = S.meta[s];
+      if (mt.q == kEnd) break;
       off = mt.off;
       n = mt.n;
       n_tma = ((n * ES) & ~15u) / ES;
+      m_chunk = m_rest = mt.m;
       remaining = __popc(mt.m);
       if constexpr (OPC == OP_RENORM) {
         s_sel = 0.0f;
@@ -416,14 +420,15 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
         }
       }
     } else {
-      const uint32_t i = mt.which - 1;
+      const uint32_t i = __ffs(m_rest) - 1;
+      m_rest &= m_rest - 1;
       const void* src = p.experts.p[i];
       if constexpr (kTiesLike<OPC>) {
         // TIES: trim test on the magnitude's bits: key(|d|) >= tau exactly when bits(|d|) >=
         // the producer's threshold (a NaN pattern, never true, when nothing is kept).
         // DARE-TIES: the delta is first dropped or rescaled by the keep mask, and every
         // nonzero result is kept (threshold = the smallest subnormal).
-        const float thr = __uint_as_float(mt.aux);
+        const float thr = __uint_as_float(OPC == OP_TIES ? S.meta[s].aux : 1u);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
@@ -477,34 +482,56 @@ __global__ void __launch_bounds__(kThreads, Geo<OPC>::kCtasPerSm)
     if (remaining == 0) {
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
+        // every lane of the warp runs the finalisation (a lane past the chunk's end holds
+        // zeros) so that the warp vote below is reached by all of them; only the store is
+        // limited to the chunk
         const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
-        if (k0 >= n) continue;
+        const bool live = k0 < n;
         float y[V];
-        if (mt.m == 0) {
+        if (m_chunk == 0) {  // uniform over the warp
           // no expert selected: every accumulator is +0, so the output is M_0 plus the
           // zero the operator adds (lambda * +0 for TIES, +0 otherwise)
           const float z = kTiesLike<OPC> ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
 #pragma unroll
           for (int e = 0; e < V; ++e) y[e] = __fadd_rn(x0[u][e], z);
-          store_vec<BF16>(p.out, off + k0, n - k0, y);
+          if (live) store_vec<BF16>(p.out, off + k0, n - k0, y);
           continue;
         }
-#pragma unroll
-        for (int e = 0; e < V; ++e) {
-          if constexpr (kTiesLike<OPC>) {
-            // one division per element: the mean of the entries whose sign was elected
-            // (S != 0 implies at least one of them, so c >= 1; otherwise +0 / 1 = +0)
+        if constexpr (kTiesLike<OPC>) {
+          // one division per element: the mean of the entries whose sign was elected
+          // (S != 0 implies at least one of them, so c >= 1; otherwise +0 / 1 = +0).  The
+          // rare numerators that need the IEEE division take it under one warp vote.
+          auto num_c = [&](int e, float& num, uint32_t& c) {
             const bool pos = Sg[u][e] > 0.0f, any = Sg[u][e] != 0.0f;
-            const float num = any ? (pos ? Pp[u][e] : Nn[u][e]) : 0.0f;
-            const uint32_t c = any ? (pos ? (cnt[u][e] & 0xFFFFu) : (cnt[u][e] >> 16)) : 0u;
+            num = any ? (pos ? Pp[u][e] : Nn[u][e]) : 0.0f;
+            c = any ? (pos ? (cnt[u][e] & 0xFFFFu) : (cnt[u][e] >> 16)) : 0u;
+          };
+          bool exact = false;
+#pragma unroll
+          for (int e = 0; e < V; ++e) {
+            float num;
+            uint32_t c;
+            num_c(e, num, c);
             const float2 cy = S.ctab[c];
-            const float mm = div_small(num, cy.x, cy.y);
-            y[e] = __fmaf_rn(p.lambda, mm, x0[u][e]);
-          } else {
-            y[e] = __fadd_rn(x0[u][e], acc[u][e]);
+            y[e] = div_small_fast(num, cy.x, cy.y);
+            exact = exact || div_small_needs_ieee(num);
           }
+          if (__any_sync(0xFFFFFFFFu, exact)) {
+#pragma unroll
+            for (int e = 0; e < V; ++e) {
+              float num;
+              uint32_t c;
+              num_c(e, num, c);
+              if (div_small_needs_ieee(num)) y[e] = __fdiv_rn(num, S.ctab[c].x);
+            }
+          }
+#pragma unroll
+          for (int e = 0; e < V; ++e) y[e] = __fmaf_rn(p.lambda, y[e], x0[u][e]);
+        } else {
+#pragma unroll
+          for (int e = 0; e < V; ++e) y[e] = __fadd_rn(x0[u][e], acc[u][e]);
         }
-        store_vec<BF16>(p.out, off + k0, n - k0, y);
+        if (live) store_vec<BF16>(p.out, off + k0, n - k0, y);
       }
     }
   }
@@ -528,7 +555,7 @@ cudaError_t launch_op(const MergeLaunch& p, cudaStream_t st) {
   uint64_t grid = (uint64_t)sms * Geo<OPC>::kCtasPerSm;
   if (grid > n_chunks) grid = n_chunks;
   if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
-  merge_tma_kernel<BF16, OPC><<<(unsigned)grid, kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
+  merge_tma_kernel<BF16, OPC><<<(unsigned)grid, Geo<OPC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
   count_launches(1);
   return cudaGetLastError();
 }

@@ -14,14 +14,21 @@
 
 namespace mp {
 
-// a / c for a small integer c given as the float c and its reciprocal y = RN(1/c)
-__device__ __forceinline__ float div_small(float a, float c, float y) {
+// the correction step alone: a / c rounded to nearest-even unless div_small_needs_ieee(a)
+__device__ __forceinline__ float div_small_fast(float a, float c, float y) {
   const float q = __fmul_rn(a, y);
   const float r = __fmaf_rn(-q, c, a);
-  float out = __fmaf_rn(r, y, q);
-  const float aa = fabsf(a);
-  if (aa < 0x1p-100f && aa > 0.0f) out = __fdiv_rn(a, c);
-  return out;
+  return __fmaf_rn(r, y, q);
+}
+
+// true for the numerators 0 < |a| < 2^-100, which take the IEEE division
+__device__ __forceinline__ bool div_small_needs_ieee(float a) {
+  return (__float_as_uint(a) & 0x7FFFFFFFu) - 1u < 0x0D7FFFFFu;  // bits of 2^-100 are 0x0D800000
+}
+
+// a / c for a small integer c given as the float c and its reciprocal y = RN(1/c)
+__device__ __forceinline__ float div_small(float a, float c, float y) {
+  return div_small_needs_ieee(a) ? __fdiv_rn(a, c) : div_small_fast(a, c, y);
 }
 
 }  // namespace mp
