@@ -437,7 +437,7 @@ def native(args, rank, world, local_rank):
 
     elapsed_ms = _max_over_ranks(elapsed_ms, world)
     ms_per_step = elapsed_ms / args.steps
-    value = world * len(budgets) * N / (ms_per_step / 1e3)
+    value = replica_value(len(budgets) * N, world, ms_per_step)
 
     line = {
         "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
@@ -492,14 +492,22 @@ def measure_h2d(pinned_src) -> float:
 
 
 def _max_over_ranks(x: float, world: int) -> float:
+    """the largest x over the replicas (the slowest rank's time is the job's time)"""
     if world == 1:
         return x
     import torch
     import torch.distributed as dist
 
-    t = torch.tensor([x], dtype=torch.float64, device="cuda")
+    dev = "cuda" if dist.get_backend() == "nccl" else "cpu"
+    t = torch.tensor([x], dtype=torch.float64, device=dev)
     dist.all_reduce(t, op=dist.ReduceOp.MAX)
     return float(t.item())
+
+
+def replica_value(units_per_rank: float, world: int, ms_per_step: float) -> float:
+    """whole-job throughput of N independent replicas: every rank processes the same units
+    per step, the step takes the slowest rank's time"""
+    return world * units_per_rank / (ms_per_step / 1e3)
 
 
 # ---- K-scaling at a fixed absolute budget (Cor. 1) --------------------------------------------------

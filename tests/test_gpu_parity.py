@@ -187,6 +187,11 @@ def fam_k17():
                         per_expert_active=True, name="k17")
 
 
+def fam_k1():
+    # K = 1, the smallest family (one-expert catalog groups, one-bit masks)
+    return synth.custom([12000, 4096, 777], dtype=synth.BF16, block_elems=2048, K=1, active_frac=0.6, name="k1")
+
+
 def fam_k32():
     # K = 32, the largest family: the access mask uses its top bit
     return synth.custom([9000, 4099, 16384], dtype=synth.BF16, block_elems=2048, K=32, active_frac=0.3,
@@ -196,7 +201,7 @@ def fam_k32():
 FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 
 
-@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17, fam_k32],
+@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17, fam_k32, fam_k1],
                          ids=lambda f: f.__name__)
 def test_parity_small_families(make):
     fam = make()
