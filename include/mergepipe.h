@@ -93,6 +93,8 @@ typedef struct {
   uint32_t K;                     /* number of experts, 1..32 */
   const void* const* experts;     /* host array of K pointers: M_1..M_K */
   uint32_t experts_location;      /* 0 = device memory, 1 = pinned host memory */
+  const uint64_t* lineage_ids;    /* optional host array of K + 1 caller ids of M_0..M_K,
+                                     recorded in the manifest (Sec. 3 "Executor"); NULL = none */
 } mp_family;
 
 /* Operator and its parameters theta (Alg. 1 records op and theta with the plan). */
@@ -235,6 +237,11 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
    MP_ERR_BUDGET if realized reads exceed the planned bytes. */
 mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_bytes_per_expert,
                            uint64_t* realized_total, uint64_t* touched_blocks, uint64_t* digest);
+
+/* The manifest's lineage (Sec. 3: the manifest records lineage): the K + 1 caller ids of
+   M_0..M_K given in mp_family.lineage_ids at merge time, copied into ids[0..K] (all zero
+   when the family gave none).  Host only; no device wait. */
+mp_status mp_manifest_lineage(const mp_manifest* man, uint64_t* ids);
 
 /* B = floor(f * C_full) with C_full = K * sum_t numel_t * element size (the full expert
    read); f in [0, 1] (clamped).  Returns 0 for an invalid family. */

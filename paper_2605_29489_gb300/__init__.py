@@ -23,7 +23,7 @@ import numpy as np
 __all__ = [
     "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
-    "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_budget_from_fraction", "mp_last_error",
+    "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_manifest_lineage", "mp_budget_from_fraction", "mp_last_error",
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "lib", "library_path",
 ]
 
@@ -47,7 +47,8 @@ class _Tensor(ctypes.Structure):
 class _Family(ctypes.Structure):
     _fields_ = [("dtype", ctypes.c_int), ("n_tensors", ctypes.c_uint32), ("tensors", ctypes.POINTER(_Tensor)),
                 ("block_elems", ctypes.c_uint32), ("base", ctypes.c_void_p), ("K", ctypes.c_uint32),
-                ("experts", ctypes.POINTER(ctypes.c_void_p)), ("experts_location", ctypes.c_uint32)]
+                ("experts", ctypes.POINTER(ctypes.c_void_p)), ("experts_location", ctypes.c_uint32),
+                ("lineage_ids", ctypes.POINTER(ctypes.c_uint64))]
 
 
 class _Op(ctypes.Structure):
@@ -79,6 +80,7 @@ def lib():
             ("mp_index_shape", [vp, vp, vp, vp]),
             ("mp_plan_info", [vp, vp, vp, vp, vp, vp, vp]),
             ("mp_manifest_info", [vp, vp, vp, vp, vp]),
+            ("mp_manifest_lineage", [vp, vp]),
         ]:
             f = getattr(L, name)
             f.restype, f.argtypes = st, args
@@ -108,13 +110,14 @@ def _stream_ptr(stream) -> int | None:
 class Family:
     """An mp_family plus the Python objects that keep its memory alive."""
 
-    def __init__(self, tensors, base, experts, block_elems, dtype, experts_location):
+    def __init__(self, tensors, base, experts, block_elems, dtype, experts_location, lineage_ids=None):
         self.tensors = [(int(o), int(n)) for o, n in tensors]
         self.base, self.experts = base, list(experts)
         self._tarr = (_Tensor * len(self.tensors))(*[_Tensor(o, n) for o, n in self.tensors])
         self._earr = (ctypes.c_void_p * len(self.experts))(*[_ptr(e) for e in self.experts])
+        self._lin = None if lineage_ids is None else (ctypes.c_uint64 * (len(self.experts) + 1))(*lineage_ids)
         self.c = _Family(dtype, len(self.tensors), self._tarr, block_elems, _ptr(base), len(self.experts),
-                         self._earr, experts_location)
+                         self._earr, experts_location, self._lin)
 
     @property
     def K(self):
@@ -132,14 +135,17 @@ def _ptr(t) -> int:
     return int(t)
 
 
-def family(tensors, base, experts, block_elems=65536, dtype=None, experts_location=None) -> Family:
-    """tensors: [(offset_elems, numel)] in checkpoint order; base/experts: flat torch tensors"""
+def family(tensors, base, experts, block_elems=65536, dtype=None, experts_location=None, lineage_ids=None) -> Family:
+    """tensors: [(offset_elems, numel)] in checkpoint order; base/experts: flat torch tensors;
+    lineage_ids: optional K + 1 integer ids of the base and the experts, kept in the manifest"""
     if dtype is None:
         import torch
         dtype = MP_BF16 if base.dtype == torch.bfloat16 else MP_F32
     if experts_location is None:
         experts_location = 0 if getattr(experts[0], "is_cuda", True) else 1
-    return Family(tensors, base, experts, block_elems, dtype, experts_location)
+    if lineage_ids is not None and len(lineage_ids) != len(experts) + 1:
+        raise ValueError("lineage_ids needs K + 1 ids (base first)")
+    return Family(tensors, base, experts, block_elems, dtype, experts_location, lineage_ids)
 
 
 class Op:
@@ -261,6 +267,13 @@ def mp_manifest_info(man: Handle, K: int, check: bool = True):
     if check:
         _check(rc)
     return dict(realized=per, realized_total=tot.value, touched=touched.value, digest=dig.value, status=rc)
+
+
+def mp_manifest_lineage(man: Handle, K: int):
+    """the K + 1 lineage ids recorded in the manifest (zeros when none were given)"""
+    ids = np.zeros(K + 1, np.uint64)
+    _check(lib().mp_manifest_lineage(ctypes.c_void_p(man.ptr), ids.ctypes.data))
+    return ids
 
 
 def mp_budget_from_fraction(fam: Family, f: float) -> int:

@@ -724,6 +724,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   mf->device = plan->device;
   mf->K = g.K;
   mf->done = nullptr;
+  for (uint32_t i = 0; i <= kMaxK; ++i) mf->lineage[i] = (family->lineage_ids && i <= g.K) ? family->lineage_ids[i] : 0u;
   const size_t counters_bytes = (size_t)kCounterSlots * g.K * 8;
   // the counters (64 slots x K), the plan summary and the error word come back in one copy
   const size_t back_bytes = counters_bytes + 64 + 16;
@@ -923,6 +924,14 @@ mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_per_expert
   if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the merge gave up");
   if (err) return fail(MP_ERR_CUDA, "merge kernels reported an error");
   if (tot > s[0]) return fail(MP_ERR_BUDGET, "realized expert reads exceed the planned bytes");
+  return MP_OK;
+}
+
+mp_status mp_manifest_lineage(const mp_manifest* man, uint64_t* ids) {
+  mp_status st;
+  if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
+  if (!ids) return fail(MP_ERR_INVALID_ARG, "ids is NULL");
+  for (uint32_t i = 0; i <= man->K; ++i) ids[i] = man->lineage[i];
   return MP_OK;
 }
 

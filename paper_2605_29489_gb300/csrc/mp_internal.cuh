@@ -110,6 +110,7 @@ struct mp_manifest_s {
   unsigned long long* h_realized;  // pinned host copy (slots summed on host)
   uint32_t* h_err;
   uint64_t planned, touched, digest;
+  uint64_t lineage[mp::kMaxK + 1];  // caller ids of M_0..M_K (zeros when none were given)
   cudaEvent_t done;
 };
 

@@ -314,3 +314,23 @@ def test_replay_is_bit_identical():
     cov = torch.from_numpy(tensor_mask(fam)).cuda()   # padding between tensors is never written
     assert torch.equal(o1.view(torch.int16)[cov], o2.view(torch.int16)[cov])
     assert mp.mp_manifest_info(m1, fam.K)["digest"] == mp.mp_manifest_info(m2, fam.K)["digest"]
+
+
+def test_manifest_records_lineage():
+    """Sec. 3: the manifest records the lineage of the merged checkpoint (the caller's ids of
+    M_0..M_K as given with the family); without ids it records zeros"""
+    fam = fam_ragged_bf16()
+    base, experts = fam.host_arrays()
+    b, ex = dev(fam, base), [dev(fam, e) for e in experts]
+    offs, nums, _ = fam.layout()
+    ids = [0xB0, 11, 22, 0xFFFFFFFFFFFFFFFF][: fam.K + 1]
+    gop = mp.make_op(mp.MP_OP_AVG, alpha=[1.0 / fam.K] * fam.K)
+    for lin in (ids, None):
+        mf = mp.family(list(zip(offs.tolist(), nums.tolist())), b, ex, fam.block_elems, fam.dtype, 0, lineage_ids=lin)
+        idx = mp.mp_index_blocks(mf, gop)
+        plan = mp.mp_plan(idx, gop, mp.mp_budget_from_fraction(mf, 0.5))
+        man = mp.mp_merge(mf, idx, plan, torch.empty_like(b))
+        got = mp.mp_manifest_lineage(man, fam.K).tolist()
+        assert got == (ids if lin is not None else [0] * (fam.K + 1))
+        for h in (man, plan, idx):
+            h.free()
