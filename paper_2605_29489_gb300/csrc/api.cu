@@ -780,6 +780,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   {
     double t = floor(plan->drop_p * 65536.0);
     p.dare_T = !(t > 0.0) ? 0u : (t > 65536.0 ? 65536u : (uint32_t)t);
+    p.dare_T16 = (p.dare_T > 65535u ? 65535u : p.dare_T) << 16;
   }
   p.seed = plan->seed;
   for (int r = 0; r < 10; ++r) {

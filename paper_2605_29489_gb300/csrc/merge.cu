@@ -156,16 +156,18 @@ __device__ __forceinline__ void ties_tally(float d, float thr, float& S, float& 
       : "f"(d), "f"(thr));
 }
 
+// bf16 -> fp32: the upper element by a mask, the lower one moved up by a multiply (which runs
+// on the FMA pipe and leaves the ALU pipe to the compares)
 template <bool BF16>
 __device__ __forceinline__ void unpack(const uint4 r, float* x) {
   if constexpr (BF16) {
-    x[0] = __uint_as_float(r.x << 16);
+    x[0] = __uint_as_float(r.x * 65536u);
     x[1] = __uint_as_float(r.x & 0xFFFF0000u);
-    x[2] = __uint_as_float(r.y << 16);
+    x[2] = __uint_as_float(r.y * 65536u);
     x[3] = __uint_as_float(r.y & 0xFFFF0000u);
-    x[4] = __uint_as_float(r.z << 16);
+    x[4] = __uint_as_float(r.z * 65536u);
     x[5] = __uint_as_float(r.z & 0xFFFF0000u);
-    x[6] = __uint_as_float(r.w << 16);
+    x[6] = __uint_as_float(r.w * 65536u);
     x[7] = __uint_as_float(r.w & 0xFFFF0000u);
   } else {
     x[0] = __uint_as_float(r.x);
@@ -379,7 +381,9 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
 #pragma unroll
     for (int e = 0; e < V; ++e) {
       const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
-      kept[e] = ((e & 1) ? (wd >> 16) : (wd & 0xFFFFu)) >= p.dare_T;
+      // word >= T, compared in the upper half of a 32-bit register: the upper word as it
+      // stands, the lower one moved up by a multiply (FMA pipe; the ALU pipe is the busy one)
+      kept[e] = ((e & 1) ? wd : wd * 65536u) >= p.dare_T16;
     }
   };
   for (uint32_t fill = 0;; ++fill) {

@@ -206,6 +206,8 @@ struct MergeLaunch {
   float lambda;
   float sigma;          // DARE rescale
   uint32_t dare_T;      // DARE keep threshold on 16-bit words
+  uint32_t dare_T16;    // min(dare_T, 65535) << 16: the same test on a word in the upper half
+                        // (p = 1 has sigma = 0, so a word kept by the clamp adds exactly +-0)
   uint32_t dare_rk[10][2];  // DARE: Philox round keys of the seed (precomputed on the host)
   uint64_t seed;
   unsigned long long* realized;  // [kCounterSlots][K]
