@@ -217,7 +217,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
   if (tid == 0) {
     for (int s = 0; s < kIxSlots; ++s) {
       mbar_init(&S.full[s], 1);
-      mbar_init(&S.empty[s], kIxConsumers / 32);
+      mbar_init(&S.empty[s], kIxConsumers);  // every consumer thread arrives
     }
     mbar_init(&S.cbar, kIxConsumers / 32);
     S.abort = 0;
@@ -298,8 +298,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
     return true;
   };
   auto release = [&](uint32_t f) {
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&S.empty[f % kIxSlots]);
+    mbar_arrive(&S.empty[f % kIxSlots]);  // every consumer thread: its own reads of the slot are done
   };
   while (alive) {
     if (!wait_full(fill)) break;

@@ -15,8 +15,8 @@
 //    mask, TIES threshold) before arming the barrier;
 //  * consumers take the slots in the same order: the base fill loads M_0 into registers,
 //    each expert fill folds Delta_i into fp32 accumulators, the last fill of a chunk
-//    writes the output with 16-byte streaming stores; each warp releases a slot on its
-//    "empty" mbarrier as soon as it has read it;
+//    writes the output with 16-byte streaming stores; every consumer thread arrives on the
+//    slot's "empty" mbarrier as soon as it has read it;
 //  * the bytes in flight are the ring (NS slots per CTA), independent of registers and of
 //    how many experts a block selects.
 // Per element, in the fixed ascending expert order:
@@ -246,7 +246,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   if (tid == 0) {
     for (int s = 0; s < kSlots; ++s) {
       mbar_init(&S.full[s], 1);
-      mbar_init(&S.empty[s], kConsumers / 32);
+      mbar_init(&S.empty[s], kConsumers);  // every consumer thread arrives
     }
     S.abort = 0;
     mbar_fence_init();
@@ -481,8 +481,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
       }
       --remaining;
     }
-    __syncwarp();
-    if (lane == 0) mbar_arrive(&S.empty[s]);
+    mbar_arrive(&S.empty[s]);  // every consumer thread: its own reads of the slot are done
     if (remaining == 0) {
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
