@@ -371,6 +371,9 @@ def native(args, rank, world, local_rank):
         for h in hs:
             h.free()
 
+    if not touched_mode:   # touched-only outputs hold only the touched blocks
+        fidelity_vs_full(fam, budgets, outs, shared_out, per_budget)
+
     peak, peak_kind = hbm_peak()
     # base read + output write of every materialised element, plus the planned expert reads
     alg_bytes = [2 * (pb["touched_elements"] if touched_mode else N) * es + pb["planned_bytes"] for pb in per_budget]
@@ -471,6 +474,44 @@ def native(args, rank, world, local_rank):
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
                                 "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
     return line
+
+
+def fidelity_vs_full(fam, budgets, outs, shared_out, per_budget):
+    """Tab. 3's fidelity columns for every budget against the full-read merge of the same
+    step (budget 1.0): relative L2 deviation ||M_A - M_full|| / ||M_full|| and the 95th
+    percentile over blocks of ||d_b|| / ||M_full[b]||.  Reporting only: computed after the
+    timed region, per tensor, in fp64 (the merge itself never runs here)."""
+    import torch
+
+    if shared_out or 1.0 not in budgets:
+        return
+    full = outs[budgets.index(1.0)]
+    offs, nums, _ = fam.layout()
+    E = fam.block_elems
+    num2 = [0.0] * len(budgets)
+    den2 = 0.0
+    blk_rel = [[] for _ in budgets]
+    for o, n in zip(offs.tolist(), nums.tolist()):
+        nb = (n + E - 1) // E
+        pad = nb * E - n
+
+        def rows(t):
+            x = t[o:o + n].double()
+            return torch.nn.functional.pad(x, (0, pad)).view(nb, E)
+
+        fr = rows(full)
+        fb2 = (fr * fr).sum(1)
+        den2 += float(fb2.sum())
+        for k in range(len(budgets)):
+            d = rows(outs[k]) - fr
+            db2 = (d * d).sum(1)
+            num2[k] += float(db2.sum())
+            blk_rel[k].append(torch.sqrt(db2 / torch.clamp(fb2, min=1e-300)))
+    for k, pb in enumerate(per_budget):
+        rel = torch.cat(blk_rel[k]).float().cpu()
+        pb["rel_l2_vs_full"] = (num2[k] / den2) ** 0.5 if den2 > 0 else 0.0
+        pb["p95_block_dev_vs_full"] = float(torch.quantile(rel, 0.95)) if rel.numel() <= (1 << 24) else \
+            float(rel.kthvalue(max(1, int(0.95 * rel.numel()))).values)
 
 
 def measure_h2d(pinned_src) -> float:
