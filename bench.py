@@ -396,6 +396,10 @@ def native(args, rank, world, local_rank):
         mf_d = mp.family(tensors, base_d, experts_d, fam.block_elems, fam.dtype, 0)
         e2e_steps = max(3, min(args.steps, 10))
 
+        # each budget's output goes back on a copy stream while the next budget is planned and
+        # merged (separate output buffers); with a shared output buffer the copies stay in order
+        copy_stream = torch.cuda.Stream() if not shared_out else stream
+
         def e2e_step():
             base_d.copy_(base_h, non_blocking=True)
             for d, h in zip(experts_d, experts_h):
@@ -403,11 +407,14 @@ def native(args, rank, world, local_rank):
             hs = []
             idx = mp.mp_index_blocks(mf_d, gop, stream)
             hs.append(idx)
+            stream.wait_stream(copy_stream)  # the previous step's copies have read the outputs
             for k, B in enumerate(Bs):
                 plan = mp.mp_plan(idx, gop, B, stream)
                 out = outs[0 if shared_out else k]
                 man = mp.mp_merge(mf_d, idx, plan, out, stream)
-                outs_h[k].copy_(out, non_blocking=True)
+                copy_stream.wait_stream(stream)
+                with torch.cuda.stream(copy_stream):
+                    outs_h[k].copy_(out, non_blocking=True)
                 hs += [plan, man]
             return hs
 
@@ -425,6 +432,7 @@ def native(args, rank, world, local_rank):
         hl = []
         for _ in range(e2e_steps):
             hl.append(e2e_step())
+        stream.wait_stream(copy_stream)  # the last copies end inside the timed region
         b.record(stream)
         torch.cuda.synchronize()
         barrier()
