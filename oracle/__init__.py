@@ -20,6 +20,7 @@ BF16, F32 = 0, 1
 AVG, TA, TIES, DARE, AVG_RENORM, DARE_TIES = 0, 1, 2, 3, 4, 5
 OK, EINVAL, EOOM, ENONFINITE = 0, -1, -3, -4
 TAU_NONE = 0x8000
+NNZ_MISSING = 0xFFFFFFFF  # catalog entry without block statistics (tensor-level fallback)
 
 _lib = None
 
@@ -53,9 +54,9 @@ def lib():
         L.orc_tau_from_hist.restype = u32
         L.orc_tau_from_hist.argtypes = [vp, u64, ctypes.c_float]
         L.orc_ties_thresholds.argtypes = [vp, ctypes.c_float, vp]
-        L.orc_plan.argtypes = [u32, u64, vp, vp, u32, u32, vp, vp, vp, vp, vp, u64, vp, vp, vp, vp, vp, vp, vp]
+        L.orc_plan.argtypes = [u32, u64, vp, vp, u32, u32, vp, vp, vp, vp, vp, u64, vp, vp, vp, vp, vp, vp, vp, vp, u32]
         L.orc_merge_block.argtypes = [ctypes.c_int, u64, u64, vp, vp, u32, u32, vp, vp, vp]
-        L.orc_merge.argtypes = [vp, vp, vp, vp, vp]
+        L.orc_merge.argtypes = [vp, vp, vp, vp, vp, vp]
         L.orc_philox4x32_10.argtypes = [vp, vp, vp]
         L.orc_dare_keep.argtypes = [u64, u32, u64, ctypes.c_double]
         L.orc_fnv1a64.restype = u64
@@ -182,7 +183,9 @@ def ties_thresholds(fam: Family, density):
 
 # ---- plan -------------------------------------------------------------------------------------
 
-def plan(K, blk_len, blk_group, n_groups, elem_size, op: Op, norm, maxabs, nnz, tau, budget):
+def plan(K, blk_len, blk_group, n_groups, elem_size, op: Op, norm, maxabs, nnz, tau, budget, blk_tensor=None):
+    """Alg. 1; blk_tensor (tensor id of each block) enables the tensor-level fallback for
+    entries whose nnz is NNZ_MISSING"""
     blk_len = np.ascontiguousarray(blk_len, np.uint32)
     blk_group = np.ascontiguousarray(blk_group, np.uint32)
     nb = blk_len.shape[0]
@@ -194,9 +197,11 @@ def plan(K, blk_len, blk_group, n_groups, elem_size, op: Op, norm, maxabs, nnz, 
     order = np.zeros(nb * K, np.uint32)
     out = [ctypes.c_uint64() for _ in range(5)]
     oc = op.c()
+    bt = None if blk_tensor is None else np.ascontiguousarray(blk_tensor, np.uint32)
+    n_t = 0 if bt is None else (int(bt.max()) + 1 if bt.size else 0)
     _check(lib().orc_plan(K, nb, _p(blk_len), _p(blk_group), n_groups, elem_size, ctypes.byref(oc),
                           _p(norm), _p(maxabs), _p(nnz), _p(tau), int(budget), _p(mask),
-                          *[ctypes.byref(o) for o in out], _p(order)))
+                          *[ctypes.byref(o) for o in out], _p(order), _p(bt), n_t))
     chat, nsel, ncand, set_hash, digest = [o.value for o in out]
     return dict(mask=mask, chat=chat, n_sel=nsel, n_cand=ncand, set_hash=set_hash, digest=digest,
                 order=order[:ncand].copy())
@@ -220,12 +225,15 @@ def merge_block(dtype, j0, base, experts, mask, op: Op, tau_k=None, known_zero=0
     return out
 
 
-def merge(fam: Family, op: Op, tau=None, mask=None, out=None):
+def merge(fam: Family, op: Op, tau=None, mask=None, out=None, nnz=None):
+    """Alg. 2; nnz: the catalog's nonzero counts [K][n_blocks] (known-zero deltas for the
+    renormalised AVG), None to derive them from the data"""
     out = np.zeros_like(fam.base) if out is None else out
     tau = None if tau is None else np.ascontiguousarray(tau, np.uint32)
     mask = None if mask is None else np.ascontiguousarray(mask, np.uint32)
+    nz = None if nnz is None else np.ascontiguousarray(nnz, np.uint32)
     c, oc = fam.c(), op.c()
-    _check(lib().orc_merge(ctypes.byref(c), ctypes.byref(oc), _p(tau), _p(mask), _p(out)))
+    _check(lib().orc_merge(ctypes.byref(c), ctypes.byref(oc), _p(tau), _p(mask), _p(out), _p(nz)))
     return out
 
 

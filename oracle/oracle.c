@@ -247,13 +247,25 @@ uint64_t orc_splitmix64(uint64_t state) {
  *     little-endian bytes of (kind, K, alpha[0..K-1] bits, lambda bits, density bits,
  *     trim_scope, drop_p bits, seed, score_mode, B, C_hat, n_sel, set_hash), where set_hash is the
  *     wrapping sum over selected units u of splitmix64(u).
+ *  - Tensor-level fallback (Sec. 3 Planner: deterministic fallback when block metadata
+ *    are missing; Alg. 1's scoring step names fallback metadata).  Reading: an entry
+ *    (i, b) whose nnz is ORC_NNZ_MISSING has no block statistics.  Every (expert i,
+ *    tensor t) holding such an entry is planned as ONE unit at tensor granularity: it is
+ *    always a candidate (nothing rules it out), its id is the unit of the tensor's first
+ *    block b0(t)*K + i, its cost is the whole tensor's bytes, and its score is
+ *    |coef_i| * sqrt(ss) with ss the fp32 chain ss = fma(n_b, n_b, ss) over the known
+ *    blocks of t in ascending order from 0 (the norm of the part of Delta_{i,t} the
+ *    catalog knows; 0 if none), divided by the tensor's bytes (converted to fp32) in the
+ *    score-per-byte mode.  The tensor's other units are not candidates.  Taking it sets
+ *    bit i on every block of t; it counts once in n_sel and set_hash.
  * Pins: brute force over all subsets on tiny inputs; the cardinality-knapsack optimum
- * when all costs are equal; Prop. 1 (C_hat <= B); full budget selects every candidate.
+ * when all costs are equal; Prop. 1 (C_hat <= B); full budget selects every candidate;
+ * for the fallback, a hand-worked catalog and the known-part norm against the deltas.
  * ------------------------------------------------------------------------------------- */
 typedef struct {
   float score;
   uint32_t unit;
-  uint32_t cost;
+  uint64_t cost;
 } orc_cand;
 
 static int cand_cmp(const void* a, const void* b) {
@@ -277,25 +289,62 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
              uint32_t n_groups, uint32_t elem_size, const orc_op* op, const float* norm,
              const float* maxabs, const uint32_t* nnz, const uint32_t* tau, uint64_t budget,
              uint32_t* mask, uint64_t* chat_out, uint64_t* n_sel_out, uint64_t* n_cand_out,
-             uint64_t* set_hash_out, uint64_t* digest_out, uint32_t* order) {
+             uint64_t* set_hash_out, uint64_t* digest_out, uint32_t* order, const uint32_t* blk_tensor,
+             uint32_t n_tensors) {
   if (!op || K == 0 || K > 32 || op->K != K || !norm || !maxabs || !nnz || !mask) return ORC_EINVAL;
   if (op->kind == ORC_TIES && (!tau || !blk_group)) return ORC_EINVAL;
   if (op->kind != ORC_TIES && op->kind != ORC_DARE_TIES && !op->alpha) return ORC_EINVAL;
   if (n_blocks * K > 0xFFFFFFFFull) return ORC_EINVAL;
+  if (blk_tensor) /* tensors in checkpoint order: the blocks of a tensor are contiguous */
+    for (uint64_t b = 0; b < n_blocks; ++b)
+      if (blk_tensor[b] >= n_tensors || (b > 0 && blk_tensor[b] < blk_tensor[b - 1])) return ORC_EINVAL;
+
+  /* fallback pairs (i, t): some entry of tensor t has no statistics for expert i */
+  uint8_t* fb = NULL;
+  if (blk_tensor) {
+    fb = (uint8_t*)calloc((size_t)K * n_tensors + 1, 1);
+    if (!fb) return ORC_EOOM;
+  }
+  for (uint32_t i = 0; i < K; ++i)
+    for (uint64_t b = 0; b < n_blocks; ++b)
+      if (nnz[(uint64_t)i * n_blocks + b] == ORC_NNZ_MISSING) {
+        if (!fb) return ORC_EINVAL; /* missing statistics need the tensor map */
+        fb[(size_t)i * n_tensors + blk_tensor[b]] = 1;
+      }
 
   orc_cand* q = (orc_cand*)malloc(sizeof(orc_cand) * (size_t)(n_blocks * K + 1));
-  if (!q) return ORC_EOOM;
+  if (!q) {
+    free(fb);
+    return ORC_EOOM;
+  }
   uint64_t nq = 0;
   for (uint64_t b = 0; b < n_blocks; ++b) {
     for (uint32_t i = 0; i < K; ++i) {
       uint64_t s = (uint64_t)i * n_blocks + b;
+      float coef = (op->kind == ORC_TIES || op->kind == ORC_DARE_TIES) ? op->lambda : op->alpha[i];
+      if (fb && fb[(size_t)i * n_tensors + blk_tensor[b]]) {
+        const uint32_t t = blk_tensor[b];
+        if (b > 0 && blk_tensor[b - 1] == t) continue; /* only the tensor's first block */
+        float ss = 0.0f;
+        uint64_t cost = 0;
+        for (uint64_t b2 = b; b2 < n_blocks && blk_tensor[b2] == t; ++b2) {
+          const uint64_t s2 = (uint64_t)i * n_blocks + b2;
+          cost += (uint64_t)blk_len[b2] * elem_size;
+          if (nnz[s2] != ORC_NNZ_MISSING) ss = fmaf(norm[s2], norm[s2], ss);
+        }
+        q[nq].score = fabsf(coef) * sqrtf(ss);
+        q[nq].unit = (uint32_t)(b * K + i);
+        q[nq].cost = cost;
+        if (op->score_mode) q[nq].score = q[nq].score / (float)cost;
+        ++nq;
+        continue;
+      }
       if (nnz[s] == 0) continue;
       if (op->kind == ORC_TIES && orc_ties_key(maxabs[s]) < tau[(size_t)i * n_groups + blk_group[b]])
         continue;
-      float coef = (op->kind == ORC_TIES || op->kind == ORC_DARE_TIES) ? op->lambda : op->alpha[i];
       q[nq].score = fabsf(coef) * norm[s];
       q[nq].unit = (uint32_t)(b * K + i);
-      q[nq].cost = blk_len[b] * elem_size;
+      q[nq].cost = (uint64_t)blk_len[b] * elem_size;
       if (op->score_mode) q[nq].score = q[nq].score / (float)q[nq].cost;
       ++nq;
     }
@@ -306,14 +355,21 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
   uint64_t chat = 0, nsel = 0, set_hash = 0;
   for (uint64_t r = 0; r < nq; ++r) {
     if (chat + q[r].cost <= budget) {
+      const uint64_t b = q[r].unit / K;
+      const uint32_t i = q[r].unit % K;
       chat += q[r].cost;
-      mask[q[r].unit / K] |= 1u << (q[r].unit % K);
+      if (fb && fb[(size_t)i * n_tensors + blk_tensor[b]]) {
+        for (uint64_t b2 = b; b2 < n_blocks && blk_tensor[b2] == blk_tensor[b]; ++b2) mask[b2] |= 1u << i;
+      } else {
+        mask[b] |= 1u << i;
+      }
       set_hash += orc_splitmix64(q[r].unit);
       ++nsel;
     }
     if (order) order[r] = q[r].unit;
   }
   free(q);
+  free(fb);
 
   uint8_t hdr[4 + 4 + 4 * 32 + 4 + 4 + 4 + 8 + 8 + 4 + 8 + 8 + 8 + 8];
   size_t o = 0;
@@ -490,9 +546,12 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
 
 /* Alg. 2 ExecuteMerge: tensors in order, blocks in order, every block materialised
    (untouched blocks are copies of the base; the paper's comparisons use full logical
-   checkpoint materialisation).  mask may be NULL for the full read A = 1 (Eq. 1). */
+   checkpoint materialisation).  mask may be NULL for the full read A = 1 (Eq. 1).
+   nnz: the catalog's nonzero counts [K][n_blocks], which tell the renormalised AVG which
+   deltas are known to be zero; NULL derives them from the data (the full catalog).  An
+   entry of ORC_NNZ_MISSING is not known to be zero. */
 int orc_merge(const orc_family* f, const orc_op* op, const uint32_t* tau, const uint32_t* mask,
-              void* out) {
+              void* out, const uint32_t* nnz) {
   if (!f || !op || !out || op->K != f->K || f->K == 0 || f->K > 32) return ORC_EINVAL;
   const uint32_t all = f->K == 32 ? 0xFFFFFFFFu : ((1u << f->K) - 1u);
   uint32_t tau_k[32];
@@ -504,7 +563,10 @@ int orc_merge(const orc_family* f, const orc_op* op, const uint32_t* tau, const 
       if (op->kind == ORC_TIES) tau_k[i] = tau[(size_t)i * f->n_groups + f->blk_group[b]];
     }
     uint32_t known_zero = 0;
-    if (op->kind == ORC_AVG_RENORM) {
+    if (op->kind == ORC_AVG_RENORM && nnz) {
+      for (uint32_t i = 0; i < f->K; ++i)
+        if (nnz[(size_t)i * f->n_blocks + b] == 0) known_zero |= 1u << i;
+    } else if (op->kind == ORC_AVG_RENORM) {
       const void* b0 = elem_ptr(f->dtype, f->base, off);
       for (uint32_t i = 0; i < f->K; ++i) {
         uint64_t k = 0;

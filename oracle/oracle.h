@@ -27,6 +27,7 @@ enum { ORC_BF16 = 0, ORC_F32 = 1 };
 enum { ORC_AVG = 0, ORC_TA = 1, ORC_TIES = 2, ORC_DARE = 3, ORC_AVG_RENORM = 4, ORC_DARE_TIES = 5 };
 enum { ORC_OK = 0, ORC_EINVAL = -1, ORC_EOOM = -3, ORC_ENONFINITE = -4 };
 #define ORC_TAU_NONE 0x8000u /* TIES threshold when k = 0: no 15-bit key reaches it */
+#define ORC_NNZ_MISSING 0xFFFFFFFFu /* catalog entry without block statistics (tensor-level fallback) */
 
 /* merge operator and its parameters theta (Alg. 1 records op and theta) */
 typedef struct {
@@ -75,7 +76,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
              uint32_t n_groups, uint32_t elem_size, const orc_op* op, const float* norm,
              const float* maxabs, const uint32_t* nnz, const uint32_t* tau, uint64_t budget,
              uint32_t* mask, uint64_t* chat, uint64_t* n_sel, uint64_t* n_cand, uint64_t* set_hash,
-             uint64_t* digest, uint32_t* order);
+             uint64_t* digest, uint32_t* order, const uint32_t* blk_tensor, uint32_t n_tensors);
 
 /* Eq. 4 budgeted merge of one block, and of a whole family (Alg. 2).  known_zero (used by
    the renormalised AVG only): bit i set when expert i's delta block is exactly zero, which
@@ -83,7 +84,7 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
 int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const void* const* experts,
                     uint32_t mask, uint32_t known_zero, const orc_op* op, const uint32_t* tau_k, void* out);
 int orc_merge(const orc_family* f, const orc_op* op, const uint32_t* tau, const uint32_t* mask,
-              void* out);
+              void* out, const uint32_t* nnz);
 
 /* generators and hashes */
 void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]);

@@ -624,3 +624,188 @@ def test_dare_ties_uses_the_dare_mask():
         v = np.float32(d[i, k] * sigma)
         want = np.float32(np.float64(np.float32(0.9)) * np.float64(v) + np.float64(x0[k]))  # one rounding (fma)
         assert out[k] == bf16_to_f32(to_bf16(np.array([want], np.float32)))[0], k
+
+
+# ---- tensor-level fallback (Sec. 3 Planner; Alg. 1 scoring with fallback metadata) -----------------------
+
+MISS = oracle.NNZ_MISSING
+
+
+def _fallback_worked_catalog():
+    """two experts over two tensors: t0 = blocks 0-2, t1 = blocks 3-4, 4 bf16 elements (8 bytes)
+    each.  Expert 0 has no statistics for block 2, expert 1 none for block 4."""
+    blk_len = np.full(5, 4, np.uint32)
+    blk_tensor = np.array([0, 0, 0, 1, 1], np.uint32)
+    norm = np.array([[3.0, 4.0, 99.0, 1.0, 2.0],
+                     [1.0, 1.0, 1.0, 6.0, 99.0]], np.float32)
+    nnz = np.array([[4, 4, MISS, 4, 4],
+                    [4, 4, 4, 4, MISS]], np.uint32)
+    return blk_len, blk_tensor, norm, nnz
+
+
+def _fallback_plan(budget, score_mode=0):
+    blk_len, bt, norm, nnz = _fallback_worked_catalog()
+    op = oracle.Op(oracle.AVG, 2, alpha=[1.0, 1.0], score_mode=score_mode)
+    return oracle.plan(2, blk_len, bt, 2, 2, op, norm, np.ones_like(norm), nnz, None, budget, blk_tensor=bt)
+
+
+def test_fallback_worked_example():
+    """Hand-worked.  The pairs (0, t0) and (1, t1) fall back to one unit each:
+    (0, t0): id 0*2+0 = 0, cost 24, score sqrt(3^2 + 4^2) = 5 (block 2's 99 is not used);
+    (1, t1): id 3*2+1 = 7, cost 16, score sqrt(6^2) = 6.
+    Block units: (1,b0) id 1, (1,b1) id 3, (1,b2) id 5, (0,b3) id 6 with score 1 and (0,b4) id
+    8 with score 2, cost 8 each.  Order by score: 7, 0, 8, then 1, 3, 5, 6.
+    B = 40: 7 (16), 0 (40), then nothing fits.  B = 30: 7 (16), 0 skipped, 8 (24), the rest
+    skipped.  Per byte the scores are 6/16, 5/24, 2/8 and 1/8: order 7, 8, 0, 1, 3, 5, 6; B = 48
+    takes 7, 8 and 0 (48).  B = 80 (everything) takes every unit."""
+    p = _fallback_plan(40)
+    assert p["order"].tolist() == [7, 0, 8, 1, 3, 5, 6] and p["n_cand"] == 7
+    assert p["mask"].tolist() == [1, 1, 1, 2, 2] and p["chat"] == 40 and p["n_sel"] == 2
+    assert p["set_hash"] == (oracle.splitmix64(7) + oracle.splitmix64(0)) % 2 ** 64
+    p = _fallback_plan(30)
+    assert p["mask"].tolist() == [0, 0, 0, 2, 3] and p["chat"] == 24 and p["n_sel"] == 2
+    p = _fallback_plan(48, score_mode=1)
+    assert p["order"].tolist() == [7, 8, 0, 1, 3, 5, 6]
+    assert p["mask"].tolist() == [1, 1, 1, 2, 3] and p["chat"] == 48
+    p = _fallback_plan(30, score_mode=1)
+    assert p["mask"].tolist() == [0, 0, 0, 2, 3] and p["chat"] == 24
+    p = _fallback_plan(80)
+    assert p["mask"].tolist() == [3] * 5 and p["chat"] == 80 and p["n_sel"] == 7
+
+
+def test_fallback_needs_the_tensor_map():
+    blk_len, bt, norm, nnz = _fallback_worked_catalog()
+    op = oracle.Op(oracle.AVG, 2, alpha=[1.0, 1.0])
+    with pytest.raises(Exception):
+        oracle.plan(2, blk_len, bt, 2, 2, op, norm, np.ones_like(norm), nnz, None, 40)
+    with pytest.raises(Exception):   # a tensor's blocks must be contiguous
+        oracle.plan(2, blk_len, bt, 2, 2, op, norm, np.ones_like(norm), nnz, None, 40,
+                    blk_tensor=np.array([0, 1, 0, 1, 1], np.uint32))
+
+
+def test_fallback_without_missing_entries_is_the_block_plan(tiny_family):
+    """the tensor map changes nothing while every entry has statistics"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    norm, maxabs, nnz = oracle.index(of)
+    _, bl, bt = fam.block_table()
+    for kind, kw in ((oracle.TA, dict(alpha=[0.3, -0.5, 0.7, 1.0][:fam.K])), (oracle.AVG, dict(alpha=[0.25] * fam.K))):
+        for sm in (0, 1):
+            op = oracle.Op(kind, fam.K, score_mode=sm, **kw)
+            for f in (0.1, 0.5, 1.0):
+                B = int(f * fam.K * fam.total_elems * 4)
+                a = oracle.plan(fam.K, bl, bt, len(fam.tensors), 4, op, norm, maxabs, nnz, None, B)
+                b = oracle.plan(fam.K, bl, bt, len(fam.tensors), 4, op, norm, maxabs, nnz, None, B, blk_tensor=bt)
+                assert a["digest"] == b["digest"] and np.array_equal(a["mask"], b["mask"])
+                assert np.array_equal(a["order"], b["order"])
+
+
+def test_fallback_score_is_the_known_part_norm_of_the_deltas(tiny_family):
+    """Against the deltas themselves: with one expert, a fallback tensor t competes with one
+    block whose catalog norm is set 0.1 % above or below ||Delta_t|| over t's known blocks
+    (fp64, from the data).  The budget fits either but not both, so the winner shows the
+    order: the block wins when above, the tensor when below."""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base[:], [experts[0]])
+    norm, maxabs, nnz = oracle.index(of)
+    bo, bl, bt = fam.block_table()
+    counts = np.bincount(bt)
+    t = int(np.argmax(counts))                      # the tensor with most blocks
+    blocks = np.nonzero(bt == t)[0]
+    assert len(blocks) >= 3
+    other = int(np.nonzero(bt != t)[0][0])
+    miss = int(blocks[1])
+    nnz = nnz.copy()
+    keep = np.zeros(nnz.shape[1], bool)
+    keep[blocks] = True
+    keep[other] = True
+    nnz[0, ~keep] = 0                               # nothing else competes
+    nnz[0, miss] = MISS
+    d = experts[0].astype(np.float64) - base.astype(np.float64)
+    known = [int(b) for b in blocks if int(b) != miss]
+    exact = math.sqrt(sum(float((d[int(bo[b]):int(bo[b] + bl[b])] ** 2).sum()) for b in known))
+    t_cost = int(bl[blocks].sum()) * 4
+    B = max(t_cost, int(bl[other]) * 4)
+    assert B < t_cost + int(bl[other]) * 4
+    op = oracle.Op(oracle.TA, 1, alpha=[1.0])
+    for factor, tensor_wins in ((1.001, False), (0.999, True)):
+        nm = norm.copy()
+        nm[0, other] = np.float32(exact * factor)
+        p = oracle.plan(1, bl, bt, len(fam.tensors), 4, op, nm, maxabs, nnz, None, B, blk_tensor=bt)
+        assert bool(p["mask"][blocks[0]]) == tensor_wins
+        assert bool(p["mask"][other]) == (not tensor_wins)
+        # all or nothing over the tensor
+        assert len(set(int(p["mask"][b]) for b in blocks)) == 1
+
+
+def test_fallback_properties_on_random_catalogs():
+    """For random catalogs with missing entries: a fallback pair is read all or nothing;
+    C_hat is the bytes the mask reads and never exceeds B (Prop. 1); the candidates are the
+    fallback pairs plus the other units with nnz > 0; the full budget reads every candidate
+    block; along the order, the greedy takes a unit iff it still fits."""
+    rng = np.random.default_rng(31)
+    for trial in range(40):
+        K = int(rng.integers(1, 5))
+        n_t = int(rng.integers(1, 6))
+        per_t = rng.integers(1, 5, n_t)
+        bt = np.repeat(np.arange(n_t), per_t).astype(np.uint32)
+        nb = bt.size
+        bl = rng.integers(1, 9, nb).astype(np.uint32)
+        norm = rng.choice([0.5, 1.0, 2.0, 3.0], (K, nb)).astype(np.float32)
+        nnz = (rng.random((K, nb)) > 0.25).astype(np.uint32) * 3
+        nnz[rng.random((K, nb)) < 0.2] = MISS
+        op = oracle.Op(oracle.TA, K, alpha=rng.choice([-1.0, 0.5, 2.0], K), score_mode=trial % 2)
+        fb = np.zeros((K, n_t), bool)
+        for i in range(K):
+            for b in range(nb):
+                fb[i, bt[b]] |= nnz[i, b] == MISS
+        first = {int(t): int(np.nonzero(bt == t)[0][0]) for t in range(n_t)}
+        cost = {}
+        for b in range(nb):
+            for i in range(K):
+                if fb[i, bt[b]]:
+                    if b == first[int(bt[b])]:
+                        cost[b * K + i] = int(bl[bt == bt[b]].sum()) * 2
+                elif nnz[i, b] > 0:
+                    cost[b * K + i] = int(bl[b]) * 2
+        total = sum(cost.values())
+        for B in (0, total // 3, total // 2, total):
+            p = oracle.plan(K, bl, np.zeros(nb, np.uint32), 1, 2, op, norm, np.ones_like(norm), nnz, None, B,
+                            blk_tensor=bt)
+            A = (p["mask"][None, :] >> np.arange(K)[:, None]) & 1
+            for i in range(K):
+                for t in range(n_t):
+                    if fb[i, t]:
+                        assert len(set(A[i, bt == t].tolist())) == 1
+            assert p["chat"] == int((A * bl[None, :]).sum()) * 2 <= B
+            assert p["n_cand"] == len(cost) and sorted(p["order"].tolist()) == sorted(cost)
+            run = 0
+            for u in p["order"].tolist():
+                b, i = u // K, u % K
+                if A[i, b]:
+                    assert run + cost[u] <= B
+                    run += cost[u]
+                else:
+                    assert run + cost[u] > B
+            assert run == p["chat"]
+            if B == total:
+                want = fb[:, bt] | ((nnz > 0) & (nnz != MISS))
+                assert np.array_equal(A.astype(bool), want)
+
+
+def test_fallback_plan_at_full_budget_merges_like_the_full_read(tiny_family):
+    """A = 1 over every block that can change the output recovers the full-read operator
+    (Eq. 5), whatever entries lack statistics"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    norm, maxabs, nnz = oracle.index(of)
+    _, bl, bt = fam.block_table()
+    rng = np.random.default_rng(32)
+    nnz = nnz.copy()
+    nnz[rng.random(nnz.shape) < 0.15] = MISS
+    for op in (oracle.Op(oracle.TA, fam.K, alpha=[0.4] * fam.K), oracle.Op(oracle.AVG_RENORM, fam.K, alpha=[1.0] * fam.K)):
+        B = fam.K * fam.total_elems * 4
+        p = oracle.plan(fam.K, bl, bt, len(fam.tensors), 4, op, norm, maxabs, nnz, None, B, blk_tensor=bt)
+        got = oracle.merge(of, op, mask=p["mask"], nnz=nnz)
+        want = oracle.merge(of, op)
+        assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
