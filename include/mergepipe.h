@@ -53,6 +53,10 @@ typedef int32_t mp_status;
 
 typedef struct CUstream_st* mp_stream;
 
+/* nnz of a catalog entry that has no block statistics (mp_index_import); no block holds
+   2^32 - 1 elements, so no count takes this value */
+#define MP_NNZ_MISSING 0xFFFFFFFFu
+
 typedef enum { MP_BF16 = 0, MP_F32 = 1 } mp_dtype;
 
 /* Merge operators (Sec. 1, App. A.1).  AVG and TA are the fixed-coefficient additive
@@ -131,6 +135,25 @@ typedef struct mp_manifest_s mp_manifest;
 mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream stream, mp_index** out);
 
 /*
+ * mp_index_import — a catalog from statistics computed earlier, without reading the
+ * experts (Sec. 3 "Catalog": the metadata are reusable, so planning needs no new scan).
+ * norm, maxabs, nnz: host arrays [K][n_blocks], expert-major, in the layout and meaning
+ * mp_index_stats returns for this family's geometry; tau: host [K][n_groups] TIES
+ * thresholds (required iff op is TIES; n_groups as for mp_index_blocks), else NULL.
+ * An entry whose nnz is MP_NNZ_MISSING has no block metadata (its norm and maxabs are
+ * ignored): mp_plan then plans every (expert, tensor) pair holding such an entry at tensor
+ * granularity (Sec. 3 "Planner", the deterministic tensor-level fallback; see mp_plan).
+ * Every other entry must be a block statistic: nnz <= the block's elements, norm and
+ * maxabs finite and >= 0; tau entries in [0, 0x8000].  The arrays are copied before the
+ * call returns; the family's buffers are not read here (only its geometry), but must be
+ * the ones the statistics describe when the index is used to merge.  The renormalised
+ * AVG treats a delta as known to be zero only where nnz = 0.
+ * Errors: MP_ERR_INVALID_ARG (bad family, op or entry), MP_ERR_OOM, MP_ERR_CUDA.
+ */
+mp_status mp_index_import(const mp_family* family, const mp_op* op, const float* norm, const float* maxabs,
+                          const uint32_t* nnz, const uint32_t* tau, mp_stream stream, mp_index** out);
+
+/*
  * mp_plan — Alg. 1 PlanGen under budget B (bytes of expert reads, Eq. 3; cost of unit
  * (i,b) = elements(b) * element size, App. A.1).
  *  candidates: units with nnz > 0 (for TIES also bf16 key of maxabs >= tau); the others
@@ -138,6 +161,14 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
  *  score:      |alpha_i| * norm (TIES: |lambda| * norm), fp32 (Prop. 2's utility);
  *  order:      decreasing score, ties by ascending unit id b*K + i;
  *  select:     greedy with skip — a candidate is taken iff C_hat + c <= B.
+ *  fallback:   (imported catalogs with MP_NNZ_MISSING entries; Sec. 3 "Planner") each
+ *              (expert i, tensor t) holding such an entry is ONE candidate with unit id
+ *              b0(t)*K + i (b0 = the tensor's first block), cost = the whole tensor's bytes
+ *              and score |coef_i| * sqrt(ss), ss = the fp32 chain fma(norm, norm, ss) over
+ *              t's known blocks in block order (0 if none); per byte in score mode 1 (the
+ *              cost converted to fp32).  t's other units of expert i are not candidates;
+ *              taking it sets bit i on every block of t.  It counts once in the number
+ *              selected and in the set hash.
  * The plan records the access mask (bit i of word b = A_{i,t,b}), C_hat, the number of
  * selected units, the traversal order and a digest (FNV-1a 64 over op, theta, B, C_hat,
  * count and the sum of splitmix64(unit) over the selected units).  Budget soundness
@@ -200,6 +231,8 @@ mp_status mp_merge_touched(const mp_family* family, const mp_index* index, const
  *  outputs (device): mask[n_blocks], order[K*n_blocks] (first n_candidates valid),
  *    summary[8] uint64 = {planned bytes, selected, candidates, selected-unit set hash,
  *    digest, touched blocks, error word, 0}.  The results equal mp_plan's bit for bit.
+ *    This call has no tensor map, so it does not plan the tensor-level fallback: an nnz
+ *    of MP_NNZ_MISSING sets bit 8 of the error word, and that entry is never read.
  * Limit: K * n_blocks <= 524288 units; larger requests return MP_ERR_INVALID_ARG and
  * launch nothing.  The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current); make that first call before any

@@ -24,7 +24,8 @@ __all__ = [
     "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_manifest_lineage", "mp_budget_from_fraction", "mp_last_error",
-    "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "lib", "library_path",
+    "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "lib",
+    "library_path",
 ]
 
 MP_OK = 0
@@ -32,6 +33,7 @@ MP_ERR = {-1: "MP_ERR_INVALID_ARG", -2: "MP_ERR_CUDA", -3: "MP_ERR_OOM", -4: "MP
           -5: "MP_ERR_BUDGET", -6: "MP_ERR_TIMEOUT", -7: "MP_ERR_UNSUPPORTED", -8: "MP_ERR_MISMATCH"}
 MP_BF16, MP_F32 = 0, 1
 MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES = 0, 1, 2, 3, 4, 5
+MP_NNZ_MISSING = 0xFFFFFFFF   # catalog entry without block statistics (tensor-level fallback)
 
 
 class MergePipeError(RuntimeError):
@@ -73,6 +75,7 @@ def lib():
         vp, u64, st = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int32
         for name, args in [
             ("mp_index_blocks", [vp, vp, vp, vp]),
+            ("mp_index_import", [vp, vp, vp, vp, vp, vp, vp, vp]),
             ("mp_plan", [vp, vp, u64, vp, vp]),
             ("mp_merge", [vp, vp, vp, vp, vp, vp]),
             ("mp_merge_touched", [vp, vp, vp, vp, vp, vp]),
@@ -191,6 +194,18 @@ def mp_index_blocks(fam: Family, op: Op | None = None, stream=None) -> Handle:
     out = ctypes.c_void_p()
     _check(lib().mp_index_blocks(fam.ref(), None if op is None else op.ref(), ctypes.c_void_p(_stream_ptr(stream)),
                                  ctypes.byref(out)))
+    return Handle(out.value, "index")
+
+
+def mp_index_import(fam: Family, op: Op | None, norm, maxabs, nnz, tau=None, stream=None) -> Handle:
+    """a catalog from saved statistics (host arrays [K, n_blocks], tau [K, n_groups] for TIES);
+    entries with nnz == MP_NNZ_MISSING have no statistics"""
+    arrs = [np.ascontiguousarray(norm, np.float32), np.ascontiguousarray(maxabs, np.float32),
+            np.ascontiguousarray(nnz, np.uint32), None if tau is None else np.ascontiguousarray(tau, np.uint32)]
+    out = ctypes.c_void_p()
+    _check(lib().mp_index_import(fam.ref(), None if op is None else op.ref(),
+                                 *[None if a is None else a.ctypes.data for a in arrs],
+                                 ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(out)))
     return Handle(out.value, "index")
 
 

@@ -1,6 +1,7 @@
 // Host side of the C ABI: argument validation, handle lifetime, block tables and the
 // launch sequence of index, plan and merge.  Every device step runs in the kernels of
 // index.cu, plan.cu and merge.cu; this file only marshals arguments and memory.
+#include <float.h>
 #include <math.h>
 #include <string.h>
 
@@ -218,6 +219,11 @@ mp_status cuda_fail(cudaError_t e, const char* what) {
   return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
 }
 
+mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t work_bytes, cudaStream_t cs,
+                    mp_index_s** out, char** work);
+cudaError_t finish_index(mp_index_s* ix, cudaStream_t cs);
+void discard_index(mp_index_s* ix, cudaStream_t cs);
+
 // ---- experts in pinned host memory: segment pipeline -------------------------------------
 //
 // The family is walked in segments of consecutive blocks (about kSegmentElems elements
@@ -406,6 +412,106 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
   return e;
 }
 
+// A new index handle for geometry g: one device allocation holding the block table
+// (offset, length, TIES trim group and tensor of each block, first block of each tensor),
+// the statistics, the error word and work_bytes of scratch for the caller (*work).  The
+// table is uploaded and the error word and tau cleared on cs.
+mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t work_bytes, cudaStream_t cs,
+                    mp_index_s** out, char** work) {
+  const bool ties = op && op->kind == MP_OP_TIES;
+  const uint32_t scope = ties ? op->trim_scope : 0u;
+  const uint32_t n_groups = scope == 0 ? g.n_tensors : 1u;
+  const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
+  std::vector<uint64_t> h_off(nb);
+  std::vector<uint32_t> h_len(nb), h_grp(nb), h_tens(nb), h_tb0(g.n_tensors + 1);
+  for (uint32_t t = 0; t < g.n_tensors; ++t) {
+    const uint64_t b0 = g.t_first_block[t], tb = (g.t_numel[t] + g.block_elems - 1) / g.block_elems;
+    h_tb0[t] = (uint32_t)b0;
+    for (uint64_t k = 0; k < tb; ++k) {
+      h_off[b0 + k] = g.t_off[t] + k * g.block_elems;
+      const uint64_t rem = g.t_numel[t] - k * g.block_elems;
+      h_len[b0 + k] = (uint32_t)(rem < g.block_elems ? rem : g.block_elems);
+      h_grp[b0 + k] = scope == 0 ? t : 0u;
+      h_tens[b0 + k] = t;
+    }
+  }
+  h_tb0[g.n_tensors] = (uint32_t)nb;
+
+  size_t o = 0;
+  auto slot = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
+  const size_t o_off = slot(nb * 8), o_len = slot(nb * 4), o_grp = slot(nb * 4), o_tens = slot(nb * 4);
+  const size_t o_tb0 = slot(((size_t)g.n_tensors + 1) * 4);
+  const size_t o_norm = slot(U * 4), o_max = slot(U * 4), o_nnz = slot(U * 4), o_tau = slot(KG * 4);
+  const size_t o_err = slot(16);
+  const size_t o_work = slot(work_bytes);
+  mp_index_s* ix = new (std::nothrow) mp_index_s();
+  if (!ix) return fail(MP_ERR_OOM, "host allocation failed");
+  ix->magic = kMagicIndex;
+  ix->id = g_next_id++;
+  cudaGetDevice(&ix->device);
+  ix->g = g;
+  ix->op_kind = op ? (int)op->kind : -1;
+  ix->density = ties ? op->density : 0.0f;
+  ix->trim_scope = scope;
+  ix->n_groups = n_groups;
+  ix->has_missing = false;
+  ix->done = nullptr;
+  mp_status st;
+  if ((st = dev_alloc(ix->mem, o, cs)) != MP_OK) {
+    delete ix;
+    return st;
+  }
+  char* m = static_cast<char*>(ix->mem.ptr);
+  ix->d_blk_off = (uint64_t*)(m + o_off);
+  ix->d_blk_len = (uint32_t*)(m + o_len);
+  ix->d_blk_group = (uint32_t*)(m + o_grp);
+  ix->d_blk_tensor = (uint32_t*)(m + o_tens);
+  ix->d_t_blk0 = (uint32_t*)(m + o_tb0);
+  ix->d_norm = (float*)(m + o_norm);
+  ix->d_maxabs = (float*)(m + o_max);
+  ix->d_nnz = (uint32_t*)(m + o_nnz);
+  ix->d_tau = (uint32_t*)(m + o_tau);
+  ix->d_err = (uint32_t*)(m + o_err);
+  cudaError_t e = cudaSuccess;
+  const char* what = "block table copy";
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_off, h_off.data(), nb * 8, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_len, h_len.data(), nb * 4, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_group, h_grp.data(), nb * 4, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_tensor, h_tens.data(), nb * 4, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess)
+    e = cudaMemcpyAsync(ix->d_t_blk0, h_tb0.data(), ((size_t)g.n_tensors + 1) * 4, cudaMemcpyHostToDevice, cs);
+  if (e == cudaSuccess) what = "memset", e = cudaMemsetAsync(ix->d_err, 0, 16, cs);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_tau, 0, KG * 4, cs);
+  if (e != cudaSuccess) {
+    mp_status r = cuda_fail(e, what);
+    discard_index(ix, cs);
+    return r;
+  }
+  if (host_pool) {
+    ix->h_blk_off = std::move(h_off);
+    ix->h_blk_len = std::move(h_len);
+  }
+  *out = ix;
+  *work = m + o_work;
+  return MP_OK;
+}
+
+// the handle is complete once the stream reaches this point
+cudaError_t finish_index(mp_index_s* ix, cudaStream_t cs) {
+  cudaError_t e;
+  if ((e = cudaEventCreateWithFlags(&ix->done, cudaEventDisableTiming)) != cudaSuccess) return e;
+  return cudaEventRecord(ix->done, cs);
+}
+
+// frees a handle whose construction failed (after the stream's work on it is done)
+void discard_index(mp_index_s* ix, cudaStream_t cs) {
+  cudaStreamSynchronize(cs);
+  cudaGetLastError();
+  dev_free(ix->mem);
+  if (ix->done) cudaEventDestroy(ix->done);
+  delete ix;
+}
+
 }  // namespace mp
 
 using namespace mp;
@@ -442,32 +548,17 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
 
   const uint32_t scope = ties ? op->trim_scope : 0u;
   const uint32_t n_groups = scope == 0 ? g.n_tensors : 1u;
-  const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
-
-  std::vector<uint64_t> h_off(nb);
-  std::vector<uint32_t> h_len(nb), h_grp(nb);
+  const uint64_t KG = (uint64_t)g.K * n_groups;
   std::vector<unsigned long long> h_kth(n_groups, 0);
-  std::vector<uint64_t> gnumel(n_groups, 0);
-  for (uint32_t t = 0; t < g.n_tensors; ++t) {
-    uint64_t b0 = g.t_first_block[t];
-    uint64_t tb = (g.t_numel[t] + g.block_elems - 1) / g.block_elems;
-    for (uint64_t k = 0; k < tb; ++k) {
-      h_off[b0 + k] = g.t_off[t] + k * g.block_elems;
-      uint64_t rem = g.t_numel[t] - k * g.block_elems;
-      h_len[b0 + k] = (uint32_t)(rem < g.block_elems ? rem : g.block_elems);
-      h_grp[b0 + k] = scope == 0 ? t : 0u;
-    }
-    gnumel[scope == 0 ? t : 0] += g.t_numel[t];
-  }
-  if (ties)
+  if (ties) {
+    std::vector<uint64_t> gnumel(n_groups, 0);
+    for (uint32_t t = 0; t < g.n_tensors; ++t) gnumel[scope == 0 ? t : 0] += g.t_numel[t];
     for (uint32_t q = 0; q < n_groups; ++q)
       h_kth[q] = (unsigned long long)floor((double)op->density * (double)gnumel[q]);
-
+  }
+  // the index kernels' work space after the handle's own arrays
   size_t o = 0;
   auto slot = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
-  const size_t o_off = slot(nb * 8), o_len = slot(nb * 4), o_grp = slot(nb * 4);
-  const size_t o_norm = slot(U * 4), o_max = slot(U * 4), o_nnz = slot(U * 4), o_tau = slot(KG * 4);
-  const size_t o_err = slot(16);
   const size_t o_work = slot(16);  // the index kernel's work counter
   size_t o_coarse = 0, o_fine = 0, o_kth = 0, o_est = 0, o_rank = 0;
   if (ties) {
@@ -477,54 +568,21 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     o_est = slot(KG * 4);
     o_rank = slot(KG * 8);
   }
-  mp_index_s* ix = new (std::nothrow) mp_index_s();
-  if (!ix) return fail(MP_ERR_OOM, "host allocation failed");
-  ix->magic = kMagicIndex;
-  ix->id = g_next_id++;
-  cudaGetDevice(&ix->device);
-  ix->g = g;
-  ix->op_kind = op ? (int)op->kind : -1;
-  ix->density = ties ? op->density : 0.0f;
-  ix->trim_scope = scope;
-  ix->n_groups = n_groups;
-  ix->done = nullptr;
-  if ((st = dev_alloc(ix->mem, o, cs)) != MP_OK) {
-    delete ix;
-    return st;
-  }
-  char* m = static_cast<char*>(ix->mem.ptr);
-  ix->d_blk_off = (uint64_t*)(m + o_off);
-  ix->d_blk_len = (uint32_t*)(m + o_len);
-  ix->d_blk_group = (uint32_t*)(m + o_grp);
-  ix->d_norm = (float*)(m + o_norm);
-  ix->d_maxabs = (float*)(m + o_max);
-  ix->d_nnz = (uint32_t*)(m + o_nnz);
-  ix->d_tau = (uint32_t*)(m + o_tau);
-  ix->d_err = (uint32_t*)(m + o_err);
+  mp_index_s* ix = nullptr;
+  char* m = nullptr;
+  if ((st = new_index(g, op, family->experts_location != 0, o, cs, &ix, &m)) != MP_OK) return st;
 
   cudaError_t e;
   auto bail = [&](cudaError_t err, const char* what) {
     mp_status r = cuda_fail(err, what);
-    cudaStreamSynchronize(cs);
-    dev_free(ix->mem);
-    if (ix->done) cudaEventDestroy(ix->done);
-    delete ix;
+    discard_index(ix, cs);
     return r;
   };
-  if ((e = cudaMemcpyAsync(ix->d_blk_off, h_off.data(), nb * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
-    return bail(e, "block table copy");
-  if ((e = cudaMemcpyAsync(ix->d_blk_len, h_len.data(), nb * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
-    return bail(e, "block table copy");
-  if ((e = cudaMemcpyAsync(ix->d_blk_group, h_grp.data(), nb * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
-    return bail(e, "block table copy");
-  if ((e = cudaMemsetAsync(ix->d_err, 0, 16, cs)) != cudaSuccess) return bail(e, "memset");
-  if ((e = cudaMemsetAsync(ix->d_tau, 0, KG * 4, cs)) != cudaSuccess) return bail(e, "memset");
-
   IndexLaunch p;
   memset(&p, 0, sizeof(p));
   p.dtype = g.dtype;
   p.K = g.K;
-  p.n_blocks = nb;
+  p.n_blocks = g.n_blocks;
   p.n_groups = n_groups;
   p.base = base;
   p.experts = ex;
@@ -549,17 +607,74 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
       return bail(e, "k copy");
   }
   p.b_begin = 0;
-  p.b_end = nb;
+  p.b_end = g.n_blocks;
   p.expert_origin = 0;
   if (family->experts_location == 0) {
     if ((e = launch_index(p, cs)) != cudaSuccess) return bail(e, "index kernels");
   } else {
-    ix->h_blk_off = h_off;
-    ix->h_blk_len = h_len;
     if ((e = index_host_pool(p, ix, cs)) != cudaSuccess) return bail(e, "index (host pool)");
   }
-  if ((e = cudaEventCreateWithFlags(&ix->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
-  if ((e = cudaEventRecord(ix->done, cs)) != cudaSuccess) return bail(e, "event record");
+  if ((e = finish_index(ix, cs)) != cudaSuccess) return bail(e, "event");
+  *out = ix;
+  return MP_OK;
+}
+
+mp_status mp_index_import(const mp_family* family, const mp_op* op, const float* norm, const float* maxabs,
+                          const uint32_t* nnz, const uint32_t* tau, mp_stream stream, mp_index** out) {
+  if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
+  *out = nullptr;
+  Geometry g;
+  mp_status st = build_geometry(family, g);
+  if (st != MP_OK) return st;
+  const bool ties = op && op->kind == MP_OP_TIES;
+  if (op && (st = check_op(op, g.K)) != MP_OK) return st;
+  if (!norm || !maxabs || !nnz) return fail(MP_ERR_INVALID_ARG, "norm, maxabs and nnz are required");
+  if (ties && !tau) return fail(MP_ERR_INVALID_ARG, "a TIES catalog needs tau");
+  const uint32_t n_groups = (ties && op->trim_scope == 1) ? 1u : g.n_tensors;
+  const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
+  // every entry is either statistics of its block or marked missing
+  bool missing = false;
+  for (uint32_t t = 0; t < g.n_tensors; ++t) {
+    const uint64_t b0 = g.t_first_block[t], tb = (g.t_numel[t] + g.block_elems - 1) / g.block_elems;
+    for (uint64_t k = 0; k < tb; ++k) {
+      const uint64_t rem = g.t_numel[t] - k * g.block_elems;
+      const uint32_t len = (uint32_t)(rem < g.block_elems ? rem : g.block_elems);
+      for (uint32_t i = 0; i < g.K; ++i) {
+        const uint64_t q = (uint64_t)i * nb + b0 + k;
+        if (nnz[q] == MP_NNZ_MISSING) {
+          missing = true;
+          continue;
+        }
+        if (nnz[q] > len || !(norm[q] >= 0.0f && norm[q] <= FLT_MAX) || !(maxabs[q] >= 0.0f && maxabs[q] <= FLT_MAX))
+          return fail(MP_ERR_INVALID_ARG, "catalog entry " + std::to_string(q) +
+                                              " is not a block statistic (nnz above the block length, or a "
+                                              "negative or non-finite norm or maxabs)");
+      }
+    }
+  }
+  if (ties)
+    for (uint64_t q = 0; q < KG; ++q)
+      if (tau[q] > 0x8000u) return fail(MP_ERR_INVALID_ARG, "tau entries must be in [0, 0x8000]");
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  mp_index_s* ix = nullptr;
+  char* m = nullptr;
+  if ((st = new_index(g, op, family->experts_location != 0, 0, cs, &ix, &m)) != MP_OK) return st;
+  ix->has_missing = missing;
+  cudaError_t e;
+  auto bail = [&](cudaError_t err, const char* what) {
+    mp_status r = cuda_fail(err, what);
+    discard_index(ix, cs);
+    return r;
+  };
+  if ((e = cudaMemcpyAsync(ix->d_norm, norm, U * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "catalog copy");
+  if ((e = cudaMemcpyAsync(ix->d_maxabs, maxabs, U * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "catalog copy");
+  if ((e = cudaMemcpyAsync(ix->d_nnz, nnz, U * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "catalog copy");
+  if (ties && (e = cudaMemcpyAsync(ix->d_tau, tau, KG * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+    return bail(e, "catalog copy");
+  if ((e = finish_index(ix, cs)) != cudaSuccess) return bail(e, "event");
   *out = ix;
   return MP_OK;
 }
@@ -625,7 +740,8 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   };
   cudaError_t e;
   if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
-  if ((e = cudaMallocAsync(&scratch.ptr, plan_scratch_bytes(U), cs)) != cudaSuccess) {
+  const uint64_t n_pairs = index->has_missing ? (uint64_t)g.K * g.n_tensors : 0ull;
+  if ((e = cudaMallocAsync(&scratch.ptr, plan_scratch_bytes(U, n_pairs), cs)) != cudaSuccess) {
     scratch.ptr = nullptr;
     return bail(e, "plan scratch");
   }
@@ -647,6 +763,10 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   p.nnz = index->d_nnz;
   p.tau = index->d_tau;
   p.index_err = index->d_err;
+  p.fallback = index->has_missing ? 1u : 0u;
+  p.n_tensors = g.n_tensors;
+  p.blk_tensor = index->d_blk_tensor;
+  p.t_blk0 = index->d_t_blk0;
   p.budget = budget_bytes;
   p.mask = pl->d_mask;
   p.order = pl->d_order;
@@ -898,6 +1018,7 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
   if (order && s[2] && (e = cudaMemcpy(order, plan->d_order, s[2] * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail(e, "copy");
   if (s[6] & kErrNonfinite) return fail(MP_ERR_NONFINITE, "the index saw a NaN or infinite delta");
+  if (s[6] & kErrMissing) return fail(MP_ERR_UNSUPPORTED, "a catalog entry without statistics and no tensor map");
   if (s[6]) return fail(MP_ERR_TIMEOUT, "index kernels reported an error");
   if (s[0] > plan->budget) return fail(MP_ERR_BUDGET, "planned bytes exceed the budget");
   return MP_OK;

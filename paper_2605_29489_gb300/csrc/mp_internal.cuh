@@ -22,7 +22,9 @@ constexpr int kMaxK = 32;
 constexpr int kCounterSlots = 64;  // realized-byte counters are spread over slots
 
 // device error word bits
-enum : uint32_t { kErrNonfinite = 1u, kErrTimeout = 2u, kErrInternal = 4u };
+enum : uint32_t { kErrNonfinite = 1u, kErrTimeout = 2u, kErrInternal = 4u, kErrMissing = 8u };
+// nnz of a catalog entry without block statistics (no block holds 2^32 - 1 elements)
+constexpr uint32_t kNnzMissing = 0xFFFFFFFFu;
 
 struct ExpertPtrs {
   const void* p[kMaxK];
@@ -67,6 +69,9 @@ struct mp_index_s {
   uint64_t* d_blk_off;     // [n_blocks] element offset of each block
   uint32_t* d_blk_len;     // [n_blocks] elements of each block
   uint32_t* d_blk_group;   // [n_blocks] TIES trim group of each block
+  uint32_t* d_blk_tensor;  // [n_blocks] tensor of each block
+  uint32_t* d_t_blk0;      // [n_tensors + 1] first block of each tensor, then n_blocks
+  bool has_missing;        // some entry has nnz == kNnzMissing (imported catalogs only)
   float* d_norm;           // [K][n_blocks]
   float* d_maxabs;         // [K][n_blocks]
   uint32_t* d_nnz;         // [K][n_blocks]
@@ -173,6 +178,13 @@ struct PlanLaunch {
   const uint32_t* nnz;
   const uint32_t* tau;
   const uint32_t* index_err;
+  // tensor-level fallback: with fallback = 1, an (expert, tensor) pair holding an entry
+  // with nnz == kNnzMissing is planned as one unit (blk_tensor, t_blk0 as in mp_index_s);
+  // with fallback = 0 such an entry is reported (kErrMissing) and never read
+  uint32_t fallback;
+  uint32_t n_tensors;
+  const uint32_t* blk_tensor;
+  const uint32_t* t_blk0;
   uint64_t budget;
   uint32_t* mask;
   uint32_t* order;
@@ -181,8 +193,9 @@ struct PlanLaunch {
   uint8_t hdr_prefix[256];
   uint32_t hdr_prefix_len;
 };
-// scratch bytes plan_run needs for n_units units
-size_t plan_scratch_bytes(uint64_t n_units);
+// scratch bytes the planner needs for n_units units and n_pairs (expert, tensor) pairs
+// (n_pairs = 0 without the tensor-level fallback)
+size_t plan_scratch_bytes(uint64_t n_units, uint64_t n_pairs);
 cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st);
 
 // ---- merge (merge.cu) -------------------------------------------------------------------

@@ -4,6 +4,11 @@
 // below together, separated by grid barriers whose waits are bounded.  Every phase
 // gives CTA c a contiguous slice of the data, so order is preserved wherever it matters.
 //
+//  0  tensor-level fallback (only for catalogs with entries lacking statistics, nnz =
+//     kNnzMissing): flag every (expert, tensor) pair holding one; then one warp per flagged
+//     pair computes its unit's cost (the whole tensor's bytes) and score (|coef_i| times
+//     the norm of the tensor's known blocks: an fp32 fma chain in block order, then sqrt).
+//     The pair's unit is b0(t)*K + i; the tensor's other units are not candidates.
 //  A  score: unit u = b*K + i is a candidate iff nnz > 0 (TIES: and key(maxabs) >= tau);
 //     score = |coef_i| * norm (fp32), divided by the block's bytes in the score-per-byte
 //     mode; sort key = ~bits(score), so ascending key order is
@@ -17,8 +22,9 @@
 //  E  after that first overflow only candidates with cost <= the remaining budget R0 can
 //     ever be taken (R only shrinks): they are compacted, then one warp of CTA 0 runs the
 //     greedy with skip over them in order, from shared memory.
-//  F  the mask, the set hash and the count are scattered from the selected positions;
-//     the last CTA counts touched blocks and computes the digest.
+//  F  the mask, the set hash and the count are scattered from the selected positions
+//     (a fallback unit sets its expert's bit on every block of the tensor); the last CTA
+//     counts touched blocks and computes the digest.
 #include "mp_internal.cuh"
 
 namespace mp {
@@ -32,7 +38,8 @@ constexpr uint32_t kBarrierLimit = 1u << 24;
 // summary words (plan handle)
 enum { S_CHAT = 0, S_NSEL = 1, S_NCAND = 2, S_SETHASH = 3, S_DIGEST = 4, S_TOUCHED = 5, S_ERR = 6 };
 // scratch scalars
-enum { X_BAR_COUNT = 0, X_BAR_GEN = 1, X_P = 2, X_PBP = 3, X_TAILSUM = 4, X_DONE = 5, X_TOTAL = 6, X_COUNT = 8 };
+enum { X_BAR_COUNT = 0, X_BAR_GEN = 1, X_P = 2, X_PBP = 3, X_TAILSUM = 4, X_DONE = 5, X_TOTAL = 6, X_MISSING = 7,
+       X_COUNT = 8 };
 
 constexpr unsigned long long kNoP = ~0ull;
 
@@ -47,11 +54,14 @@ struct Scratch {
   unsigned long long* cta_a;    // [kMaxGrid]
   unsigned long long* cta_b;    // [kMaxGrid]
   unsigned long long* x;        // [X_COUNT]
+  uint32_t* pair_flag;          // [K * n_tensors] (fallback only; cleared by the host)
+  uint32_t* pair_key;           // [K * n_tensors]
+  unsigned long long* pair_cost;  // [K * n_tensors]
 };
 
 inline size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
 
-size_t carve(void* base, uint64_t U, Scratch* s) {
+size_t carve(void* base, uint64_t U, uint64_t n_pairs, Scratch* s) {
   char* p = static_cast<char*>(base);
   size_t o = 0;
   auto take = [&](size_t bytes) { char* r = p + o; o += align_up(bytes); return r; };
@@ -66,6 +76,9 @@ size_t carve(void* base, uint64_t U, Scratch* s) {
   t.cta_a = (unsigned long long*)take(kMaxGrid * 8);
   t.cta_b = (unsigned long long*)take(kMaxGrid * 8);
   t.x = (unsigned long long*)take(X_COUNT * 8);
+  t.pair_flag = (uint32_t*)take(n_pairs * 4);
+  t.pair_key = (uint32_t*)take(n_pairs * 4);
+  t.pair_cost = (unsigned long long*)take(n_pairs * 8);
   if (s) *s = t;
   return o;
 }
@@ -169,11 +182,17 @@ struct Unit {
   uint32_t key;
 };
 
-__device__ __forceinline__ Unit score_unit(const PlanLaunch& p, uint64_t u) {
+__device__ __forceinline__ Unit score_unit(const PlanLaunch& p, const Scratch& s, uint64_t u) {
   const uint64_t b = u / p.K;
   const uint32_t i = (uint32_t)(u % p.K);
   const uint64_t st = (uint64_t)i * p.n_blocks + b;
-  bool cand = p.nnz[st] != 0u;
+  if (p.fallback) {
+    const uint32_t t = p.blk_tensor[b];
+    const uint32_t pr = i * p.n_tensors + t;
+    if (s.pair_flag[pr]) return Unit{b == p.t_blk0[t], s.pair_key[pr]};
+  }
+  const uint32_t nz = p.nnz[st];
+  bool cand = nz != 0u && nz != kNnzMissing;
   if (cand && p.op_kind == MP_OP_TIES)
     cand = ties_key(p.maxabs[st]) >= p.tau[(uint64_t)i * p.n_groups + p.blk_group[b]];
   float score = __fmul_rn(p.coef[i], p.norm[st]);
@@ -182,8 +201,47 @@ __device__ __forceinline__ Unit score_unit(const PlanLaunch& p, uint64_t u) {
   return Unit{cand, ~__float_as_uint(score)};
 }
 
-__device__ __forceinline__ unsigned long long unit_cost(const PlanLaunch& p, uint32_t u) {
-  return (unsigned long long)p.blk_len[u / p.K] * p.elem_size;
+__device__ __forceinline__ unsigned long long unit_cost(const PlanLaunch& p, const Scratch& s, uint32_t u) {
+  const uint32_t b = u / p.K;
+  if (p.fallback) {
+    const uint32_t pr = (u % p.K) * p.n_tensors + p.blk_tensor[b];
+    if (s.pair_flag[pr]) return s.pair_cost[pr];
+  }
+  return (unsigned long long)p.blk_len[b] * p.elem_size;
+}
+
+// phase 0b for one flagged pair (i, t), by one warp: cost = the tensor's bytes, key from
+// |coef_i| * sqrt(ss), ss the fp32 chain fma(n, n, ss) over the known blocks in block order
+__device__ __forceinline__ void fallback_pair(const PlanLaunch& p, const Scratch& s, uint32_t pr, uint32_t lane) {
+  const uint32_t i = pr / p.n_tensors, t = pr % p.n_tensors;
+  const uint32_t b0 = p.t_blk0[t], b1 = p.t_blk0[t + 1];
+  const float* nrm = p.norm + (uint64_t)i * p.n_blocks;
+  const uint32_t* nz = p.nnz + (uint64_t)i * p.n_blocks;
+  float ss = 0.0f;
+  unsigned long long cost = 0;
+  for (uint32_t bb = b0; bb < b1; bb += 32) {
+    const uint32_t b = bb + lane;
+    float n = 0.0f;
+    int known = 0;
+    if (b < b1) {
+      n = nrm[b];
+      known = nz[b] != kNnzMissing;
+      cost += (unsigned long long)p.blk_len[b] * p.elem_size;
+    }
+    const uint32_t m = b1 - bb < 32u ? b1 - bb : 32u;  // uniform over the warp
+    for (uint32_t j = 0; j < m; ++j) {
+      const float nj = __shfl_sync(0xFFFFFFFFu, n, j);
+      if (__shfl_sync(0xFFFFFFFFu, known, j)) ss = __fmaf_rn(nj, nj, ss);
+    }
+  }
+#pragma unroll
+  for (int sh = 16; sh > 0; sh >>= 1) cost += __shfl_xor_sync(0xFFFFFFFFu, cost, sh);
+  float score = __fmul_rn(p.coef[i], __fsqrt_rn(ss));
+  if (p.score_mode) score = __fdiv_rn(score, __ull2float_rn(cost));
+  if (lane == 0) {
+    s.pair_key[pr] = ~__float_as_uint(score);
+    s.pair_cost[pr] = cost;
+  }
 }
 
 __device__ __forceinline__ void slice(uint64_t n, uint64_t& a, uint64_t& b) {
@@ -194,7 +252,7 @@ __device__ __forceinline__ void slice(uint64_t n, uint64_t& a, uint64_t& b) {
 __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s) {
   __shared__ uint32_t s_run[256];
   __shared__ uint32_t s_wcnt[kPT / 32][256];
-  __shared__ uint32_t s_cost[kTailChunk];
+  __shared__ unsigned long long s_cost[kTailChunk];
   __shared__ unsigned long long s_bcast[1];
   const uint32_t tid = threadIdx.x, lane = tid & 31u, warp = tid >> 5;
   const uint32_t G = gridDim.x, c = blockIdx.x;
@@ -208,9 +266,30 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   if (c == 0 && tid == 0) s.x[X_P] = kNoP;
   uint64_t u0, u1;
   slice(U, u0, u1);
+  if (p.fallback) {
+    // 0a: flag the pairs holding an entry without statistics
+    for (uint64_t u = u0 + tid; u < u1; u += kPT) {
+      const uint64_t b = u / p.K;
+      const uint32_t i = (uint32_t)(u % p.K);
+      if (p.nnz[(uint64_t)i * p.n_blocks + b] == kNnzMissing)
+        atomicOr(&s.pair_flag[i * p.n_tensors + p.blk_tensor[b]], 1u);
+    }
+    if (!grid_sync(s.x, gen, p.summary)) return;
+    // 0b: the flagged pairs' units, one warp each
+    const uint32_t n_pairs = p.K * p.n_tensors, nw = G * (kPT / 32);
+    for (uint32_t pr = c * (kPT / 32) + warp; pr < n_pairs; pr += nw)
+      if (s.pair_flag[pr]) fallback_pair(p, s, pr, lane);
+    if (!grid_sync(s.x, gen, p.summary)) return;
+  }
   {
+    // without the fallback an entry lacking statistics cannot be planned: it is reported
     unsigned long long cnt = 0;
-    for (uint64_t u = u0 + tid; u < u1; u += kPT) cnt += score_unit(p, u).cand ? 1ull : 0ull;
+    bool miss = false;
+    for (uint64_t u = u0 + tid; u < u1; u += kPT) {
+      cnt += score_unit(p, s, u).cand ? 1ull : 0ull;
+      miss |= !p.fallback && p.nnz[(u % p.K) * p.n_blocks + u / p.K] == kNnzMissing;
+    }
+    if (__syncthreads_or(miss) && tid == 0) s.x[X_MISSING] = 1ull;
     cnt = block_sum<unsigned long long>(cnt);
     if (tid == 0) s.cta_a[c] = cnt;
   }
@@ -224,7 +303,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     unsigned long long run = before;
     for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
       const uint64_t u = t0 + tid;
-      Unit x = u < u1 ? score_unit(p, u) : Unit{false, 0u};
+      Unit x = u < u1 ? score_unit(p, s, u) : Unit{false, 0u};
       uint32_t tot;
       const uint32_t pos = block_scan<uint32_t>(x.cand ? 1u : 0u, tot);
       if (x.cand) {
@@ -320,7 +399,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   // ---- D: cost prefix in sorted order; the first position where it exceeds B ----
   {
     unsigned long long sum = 0;
-    for (uint64_t j = q0 + tid; j < q1; j += kPT) sum += unit_cost(p, order[j]);
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) sum += unit_cost(p, s, order[j]);
     sum = block_sum<unsigned long long>(sum);
     if (tid == 0) s.cta_b[c] = sum;
   }
@@ -331,7 +410,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     if (c == 0 && tid == 0) s.x[X_TOTAL] = total_cost;
     for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
       const uint64_t j = t0 + tid;
-      const unsigned long long cj = j < q1 ? unit_cost(p, order[j]) : 0ull;
+      const unsigned long long cj = j < q1 ? unit_cost(p, s, order[j]) : 0ull;
       unsigned long long tot;
       const unsigned long long before = run + block_scan<unsigned long long>(cj, tot);
       if (j < q1 && before + cj > p.budget && before <= p.budget) {  // unique: prefixes only grow
@@ -349,7 +428,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   if (P != kNoP) {
     {
       unsigned long long cnt = 0;
-      for (uint64_t j = q0 + tid; j < q1; j += kPT) cnt += (j > P && unit_cost(p, order[j]) <= R0) ? 1ull : 0ull;
+      for (uint64_t j = q0 + tid; j < q1; j += kPT) cnt += (j > P && unit_cost(p, s, order[j]) <= R0) ? 1ull : 0ull;
       cnt = block_sum<unsigned long long>(cnt);
       if (tid == 0) s.cta_a[c] = cnt;
     }
@@ -359,7 +438,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
       unsigned long long run = block_sum_prefix(s.cta_a, c);
       for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
         const uint64_t j = t0 + tid;
-        const bool f = j < q1 && j > P && unit_cost(p, order[j]) <= R0;
+        const bool f = j < q1 && j > P && unit_cost(p, s, order[j]) <= R0;
         uint32_t tot;
         const uint32_t pos = block_scan<uint32_t>(f ? 1u : 0u, tot);
         if (f) s.tail_pos[run + pos] = (uint32_t)j;
@@ -372,7 +451,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
       unsigned long long R = R0;
       for (unsigned long long k0 = 0; k0 < L; k0 += kTailChunk) {
         const uint32_t n = (uint32_t)min((unsigned long long)kTailChunk, L - k0);
-        for (uint32_t k = tid; k < n; k += kPT) s_cost[k] = (uint32_t)unit_cost(p, order[s.tail_pos[k0 + k]]);
+        for (uint32_t k = tid; k < n; k += kPT) s_cost[k] = unit_cost(p, s, order[s.tail_pos[k0 + k]]);
         __syncthreads();
         if (warp == 0) {
           for (uint32_t b0 = 0; b0 < n; b0 += 32) {
@@ -404,7 +483,13 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     for (uint64_t j = q0 + tid; j < q1; j += kPT) {
       if ((P == kNoP || j < P) || s.tailsel[j]) {
         const uint32_t u = order[j];
-        atomicOr(&p.mask[u / p.K], 1u << (u % p.K));
+        const uint32_t b = u / p.K, i = u % p.K;
+        const uint32_t t = p.fallback ? p.blk_tensor[b] : 0u;
+        if (p.fallback && s.pair_flag[i * p.n_tensors + t]) {
+          for (uint32_t bb = b; bb < p.t_blk0[t + 1]; ++bb) atomicOr(&p.mask[bb], 1u << i);
+        } else {
+          atomicOr(&p.mask[b], 1u << i);
+        }
         h += splitmix64(u);
         ++n;
       }
@@ -451,18 +536,20 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   sum[S_CHAT] = chat;
   sum[S_NCAND] = Q;
   sum[S_DIGEST] = h;
-  sum[S_ERR] = sum[S_ERR] | (unsigned long long)*p.index_err;
+  sum[S_ERR] = sum[S_ERR] | (unsigned long long)*p.index_err | (s.x[X_MISSING] ? (unsigned long long)kErrMissing : 0ull);
 }
 
 }  // namespace
 
-size_t plan_scratch_bytes(uint64_t n_units) { return carve(nullptr, n_units, nullptr); }
+size_t plan_scratch_bytes(uint64_t n_units, uint64_t n_pairs) { return carve(nullptr, n_units, n_pairs, nullptr); }
 
 cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st) {
   const uint64_t U = (uint64_t)p.K * p.n_blocks;
   if (U > 0xFFFFFFFFull) return cudaErrorInvalidValue;
+  const uint64_t n_pairs = p.fallback ? (uint64_t)p.K * p.n_tensors : 0ull;
+  if (p.fallback && (!p.blk_tensor || !p.t_blk0 || n_pairs == 0)) return cudaErrorInvalidValue;
   Scratch s;
-  carve(scratch, U, &s);
+  carve(scratch, U, n_pairs, &s);
   int dev = 0, sms = 0, per_sm = 0;
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
@@ -476,6 +563,7 @@ cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st) {
   if (grid > kMaxGrid) grid = kMaxGrid;
   if (grid < 1) grid = 1;
   if ((e = cudaMemsetAsync(s.x, 0, X_COUNT * sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if (n_pairs && (e = cudaMemsetAsync(s.pair_flag, 0, n_pairs * 4, st)) != cudaSuccess) return e;
   PlanLaunch pc = p;
   void* args[] = {&pc, &s};
   if ((e = cudaLaunchCooperativeKernel((const void*)plan_kernel, dim3((unsigned)grid), dim3(kPT), args, 0, st)) !=

@@ -78,7 +78,7 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   if (n_blocks == 0 || n_groups == 0) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: empty geometry");
   if (dtype != MP_BF16 && dtype != MP_F32) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: bad dtype");
   const uint64_t U = (uint64_t)K * n_blocks;
-  if (U > kNoAllocMaxUnits || mp::plan_scratch_bytes(U) > kNoAllocScratchBytes)
+  if (U > kNoAllocMaxUnits || mp::plan_scratch_bytes(U, 0) > kNoAllocScratchBytes)
     return fail_static(MP_ERR_INVALID_ARG,
                        "mp_plan_noalloc: K * n_blocks exceeds the static scratch limit of 524288 units");
   if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_DARE_TIES)

@@ -64,3 +64,32 @@ def test_budget_from_fraction_host_only():
     assert mp.mp_budget_from_fraction(fam, 0.1) == int(np.floor(0.1 * full))
     assert mp.mp_budget_from_fraction(fam, 0.0) == 0
     assert mp.mp_budget_from_fraction(fam, 2.0) == full
+
+
+def test_index_import_refuses_bad_entries_before_any_device_work():
+    """mp_index_import checks every entry on the host: an nnz above the block's length, a
+    negative norm, or a TIES catalog without tau is refused before any CUDA call"""
+    import numpy as np
+    import paper_2605_29489_gb300 as mp
+
+    base = np.zeros(4096 + 300, np.uint16)
+    experts = [np.zeros_like(base) for _ in range(2)]
+    fam = mp.family([(0, 4096), (4096, 300)], base, experts, block_elems=1024, dtype=mp.MP_BF16, experts_location=0)
+    K, nb = 2, 5
+    norm = np.ones((K, nb), np.float32)
+    maxabs = np.ones((K, nb), np.float32)
+    nnz = np.full((K, nb), 3, np.uint32)
+    op = mp.make_op(mp.MP_OP_TA, alpha=[0.5, 0.5])
+    bad = nnz.copy()
+    bad[1, 4] = 301                      # the last block holds 300 elements
+    with pytest.raises(mp.MergePipeError) as e:
+        mp.mp_index_import(fam, op, norm, maxabs, bad, stream=0)
+    assert e.value.status == -1
+    neg = norm.copy()
+    neg[0, 1] = -0.5
+    with pytest.raises(mp.MergePipeError) as e:
+        mp.mp_index_import(fam, op, neg, maxabs, nnz, stream=0)
+    assert e.value.status == -1
+    with pytest.raises(mp.MergePipeError) as e:
+        mp.mp_index_import(fam, mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2), norm, maxabs, nnz, None, stream=0)
+    assert e.value.status == -1
