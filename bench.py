@@ -74,6 +74,12 @@ def workloads():
                                         budgets=[1.0, 0.5, 0.25, 0.1], touched=True,
                                         desc="as qwen2.5-0.5b-ta, merged with mp_merge_touched: only touched blocks "
                                              "are read and written (Alg. 2 WriteBlockOrReference)"),
+        "llama-3-8b-ta-fallback": dict(make=lambda: synth.llama3_8b(), op="ta", lam=0.3,
+                                       budgets=[1.0, 0.5, 0.25, 0.1], fallback=True,
+                                       desc="Llama-3-8B-shaped bf16 family, K=4, TA lambda=0.3, planned from an "
+                                            "imported catalog without statistics for 10 % of the (expert, tensor) "
+                                            "pairs (the embedding of expert 0 among them) and 0.1 % of the other "
+                                            "entries: tensor-level fallback plan (Sec. 3 Planner)"),
         "tiny-avg": dict(make=lambda: synth.tiny(), op="avg", budgets=[1.0, 0.5, 0.25],
                          desc="8 fp32 512x512 tensors, K=4, AVG, 4Ki-element blocks"),
     }
@@ -106,6 +112,20 @@ def make_ops(w, K):
         return (mp.make_op(mp.MP_OP_DARE_TIES, lam=1.0, drop_p=w["drop_p"], seed=20260),
                 oracle.Op(oracle.DARE_TIES, K, lam=1.0, drop_p=w["drop_p"], seed=20260))
     raise ValueError(w["op"])
+
+
+def fallback_missing(fam, K):
+    """the seeded pattern of catalog entries without statistics of the fallback workloads:
+    every entry of 10 % of the (expert, tensor) pairs (always the largest tensor of expert 0)
+    and 0.1 % of the other entries; bool [K, n_blocks]"""
+    import numpy as np
+
+    _, _, bt = fam.block_table()
+    rng = np.random.default_rng(2605)
+    n_t = int(bt.max()) + 1
+    pairs = rng.random((K, n_t)) < 0.10
+    pairs[0, int(np.argmax(np.bincount(bt)))] = True
+    return pairs[:, bt] | (rng.random((K, bt.size)) < 0.001)
 
 
 # ---- clocks ---------------------------------------------------------------------------------------
@@ -213,6 +233,7 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
     _, oop = make_ops(w, fam.K)
     bo, bl, bt = fam.block_table()
     budgets = w["budgets"]
+    miss_all = fallback_missing(fam, fam.K) if w.get("fallback") else None
 
     def run(blocks):
         data = [fam.block_host(int(b)) for b in blocks]
@@ -228,12 +249,21 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
         of = oracle.Family(fam.dtype, offs, lens, groups, 1, base, experts)
         es = fam.elem_size
         full = fam.K * int(lens.sum()) * es
+        if miss_all is not None:
+            # the catalog is imported, not computed: build it before the clock starts
+            norm, maxabs, nnz = oracle.index(of)
+            nnz = nnz.copy()
+            nnz[miss_all[:, blocks]] = oracle.NNZ_MISSING
+            tmap = np.unique(bt[blocks], return_inverse=True)[1].astype(np.uint32)
         t0 = time.perf_counter()
-        norm, maxabs, nnz = oracle.index(of)
+        if miss_all is None:
+            norm, maxabs, nnz = oracle.index(of)
+            tmap = None
         tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
         for f in budgets:
-            pl = oracle.plan(fam.K, lens, groups, 1, es, oop, norm, maxabs, nnz, tau, math.floor(f * full))
-            oracle.merge(of, oop, tau=tau, mask=pl["mask"])
+            pl = oracle.plan(fam.K, lens, groups, 1, es, oop, norm, maxabs, nnz, tau, math.floor(f * full),
+                             blk_tensor=tmap)
+            oracle.merge(of, oop, tau=tau, mask=pl["mask"], nnz=nnz if tmap is not None else None)
         dt = time.perf_counter() - t0
         return dt, int(lens.sum())
 
@@ -244,8 +274,9 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
     n = max(1, min(nb, int(target_s / max(dt1 / len(probe), 1e-6))))
     blocks = sorted(set(int(x) for x in np.linspace(0, nb - 1, n)))
     dt, params = run(blocks)
+    first = "catalog imported (computed before timing)" if miss_all is not None else "oracle index"
     desc = (f"{len(blocks)} of {nb} blocks ({params} params) evenly spaced over the family, regenerated on the "
-            f"host; oracle index + plan and merge at budgets {budgets} (budget relative to the sample)")
+            f"host; {first} + plan and merge at budgets {budgets} (budget relative to the sample)")
     return len(budgets) * params / dt, dt, desc
 
 
@@ -298,12 +329,25 @@ def native(args, rank, world, local_rank):
     stream = torch.cuda.current_stream()
     touched_mode = bool(W.get("touched"))
     merge_fn = mp.mp_merge_touched if touched_mode else mp.mp_merge
+    catalog = None
+    if W.get("fallback"):
+        # a catalog saved earlier, with entries lacking statistics; each step imports it
+        idx0 = mp.mp_index_blocks(mf, gop)
+        c_norm, c_max, c_nnz, c_tau = mp.mp_index_stats(idx0)
+        idx0.free()
+        c_nnz[fallback_missing(fam, fam.K)] = mp.MP_NNZ_MISSING
+        catalog = (c_norm, c_max, c_nnz, c_tau if gop.kind == mp.MP_OP_TIES else None)
+
+    def make_index(fam_c):
+        if catalog is not None:
+            return mp.mp_index_import(fam_c, gop, *catalog, stream=stream)
+        return mp.mp_index_blocks(fam_c, gop, stream)
 
     def step(fam_c, ev=None):
         hs = []
         if ev is not None:
             ev["i0"].record(stream)
-        idx = mp.mp_index_blocks(fam_c, gop, stream)
+        idx = make_index(fam_c)
         hs.append(idx)
         if ev is not None:
             ev["i1"].record(stream)
@@ -405,7 +449,7 @@ def native(args, rank, world, local_rank):
             for d, h in zip(experts_d, experts_h):
                 d.copy_(h, non_blocking=True)
             hs = []
-            idx = mp.mp_index_blocks(mf_d, gop, stream)
+            idx = make_index(mf_d)
             hs.append(idx)
             stream.wait_stream(copy_stream)  # the previous step's copies have read the outputs
             for k, B in enumerate(Bs):
@@ -457,7 +501,7 @@ def native(args, rank, world, local_rank):
         "config": {"workload": args.workload, "description": W["desc"], "params": N, "K": fam.K,
                    "blocks": fam.n_blocks, "block_elems": fam.block_elems, "budgets": budgets,
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (no flush)",
-                   "step": "index + (plan + merge) per budget"},
+                   "step": ("catalog import" if catalog is not None else "index") + " + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
         "index_ms": idx_ms, "per_budget": per_budget,
         "roofline": {"bound": "hbm", "kernel": "merge_tma_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
@@ -476,6 +520,14 @@ def native(args, rank, world, local_rank):
         "clocks": clk,
         "e2e": e2e,
     }
+    if catalog is not None:
+        miss = catalog[2] == mp.MP_NNZ_MISSING
+        bt = np.asarray(fam.block_table()[2])
+        pairs = np.zeros((fam.K, int(bt.max()) + 1), bool)
+        for i in range(fam.K):
+            pairs[i, np.unique(bt[miss[i]])] = True
+        line["config"]["catalog"] = {"entries_missing": int(miss.sum()), "entries": int(miss.size),
+                                     "fallback_pairs": int(pairs.sum()), "pairs": int(pairs.size)}
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
         v, dt, desc = oracle_sample_run(W, fam, args.cpu_seconds)
         model, ncpu = cpu_info()

@@ -23,8 +23,9 @@
 //     ever be taken (R only shrinks): they are compacted, then one warp of CTA 0 runs the
 //     greedy with skip over them in order, from shared memory.
 //  F  the mask, the set hash and the count are scattered from the selected positions
-//     (a fallback unit sets its expert's bit on every block of the tensor); the last CTA
-//     counts touched blocks and computes the digest.
+//     (a taken fallback unit sets its expert's bit in a per-tensor word, which the
+//     touched-block pass ORs into every block of the tensor); the last CTA computes the
+//     digest.
 #include "mp_internal.cuh"
 
 namespace mp {
@@ -39,7 +40,7 @@ constexpr uint32_t kBarrierLimit = 1u << 24;
 enum { S_CHAT = 0, S_NSEL = 1, S_NCAND = 2, S_SETHASH = 3, S_DIGEST = 4, S_TOUCHED = 5, S_ERR = 6 };
 // scratch scalars
 enum { X_BAR_COUNT = 0, X_BAR_GEN = 1, X_P = 2, X_PBP = 3, X_TAILSUM = 4, X_DONE = 5, X_TOTAL = 6, X_MISSING = 7,
-       X_COUNT = 8 };
+       X_TAILMIN = 8, X_COUNT = 16 };
 
 constexpr unsigned long long kNoP = ~0ull;
 
@@ -48,6 +49,7 @@ struct Scratch {
   uint32_t* keys_b;             // [U]
   uint32_t* vals_b;             // [U]
   uint32_t* tail_pos;           // [U]
+  unsigned long long* tail_cost;  // [U] costs of the compacted tail, in order
   uint8_t* tailsel;             // [U]
   uint32_t* hist;               // [256][kMaxGrid]
   uint32_t* tot;                // [256]
@@ -57,6 +59,7 @@ struct Scratch {
   uint32_t* pair_flag;          // [K * n_tensors] (fallback only; cleared by the host)
   uint32_t* pair_key;           // [K * n_tensors]
   unsigned long long* pair_cost;  // [K * n_tensors]
+  uint32_t* sel_bits;           // [n_tensors] experts whose fallback unit of the tensor was taken (cleared by the host)
 };
 
 inline size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
@@ -70,6 +73,7 @@ size_t carve(void* base, uint64_t U, uint64_t n_pairs, Scratch* s) {
   t.keys_b = (uint32_t*)take(U * 4);
   t.vals_b = (uint32_t*)take(U * 4);
   t.tail_pos = (uint32_t*)take(U * 4);
+  t.tail_cost = (unsigned long long*)take(U * 8);
   t.tailsel = (uint8_t*)take(U);
   t.hist = (uint32_t*)take((size_t)256 * kMaxGrid * 4);
   t.tot = (uint32_t*)take(256 * 4);
@@ -79,6 +83,7 @@ size_t carve(void* base, uint64_t U, uint64_t n_pairs, Scratch* s) {
   t.pair_flag = (uint32_t*)take(n_pairs * 4);
   t.pair_key = (uint32_t*)take(n_pairs * 4);
   t.pair_cost = (unsigned long long*)take(n_pairs * 8);
+  t.sel_bits = (uint32_t*)take(n_pairs * 4);  // n_tensors words used (n_pairs >= n_tensors)
   if (s) *s = t;
   return o;
 }
@@ -211,7 +216,11 @@ __device__ __forceinline__ unsigned long long unit_cost(const PlanLaunch& p, con
 }
 
 // phase 0b for one flagged pair (i, t), by one warp: cost = the tensor's bytes, key from
-// |coef_i| * sqrt(ss), ss the fp32 chain fma(n, n, ss) over the known blocks in block order
+// |coef_i| * sqrt(ss), ss the fp32 chain fma(n, n, ss) over the known blocks in block order.
+// The lanes load a batch of kFbChunks chunks of 32 consecutive entries at once (one load
+// latency per batch); every lane then runs the same chain over them in block order.
+constexpr int kFbChunks = 8;
+
 __device__ __forceinline__ void fallback_pair(const PlanLaunch& p, const Scratch& s, uint32_t pr, uint32_t lane) {
   const uint32_t i = pr / p.n_tensors, t = pr % p.n_tensors;
   const uint32_t b0 = p.t_blk0[t], b1 = p.t_blk0[t + 1];
@@ -219,19 +228,29 @@ __device__ __forceinline__ void fallback_pair(const PlanLaunch& p, const Scratch
   const uint32_t* nz = p.nnz + (uint64_t)i * p.n_blocks;
   float ss = 0.0f;
   unsigned long long cost = 0;
-  for (uint32_t bb = b0; bb < b1; bb += 32) {
-    const uint32_t b = bb + lane;
-    float n = 0.0f;
-    int known = 0;
-    if (b < b1) {
-      n = nrm[b];
-      known = nz[b] != kNnzMissing;
-      cost += (unsigned long long)p.blk_len[b] * p.elem_size;
+  for (uint32_t bb = b0; bb < b1; bb += 32u * kFbChunks) {
+    float n[kFbChunks];
+    bool known[kFbChunks];
+#pragma unroll
+    for (int c = 0; c < kFbChunks; ++c) {
+      const uint32_t b = bb + 32u * c + lane;
+      n[c] = 0.0f;
+      known[c] = false;
+      if (b < b1) {
+        n[c] = __ldg(nrm + b);
+        known[c] = __ldg(nz + b) != kNnzMissing;
+        cost += (unsigned long long)__ldg(p.blk_len + b) * p.elem_size;
+      }
     }
-    const uint32_t m = b1 - bb < 32u ? b1 - bb : 32u;  // uniform over the warp
-    for (uint32_t j = 0; j < m; ++j) {
-      const float nj = __shfl_sync(0xFFFFFFFFu, n, j);
-      if (__shfl_sync(0xFFFFFFFFu, known, j)) ss = __fmaf_rn(nj, nj, ss);
+#pragma unroll
+    for (int c = 0; c < kFbChunks; ++c) {
+      // an entry without statistics adds fma(0, 0, ss) = ss exactly (ss >= +0)
+      const float nv = known[c] ? n[c] : 0.0f;
+#pragma unroll
+      for (int j = 0; j < 32; ++j) {
+        const float nj = __shfl_sync(0xFFFFFFFFu, nv, j);
+        ss = __fmaf_rn(nj, nj, ss);
+      }
     }
   }
 #pragma unroll
@@ -263,16 +282,24 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   for (uint64_t k = (uint64_t)c * kPT + tid; k < p.n_blocks; k += (uint64_t)G * kPT) p.mask[k] = 0u;
   for (uint64_t k = (uint64_t)c * kPT + tid; k < U; k += (uint64_t)G * kPT) s.tailsel[k] = 0;
   if (c == 0 && tid < 8) p.summary[tid] = 0;
-  if (c == 0 && tid == 0) s.x[X_P] = kNoP;
+  if (c == 0 && tid == 0) {
+    s.x[X_P] = kNoP;
+    s.x[X_TAILMIN] = ~0ull;
+  }
   uint64_t u0, u1;
   slice(U, u0, u1);
   if (p.fallback) {
-    // 0a: flag the pairs holding an entry without statistics
-    for (uint64_t u = u0 + tid; u < u1; u += kPT) {
-      const uint64_t b = u / p.K;
-      const uint32_t i = (uint32_t)(u % p.K);
-      if (p.nnz[(uint64_t)i * p.n_blocks + b] == kNnzMissing)
-        atomicOr(&s.pair_flag[i * p.n_tensors + p.blk_tensor[b]], 1u);
+    // 0a: flag the pairs holding an entry without statistics (one atomic per pair and warp)
+    for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
+      const uint64_t u = t0 + tid;
+      uint32_t pr = 0xFFFFFFFFu;
+      if (u < u1) {
+        const uint64_t b = u / p.K;
+        const uint32_t i = (uint32_t)(u % p.K);
+        if (p.nnz[(uint64_t)i * p.n_blocks + b] == kNnzMissing) pr = i * p.n_tensors + p.blk_tensor[b];
+      }
+      const uint32_t peers = __match_any_sync(0xFFFFFFFFu, pr);
+      if (pr != 0xFFFFFFFFu && lane == (uint32_t)(__ffs(peers) - 1)) atomicOr(&s.pair_flag[pr], 1u);
     }
     if (!grid_sync(s.x, gen, p.summary)) return;
     // 0b: the flagged pairs' units, one warp each
@@ -436,25 +463,39 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     const unsigned long long L = block_sum_prefix(s.cta_a, G);
     {
       unsigned long long run = block_sum_prefix(s.cta_a, c);
+      unsigned long long cmin = ~0ull;
       for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
         const uint64_t j = t0 + tid;
-        const bool f = j < q1 && j > P && unit_cost(p, s, order[j]) <= R0;
+        const unsigned long long cj = j < q1 ? unit_cost(p, s, order[j]) : ~0ull;
+        const bool f = j < q1 && j > P && cj <= R0;
         uint32_t tot;
         const uint32_t pos = block_scan<uint32_t>(f ? 1u : 0u, tot);
-        if (f) s.tail_pos[run + pos] = (uint32_t)j;
+        if (f) {
+          s.tail_pos[run + pos] = (uint32_t)j;
+          s.tail_cost[run + pos] = cj;
+          cmin = cj < cmin ? cj : cmin;
+        }
         run += tot;
       }
+#pragma unroll
+      for (int sh = 16; sh > 0; sh >>= 1) {
+        const unsigned long long o = __shfl_xor_sync(0xFFFFFFFFu, cmin, sh);
+        cmin = o < cmin ? o : cmin;
+      }
+      if (lane == 0 && cmin != ~0ull) atomicMin(&s.x[X_TAILMIN], cmin);
     }
     if (!grid_sync(s.x, gen, p.summary)) return;
     if (c == 0) {
-      // greedy with skip over the compacted tail, in order, from shared memory
+      // greedy with skip over the compacted tail, in order, from shared memory; once R is
+      // below the smallest tail cost nothing more can be taken
+      const unsigned long long cmin = __ldcg(&s.x[X_TAILMIN]);
       unsigned long long R = R0;
-      for (unsigned long long k0 = 0; k0 < L; k0 += kTailChunk) {
+      for (unsigned long long k0 = 0; k0 < L && R >= cmin; k0 += kTailChunk) {
         const uint32_t n = (uint32_t)min((unsigned long long)kTailChunk, L - k0);
-        for (uint32_t k = tid; k < n; k += kPT) s_cost[k] = unit_cost(p, s, order[s.tail_pos[k0 + k]]);
+        for (uint32_t k = tid; k < n; k += kPT) s_cost[k] = __ldcg(s.tail_cost + k0 + k);
         __syncthreads();
         if (warp == 0) {
-          for (uint32_t b0 = 0; b0 < n; b0 += 32) {
+          for (uint32_t b0 = 0; b0 < n && R >= cmin; b0 += 32) {
             const uint32_t k = b0 + lane;
             const unsigned long long ck = k < n ? s_cost[k] : ~0ull;
             uint32_t done = 0u;
@@ -486,7 +527,7 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
         const uint32_t b = u / p.K, i = u % p.K;
         const uint32_t t = p.fallback ? p.blk_tensor[b] : 0u;
         if (p.fallback && s.pair_flag[i * p.n_tensors + t]) {
-          for (uint32_t bb = b; bb < p.t_blk0[t + 1]; ++bb) atomicOr(&p.mask[bb], 1u << i);
+          atomicOr(&s.sel_bits[t], 1u << i);  // every block of t gets bit i in the next pass
         } else {
           atomicOr(&p.mask[b], 1u << i);
         }
@@ -506,7 +547,17 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     uint64_t b0, b1;
     slice(p.n_blocks, b0, b1);
     unsigned long long t = 0;
-    for (uint64_t b = b0 + tid; b < b1; b += kPT) t += p.mask[b] != 0u ? 1ull : 0ull;
+    for (uint64_t b = b0 + tid; b < b1; b += kPT) {
+      uint32_t m = p.mask[b];
+      if (p.fallback) {
+        const uint32_t sb = __ldcg(s.sel_bits + p.blk_tensor[b]);
+        if (sb) {
+          m |= sb;
+          p.mask[b] = m;  // one thread per block in this pass
+        }
+      }
+      t += m != 0u ? 1ull : 0ull;
+    }
     t = block_sum<unsigned long long>(t);
     __shared__ bool last;
     if (tid == 0) {
@@ -564,6 +615,7 @@ cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st) {
   if (grid < 1) grid = 1;
   if ((e = cudaMemsetAsync(s.x, 0, X_COUNT * sizeof(unsigned long long), st)) != cudaSuccess) return e;
   if (n_pairs && (e = cudaMemsetAsync(s.pair_flag, 0, n_pairs * 4, st)) != cudaSuccess) return e;
+  if (n_pairs && (e = cudaMemsetAsync(s.sel_bits, 0, (size_t)p.n_tensors * 4, st)) != cudaSuccess) return e;
   PlanLaunch pc = p;
   void* args[] = {&pc, &s};
   if ((e = cudaLaunchCooperativeKernel((const void*)plan_kernel, dim3((unsigned)grid), dim3(kPT), args, 0, st)) !=
