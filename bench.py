@@ -428,6 +428,7 @@ def native(args, rank, world, local_rank):
                   hbm_frac_nominal=ab / s / 1e9 / NOMINAL_HBM_GBS)
     merge_total_s = sum(merge_ms) / 1e3
     achieved = sum(alg_bytes) / merge_total_s / 1e9
+    t_model = time_model_fit(budgets, per_budget, N * es, fam.K * N * es, peak, touched_mode) if not host_pool else None
 
     # ---- e2e: pinned host inputs in, merged outputs back, inside the timed region ----
     e2e = None
@@ -503,7 +504,7 @@ def native(args, rank, world, local_rank):
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (no flush)",
                    "step": ("catalog import" if catalog is not None else "index") + " + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
-        "index_ms": idx_ms, "per_budget": per_budget,
+        "index_ms": idx_ms, "per_budget": per_budget, "time_model": t_model,
         "roofline": {"bound": "hbm", "kernel": "merge_tma_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
@@ -534,6 +535,30 @@ def native(args, rank, world, local_rank):
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
                                 "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
     return line
+
+
+def time_model_fit(budgets, per_budget, ckpt_bytes, c_full, peak_gbs, touched_mode):
+    """The merge time against the affine model T(f) = (2 N s + f C_full) / BW: a least-squares
+    line through the measured (planned fraction, merge ms) points, next to the model's slope
+    C_full / BW and intercept 2 N s / BW at the measured copy bandwidth."""
+    if len(budgets) < 2:
+        return None
+    x = [pb["planned_bytes"] / c_full for pb in per_budget]
+    y = [pb["merge_ms"] for pb in per_budget]
+    n = len(x)
+    mx, my = sum(x) / n, sum(y) / n
+    sxx = sum((a - mx) ** 2 for a in x)
+    if sxx <= 0:
+        return None
+    slope = sum((a - mx) * (b - my) for a, b in zip(x, y)) / sxx
+    icpt = my - slope * mx
+    res = [b - (icpt + slope * a) for a, b in zip(x, y)]
+    ss_tot = sum((b - my) ** 2 for b in y)
+    r2 = 1.0 - sum(r * r for r in res) / ss_tot if ss_tot > 0 else 1.0
+    return {"x": "planned expert bytes / C_full", "slope_ms": slope, "intercept_ms": icpt, "r2": r2,
+            "model_slope_ms": c_full / (peak_gbs * 1e9) * 1e3,
+            "model_intercept_ms": None if touched_mode else 2 * ckpt_bytes / (peak_gbs * 1e9) * 1e3,
+            "bw_from_slope_gbs": c_full / (slope / 1e3) / 1e9 if slope > 0 else None}
 
 
 def fidelity_vs_full(fam, budgets, outs, shared_out, per_budget):
