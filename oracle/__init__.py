@@ -63,6 +63,10 @@ def lib():
         L.orc_fnv1a64.argtypes = [vp, ctypes.c_size_t]
         L.orc_splitmix64.restype = u64
         L.orc_splitmix64.argtypes = [u64]
+        for nm in ("orc_block_hash", "orc_block_hash_sum"):
+            getattr(L, nm).restype = u64
+            getattr(L, nm).argtypes = [vp, u64]
+        L.orc_index_hashes.argtypes = [vp, vp, vp]
         _lib = L
     return _lib
 
@@ -258,6 +262,27 @@ def fnv1a64(data: bytes) -> int:
 
 def splitmix64(state: int) -> int:
     return int(lib().orc_splitmix64(state & 0xFFFFFFFFFFFFFFFF))
+
+
+def block_hash(data: bytes) -> int:
+    """the catalog's content hash of one block's bytes"""
+    buf = ctypes.create_string_buffer(bytes(data), max(1, len(data)))
+    return int(lib().orc_block_hash(ctypes.cast(buf, ctypes.c_void_p), len(data)))
+
+
+def block_hash_sum(data: bytes) -> int:
+    """the multilinear sum H of the block hash (before the final mix)"""
+    buf = ctypes.create_string_buffer(bytes(data), max(1, len(data)))
+    return int(lib().orc_block_hash_sum(ctypes.cast(buf, ctypes.c_void_p), len(data)))
+
+
+def index_hashes(fam: Family):
+    """(base_hash [n_blocks], expert_hash [K, n_blocks]) uint64"""
+    bh = np.zeros(fam.n_blocks, np.uint64)
+    eh = np.zeros((fam.K, fam.n_blocks), np.uint64)
+    c = fam.c()
+    _check(lib().orc_index_hashes(ctypes.byref(c), _p(bh), _p(eh)))
+    return bh, eh
 
 
 def f32_bits(x: float) -> int:

@@ -229,6 +229,56 @@ uint64_t orc_splitmix64(uint64_t state) {
 }
 
 /* ---------------------------------------------------------------------------------------
+ * Block content hash (Sec. 3 "Catalog": the catalog stores hashes of every block; Alg. 2
+ * validates hashes before the manifest is built).  The paper names no function.  Reading:
+ * the block's L bytes, zero-padded to a multiple of 16, are vectors q = 0, 1, ... of two
+ * little-endian 64-bit words (lo_q, hi_q); with k_q = SplitMix64(q), a_q = k_q | 1 and
+ * b_q = rotl(k_q, 32) | 1,
+ *     H = sum_q (lo_q * a_q + hi_q * b_q)  mod 2^64,      hash = SplitMix64(H xor L).
+ * q counts from the block's start, so equal blocks hash equal wherever they sit.  A
+ * multilinear sum with odd keys: any change of a single word changes H (odd keys are units
+ * mod 2^64), and the sum can be formed in any order.  It detects changed or corrupted
+ * blocks; it is not a cryptographic hash.
+ * Pins: every single-word change is detected (including a change by 2^63); swapping two
+ * different vectors or the two words of a vector changes the hash; H is additive over
+ * blocks with disjoint support; the length is part of the hash; the GPU catalog matches.
+ * ------------------------------------------------------------------------------------- */
+static uint64_t rd_le64(const uint8_t* p) {
+  uint64_t v = 0;
+  for (int k = 7; k >= 0; --k) v = (v << 8) | p[k];
+  return v;
+}
+
+uint64_t orc_block_hash_sum(const void* bytes, uint64_t len) {
+  const uint8_t* src = (const uint8_t*)bytes;
+  uint64_t H = 0;
+  for (uint64_t q = 0; q * 16 < len; ++q) {
+    uint8_t v[16] = {0};
+    const uint64_t m = len - q * 16 < 16 ? len - q * 16 : 16;
+    memcpy(v, src + q * 16, (size_t)m);
+    const uint64_t k = orc_splitmix64(q);
+    const uint64_t a = k | 1u, b = ((k << 32) | (k >> 32)) | 1u;
+    H += rd_le64(v) * a + rd_le64(v + 8) * b;
+  }
+  return H;
+}
+
+uint64_t orc_block_hash(const void* bytes, uint64_t len) { return orc_splitmix64(orc_block_hash_sum(bytes, len) ^ len); }
+
+/* the catalog's hashes of a family: base_hash[b], expert_hash[i * n_blocks + b] */
+int orc_index_hashes(const orc_family* f, uint64_t* base_hash, uint64_t* expert_hash) {
+  if (!f || !base_hash || !expert_hash) return ORC_EINVAL;
+  const uint64_t es = f->dtype == ORC_BF16 ? 2u : 4u;
+  for (uint64_t b = 0; b < f->n_blocks; ++b) {
+    const uint64_t len = (uint64_t)f->blk_len[b] * es;
+    base_hash[b] = orc_block_hash(elem_ptr(f->dtype, f->base, f->blk_off[b]), len);
+    for (uint32_t i = 0; i < f->K; ++i)
+      expert_hash[(uint64_t)i * f->n_blocks + b] = orc_block_hash(elem_ptr(f->dtype, f->experts[i], f->blk_off[b]), len);
+  }
+  return ORC_OK;
+}
+
+/* ---------------------------------------------------------------------------------------
  * Alg. 1 PlanGen (Sec. 3), cost model Eq. 3 and App. A.1.
  *  - Candidates Q: units (i, b) whose delta can change the output.  Reading: a unit
  *    with nnz = 0 contributes exactly nothing to any operator, and under TIES a unit

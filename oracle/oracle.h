@@ -92,6 +92,11 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p);
 uint64_t orc_fnv1a64(const uint8_t* data, size_t n);
 uint64_t orc_splitmix64(uint64_t state);
 
+/* block content hash (catalog hashes; Alg. 2 validation): the multilinear sum H and the hash */
+uint64_t orc_block_hash_sum(const void* bytes, uint64_t len);
+uint64_t orc_block_hash(const void* bytes, uint64_t len);
+int orc_index_hashes(const orc_family* f, uint64_t* base_hash, uint64_t* expert_hash);
+
 #ifdef __cplusplus
 }
 #endif

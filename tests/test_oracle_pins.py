@@ -809,3 +809,79 @@ def test_fallback_plan_at_full_budget_merges_like_the_full_read(tiny_family):
         got = oracle.merge(of, op, mask=p["mask"], nnz=nnz)
         want = oracle.merge(of, op)
         assert np.array_equal(got.view(np.uint32), want.view(np.uint32))
+
+
+# ---- block content hash (catalog hashes; Alg. 2 validates them) -------------------------------------------
+
+M64 = 2 ** 64
+
+
+def _words_to_bytes(words):
+    return np.asarray(words, np.uint64).tobytes()
+
+
+def test_block_hash_detects_every_single_word_change():
+    """odd keys are units mod 2^64: changing any one 64-bit word by any nonzero amount
+    (including 2^63, which an even key would annihilate) changes the hash"""
+    rng = np.random.default_rng(41)
+    words = rng.integers(0, 2 ** 63, 64, dtype=np.uint64) * np.uint64(2) + np.uint64(1)
+    h0 = oracle.block_hash(_words_to_bytes(words))
+    for j in range(words.size):
+        for d in (1, 2 ** 63, int(rng.integers(1, 2 ** 62))):
+            w = words.copy()
+            w[j] = np.uint64((int(w[j]) + d) % M64)
+            assert oracle.block_hash(_words_to_bytes(w)) != h0, (j, d)
+
+
+def test_block_hash_depends_on_position_and_word_order():
+    rng = np.random.default_rng(42)
+    words = rng.integers(0, 2 ** 63, 32, dtype=np.uint64)
+    h0 = oracle.block_hash(_words_to_bytes(words))
+    sw = words.copy()
+    sw[[0, 1, 2, 3]] = sw[[2, 3, 0, 1]]           # swap vectors 0 and 1
+    assert oracle.block_hash(_words_to_bytes(sw)) != h0
+    hl = words.copy()
+    hl[[4, 5]] = hl[[5, 4]]                       # swap the two words of vector 2
+    assert oracle.block_hash(_words_to_bytes(hl)) != h0
+
+
+def test_block_hash_sum_is_additive_over_disjoint_support():
+    """H is a sum of per-word terms, so blocks with disjoint nonzero words add (mod 2^64),
+    and an all-zero block has H = 0 (its hash is SplitMix64 of the length alone)"""
+    rng = np.random.default_rng(43)
+    for n_words in (2, 6, 64, 2 * 257):
+        a = rng.integers(0, 2 ** 63, n_words, dtype=np.uint64)
+        pick = rng.random(n_words) < 0.5
+        x = np.where(pick, a, 0).astype(np.uint64)
+        y = np.where(pick, 0, a).astype(np.uint64)
+        hx, hy, ha = (oracle.block_hash_sum(_words_to_bytes(v)) for v in (x, y, a))
+        assert (hx + hy) % M64 == ha
+        assert oracle.block_hash_sum(bytes(8 * n_words)) == 0
+        assert oracle.block_hash(bytes(8 * n_words)) == oracle.splitmix64(8 * n_words)
+
+
+def test_block_hash_pads_to_vectors_and_mixes_the_length():
+    """a ragged block is hashed as if zero-padded to 16 bytes (same H), but the length is
+    mixed in, so the padded and unpadded blocks differ"""
+    data = bytes(range(1, 23))                    # 22 bytes: one full vector and 6 bytes
+    padded = data + bytes(10)
+    assert oracle.block_hash_sum(data) == oracle.block_hash_sum(padded)
+    assert oracle.block_hash(data) != oracle.block_hash(padded)
+
+
+def test_index_hashes_are_content_addressed(tiny_family):
+    """the catalog's hash of a block depends on its bytes only: an expert block equal to the
+    base block has the base's hash, and every block matches hashing its bytes directly"""
+    fam, base, experts = tiny_family
+    e0 = experts[0].copy()
+    bo, bl, _ = fam.block_table()
+    s0 = slice(int(bo[1]), int(bo[1] + bl[1]))
+    e0[s0] = base[s0]
+    of = oracle_family(fam, base, [e0] + list(experts[1:]))
+    bh, eh = oracle.index_hashes(of)
+    assert eh[0, 1] == bh[1]
+    for b in (0, 1, fam.n_blocks - 1):
+        s = slice(int(bo[b]), int(bo[b] + bl[b]))
+        assert bh[b] == oracle.block_hash(base[s].tobytes())
+        assert eh[1, b] == oracle.block_hash(experts[1][s].tobytes())
+    assert len(set(bh.tolist())) > fam.n_blocks // 2
