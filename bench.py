@@ -411,6 +411,9 @@ def native(args, rank, world, local_rank):
                                touched_ratio=pi["chat"] / (fam.K * N * es), plan_ms=plan_ms[k], merge_ms=merge_ms[k]))
         if touched_mode:
             per_budget[-1]["touched_elements"] = int(np.asarray(blk_len)[np.asarray(pi["mask"]) != 0].sum())
+    hashes = None
+    if not host_pool and not args.no_hash:
+        hashes = time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream)
     for hs in handles:
         for h in hs:
             h.free()
@@ -504,7 +507,7 @@ def native(args, rank, world, local_rank):
                    "parallelism": f"replicas x{world}", "l2": "inputs larger than L2 (no flush)",
                    "step": ("catalog import" if catalog is not None else "index") + " + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
-        "index_ms": idx_ms, "per_budget": per_budget, "time_model": t_model,
+        "index_ms": idx_ms, "per_budget": per_budget, "time_model": t_model, "block_hashes": hashes,
         "roofline": {"bound": "hbm", "kernel": "merge_tma_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
@@ -535,6 +538,43 @@ def native(args, rank, world, local_rank):
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
                                 "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
     return line
+
+
+def time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream, reps=3):
+    """The catalog's block hashes (one pass over the K + 1 checkpoints) and Alg. 2's hash
+    validation of the last budget's merge (base + selected expert blocks + output), timed
+    with CUDA events after the timed region; not part of the step."""
+    import torch
+
+    idx, k = last[0], len(per_budget) - 1
+    plan, man = last[1 + 2 * k], last[2 + 2 * k]
+    out = outs[0 if shared_out else k]
+    es, N = fam.elem_size, fam.n_params
+    E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    mp.mp_index_hashes(mf, idx, stream)
+    mp.mp_manifest_validate(mf, idx, plan, out, man, stream)
+    torch.cuda.synchronize()
+    t_cat, t_val = [], []
+    for _ in range(reps):
+        a, b, c = E(), E(), E()
+        a.record(stream)
+        mp.mp_index_hashes(mf, idx, stream)
+        b.record(stream)
+        mp.mp_manifest_validate(mf, idx, plan, out, man, stream)
+        c.record(stream)
+        torch.cuda.synchronize()
+        t_cat.append(a.elapsed_time(b))
+        t_val.append(b.elapsed_time(c))
+    v = mp.mp_manifest_validation(man, fam.n_blocks)
+    peak, _ = hbm_peak()
+    cat_bytes = (fam.K + 1) * N * es
+    val_bytes = 2 * N * es + per_budget[k]["planned_bytes"]
+    cat_ms, val_ms = statistics.median(t_cat), statistics.median(t_val)
+    return {"catalog_ms": cat_ms, "catalog_bytes": cat_bytes, "catalog_gbs": cat_bytes / cat_ms / 1e6,
+            "catalog_frac": cat_bytes / cat_ms / 1e6 / peak, "validate_f": per_budget[k]["f"],
+            "validate_ms": val_ms, "validate_bytes": val_bytes, "validate_gbs": val_bytes / val_ms / 1e6,
+            "validate_frac": val_bytes / val_ms / 1e6 / peak, "blocks_checked": v["checked"],
+            "mismatched": v["mismatched"]}
 
 
 def time_model_fit(budgets, per_budget, ckpt_bytes, c_full, peak_gbs, touched_mode):
@@ -750,6 +790,7 @@ def main():
     ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads().keys()))
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-hash", action="store_true", help="skip timing the block-hash passes")
     ap.add_argument("--cpu-seconds", type=float, default=15.0)
     ap.add_argument("--k-sweep", action="store_true",
                     help="K-scaling at a fixed absolute budget (Cor. 1) instead of the workload sweep")

@@ -144,14 +144,35 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
  * ignored): mp_plan then plans every (expert, tensor) pair holding such an entry at tensor
  * granularity (Sec. 3 "Planner", the deterministic tensor-level fallback; see mp_plan).
  * Every other entry must be a block statistic: nnz <= the block's elements, norm and
- * maxabs finite and >= 0; tau entries in [0, 0x8000].  The arrays are copied before the
- * call returns; the family's buffers are not read here (only its geometry), but must be
- * the ones the statistics describe when the index is used to merge.  The renormalised
- * AVG treats a delta as known to be zero only where nnz = 0.
+ * maxabs finite and >= 0; tau entries in [0, 0x8000].  base_hash [n_blocks] and
+ * expert_hash [K][n_blocks] (host, optional, both or neither) are the catalog's block
+ * hashes as mp_index_hash_values returns them.  The arrays are copied before the call
+ * returns; the family's buffers are not read here (only its geometry), but must be the
+ * ones the statistics describe when the index is used to merge.  The renormalised AVG
+ * treats a delta as known to be zero only where nnz = 0.
  * Errors: MP_ERR_INVALID_ARG (bad family, op or entry), MP_ERR_OOM, MP_ERR_CUDA.
  */
 mp_status mp_index_import(const mp_family* family, const mp_op* op, const float* norm, const float* maxabs,
-                          const uint32_t* nnz, const uint32_t* tau, mp_stream stream, mp_index** out);
+                          const uint32_t* nnz, const uint32_t* tau, const uint64_t* base_hash,
+                          const uint64_t* expert_hash, mp_stream stream, mp_index** out);
+
+/*
+ * mp_index_hashes — the catalog's block content hashes (Sec. 3 "Catalog" stores hashes of
+ * every block; Alg. 2 validates them).  For the base and every expert, each block's bytes
+ * (L of them, zero-padded to 16-byte vectors q of two little-endian 64-bit words lo_q,
+ * hi_q) hash to SplitMix64(H xor L), H = sum_q lo_q * (k_q | 1) + hi_q * (rotl(k_q, 32) | 1)
+ * mod 2^64 with k_q = SplitMix64(q) counted from the block's start: equal blocks hash
+ * equal, and any change of one 64-bit word changes the hash (not a cryptographic hash).
+ * One pass over (K + 1) N s bytes, enqueued on stream after the index's own work; the
+ * hashes are stored in the index.  family must be the index's family (same geometry).
+ * Errors: MP_ERR_INVALID_ARG, MP_ERR_MISMATCH, MP_ERR_OOM, MP_ERR_CUDA.
+ */
+mp_status mp_index_hashes(const mp_family* family, mp_index* index, mp_stream stream);
+
+/* Host copies of the catalog's block hashes: base_hash [n_blocks], expert_hash [K][n_blocks]
+   (either may be NULL).  Waits for the index work.  MP_ERR_INVALID_ARG if the index holds
+   no hashes. */
+mp_status mp_index_hash_values(const mp_index* index, uint64_t* base_hash, uint64_t* expert_hash);
 
 /*
  * mp_plan — Alg. 1 PlanGen under budget B (bytes of expert reads, Eq. 3; cost of unit
@@ -270,6 +291,28 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
    MP_ERR_BUDGET if realized reads exceed the planned bytes. */
 mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_bytes_per_expert,
                            uint64_t* realized_total, uint64_t* touched_blocks, uint64_t* digest);
+
+/*
+ * mp_manifest_validate — Alg. 2's hash validation before the manifest is final: after the
+ * merge recorded in man (stream-ordered after it), hash every base block, every expert
+ * block the plan selected (exactly the blocks the merge read) and every block of out (the
+ * buffer the merge wrote), with the function of mp_index_hashes.  The inputs are compared
+ * with the catalog's hashes, which detects a base or expert buffer changed since the index
+ * was built; the output's hashes are recorded in the manifest (a merged checkpoint can be
+ * checked against them later).  Reads N s + C_hat + N s bytes.  index must hold hashes.
+ * Errors: MP_ERR_UNSUPPORTED (no catalog hashes), MP_ERR_MISMATCH (handles or geometry do
+ * not belong together), MP_ERR_INVALID_ARG, MP_ERR_OOM, MP_ERR_CUDA.  Mismatches are
+ * reported by mp_manifest_validation.
+ */
+mp_status mp_manifest_validate(const mp_family* family, const mp_index* index, const mp_plan_t* plan, const void* out,
+                               mp_stream stream, mp_manifest* man);
+
+/* Results of mp_manifest_validate (waits for it): blocks checked against the catalog,
+   mismatches, and out_hash [n_blocks] the merged output's block hashes (any pointer may be
+   NULL).  Returns MP_ERR_MISMATCH when a block read by the merge differs from the catalog
+   (the message names the first one), MP_ERR_INVALID_ARG if the manifest was not
+   validated. */
+mp_status mp_manifest_validation(const mp_manifest* man, uint64_t* checked, uint64_t* mismatched, uint64_t* out_hash);
 
 /* The manifest's lineage (Sec. 3: the manifest records lineage): the K + 1 caller ids of
    M_0..M_K given in mp_family.lineage_ids at merge time, copied into ids[0..K] (all zero

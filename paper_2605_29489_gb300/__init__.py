@@ -24,7 +24,8 @@ __all__ = [
     "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_manifest_lineage", "mp_budget_from_fraction", "mp_last_error",
-    "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "lib",
+    "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "mp_index_hashes",
+    "mp_index_hash_values", "mp_manifest_validate", "mp_manifest_validation", "lib",
     "library_path",
 ]
 
@@ -75,7 +76,11 @@ def lib():
         vp, u64, st = ctypes.c_void_p, ctypes.c_uint64, ctypes.c_int32
         for name, args in [
             ("mp_index_blocks", [vp, vp, vp, vp]),
-            ("mp_index_import", [vp, vp, vp, vp, vp, vp, vp, vp]),
+            ("mp_index_import", [vp, vp, vp, vp, vp, vp, vp, vp, vp, vp]),
+            ("mp_index_hashes", [vp, vp, vp]),
+            ("mp_index_hash_values", [vp, vp, vp]),
+            ("mp_manifest_validate", [vp, vp, vp, vp, vp, vp]),
+            ("mp_manifest_validation", [vp, vp, vp, vp]),
             ("mp_plan", [vp, vp, u64, vp, vp]),
             ("mp_merge", [vp, vp, vp, vp, vp, vp]),
             ("mp_merge_touched", [vp, vp, vp, vp, vp, vp]),
@@ -197,16 +202,52 @@ def mp_index_blocks(fam: Family, op: Op | None = None, stream=None) -> Handle:
     return Handle(out.value, "index")
 
 
-def mp_index_import(fam: Family, op: Op | None, norm, maxabs, nnz, tau=None, stream=None) -> Handle:
-    """a catalog from saved statistics (host arrays [K, n_blocks], tau [K, n_groups] for TIES);
-    entries with nnz == MP_NNZ_MISSING have no statistics"""
+def mp_index_import(fam: Family, op: Op | None, norm, maxabs, nnz, tau=None, stream=None, base_hash=None,
+                    expert_hash=None) -> Handle:
+    """a catalog from saved statistics (host arrays [K, n_blocks], tau [K, n_groups] for TIES,
+    optional block hashes [n_blocks] and [K, n_blocks]); entries with nnz == MP_NNZ_MISSING
+    have no statistics"""
     arrs = [np.ascontiguousarray(norm, np.float32), np.ascontiguousarray(maxabs, np.float32),
-            np.ascontiguousarray(nnz, np.uint32), None if tau is None else np.ascontiguousarray(tau, np.uint32)]
+            np.ascontiguousarray(nnz, np.uint32), None if tau is None else np.ascontiguousarray(tau, np.uint32),
+            None if base_hash is None else np.ascontiguousarray(base_hash, np.uint64),
+            None if expert_hash is None else np.ascontiguousarray(expert_hash, np.uint64)]
     out = ctypes.c_void_p()
     _check(lib().mp_index_import(fam.ref(), None if op is None else op.ref(),
                                  *[None if a is None else a.ctypes.data for a in arrs],
                                  ctypes.c_void_p(_stream_ptr(stream)), ctypes.byref(out)))
     return Handle(out.value, "index")
+
+
+def mp_index_hashes(fam: Family, index: Handle, stream=None):
+    """add the catalog's block content hashes to an index (one pass over every checkpoint)"""
+    _check(lib().mp_index_hashes(fam.ref(), ctypes.c_void_p(index.ptr), ctypes.c_void_p(_stream_ptr(stream))))
+
+
+def mp_index_hash_values(index: Handle):
+    """(base_hash [n_blocks], expert_hash [K, n_blocks]) uint64"""
+    nb, nu, _ = mp_index_shape(index)
+    bh = np.zeros(nb, np.uint64)
+    eh = np.zeros((nu // nb, nb), np.uint64)
+    _check(lib().mp_index_hash_values(ctypes.c_void_p(index.ptr), bh.ctypes.data, eh.ctypes.data))
+    return bh, eh
+
+
+def mp_manifest_validate(fam: Family, index: Handle, plan: Handle, out, man: Handle, stream=None):
+    """Alg. 2's hash validation of the blocks a merge read, and the output's block hashes"""
+    _check(lib().mp_manifest_validate(fam.ref(), ctypes.c_void_p(index.ptr), ctypes.c_void_p(plan.ptr),
+                                      ctypes.c_void_p(_ptr(out)), ctypes.c_void_p(_stream_ptr(stream)),
+                                      ctypes.c_void_p(man.ptr)))
+
+
+def mp_manifest_validation(man: Handle, n_blocks: int, check: bool = True):
+    """dict(checked, mismatched, out_hash, status) of mp_manifest_validate"""
+    c, m = ctypes.c_uint64(), ctypes.c_uint64()
+    oh = np.zeros(n_blocks, np.uint64)
+    rc = lib().mp_manifest_validation(ctypes.c_void_p(man.ptr), ctypes.byref(c), ctypes.byref(m), oh.ctypes.data)
+    if check:
+        _check(rc)
+    return dict(checked=c.value, mismatched=m.value, out_hash=oh, status=rc,
+                error=mp_last_error() if rc != MP_OK else "")
 
 
 def mp_plan(index: Handle, op: Op, budget_bytes: int, stream=None) -> Handle:

@@ -223,6 +223,7 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
                     mp_index_s** out, char** work);
 cudaError_t finish_index(mp_index_s* ix, cudaStream_t cs);
 void discard_index(mp_index_s* ix, cudaStream_t cs);
+mp_status alloc_hashes(mp_index_s* ix, cudaStream_t cs);
 
 // ---- experts in pinned host memory: segment pipeline -------------------------------------
 //
@@ -503,10 +504,22 @@ cudaError_t finish_index(mp_index_s* ix, cudaStream_t cs) {
   return cudaEventRecord(ix->done, cs);
 }
 
+// the catalog's hash arrays (base, then K experts), allocated once per index
+mp_status alloc_hashes(mp_index_s* ix, cudaStream_t cs) {
+  if (ix->hash_mem.ptr) return MP_OK;
+  const uint64_t nb = ix->g.n_blocks;
+  mp_status st = dev_alloc(ix->hash_mem, (size_t)(ix->g.K + 1) * nb * 8, cs);
+  if (st != MP_OK) return st;
+  ix->d_base_hash = static_cast<unsigned long long*>(ix->hash_mem.ptr);
+  ix->d_expert_hash = ix->d_base_hash + nb;
+  return MP_OK;
+}
+
 // frees a handle whose construction failed (after the stream's work on it is done)
 void discard_index(mp_index_s* ix, cudaStream_t cs) {
   cudaStreamSynchronize(cs);
   cudaGetLastError();
+  dev_free(ix->hash_mem);
   dev_free(ix->mem);
   if (ix->done) cudaEventDestroy(ix->done);
   delete ix;
@@ -620,7 +633,8 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
 }
 
 mp_status mp_index_import(const mp_family* family, const mp_op* op, const float* norm, const float* maxabs,
-                          const uint32_t* nnz, const uint32_t* tau, mp_stream stream, mp_index** out) {
+                          const uint32_t* nnz, const uint32_t* tau, const uint64_t* base_hash,
+                          const uint64_t* expert_hash, mp_stream stream, mp_index** out) {
   if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
   Geometry g;
@@ -630,6 +644,8 @@ mp_status mp_index_import(const mp_family* family, const mp_op* op, const float*
   if (op && (st = check_op(op, g.K)) != MP_OK) return st;
   if (!norm || !maxabs || !nnz) return fail(MP_ERR_INVALID_ARG, "norm, maxabs and nnz are required");
   if (ties && !tau) return fail(MP_ERR_INVALID_ARG, "a TIES catalog needs tau");
+  if ((base_hash == nullptr) != (expert_hash == nullptr))
+    return fail(MP_ERR_INVALID_ARG, "block hashes come as base_hash and expert_hash together");
   const uint32_t n_groups = (ties && op->trim_scope == 1) ? 1u : g.n_tensors;
   const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
   // every entry is either statistics of its block or marked missing
@@ -674,6 +690,16 @@ mp_status mp_index_import(const mp_family* family, const mp_op* op, const float*
     return bail(e, "catalog copy");
   if (ties && (e = cudaMemcpyAsync(ix->d_tau, tau, KG * 4, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
     return bail(e, "catalog copy");
+  if (base_hash) {
+    if ((st = alloc_hashes(ix, cs)) != MP_OK) {
+      discard_index(ix, cs);
+      return st;
+    }
+    if ((e = cudaMemcpyAsync(ix->d_base_hash, base_hash, nb * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+      return bail(e, "hash copy");
+    if ((e = cudaMemcpyAsync(ix->d_expert_hash, expert_hash, U * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+      return bail(e, "hash copy");
+  }
   if ((e = finish_index(ix, cs)) != cudaSuccess) return bail(e, "event");
   *out = ix;
   return MP_OK;
@@ -843,7 +869,9 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   mf->plan_id = plan->id;
   mf->device = plan->device;
   mf->K = g.K;
+  mf->n_blocks = g.n_blocks;
   mf->done = nullptr;
+  mf->valid_done = nullptr;
   for (uint32_t i = 0; i <= kMaxK; ++i) mf->lineage[i] = (family->lineage_ids && i <= g.K) ? family->lineage_ids[i] : 0u;
   const size_t counters_bytes = (size_t)kCounterSlots * g.K * 8;
   // the counters (64 slots x K), the plan summary and the error word come back in one copy
@@ -951,6 +979,7 @@ void mp_free(void* handle) {
   if (magic == kMagicIndex) {
     mp_index_s* ix = static_cast<mp_index_s*>(handle);
     if (ix->done) cudaEventSynchronize(ix->done), cudaEventDestroy(ix->done);
+    dev_free(ix->hash_mem);
     dev_free(ix->mem);
     ix->magic = 0;
     delete ix;
@@ -964,6 +993,8 @@ void mp_free(void* handle) {
   } else if (magic == kMagicManifest) {
     mp_manifest_s* mf = static_cast<mp_manifest_s*>(handle);
     if (mf->done) cudaEventSynchronize(mf->done), cudaEventDestroy(mf->done);
+    if (mf->valid_done) cudaEventSynchronize(mf->valid_done), cudaEventDestroy(mf->valid_done);
+    dev_free(mf->valid_mem);
     dev_free(mf->mem);
     pin_put(mf->h_realized, (size_t)kCounterSlots * mf->K * 8 + 64 + 16);
     mf->magic = 0;
@@ -1046,6 +1077,123 @@ mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_per_expert
   if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the merge gave up");
   if (err) return fail(MP_ERR_CUDA, "merge kernels reported an error");
   if (tot > s[0]) return fail(MP_ERR_BUDGET, "realized expert reads exceed the planned bytes");
+  return MP_OK;
+}
+
+mp_status mp_index_hashes(const mp_family* family, mp_index* index, mp_stream stream) {
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  Geometry g;
+  if ((st = build_geometry(family, g)) != MP_OK) return st;
+  if (!g.same_as(index->g)) return fail(MP_ERR_MISMATCH, "family geometry differs from the index's");
+  const void* base;
+  ExpertPtrs ex;
+  if ((st = resolve_pointers(family, base, ex)) != MP_OK) return st;
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  // after whatever built the index; the index's event then covers the hashes too
+  if (index->done && (e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  if ((st = alloc_hashes(index, cs)) != MP_OK) return st;
+  HashLaunch p;
+  memset(&p, 0, sizeof(p));
+  p.K = g.K;
+  p.elem_size = g.elem_size;
+  p.n_blocks = g.n_blocks;
+  p.blk_off = index->d_blk_off;
+  p.blk_len = index->d_blk_len;
+  p.base = base;
+  p.experts = ex;
+  p.base_hash = index->d_base_hash;
+  p.expert_hash = index->d_expert_hash;
+  if ((e = launch_hash(p, cs)) != cudaSuccess) return cuda_fail(e, "hash kernel");
+  if ((e = cudaEventRecord(index->done, cs)) != cudaSuccess) return cuda_fail(e, "event record");
+  return MP_OK;
+}
+
+mp_status mp_index_hash_values(const mp_index* index, uint64_t* base_hash, uint64_t* expert_hash) {
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  if (!index->hash_mem.ptr) return fail(MP_ERR_INVALID_ARG, "the index holds no block hashes (mp_index_hashes)");
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(index->done)) != cudaSuccess) return cuda_fail(e, "index work");
+  const uint64_t nb = index->g.n_blocks;
+  if (base_hash && (e = cudaMemcpy(base_hash, index->d_base_hash, nb * 8, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (expert_hash && (e = cudaMemcpy(expert_hash, index->d_expert_hash, nb * index->g.K * 8,
+                                     cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  return MP_OK;
+}
+
+mp_status mp_manifest_validate(const mp_family* family, const mp_index* index, const mp_plan_t* plan, const void* out,
+                               mp_stream stream, mp_manifest* man) {
+  mp_status st;
+  if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
+  if ((st = check_handle(plan, kMagicPlan, "plan")) != MP_OK) return st;
+  if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
+  if (plan->index_id != index->id || man->plan_id != plan->id)
+    return fail(MP_ERR_MISMATCH, "index, plan and manifest do not belong together");
+  if (!index->hash_mem.ptr)
+    return fail(MP_ERR_UNSUPPORTED, "the index holds no block hashes to validate against (mp_index_hashes)");
+  Geometry g;
+  if ((st = build_geometry(family, g)) != MP_OK) return st;
+  if (!g.same_as(index->g)) return fail(MP_ERR_MISMATCH, "family geometry differs from the index's");
+  if (!out || reinterpret_cast<uintptr_t>(out) % 16 != 0 || !is_device_ptr(out))
+    return fail(MP_ERR_INVALID_ARG, "out must be the 16-byte aligned device buffer the merge wrote");
+  const void* base;
+  ExpertPtrs ex;
+  if ((st = resolve_pointers(family, base, ex)) != MP_OK) return st;
+  cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  cudaError_t e;
+  if (!man->valid_mem.ptr) {
+    if ((st = dev_alloc(man->valid_mem, 32 + (size_t)g.n_blocks * 8, cs)) != MP_OK) return st;
+    man->d_vresult = static_cast<unsigned long long*>(man->valid_mem.ptr);
+    man->d_out_hash = man->d_vresult + 4;
+  }
+  if ((e = cudaStreamWaitEvent(cs, man->done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  if ((e = cudaMemsetAsync(man->d_vresult, 0, 16, cs)) != cudaSuccess) return cuda_fail(e, "memset");
+  if ((e = cudaMemsetAsync(man->d_vresult + 2, 0xFF, 8, cs)) != cudaSuccess) return cuda_fail(e, "memset");
+  HashLaunch p;
+  memset(&p, 0, sizeof(p));
+  p.K = g.K;
+  p.elem_size = g.elem_size;
+  p.n_blocks = g.n_blocks;
+  p.blk_off = index->d_blk_off;
+  p.blk_len = index->d_blk_len;
+  p.base = base;
+  p.experts = ex;
+  p.out = out;
+  p.mask = plan->d_mask;
+  p.validate = 1;
+  p.base_hash = index->d_base_hash;
+  p.expert_hash = index->d_expert_hash;
+  p.out_hash = man->d_out_hash;
+  p.result = man->d_vresult;
+  if ((e = launch_hash(p, cs)) != cudaSuccess) return cuda_fail(e, "hash kernel");
+  if (!man->valid_done && (e = cudaEventCreateWithFlags(&man->valid_done, cudaEventDisableTiming)) != cudaSuccess)
+    return cuda_fail(e, "event");
+  if ((e = cudaEventRecord(man->valid_done, cs)) != cudaSuccess) return cuda_fail(e, "event record");
+  return MP_OK;
+}
+
+mp_status mp_manifest_validation(const mp_manifest* man, uint64_t* checked, uint64_t* mismatched, uint64_t* out_hash) {
+  mp_status st;
+  if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
+  if (!man->valid_done) return fail(MP_ERR_INVALID_ARG, "the manifest was not validated (mp_manifest_validate)");
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(man->valid_done)) != cudaSuccess) return cuda_fail(e, "validation work");
+  unsigned long long r[3];
+  if ((e = cudaMemcpy(r, man->d_vresult, sizeof(r), cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
+  if (out_hash && (e = cudaMemcpy(out_hash, man->d_out_hash, man->n_blocks * 8, cudaMemcpyDeviceToHost)) != cudaSuccess)
+    return cuda_fail(e, "copy");
+  if (checked) *checked = r[0];
+  if (mismatched) *mismatched = r[1];
+  if (r[1]) {
+    const uint64_t k = r[2] / man->n_blocks, b = r[2] % man->n_blocks;
+    return fail(MP_ERR_MISMATCH, std::to_string(r[1]) + " block(s) read by the merge differ from the catalog; first: " +
+                                     (k == 0 ? std::string("base") : "expert " + std::to_string(k - 1)) + " block " +
+                                     std::to_string(b));
+  }
   return MP_OK;
 }
 

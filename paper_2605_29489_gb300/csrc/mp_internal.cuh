@@ -72,6 +72,9 @@ struct mp_index_s {
   uint32_t* d_blk_tensor;  // [n_blocks] tensor of each block
   uint32_t* d_t_blk0;      // [n_tensors + 1] first block of each tensor, then n_blocks
   bool has_missing;        // some entry has nnz == kNnzMissing (imported catalogs only)
+  mp::Alloc hash_mem;      // the catalog's block hashes, once computed or imported
+  unsigned long long* d_base_hash;    // [n_blocks]
+  unsigned long long* d_expert_hash;  // [K][n_blocks]
   float* d_norm;           // [K][n_blocks]
   float* d_maxabs;         // [K][n_blocks]
   uint32_t* d_nnz;         // [K][n_blocks]
@@ -117,6 +120,13 @@ struct mp_manifest_s {
   uint64_t planned, touched, digest;
   uint64_t lineage[mp::kMaxK + 1];  // caller ids of M_0..M_K (zeros when none were given)
   cudaEvent_t done;
+  // hash validation (mp_manifest_validate): checked / mismatched / first bad item, and
+  // the output's block hashes
+  mp::Alloc valid_mem;
+  unsigned long long* d_vresult;   // [3]
+  unsigned long long* d_out_hash;  // [n_blocks]
+  uint64_t n_blocks;
+  cudaEvent_t valid_done;
 };
 
 namespace mp {
@@ -247,5 +257,28 @@ struct GatherLaunch {
   unsigned long long* gathered;  // bytes copied, accumulated (may be NULL)
 };
 cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st);
+
+// ---- block content hashes (hash.cu) --------------------------------------------------------
+// catalog mode (validate = 0): hash every block of the base and of each expert into
+// base_hash / expert_hash.  Validation: hash the base, the expert blocks selected by mask
+// and every block of out; compare the first two with the catalog (result[0] += blocks
+// checked, result[1] += mismatches, result[2] = min mismatching item), write out_hash.
+struct HashLaunch {
+  uint32_t K;
+  uint32_t elem_size;
+  uint64_t n_blocks;
+  const uint64_t* blk_off;
+  const uint32_t* blk_len;
+  const void* base;
+  ExpertPtrs experts;
+  const void* out;
+  const uint32_t* mask;
+  uint32_t validate;
+  unsigned long long* base_hash;    // [n_blocks]
+  unsigned long long* expert_hash;  // [K][n_blocks]
+  unsigned long long* out_hash;     // [n_blocks]
+  unsigned long long* result;       // [3]
+};
+cudaError_t launch_hash(const HashLaunch& p, cudaStream_t st);
 
 }  // namespace mp
