@@ -509,9 +509,11 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  *                                    out = round(M_0 + acc)
  *  DARE: v_i = keep_i ? delta_i * sigma : 0, sigma = fp32(1/(1-p));
  *        acc = sum_i fma(alpha_i, A_i v_i, acc); out = round(M_0 + acc)
- *  TIES: d^_i = A_i delta_i if key(delta_i) >= tau_i else 0;  S = sum_i d^_i;
- *        gamma = sign(S);  m = (sum of d^_i with sign gamma) / (their count), 0 if S = 0;
- *        out = round(fma(lambda, m, M_0))
+ *  TIES: d^_i = A_i delta_i if key(delta_i) >= tau_i else 0;  P = sum of the d^_i > 0,
+ *        N = sum of the d^_i < 0 (each an ascending fp32 chain from +0), c+ and c- their
+ *        counts;  gamma = sign(P + N), taken exactly as P > -N, P < -N or P = -N (the
+ *        rounded sum fl(P + N) has the sign of P + N);  m = P / c+ if gamma > 0, N / c- if
+ *        gamma < 0, else 0;  out = round(fma(lambda, m, M_0))
  *  AVG, renormalised over the selected experts (App. A.1, the selected-only variant with
  *        coefficients beta_i(A) = 0 when A_i = 0): s = sum of alpha_j over the experts j that
  *        are selected or whose delta block is exactly zero (ascending fp32 adds from +0);
@@ -519,7 +521,7 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  *        acc = sum_i fma(beta_i, A_i delta_i, acc); out = round(M_0 + acc)
  *  DARE-TIES: DARE's drop and rescale with the same mask omega, then TIES's election and
  *        disjoint mean without magnitude trimming: d^_i = A_i (keep_i ? delta_i * sigma : 0),
- *        then S, gamma, m and out as TIES
+ *        then P, N, gamma, m and out as TIES
  * round = bf16 round-to-nearest-even, or none for fp32 checkpoints.
  * Pins: hand-computed TIES, AVG and renormalised-AVG examples; Eq. 5 against an fp64
  * restatement of the unmasked operator (within one bf16 ulp); Prop. 2 bound and the
@@ -553,7 +555,7 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
     float x0 = load_elem(dtype, base, k);
     float res;
     if (ties_like) {
-      float S = 0.0f, P = 0.0f, Nn = 0.0f;
+      float P = 0.0f, Nn = 0.0f;
       uint32_t cp = 0, cn = 0;
       for (uint32_t i = 0; i < K; ++i) {
         float dh = 0.0f;
@@ -565,7 +567,6 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
             dh = d * sigma;
           }
         }
-        S = S + dh;
         if (dh > 0.0f) {
           P = P + dh;
           ++cp;
@@ -575,8 +576,8 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
         }
       }
       float m = 0.0f;
-      if (S > 0.0f) m = P / (float)cp;
-      else if (S < 0.0f) m = Nn / (float)cn;
+      if (P > -Nn) m = P / (float)cp;
+      else if (P < -Nn) m = Nn / (float)cn;
       res = fmaf(op->lambda, m, x0);
     } else {
       float acc = 0.0f;

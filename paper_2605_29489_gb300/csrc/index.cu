@@ -81,6 +81,7 @@ __device__ __forceinline__ uint32_t ties_key(float d) {
 // combined by the xor butterfly.
 constexpr int kIxConsumers = 256;
 constexpr int kIxThreads = kIxConsumers + 32;
+static_assert(kIxConsumers == 256, "one consumer thread per coarse TIES bin at the end of a block");
 constexpr uint32_t kIxEnd = 0xFFFFFFFFu;
 
 // ring geometry.  The plain catalog is bound by HBM: two CTAs per SM with twelve 8 KiB
@@ -112,7 +113,6 @@ struct __align__(128) IxSmem {
   float red_ss[KG][8];
   float red_mx[KG][8];
   uint32_t red_nz[KG][8];
-  uint32_t nnz_tot[KG];
   uint64_t cbar;  // consumer-only barrier (one arrival per consumer warp)
   int abort;
 };
@@ -142,30 +142,36 @@ __device__ __forceinline__ bool same_vec(const uint4 a, const uint4 b) {
 // TIES coarse bins of two deltas: bin = upper 8 bits of the 15-bit key bits(bf16(|d|)),
 // i.e. bits 7..14 of the round-to-nearest-even bf16 of d (the sign bit 15 is masked off);
 // both are converted by one packed cvt.  A nonzero delta adds 1 to its bin of the
-// shared histogram at hist (byte address in the shared window) and 1 to nz; a zero delta
-// adds nothing.  Predicated, so that no branch is taken per element.
-__device__ __forceinline__ void ties_bin2(float d0, float d1, uint32_t hist, uint32_t& nz) {
+// shared histogram at hist (byte address in the shared window); a zero delta adds
+// nothing, so the histogram's total is the block's nonzero count.  Predicated, so that no
+// branch is taken per element.
+__device__ __forceinline__ void ties_bin2(float d0, float d1, uint32_t hist) {
   asm volatile(
       "{\n"
       " .reg .pred p0, p1;\n"
       " .reg .b32 w, a0, a1;\n"
-      " cvt.rn.bf16x2.f32 w, %3, %2;\n"
-      " setp.ne.f32 p0, %2, 0f00000000;\n"
-      " setp.ne.f32 p1, %3, 0f00000000;\n"
+      " cvt.rn.bf16x2.f32 w, %2, %1;\n"
+      " setp.ne.f32 p0, %1, 0f00000000;\n"
+      " setp.ne.f32 p1, %2, 0f00000000;\n"
       " shr.b32 a0, w, 5;\n"
       " and.b32 a0, a0, 1020;\n"
-      " add.u32 a0, a0, %1;\n"
+      " add.u32 a0, a0, %0;\n"
       " shr.b32 a1, w, 21;\n"
       " and.b32 a1, a1, 1020;\n"
-      " add.u32 a1, a1, %1;\n"
+      " add.u32 a1, a1, %0;\n"
       " @p0 red.shared.add.u32 [a0], 1;\n"
       " @p1 red.shared.add.u32 [a1], 1;\n"
-      " @p0 add.u32 %0, %0, 1;\n"
-      " @p1 add.u32 %0, %0, 1;\n"
-      "}\n"
-      : "+r"(nz)
-      : "r"(hist), "f"(d0), "f"(d1)
+      "}\n" ::"r"(hist),
+      "f"(d0), "f"(d1)
       : "memory");
+}
+
+// (d0, d1) = (a0 - b0, a1 - b1), each rounded to nearest: one packed subtract
+__device__ __forceinline__ void f2_sub(float a0, float a1, float b0, float b1, float& d0, float& d1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n sub.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
 // TIES fine bins of two deltas: a nonzero delta whose coarse bin (key bits 7..14) is es
@@ -353,7 +359,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
           unpack<BF16>(re[u], xe);
           float d[V];
 #pragma unroll
-          for (int e = 0; e < V; ++e) d[e] = __fsub_rn(xe[e], xb[u][e]);
+          for (int e = 0; e < V; e += 2) f2_sub(xe[e], xe[e + 1], xb[u][e], xb[u][e + 1], d[e], d[e + 1]);
           // the sum of squares is one fma chain in element order (the canonical order);
           // max |d| and the counts are exact in any order, so they take a tree
 #pragma unroll
@@ -369,7 +375,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
             if constexpr (TIES) {
-              ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]), nz[k]);
+              ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]));
             } else {
               nz[k] += d[e] != 0.0f ? 1u : 0u;
               nz[k] += d[e + 1] != 0.0f ? 1u : 0u;
@@ -422,8 +428,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
           const uint64_t u = (uint64_t)(i0 + k) * p.n_blocks + b;
           p.norm[u] = __fsqrt_rn(a);
           p.maxabs[u] = m;
-          p.nnz[u] = c;
-          S.nnz_tot[k] = c;
+          if constexpr (!TIES) p.nnz[u] = c;
           // a NaN delta makes the sum of squares NaN; an infinite one makes max |delta| infinite
           if (isnan(a) || isinf(m)) bad = 1u;
         }
@@ -431,20 +436,41 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
       if (lane == 0 && bad) atomicOr(p.err, kErrNonfinite);
     }
     if constexpr (TIES) {
+      // every nonzero delta added 1 to exactly one bin: the histogram's total is nnz
       if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
-      atomicOr(p.err, kErrTimeout);
-      S.abort = 1;
-      break;
-    }
+        atomicOr(p.err, kErrTimeout);
+        S.abort = 1;
+        break;
+      }
+      uint32_t hc[KG];
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        hc[k] = S.hist[k][tid];
+        S.hist[k][tid] = 0u;
+        uint32_t w = hc[k];
+#pragma unroll
+        for (int s = 16; s >= 1; s >>= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, s);
+        if (lane == 0) S.red_nz[k][warp] = w;
+      }
+      if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+        atomicOr(p.err, kErrTimeout);
+        S.abort = 1;
+        break;
+      }
       const uint32_t grp = p.blk_group[b];
       const uint32_t len = p.blk_len[b];
-      for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += kIxConsumers) {
-        const uint32_t k = x >> 8, e = x & 255u;
-        unsigned long long c = S.hist[k][e];
-        S.hist[k][e] = 0u;
-        if (k >= kc) continue;
-        if (e == 0) c += len - S.nnz_tot[k];  // zero deltas have key 0
-        if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + e], c);
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        if ((uint32_t)k >= kc) break;
+        uint32_t nzk = 0;
+#pragma unroll
+        for (int w = 0; w < kIxConsumers / 32; ++w) nzk += S.red_nz[k][w];
+        unsigned long long c = hc[k];
+        if (tid == 0) {
+          p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
+          c += len - nzk;  // zero deltas have key 0
+        }
+        if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + tid], c);
       }
     }
     if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {

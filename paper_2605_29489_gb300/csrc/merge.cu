@@ -134,25 +134,25 @@ __host__ __device__ __forceinline__ uint32_t ties_bits_threshold(uint32_t tau) {
 }
 
 // One expert's contribution to an element's TIES tally, with predicated adds: the delta d
-// is kept when |d| >= thr; a kept d goes into S, and into P (with count +1) when positive
-// or into N (count + 0x10000) otherwise.  thr is at least the smallest subnormal, so a kept
-// d is never zero and "not positive" means negative; one compare with two destination
+// is kept when |d| >= thr; a kept d goes into P (with count +1) when positive or into N
+// (count + 0x10000) otherwise.  thr is at least the smallest subnormal, so a kept d is
+// never zero and "not positive" means negative; one compare with two destination
 // predicates splits the kept entries by sign.  A skipped add is the same as adding the +0
-// of a trimmed entry: S, P and N are never -0, so +0 leaves them unchanged.
-__device__ __forceinline__ void ties_tally(float d, float thr, float& S, float& P, float& N, uint32_t& cnt) {
+// of a trimmed entry: P and N are never -0, so +0 leaves them unchanged.  The elected
+// sign is that of P + N (compared exactly at the end).
+__device__ __forceinline__ void ties_tally(float d, float thr, float& P, float& N, uint32_t& cnt) {
   asm("{\n"
       " .reg .pred pk, pp, pn;\n"
       " .reg .f32 ad;\n"
-      " abs.f32 ad, %4;\n"
-      " setp.ge.f32 pk, ad, %5;\n"
-      " setp.gt.and.f32 pp|pn, %4, 0f00000000, pk;\n"
-      " @pk add.rn.f32 %0, %0, %4;\n"
-      " @pp add.rn.f32 %1, %1, %4;\n"
-      " @pn add.rn.f32 %2, %2, %4;\n"
-      " @pp add.u32 %3, %3, 1;\n"
-      " @pn add.u32 %3, %3, 65536;\n"
+      " abs.f32 ad, %3;\n"
+      " setp.ge.f32 pk, ad, %4;\n"
+      " setp.gt.and.f32 pp|pn, %3, 0f00000000, pk;\n"
+      " @pp add.rn.f32 %0, %0, %3;\n"
+      " @pn add.rn.f32 %1, %1, %3;\n"
+      " @pp add.u32 %2, %2, 1;\n"
+      " @pn add.u32 %2, %2, 65536;\n"
       "}\n"
-      : "+f"(S), "+f"(P), "+f"(N), "+r"(cnt)
+      : "+f"(P), "+f"(N), "+r"(cnt)
       : "f"(d), "f"(thr));
 }
 
@@ -364,7 +364,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   }
 
   // ---------------- consumers ----------------
-  float x0[VPT][V], acc[VPT][V], Sg[VPT][V], Pp[VPT][V], Nn[VPT][V];
+  float x0[VPT][V], acc[VPT][V], Pp[VPT][V], Nn[VPT][V];
   uint32_t cnt[VPT][V];  // TIES: positive count | negative count << 16
   uint64_t off = 0;
   uint32_t n = 0, n_tma = 0, remaining = 0;
@@ -416,7 +416,6 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
 #pragma unroll
           for (int e = 0; e < V; ++e) {
             acc[u][e] = 0.0f;
-            Sg[u][e] = 0.0f;
             Pp[u][e] = 0.0f;
             Nn[u][e] = 0.0f;
             cnt[u][e] = 0u;
@@ -451,8 +450,8 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
               d0 = kept[e] ? s0 : 0.0f;
               d1 = kept[e + 1] ? s1 : 0.0f;
             }
-            ties_tally(d0, thr, Sg[u][e], Pp[u][e], Nn[u][e], cnt[u][e]);
-            ties_tally(d1, thr, Sg[u][e + 1], Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
+            ties_tally(d0, thr, Pp[u][e], Nn[u][e], cnt[u][e]);
+            ties_tally(d1, thr, Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
           }
         }
       } else {
@@ -501,11 +500,12 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
           continue;
         }
         if constexpr (kTiesLike<OPC>) {
-          // one division per element: the mean of the entries whose sign was elected
-          // (S != 0 implies at least one of them, so c >= 1; otherwise +0 / 1 = +0).  The
-          // rare numerators that need the IEEE division take it under one warp vote.
+          // one division per element: the mean of the entries whose sign was elected, the
+          // sign of P + N taken exactly as P > -N or P < -N (then that side holds at least
+          // one entry, so c >= 1; otherwise +0 / 1 = +0).  The rare numerators that need the
+          // IEEE division take it under one warp vote.
           auto num_c = [&](int e, float& num, uint32_t& c) {
-            const bool pos = Sg[u][e] > 0.0f, any = Sg[u][e] != 0.0f;
+            const bool pos = Pp[u][e] > -Nn[u][e], any = Pp[u][e] != -Nn[u][e];
             num = any ? (pos ? Pp[u][e] : Nn[u][e]) : 0.0f;
             c = any ? (pos ? (cnt[u][e] & 0xFFFFu) : (cnt[u][e] >> 16)) : 0u;
           };
