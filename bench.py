@@ -115,17 +115,10 @@ def make_ops(w, K):
 
 
 def fallback_missing(fam, K):
-    """the seeded pattern of catalog entries without statistics of the fallback workloads:
-    every entry of 10 % of the (expert, tensor) pairs (always the largest tensor of expert 0)
-    and 0.1 % of the other entries; bool [K, n_blocks]"""
-    import numpy as np
+    """the fallback workloads' catalog entries without statistics (seeded; bool [K, n_blocks])"""
+    from paper_2605_29489_gb300 import synth
 
-    _, _, bt = fam.block_table()
-    rng = np.random.default_rng(2605)
-    n_t = int(bt.max()) + 1
-    pairs = rng.random((K, n_t)) < 0.10
-    pairs[0, int(np.argmax(np.bincount(bt)))] = True
-    return pairs[:, bt] | (rng.random((K, bt.size)) < 0.001)
+    return synth.missing_entries(fam, K)
 
 
 # ---- clocks ---------------------------------------------------------------------------------------

@@ -287,6 +287,20 @@ def qwen25_15b(seed: int = 0, K: int = 16, layers: int = 28) -> Family:
                   active_frac=0.25, log_mu=math.log(1e-3), log_sigma=1.0, per_expert_active=True, seed=seed)
 
 
+def missing_entries(fam: Family, K: int, seed: int = 2605, pair_frac: float = 0.10,
+                    entry_frac: float = 0.001) -> np.ndarray:
+    """A seeded pattern of catalog entries without statistics, bool [K, n_blocks]: every entry
+    of a pair_frac share of the (expert, tensor) pairs (always the largest tensor of expert
+    0) and an entry_frac share of the other entries.  Input generation only: which entries
+    a saved catalog lacks."""
+    _, _, bt = fam.block_table()
+    rng = np.random.default_rng(seed)
+    n_t = int(bt.max()) + 1
+    pairs = rng.random((K, n_t)) < pair_frac
+    pairs[0, int(np.argmax(np.bincount(bt)))] = True
+    return pairs[:, bt] | (rng.random((K, bt.size)) < entry_frac)
+
+
 def custom(shapes, dtype=BF16, block_elems=4096, K=3, active_frac=0.5, log_mu=math.log(1e-2),
            log_sigma=1.0, per_expert_active=False, seed=0, name="custom") -> Family:
     """A small family for tests: shapes is a list of element counts"""

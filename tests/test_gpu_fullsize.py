@@ -41,8 +41,22 @@ def pool():
     ex.shutdown(cancel_futures=True)
 
 
+_CATALOGS = {}  # the oracle's statistics of a family, kept for the later tests of this module
+
+
 def oracle_catalog(pool, spec, fam, ties_density=None):
     """oracle statistics [K, n_blocks] (and tau [K, n_tensors] for TIES) of the whole family"""
+    if (spec, ties_density) in _CATALOGS:
+        return _CATALOGS[(spec, ties_density)]
+    if ties_density is None:   # the statistics do not depend on the operator
+        for (sp, _), cat in _CATALOGS.items():
+            if sp == spec:
+                return cat[:3] + (None,)
+    _CATALOGS[(spec, ties_density)] = cat = _oracle_catalog(pool, spec, fam, ties_density)
+    return cat
+
+
+def _oracle_catalog(pool, spec, fam, ties_density=None):
     K, nb = fam.K, fam.n_blocks
     norm = np.zeros((K, nb), np.float32)
     maxabs = np.zeros((K, nb), np.float32)
@@ -160,3 +174,55 @@ def test_fullsize_llama3_8b_ties(pool):
         pytest.skip("needs about 100 GB of device memory")
     run_family(pool, ("llama3_8b", ()), mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2),
                oracle.Op(oracle.TIES, K, lam=1.0, density=0.2), [1.0, 0.5, 0.25, 0.1], ties_density=0.2)
+
+
+def test_fullsize_llama3_8b_fallback_plan(pool):
+    """Llama-3-8B-shaped family, K=4, TA lambda=0.3, planned from the oracle's own catalog
+    imported with the bench's missing entries (tensor-level fallback), budgets 1.0 / 0.5 /
+    0.25 / 0.1: plan bit-exact against the oracle's fallback plan; realized = planned; the
+    merge of sampled blocks (the fallback tensors' first and last blocks among them) equal
+    to the oracle's under the same mask"""
+    K = 4
+    if torch.cuda.get_device_properties(0).total_memory < 120 * 2 ** 30:
+        pytest.skip("needs about 100 GB of device memory")
+    spec = ("llama3_8b", ())
+    fam = ow.family(spec)
+    es = fam.elem_size
+    o_norm, o_max, o_nnz, _ = oracle_catalog(pool, spec, fam)
+    miss = synth.missing_entries(fam, K)
+    nz = o_nnz.copy()
+    nz[miss] = mp.MP_NNZ_MISSING
+    gop = mp.make_op(mp.MP_OP_TA, alpha=[0.3] * K)
+    oop = oracle.Op(oracle.TA, K, alpha=[0.3] * K)
+    base, experts = fam.device_arrays()
+    offs, nums, _ = fam.layout()
+    mf = mp.family(list(zip(offs.tolist(), nums.tolist())), base, experts, fam.block_elems, fam.dtype, 0)
+    imp = mp.mp_index_import(mf, gop, o_norm, o_max, nz)
+    bo, bl, bt = fam.block_table()
+    big = int(np.argmax(np.bincount(bt)))
+    big_blocks = np.nonzero(bt == big)[0]
+    samples = sorted(set(sample_blocks(fam)) | {int(big_blocks[0]), int(big_blocks[-1])})
+    out = torch.empty_like(base)
+    for f in (1.0, 0.5, 0.25, 0.1):
+        B = mp.mp_budget_from_fraction(mf, f)
+        plan = mp.mp_plan(imp, gop, B)
+        pi = mp.mp_plan_info(plan, imp)
+        opl = oracle.plan(K, bl, bt, len(fam.tensors), es, oop, o_norm, o_max, nz, None, B, blk_tensor=bt)
+        assert (pi["chat"], pi["n_sel"], pi["n_cand"], pi["digest"]) == (opl["chat"], opl["n_sel"], opl["n_cand"],
+                                                                         opl["digest"]), f
+        assert np.array_equal(pi["mask"], opl["mask"]), f
+        assert np.array_equal(pi["order"], opl["order"]), f
+        man = mp.mp_merge(mf, imp, plan, out)
+        mi = mp.mp_manifest_info(man, K)
+        assert mi["realized_total"] == opl["chat"] <= B
+        for b in samples:
+            hb, hex_ = fam.block_host(b)
+            s = slice(int(bo[b]), int(bo[b] + bl[b]))
+            want = oracle.merge_block(fam.dtype, int(bo[b]), hb, hex_, int(opl["mask"][b]), oop)
+            got = out[s].view(torch.int16).cpu().numpy().view(np.uint16)
+            assert np.array_equal(got, want), (f, b)
+        man.free()
+        plan.free()
+    imp.free()
+    del base, experts, out
+    torch.cuda.empty_cache()
