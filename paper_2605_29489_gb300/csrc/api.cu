@@ -1150,7 +1150,9 @@ mp_status mp_manifest_validate(const mp_family* family, const mp_index* index, c
     man->d_vresult = static_cast<unsigned long long*>(man->valid_mem.ptr);
     man->d_out_hash = man->d_vresult + 4;
   }
+  // after the merge (its output) and the index's own work (the hashes, perhaps added later)
   if ((e = cudaStreamWaitEvent(cs, man->done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
+  if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return cuda_fail(e, "stream wait");
   if ((e = cudaMemsetAsync(man->d_vresult, 0, 16, cs)) != cudaSuccess) return cuda_fail(e, "memset");
   if ((e = cudaMemsetAsync(man->d_vresult + 2, 0xFF, 8, cs)) != cudaSuccess) return cuda_fail(e, "memset");
   HashLaunch p;
