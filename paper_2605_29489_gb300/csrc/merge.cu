@@ -156,6 +156,26 @@ __device__ __forceinline__ void ties_tally(float d, float thr, float& P, float& 
       : "f"(d), "f"(thr));
 }
 
+// One expert's contribution to an element's DARE-TIES tally: the rescaled delta s enters
+// when its keep word kw (the 16-bit word in the upper half of a 32-bit register) reaches
+// T16 and s is nonzero, into P (count +1) when positive or N (count + 0x10000) when
+// negative; no magnitude trim.  A dropped or zero entry adds nothing (the +0 of Eq. 4's
+// dropped delta leaves P and N unchanged).
+__device__ __forceinline__ void dties_tally(float s, uint32_t kw, uint32_t T16, float& P, float& N, uint32_t& cnt) {
+  asm("{\n"
+      " .reg .pred pk, pp, pn;\n"
+      " setp.ge.u32 pk, %4, %5;\n"
+      " setp.gt.and.f32 pp, %3, 0f00000000, pk;\n"
+      " setp.lt.and.f32 pn, %3, 0f00000000, pk;\n"
+      " @pp add.rn.f32 %0, %0, %3;\n"
+      " @pn add.rn.f32 %1, %1, %3;\n"
+      " @pp add.u32 %2, %2, 1;\n"
+      " @pn add.u32 %2, %2, 65536;\n"
+      "}\n"
+      : "+f"(P), "+f"(N), "+r"(cnt)
+      : "f"(s), "r"(kw), "r"(T16));
+}
+
 // bf16 -> fp32: the upper element by a mask, the lower one moved up by a multiply (which runs
 // on the FMA pipe and leaves the ALU pipe to the compares)
 template <bool BF16>
@@ -374,17 +394,24 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is exactly
   // the 8 words of one call (chunk and tensor offsets are multiples of 8 elements); an
   // fp32 vector is half of one.
-  auto dare_kept = [&](uint32_t i, uint64_t j0, bool (&kept)[V]) {
+  // word j mod 8 of element j, in the upper half of a 32-bit register: the upper word as it
+  // stands, the lower one moved up by a multiply (FMA pipe; the ALU pipe is the busy one);
+  // it is kept iff that register >= T << 16
+  auto dare_words = [&](uint32_t i, uint64_t j0, uint32_t (&kw)[V]) {
     const uint64_t g = j0 >> 3;
     const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
     const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
 #pragma unroll
     for (int e = 0; e < V; ++e) {
       const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
-      // word >= T, compared in the upper half of a 32-bit register: the upper word as it
-      // stands, the lower one moved up by a multiply (FMA pipe; the ALU pipe is the busy one)
-      kept[e] = ((e & 1) ? wd : wd * 65536u) >= p.dare_T16;
+      kw[e] = (e & 1) ? wd : wd * 65536u;
     }
+  };
+  auto dare_kept = [&](uint32_t i, uint64_t j0, bool (&kept)[V]) {
+    uint32_t kw[V];
+    dare_words(i, j0, kw);
+#pragma unroll
+    for (int e = 0; e < V; ++e) kept[e] = kw[e] >= p.dare_T16;
   };
   for (uint32_t fill = 0;; ++fill) {
     const uint32_t s = fill % kSlots, r = fill / kSlots;
@@ -429,16 +456,16 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
       if constexpr (kTiesLike<OPC>) {
         // TIES: trim test on the magnitude's bits: key(|d|) >= tau exactly when bits(|d|) >=
         // the producer's threshold (a NaN pattern, never true, when nothing is kept).
-        // DARE-TIES: the delta is first dropped or rescaled by the keep mask, and every
-        // nonzero result is kept (threshold = the smallest subnormal).
+        // DARE-TIES: the delta is rescaled, and it enters when its keep word passes and the
+        // result is nonzero (no magnitude trim).
         const float thr = __uint_as_float(OPC == OP_TIES ? S.meta[s].aux : 1u);
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           const uint32_t k0 = (tid + (uint32_t)u * kConsumers) * V;
           float xe[V];
           read_vec<BF16>(slot, src, off - p.expert_origin, k0, n, n_tma, xe);
-          bool kept[V];
-          if constexpr (OPC == OP_DTIES) dare_kept(i, off + k0, kept);
+          uint32_t kw[V];
+          if constexpr (OPC == OP_DTIES) dare_words(i, off + k0, kw);
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
             // the deltas of an element pair in one packed fp32x2 subtract
@@ -447,11 +474,12 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
             if constexpr (OPC == OP_DTIES) {
               float s0, s1;
               f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
-              d0 = kept[e] ? s0 : 0.0f;
-              d1 = kept[e + 1] ? s1 : 0.0f;
+              dties_tally(s0, kw[e], p.dare_T16, Pp[u][e], Nn[u][e], cnt[u][e]);
+              dties_tally(s1, kw[e + 1], p.dare_T16, Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
+            } else {
+              ties_tally(d0, thr, Pp[u][e], Nn[u][e], cnt[u][e]);
+              ties_tally(d1, thr, Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
             }
-            ties_tally(d0, thr, Pp[u][e], Nn[u][e], cnt[u][e]);
-            ties_tally(d1, thr, Pp[u][e + 1], Nn[u][e + 1], cnt[u][e + 1]);
           }
         }
       } else {
