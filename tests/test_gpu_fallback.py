@@ -1,8 +1,8 @@
 """Imported catalogs and the tensor-level fallback plan (Sec. 3 "Catalog" and "Planner")
 on the GPU, through the C ABI, against the oracle.
 
-* A catalog exported with mp_index_stats and imported again with mp_index_import plans and
-  merges exactly like the index it came from.
+* The oracle's catalog imported with mp_index_import plans and merges exactly like the
+  GPU's own index of the same family (which equals it bit for bit).
 * Entries marked MP_NNZ_MISSING: the plan (mask, order, C_hat, counts, digest) equals the
   oracle's tensor-level fallback plan bit for bit, and the merge with that plan equals the
   oracle's merge with the same mask and the same catalog nnz.  Seeded missing patterns:
@@ -61,8 +61,8 @@ def run_fallback(fam, kinds=KINDS, fracs=FRACS, seed=0):
         scope = oop.trim_scope if oop.kind == oracle.TIES else 0
         of = oracle_family(fam, base, experts, trim_scope=scope)
         idx = mp.mp_index_blocks(mf, gop)
-        norm, maxabs, nnz, tau = mp.mp_index_stats(idx)
-        o_tau = tau if oop.kind == oracle.TIES else None
+        norm, maxabs, nnz = oracle.index(of)       # the oracle's catalog, imported into the GPU
+        o_tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
         for pname, miss in pats.items():
             nz = nnz.copy()
             nz[miss] = MISS
@@ -115,10 +115,10 @@ def test_fallback_full_budget_reproduces_the_full_read():
     for name, gop, oop in ops_for(fam.K, ("ta", "ties", "avg_renorm")):
         of = oracle_family(fam, base, experts)
         idx = mp.mp_index_blocks(mf, gop)
-        norm, maxabs, nnz, tau = mp.mp_index_stats(idx)
+        norm, maxabs, nnz = oracle.index(of)
         nz = nnz.copy()
         nz[rng.random(nz.shape) < 0.3] = MISS
-        o_tau = tau if oop.kind == oracle.TIES else None
+        o_tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
         imp = mp.mp_index_import(mf, gop, norm, maxabs, nz, o_tau)
         plan = mp.mp_plan(imp, gop, mp.mp_budget_from_fraction(mf, 1.0))
         out = torch.empty_like(b)
@@ -138,7 +138,7 @@ def test_noalloc_reports_missing_entries_and_skips_them():
     gop = mp.make_op(mp.MP_OP_TA, alpha=[0.3] * fam.K)
     oop = oracle.Op(oracle.TA, fam.K, alpha=[0.3] * fam.K)
     idx = mp.mp_index_blocks(mf, gop)
-    norm, maxabs, nnz, _ = mp.mp_index_stats(idx)
+    norm, maxabs, nnz = oracle.index(oracle_family(fam, base, experts))
     nz = nnz.copy()
     nz[np.random.default_rng(3).random(nz.shape) < 0.2] = MISS
     K, nb = fam.K, bl.size
@@ -181,3 +181,37 @@ def test_import_refuses_entries_that_are_not_statistics():
     with pytest.raises(mp.MergePipeError):
         mp.mp_index_import(mf, ties, norm, maxabs, nnz, None)
     idx.free()
+
+
+def test_fallback_with_a_host_resident_pool():
+    """an imported catalog with missing entries plans and merges the same when the experts
+    live in pinned host memory (the segment pipeline gathers the planned blocks)"""
+    fam = fam_k9()
+    base, experts = fam.host_arrays()
+    mf_d, b_d, _ = upload(fam, base, experts)
+    mf_h, b_h, _ = upload(fam, base, experts, host_experts=True)
+    covered = tensor_mask(fam)
+    _, bl, bt = fam.block_table()
+    of = oracle_family(fam, base, experts)
+    for name, gop, oop in ops_for(fam.K, ("ta", "avg_renorm")):
+        idx = mp.mp_index_blocks(mf_d, gop)
+        norm, maxabs, nnz = oracle.index(of)
+        nz = nnz.copy()
+        nz[missing_patterns(fam, fam.K, np.random.default_rng(9))["dense"]] = MISS
+        imp_h = mp.mp_index_import(mf_h, gop, norm, maxabs, nz)
+        for f in (0.3, 1.0):
+            B = mp.mp_budget_from_fraction(mf_h, f)
+            plan = mp.mp_plan(imp_h, gop, B)
+            pi = mp.mp_plan_info(plan, imp_h)
+            opl = oracle.plan(fam.K, bl, of.blk_group, of.n_groups, fam.elem_size, oop, norm, maxabs, nz, None, B,
+                              blk_tensor=bt)
+            assert pi["digest"] == opl["digest"] and np.array_equal(pi["mask"], opl["mask"]), (name, f)
+            out = torch.full_like(b_h, float("nan"))
+            man = mp.mp_merge(mf_h, imp_h, plan, out)
+            assert mp.mp_manifest_info(man, fam.K)["realized_total"] == opl["chat"]
+            want = oracle.merge(of, oop, mask=opl["mask"], nnz=nz)
+            assert_merge_close(fam, host(fam, out)[covered], want[covered], f"{name}/host/f={f}")
+            man.free()
+            plan.free()
+        imp_h.free()
+        idx.free()

@@ -50,25 +50,29 @@ def test_validate_after_merge_checks_what_was_read_and_hashes_the_output():
     base, experts = fam.host_arrays()
     mf, b, ex, _, idx = catalog(fam, base, experts)
     of = oracle_family(fam, base, experts)
-    bo, bl, _ = fam.block_table()
+    o_norm, o_max, o_nnz = oracle.index(of)
+    bo, bl, bt = fam.block_table()
     for name, gop, oop in ops_for(fam.K, ("ta", "ties", "dare")):
         if oop.kind == oracle.TIES:
             idx_t = mp.mp_index_blocks(mf, gop)
             mp.mp_index_hashes(mf, idx_t)
-            use, tau = idx_t, mp.mp_index_stats(idx_t)[3]
+            use, tau = idx_t, oracle.ties_thresholds(of, oop.density)
         else:
             use, tau = idx, None
         for f in (0.3, 1.0):
-            plan = mp.mp_plan(use, gop, mp.mp_budget_from_fraction(mf, f))
+            B = mp.mp_budget_from_fraction(mf, f)
+            plan = mp.mp_plan(use, gop, B)
             pi = mp.mp_plan_info(plan, use)
+            opl = oracle.plan(fam.K, bl, of.blk_group, of.n_groups, fam.elem_size, oop, o_norm, o_max, o_nnz, tau, B)
+            assert pi["digest"] == opl["digest"] and np.array_equal(pi["mask"], opl["mask"]), (name, f)
             out = torch.empty_like(b)
             man = mp.mp_merge(mf, use, plan, out)
             mp.mp_manifest_validate(mf, use, plan, out, man)
             v = mp.mp_manifest_validation(man, fam.n_blocks)
-            n_sel_blocks = int(sum(bin(int(m)).count("1") for m in pi["mask"]))
+            n_sel_blocks = int(sum(bin(int(m)).count("1") for m in opl["mask"]))
             assert v["mismatched"] == 0
             assert v["checked"] == fam.n_blocks + n_sel_blocks, (name, f)
-            want = oracle.merge(of, oop, tau=tau, mask=pi["mask"])
+            want = oracle.merge(of, oop, tau=tau, mask=opl["mask"])
             for blk in range(fam.n_blocks):
                 s = slice(int(bo[blk]), int(bo[blk] + bl[blk]))
                 assert int(v["out_hash"][blk]) == oracle.block_hash(want[s].tobytes()), (name, f, blk)

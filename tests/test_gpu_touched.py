@@ -43,22 +43,25 @@ def check_family(fam, kinds, fracs, host_experts=False):
     for name, gop, oop in ops_for(fam.K, kinds):
         scope = oop.trim_scope if oop.kind == oracle.TIES else 0
         of = oracle_family(fam, base, experts, trim_scope=scope)
+        o_norm, o_max, o_nnz = oracle.index(of)
+        tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
         idx = mp.mp_index_blocks(mf, gop)
-        tau = mp.mp_index_stats(idx)[3] if oop.kind == oracle.TIES else None
         for f in fracs:
             B = mp.mp_budget_from_fraction(mf, f)
             plan = mp.mp_plan(idx, gop, B)
             pi = mp.mp_plan_info(plan, idx)
             what = f"{fam.name}/{name}/f={f}"
-            touched = touched_elements(fam, pi["mask"])
-            want = oracle.merge(of, oop, tau=tau, mask=pi["mask"])
+            opl = oracle.plan(fam.K, bl, of.blk_group, of.n_groups, fam.elem_size, oop, o_norm, o_max, o_nnz, tau, B)
+            assert pi["digest"] == opl["digest"] and np.array_equal(pi["mask"], opl["mask"]), what
+            touched = touched_elements(fam, opl["mask"])
+            want = oracle.merge(of, oop, tau=tau, mask=opl["mask"])
 
             out = sentinel_like(b)
             before = host(fam, out).copy()
             man = mp.mp_merge_touched(mf, idx, plan, out)
             mi = mp.mp_manifest_info(man, fam.K)
-            assert mi["realized_total"] == pi["chat"] <= B, what
-            assert mi["touched"] == int((pi["mask"] != 0).sum()), what
+            assert mi["realized_total"] == opl["chat"] <= B, what
+            assert mi["touched"] == int((opl["mask"] != 0).sum()), what
             got = host(fam, out)
             assert_merge_close(fam, got[touched], want[touched], what)
             assert np.array_equal(got[~touched].view(np.uint8), before[~touched].view(np.uint8)), what
