@@ -55,15 +55,17 @@ constexpr bool kAddGeo = OPC == OP_ADD || OPC == OP_RENORM;
 
 // slot geometry per operator.  The additive merges are bound by HBM: two CTAs per SM with a
 // 96 KiB ring each (two 16-byte vectors per consumer thread and fill).  TIES, DARE and
-// DARE-TIES spend more arithmetic per byte: three CTAs per SM (more warps to hide it; measured
-// better than fewer consumer threads with more work each) with a 64 KiB ring of 4 KiB slots
-// (one vector per consumer thread and fill, so that their state fits the register budget).
+// DARE-TIES spend more arithmetic per byte, so they run more warps per SM to hide latency
+// (measured better than fewer consumer threads with more work each), with 4 KiB slots (one
+// vector per consumer thread and fill, so that their state fits the register budget): TIES
+// and DARE four CTAs per SM with a 44 KiB ring (their state fits 56 registers), DARE-TIES
+// three with a 64 KiB ring (it would spill at 56).
 template <int OPC>
 struct Geo {
   static constexpr int kConsumers = 256;
   static constexpr int kThreads = kConsumers + 32;  // + one producer warp
-  static constexpr int kCtasPerSm = kAddGeo<OPC> ? 2 : 3;
-  static constexpr uint32_t kRingBytes = kAddGeo<OPC> ? 98304u : 65536u;
+  static constexpr int kCtasPerSm = kAddGeo<OPC> ? 2 : (OPC == OP_DTIES ? 3 : 4);
+  static constexpr uint32_t kRingBytes = kAddGeo<OPC> ? 98304u : (OPC == OP_DTIES ? 65536u : 45056u);
   static constexpr uint32_t kSlotBytes = kAddGeo<OPC> ? 8192u : 4096u;  // one chunk of one checkpoint
   static constexpr int kSlots = (int)(kRingBytes / kSlotBytes);
   static constexpr uint32_t kGrab = 8;  // chunks taken per counter increment (<= 32)
