@@ -86,13 +86,14 @@ constexpr uint32_t kIxEnd = 0xFFFFFFFFu;
 
 // ring geometry.  The plain catalog is bound by HBM: two CTAs per SM with twelve 8 KiB
 // slots.  The TIES catalog also bins every delta, which makes it bound by instruction
-// latency: three CTAs per SM (more warps to hide it) with sixteen 4 KiB slots (one vector
-// per consumer thread and fill, so that the state fits the smaller register budget).
+// latency: four CTAs per SM (more warps to hide it; the state fits 56 registers) with twelve
+// 4 KiB slots (one vector per consumer thread and fill).  With eight experts per item the
+// histograms make a CTA too large for four per SM, and three run.
 template <bool TIES>
 struct IxGeo {
-  static constexpr int kCtasPerSm = TIES ? 3 : 2;
+  static constexpr int kCtasPerSm = TIES ? 4 : 2;
   static constexpr uint32_t kSlotBytes = TIES ? 4096u : 8192u;
-  static constexpr int kSlots = TIES ? 16 : 12;
+  static constexpr int kSlots = 12;
 };
 
 struct IxMeta {
