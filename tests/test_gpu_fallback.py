@@ -215,3 +215,39 @@ def test_fallback_with_a_host_resident_pool():
             plan.free()
         imp_h.free()
         idx.free()
+
+
+def test_fallback_plan_with_touched_only_merge():
+    """a fallback plan merged with mp_merge_touched: touched blocks (whole fallback tensors
+    among them) equal the oracle's merge, every other byte keeps the sentinel"""
+    fam = fam_many_blocks()
+    base, experts = fam.host_arrays()
+    mf, b, ex = upload(fam, base, experts)
+    bo, bl, bt = fam.block_table()
+    of = oracle_family(fam, base, experts)
+    norm, maxabs, nnz = oracle.index(of)
+    nz = nnz.copy()
+    nz[missing_patterns(fam, fam.K, np.random.default_rng(11))["whole-tensor"]] = MISS
+    gop = mp.make_op(mp.MP_OP_TA, alpha=[0.3] * fam.K)
+    oop = oracle.Op(oracle.TA, fam.K, alpha=[0.3] * fam.K)
+    imp = mp.mp_index_import(mf, gop, norm, maxabs, nz)
+    for f in (0.2, 0.6):
+        B = mp.mp_budget_from_fraction(mf, f)
+        plan = mp.mp_plan(imp, gop, B)
+        opl = oracle.plan(fam.K, bl, of.blk_group, of.n_groups, fam.elem_size, oop, norm, maxabs, nz, None, B,
+                          blk_tensor=bt)
+        assert np.array_equal(mp.mp_plan_info(plan, imp)["mask"], opl["mask"]), f
+        out = torch.empty_like(b)
+        out.view(torch.uint8).fill_(0x5A)
+        man = mp.mp_merge_touched(mf, imp, plan, out)
+        assert mp.mp_manifest_info(man, fam.K)["touched"] == int((opl["mask"] != 0).sum())
+        got = host(fam, out)
+        want = oracle.merge(of, oop, mask=opl["mask"])
+        touched = np.zeros(got.size, bool)
+        for blk in np.nonzero(opl["mask"])[0].tolist():
+            touched[int(bo[blk]):int(bo[blk] + bl[blk])] = True
+        assert_merge_close(fam, got[touched], want[touched], f"touched/f={f}")
+        assert bool((got[~touched].view(np.uint8) == 0x5A).all())
+        man.free()
+        plan.free()
+    imp.free()
