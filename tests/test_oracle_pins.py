@@ -885,3 +885,20 @@ def test_index_hashes_are_content_addressed(tiny_family):
         assert bh[b] == oracle.block_hash(base[s].tobytes())
         assert eh[1, b] == oracle.block_hash(experts[1][s].tobytes())
     assert len(set(bh.tolist())) > fam.n_blocks // 2
+
+
+def test_avg_single_expert_unit_weight_reproduces_the_expert():
+    """K = 1, AVG with alpha = 1: out = round(M_0 + (M_1 - M_0)) is M_1 itself wherever the
+    fp32 delta is exact (checked against fp64), bit for bit, masked-in; masked out it is M_0"""
+    rng = np.random.default_rng(51)
+    n = 5000
+    base = to_bf16(rng.standard_normal(n) * 0.02)
+    ex = to_bf16(bf16_to_f32(base) + (rng.standard_normal(n) * 1e-3).astype(np.float32))
+    b64, e64 = bf16_to_f32(base).astype(np.float64), bf16_to_f32(ex).astype(np.float64)
+    exact = (bf16_to_f32(ex) - bf16_to_f32(base)).astype(np.float64) == e64 - b64
+    assert exact.mean() > 0.99
+    op = oracle.Op(oracle.AVG, 1, alpha=[1.0])
+    out = oracle.merge_block(oracle.BF16, 0, base, [ex], 1, op)
+    assert np.array_equal(out[exact], ex[exact])
+    out0 = oracle.merge_block(oracle.BF16, 0, base, [ex], 0, op)
+    assert np.array_equal(out0.view(np.uint16) & 0x7FFF, base.view(np.uint16) & 0x7FFF)
