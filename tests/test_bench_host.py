@@ -1,0 +1,46 @@
+"""Host logic of bench.py that needs no GPU: the affine read-time model fit and the seeded
+pattern of catalog entries without statistics."""
+import math
+import os
+import sys
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+sys.path.insert(0, ROOT)
+
+
+def test_time_model_fit_recovers_an_affine_model():
+    """merge times generated from T(f) = a + b f are fitted back exactly (r^2 = 1), and the
+    model's slope and intercept follow from C_full, 2 N s and the bandwidth"""
+    import bench
+
+    c_full, ckpt = 8_000_000_000, 1_000_000_000
+    a, b = 0.31, 1.07
+    per = [{"planned_bytes": int(f * c_full), "merge_ms": a + b * f} for f in (1.0, 0.5, 0.25, 0.1)]
+    fit = bench.time_model_fit([1.0, 0.5, 0.25, 0.1], per, ckpt, c_full, 6800.0, False)
+    assert math.isclose(fit["slope_ms"], b, rel_tol=1e-9) and math.isclose(fit["intercept_ms"], a, rel_tol=1e-9)
+    assert math.isclose(fit["r2"], 1.0, rel_tol=1e-12)
+    assert math.isclose(fit["model_slope_ms"], c_full / 6800e9 * 1e3)
+    assert math.isclose(fit["model_intercept_ms"], 2 * ckpt / 6800e9 * 1e3)
+    assert math.isclose(fit["bw_from_slope_gbs"], c_full / (b / 1e3) / 1e9)
+    # the touched-only merge has no fixed 2 N s term; one budget gives no line
+    assert bench.time_model_fit([1.0, 0.5], per[:2], ckpt, c_full, 6800.0, True)["model_intercept_ms"] is None
+    assert bench.time_model_fit([1.0], per[:1], ckpt, c_full, 6800.0, False) is None
+
+
+def test_missing_entries_pattern_is_seeded_and_pair_dominated():
+    """the same pattern on every call; the largest tensor of expert 0 is missing whole; every
+    tensor with a missing pair is missing for all its blocks of that expert"""
+    from paper_2605_29489_gb300 import synth
+
+    fam = synth.qwen25_05b(layers=2)
+    a = synth.missing_entries(fam, fam.K)
+    b = synth.missing_entries(fam, fam.K)
+    assert a.shape == (fam.K, fam.n_blocks) and np.array_equal(a, b)
+    _, _, bt = fam.block_table()
+    big = int(np.argmax(np.bincount(bt)))
+    assert a[0, bt == big].all()
+    c = synth.missing_entries(fam, fam.K, pair_frac=0.0, entry_frac=0.0)
+    assert c.sum() == int((bt == big).sum())     # only the forced pair
+    assert 0.0 < a.mean() < 0.5
