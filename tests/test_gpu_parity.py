@@ -198,6 +198,18 @@ def fam_k32():
                         per_expert_active=True, name="k32")
 
 
+def fam_big_blocks():
+    # 4 Mi-element blocks (a whole block is thousands of chunks), ragged tails, K = 2
+    return synth.custom([(1 << 22) + (1 << 20) + 5, 3000, 1 << 22], dtype=synth.BF16, block_elems=1 << 22, K=2,
+                        active_frac=0.7, name="big-blocks")
+
+
+def fam_max_block():
+    # the largest block the ABI allows (2^24 elements), one expert, fp32
+    return synth.custom([(1 << 24) + 12], dtype=synth.F32, block_elems=1 << 24, K=1, active_frac=1.0, name="max-block",
+                        log_mu=math.log(1e-3))
+
+
 FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 
 
@@ -208,6 +220,15 @@ def test_parity_small_families(make):
     base, experts = fam.host_arrays()
     run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb", "avg_renorm", "dare_ties"),
              FRACS)
+
+
+@pytest.mark.parametrize("make", [fam_big_blocks, fam_max_block], ids=lambda f: f.__name__)
+def test_parity_largest_blocks(make):
+    """blocks of 2^22 and 2^24 elements: the canonical norm order over thousands of chunks,
+    TIES thresholds and DARE masks at block offsets beyond 2^24"""
+    fam = make()
+    base, experts = fam.host_arrays()
+    run_case(fam, base, experts, ("avg", "ta", "ties", "dare", "ta_pb"), [0.3, 0.6, 1.0])
 
 
 def test_parity_tiny_config():
