@@ -96,3 +96,39 @@ def test_noalloc_rejects_requests_beyond_the_static_limit():
         mp.mp_plan_noalloc(2, 1 << 19, 1, mp.MP_BF16, t, t, t, t, t, None, t, op, 100, t, t, t)
     assert ei.value.status == -1
     assert "524288" in str(ei.value)
+
+
+def test_noalloc_plan_at_the_static_limit_matches_oracle():
+    """exactly K * n_blocks = 524288 units (K = 32, 16384 blocks of mixed lengths) from a
+    seeded synthetic catalog: the plan equals the oracle's bit for bit"""
+    import oracle
+
+    K, nb = 32, 1 << 14
+    rng = np.random.default_rng(77)
+    blk_len = rng.choice([4096, 4096, 4096, 1000, 7], nb).astype(np.uint32)
+    norm = rng.lognormal(size=(K, nb)).astype(np.float32)
+    norm[:, ::5] = norm[:, 1::5][:, : norm[:, ::5].shape[1]]       # equal scores: the tie-break decides
+    maxabs = norm.copy()
+    nnz = np.minimum(rng.integers(0, 5000, (K, nb)), blk_len[None, :]).astype(np.uint32)
+    nnz[rng.random((K, nb)) < 0.1] = 0
+    alpha = [0.1 + 0.01 * i for i in range(K)]
+    gop = mp.make_op(mp.MP_OP_TA, alpha=alpha)
+    oop = oracle.Op(oracle.TA, K, alpha=alpha)
+    d_len, d_norm, d_max, d_nnz = _dev(blk_len, np.int32), _dev(norm, np.float32), _dev(maxabs, np.float32), \
+        _dev(nnz, np.int32)
+    d_err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    mask = torch.empty(nb, dtype=torch.int32, device="cuda")
+    order = torch.empty(K * nb, dtype=torch.int32, device="cuda")
+    summary = torch.empty(8, dtype=torch.int64, device="cuda")
+    full = K * int(blk_len.sum()) * 2
+    for f in (0.05, 0.5):
+        B = int(f * full)
+        mp.mp_plan_noalloc(K, nb, 1, mp.MP_BF16, d_len, None, d_norm, d_max, d_nnz, None, d_err, gop, B, mask,
+                           order, summary)
+        torch.cuda.synchronize()
+        opl = oracle.plan(K, blk_len, np.zeros(nb, np.uint32), 1, 2, oop, norm, maxabs, nnz, None, B)
+        s = summary.cpu().numpy().view(np.uint64)
+        assert (int(s[0]), int(s[1]), int(s[2]), int(s[4])) == (opl["chat"], opl["n_sel"], opl["n_cand"],
+                                                                opl["digest"]), f
+        assert np.array_equal(mask.cpu().numpy().view(np.uint32), opl["mask"]), f
+        assert np.array_equal(order.cpu().numpy().view(np.uint32)[: opl["n_cand"]], opl["order"]), f
