@@ -62,6 +62,10 @@ def workloads():
                                             "per-expert active sets"),
         "qwen2.5-1.5b-dare-2l": dict(make=lambda: synth.qwen25_15b(layers=2), op="dare", drop_p=0.9, budgets=[0.25],
                                      desc="Qwen2.5-1.5B shapes cut to 2 layers (profiling case), K=16, DARE p=0.9"),
+        "qwen2.5-1.5b-dare-ties-2l": dict(make=lambda: synth.qwen25_15b(layers=2), op="dare_ties", drop_p=0.9,
+                                          budgets=[0.25],
+                                          desc="Qwen2.5-1.5B shapes cut to 2 layers (profiling case), K=16, DARE-TIES "
+                                               "p=0.9"),
         "llama-3-8b-hostpool-avg": dict(make=lambda: synth.llama3_8b(K=8), op="avg", budgets=[1.0, 0.25, 0.1],
                                         host_pool=True,
                                         desc="Llama-3-8B-shaped bf16 base in HBM, K=8 experts (128 GB) in pinned host "
