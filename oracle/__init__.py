@@ -17,7 +17,7 @@ import numpy as np
 from . import build as _build
 
 BF16, F32 = 0, 1
-AVG, TA, TIES, DARE, AVG_RENORM, DARE_TIES = 0, 1, 2, 3, 4, 5
+AVG, TA, TIES, DARE, AVG_RENORM, DARE_TIES, TIES_MASKED = 0, 1, 2, 3, 4, 5, 6
 OK, EINVAL, EOOM, ENONFINITE = 0, -1, -3, -4
 TAU_NONE = 0x8000
 NNZ_MISSING = 0xFFFFFFFF  # catalog entry without block statistics (tensor-level fallback)
@@ -54,6 +54,7 @@ def lib():
         L.orc_tau_from_hist.restype = u32
         L.orc_tau_from_hist.argtypes = [vp, u64, ctypes.c_float]
         L.orc_ties_thresholds.argtypes = [vp, ctypes.c_float, vp]
+        L.orc_ties_masked_thresholds.argtypes = [vp, ctypes.c_float, vp, vp]
         L.orc_plan.argtypes = [u32, u64, vp, vp, u32, u32, vp, vp, vp, vp, vp, u64, vp, vp, vp, vp, vp, vp, vp, vp, u32]
         L.orc_merge_block.argtypes = [ctypes.c_int, u64, u64, vp, vp, u32, u32, vp, vp, vp]
         L.orc_merge.argtypes = [vp, vp, vp, vp, vp, vp]
@@ -182,6 +183,15 @@ def ties_thresholds(fam: Family, density):
     tau = np.zeros((fam.K, fam.n_groups), np.uint32)
     c = fam.c()
     _check(lib().orc_ties_thresholds(ctypes.byref(c), ctypes.c_float(density), _p(tau)))
+    return tau
+
+
+def ties_masked_thresholds(fam: Family, density, mask):
+    """TIES after masking: thresholds of the zero-completed masked deltas [K, n_groups]"""
+    tau = np.zeros((fam.K, fam.n_groups), np.uint32)
+    m = np.ascontiguousarray(mask, np.uint32)
+    c = fam.c()
+    _check(lib().orc_ties_masked_thresholds(ctypes.byref(c), ctypes.c_float(density), _p(m), _p(tau)))
     return tau
 
 

@@ -207,6 +207,41 @@ int orc_ties_thresholds(const orc_family* f, float density, uint32_t* tau) {
   return rc;
 }
 
+/* TIES after masking (App. A.1: TIES trims, elects signs and averages sign-consistent
+ * entries after masking).  Reading: the trim threshold of each (expert, group) is that of
+ * the zero-completed masked deltas A_i Delta_i: the k-th largest key, k = floor(density *
+ * numel_group), over the entries of the selected blocks together with a zero (key 0) for
+ * every entry of an unselected block.  With every block selected it is orc_ties_thresholds.
+ * mask: the access mask, one word per block (bit i = expert i). */
+int orc_ties_masked_thresholds(const orc_family* f, float density, const uint32_t* mask, uint32_t* tau) {
+  if (!f || !tau || !mask || f->n_groups == 0) return ORC_EINVAL;
+  uint64_t* hist = (uint64_t*)calloc((size_t)f->n_groups * 32768u, sizeof(uint64_t));
+  uint64_t* numel = (uint64_t*)calloc(f->n_groups, sizeof(uint64_t));
+  if (!hist || !numel) {
+    free(hist);
+    free(numel);
+    return ORC_EOOM;
+  }
+  for (uint64_t b = 0; b < f->n_blocks; ++b) numel[f->blk_group[b]] += f->blk_len[b];
+  int rc = ORC_OK;
+  for (uint32_t i = 0; i < f->K && rc == ORC_OK; ++i) {
+    memset(hist, 0, (size_t)f->n_groups * 32768u * sizeof(uint64_t));
+    for (uint64_t b = 0; b < f->n_blocks && rc == ORC_OK; ++b) {
+      uint64_t* h = hist + (size_t)f->blk_group[b] * 32768u;
+      if ((mask[b] >> i) & 1u)
+        rc = orc_key_hist(f->dtype, f->blk_len[b], elem_ptr(f->dtype, f->base, f->blk_off[b]),
+                          elem_ptr(f->dtype, f->experts[i], f->blk_off[b]), h);
+      else
+        h[0] += f->blk_len[b]; /* omitted: zero entries, key 0, never read */
+    }
+    for (uint32_t g = 0; g < f->n_groups && rc == ORC_OK; ++g)
+      tau[(size_t)i * f->n_groups + g] = orc_tau_from_hist(hist + (size_t)g * 32768u, numel[g], density);
+  }
+  free(hist);
+  free(numel);
+  return rc;
+}
+
 /* ---------------------------------------------------------------------------------------
  * Hashes.  FNV-1a 64 (Fowler, Noll, Vo): offset basis 14695981039346656037, prime
  * 1099511628211.  SplitMix64 output function (Steele, Lea, Flood, OOPSLA 2014).
@@ -343,7 +378,8 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
              uint32_t n_tensors) {
   if (!op || K == 0 || K > 32 || op->K != K || !norm || !maxabs || !nnz || !mask) return ORC_EINVAL;
   if (op->kind == ORC_TIES && (!tau || !blk_group)) return ORC_EINVAL;
-  if (op->kind != ORC_TIES && op->kind != ORC_DARE_TIES && !op->alpha) return ORC_EINVAL;
+  if (op->kind != ORC_TIES && op->kind != ORC_DARE_TIES && op->kind != ORC_TIES_MASKED && !op->alpha)
+    return ORC_EINVAL;
   if (n_blocks * K > 0xFFFFFFFFull) return ORC_EINVAL;
   if (blk_tensor) /* tensors in checkpoint order: the blocks of a tensor are contiguous */
     for (uint64_t b = 0; b < n_blocks; ++b)
@@ -371,7 +407,8 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
   for (uint64_t b = 0; b < n_blocks; ++b) {
     for (uint32_t i = 0; i < K; ++i) {
       uint64_t s = (uint64_t)i * n_blocks + b;
-      float coef = (op->kind == ORC_TIES || op->kind == ORC_DARE_TIES) ? op->lambda : op->alpha[i];
+      float coef = (op->kind == ORC_TIES || op->kind == ORC_DARE_TIES || op->kind == ORC_TIES_MASKED) ? op->lambda
+                                                                                                    : op->alpha[i];
       if (fb && fb[(size_t)i * n_tensors + blk_tensor[b]]) {
         const uint32_t t = blk_tensor[b];
         if (b > 0 && blk_tensor[b - 1] == t) continue; /* only the tensor's first block */
@@ -519,6 +556,8 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  *        are selected or whose delta block is exactly zero (ascending fp32 adds from +0);
  *        beta_i = alpha_i / s;
  *        acc = sum_i fma(beta_i, A_i delta_i, acc); out = round(M_0 + acc)
+ *  TIES after masking: as TIES, with tau the threshold of the masked deltas
+ *        (orc_ties_masked_thresholds)
  *  DARE-TIES: DARE's drop and rescale with the same mask omega, then TIES's election and
  *        disjoint mean without magnitude trimming: d^_i = A_i (keep_i ? delta_i * sigma : 0),
  *        then P, N, gamma, m and out as TIES
@@ -534,8 +573,9 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
   const uint32_t K = op->K;
   for (uint32_t i = 0; i < K; ++i)
     if (((mask >> i) & 1u) && !experts[i]) return ORC_EINVAL;
-  const int ties_like = op->kind == ORC_TIES || op->kind == ORC_DARE_TIES;
-  if (op->kind == ORC_TIES && !tau_k) return ORC_EINVAL;
+  const int ties_like = op->kind == ORC_TIES || op->kind == ORC_DARE_TIES || op->kind == ORC_TIES_MASKED;
+  const int trims = op->kind == ORC_TIES || op->kind == ORC_TIES_MASKED;
+  if (trims && !tau_k) return ORC_EINVAL;
   if (!ties_like && !op->alpha) return ORC_EINVAL;
   float sigma = op->drop_p < 1.0 ? (float)(1.0 / (1.0 - op->drop_p)) : 0.0f;
   /* renormalised AVG: the sum, ascending, of the coefficients of the experts that take part:
@@ -561,7 +601,7 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
         float dh = 0.0f;
         if ((mask >> i) & 1u) {
           float d = load_elem(dtype, experts[i], k) - x0;
-          if (op->kind == ORC_TIES) {
+          if (trims) {
             if (orc_ties_key(d) >= tau_k[i]) dh = d;
           } else if (orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) {
             dh = d * sigma;
@@ -611,7 +651,7 @@ int orc_merge(const orc_family* f, const orc_op* op, const uint32_t* tau, const 
     uint64_t off = f->blk_off[b];
     for (uint32_t i = 0; i < f->K; ++i) {
       ex[i] = elem_ptr(f->dtype, f->experts[i], off);
-      if (op->kind == ORC_TIES) tau_k[i] = tau[(size_t)i * f->n_groups + f->blk_group[b]];
+      if (op->kind == ORC_TIES || op->kind == ORC_TIES_MASKED) tau_k[i] = tau[(size_t)i * f->n_groups + f->blk_group[b]];
     }
     uint32_t known_zero = 0;
     if (op->kind == ORC_AVG_RENORM && nnz) {

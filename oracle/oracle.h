@@ -24,14 +24,14 @@ extern "C" {
 #endif
 
 enum { ORC_BF16 = 0, ORC_F32 = 1 };
-enum { ORC_AVG = 0, ORC_TA = 1, ORC_TIES = 2, ORC_DARE = 3, ORC_AVG_RENORM = 4, ORC_DARE_TIES = 5 };
+enum { ORC_AVG = 0, ORC_TA = 1, ORC_TIES = 2, ORC_DARE = 3, ORC_AVG_RENORM = 4, ORC_DARE_TIES = 5, ORC_TIES_MASKED = 6 };
 enum { ORC_OK = 0, ORC_EINVAL = -1, ORC_EOOM = -3, ORC_ENONFINITE = -4 };
 #define ORC_TAU_NONE 0x8000u /* TIES threshold when k = 0: no 15-bit key reaches it */
 #define ORC_NNZ_MISSING 0xFFFFFFFFu /* catalog entry without block statistics (tensor-level fallback) */
 
 /* merge operator and its parameters theta (Alg. 1 records op and theta) */
 typedef struct {
-  int kind;            /* ORC_AVG / ORC_TA / ORC_TIES / ORC_DARE / ORC_AVG_RENORM / ORC_DARE_TIES */
+  int kind;            /* ORC_AVG / ORC_TA / ORC_TIES / ORC_DARE / ORC_AVG_RENORM / ORC_DARE_TIES / ORC_TIES_MASKED */
   uint32_t K;          /* number of experts */
   const float* alpha;  /* K coefficients (AVG, TA, DARE); may be NULL for TIES */
   float lambda;        /* TIES: scale of the merged task vector */
@@ -70,6 +70,8 @@ int orc_index(const orc_family* f, float* norm, float* maxabs, uint32_t* nnz);
 int orc_key_hist(int dtype, uint64_t n, const void* base, const void* expert, uint64_t* hist32768);
 uint32_t orc_tau_from_hist(const uint64_t* hist32768, uint64_t numel, float density);
 int orc_ties_thresholds(const orc_family* f, float density, uint32_t* tau);
+/* thresholds of the zero-completed masked deltas (TIES after masking) */
+int orc_ties_masked_thresholds(const orc_family* f, float density, const uint32_t* mask, uint32_t* tau);
 
 /* Alg. 1 PlanGen */
 int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint32_t* blk_group,

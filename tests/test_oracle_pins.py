@@ -902,3 +902,47 @@ def test_avg_single_expert_unit_weight_reproduces_the_expert():
     assert np.array_equal(out[exact], ex[exact])
     out0 = oracle.merge_block(oracle.BF16, 0, base, [ex], 0, op)
     assert np.array_equal(out0.view(np.uint16) & 0x7FFF, base.view(np.uint16) & 0x7FFF)
+
+
+# ---- TIES after masking (App. A.1) ----------------------------------------------------------------------
+
+def test_ties_masked_thresholds_brute_force(tiny_family):
+    """the threshold of the zero-completed masked deltas is the k-th largest key when every
+    entry of an unselected block counts as a zero (sorted directly in numpy from the
+    deltas' bf16 keys); the full mask gives the ordinary thresholds, the empty mask keys 0"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    bo, bl, bt = fam.block_table()
+    rng = np.random.default_rng(61)
+    for density in (0.05, 0.2, 0.6):
+        full = oracle.ties_thresholds(of, density)
+        assert np.array_equal(oracle.ties_masked_thresholds(of, density, np.full(fam.n_blocks, 0xF, np.uint32)), full)
+        for trial in range(2):
+            mask = rng.integers(0, 16, fam.n_blocks).astype(np.uint32)
+            got = oracle.ties_masked_thresholds(of, density, mask)
+            for i in range(fam.K):
+                d = experts[i].astype(np.float32) - base.astype(np.float32)
+                keys = bf16_bits_torch(np.abs(d)).astype(np.int64) & 0x7FFF
+                for t in range(len(fam.tensors)):
+                    parts = []
+                    for b in np.nonzero(bt == t)[0]:
+                        s_ = slice(int(bo[b]), int(bo[b] + bl[b]))
+                        parts.append(keys[s_] if (mask[b] >> i) & 1 else np.zeros(int(bl[b]), np.int64))
+                    allk = np.sort(np.concatenate(parts))[::-1]
+                    k = int(math.floor(density * allk.size))
+                    want = oracle.TAU_NONE if k == 0 else int(allk[k - 1])
+                    assert got[i, t] == want, (density, i, t)
+        zero = oracle.ties_masked_thresholds(of, density, np.zeros(fam.n_blocks, np.uint32))
+        assert (zero == 0).all()
+
+
+def test_ties_masked_full_mask_merges_like_ties(tiny_family):
+    """with every block selected the masked operator is standard TIES (Eq. 5)"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    full_mask = np.full(fam.n_blocks, 0xF, np.uint32)
+    tau = oracle.ties_thresholds(of, 0.2)
+    tm = oracle.ties_masked_thresholds(of, 0.2, full_mask)
+    a = oracle.merge(of, oracle.Op(oracle.TIES, fam.K, lam=1.0, density=0.2), tau=tau, mask=full_mask)
+    b = oracle.merge(of, oracle.Op(oracle.TIES_MASKED, fam.K, lam=1.0, density=0.2), tau=tm, mask=full_mask)
+    assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
