@@ -66,14 +66,19 @@ typedef enum { MP_BF16 = 0, MP_F32 = 1 } mp_dtype;
    experts), 0 for an omitted expert (the coefficient-drift bound of App. A.1 applies, not
    Prop. 2); every alpha_i must be > 0.  DARE_TIES drops and rescales like DARE (same
    mask omega), then elects signs and takes the disjoint mean like TIES, without the
-   magnitude trim (lambda, drop_p and seed are used; no tau). */
+   magnitude trim (lambda, drop_p and seed are used; no tau).  TIES_MASKED is TIES applied
+   after masking (App. A.1): its trim threshold is that of the zero-completed masked
+   deltas A_i Delta_i (the k-th largest key, k = floor(density * numel) of the group, an
+   omitted entry counting as a zero), so it depends on the plan; lambda, density and
+   trim_scope are used.  With every block selected it is TIES. */
 typedef enum {
   MP_OP_AVG = 0,
   MP_OP_TA = 1,
   MP_OP_TIES = 2,
   MP_OP_DARE = 3,
   MP_OP_AVG_RENORM = 4,
-  MP_OP_DARE_TIES = 5
+  MP_OP_DARE_TIES = 5,
+  MP_OP_TIES_MASKED = 6
 } mp_op_kind;
 
 /* One tensor of the tensor set T (Sec. 2), as a span of the flat checkpoint buffers. */
@@ -220,6 +225,11 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
  */
 mp_status mp_merge(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out,
                    mp_stream stream, mp_manifest** man);
+/* (TIES_MASKED, in mp_merge and mp_merge_touched: before the merge the threshold of the
+   masked deltas is found from the catalog's per-block coarse key histograms of the selected
+   blocks and one pass over the selected expert blocks that can hold keys in its coarse bin;
+   those expert bytes are reported by mp_manifest_threshold_reads, apart from the planned
+   reads the budget bounds.) */
 
 /*
  * mp_merge_touched — Alg. 2 with WriteBlockOrReference: only the touched blocks (at least
@@ -313,6 +323,11 @@ mp_status mp_manifest_validate(const mp_family* family, const mp_index* index, c
    (the message names the first one), MP_ERR_INVALID_ARG if the manifest was not
    validated. */
 mp_status mp_manifest_validation(const mp_manifest* man, uint64_t* checked, uint64_t* mismatched, uint64_t* out_hash);
+
+/* Expert bytes read to find the TIES_MASKED threshold (0 for every other operator): a
+   subset of the selected blocks read a second time, reported apart from the realized reads
+   that the budget bounds.  Waits for the merge. */
+mp_status mp_manifest_threshold_reads(const mp_manifest* man, uint64_t* bytes);
 
 /* The manifest's lineage (Sec. 3: the manifest records lineage): the K + 1 caller ids of
    M_0..M_K given in mp_family.lineage_ids at merge time, copied into ids[0..K] (all zero

@@ -21,7 +21,8 @@ import os
 import numpy as np
 
 __all__ = [
-    "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES", "MergePipeError",
+    "MP_OK", "MP_BF16", "MP_F32", "MP_OP_AVG", "MP_OP_TA", "MP_OP_TIES", "MP_OP_DARE", "MP_OP_AVG_RENORM", "MP_OP_DARE_TIES",
+    "MP_OP_TIES_MASKED", "mp_manifest_threshold_reads", "MergePipeError",
     "family", "make_op", "mp_index_blocks", "mp_plan", "mp_merge", "mp_merge_touched", "mp_free", "mp_index_stats",
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_manifest_lineage", "mp_budget_from_fraction", "mp_last_error",
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "mp_index_hashes",
@@ -33,7 +34,7 @@ MP_OK = 0
 MP_ERR = {-1: "MP_ERR_INVALID_ARG", -2: "MP_ERR_CUDA", -3: "MP_ERR_OOM", -4: "MP_ERR_NONFINITE",
           -5: "MP_ERR_BUDGET", -6: "MP_ERR_TIMEOUT", -7: "MP_ERR_UNSUPPORTED", -8: "MP_ERR_MISMATCH"}
 MP_BF16, MP_F32 = 0, 1
-MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES = 0, 1, 2, 3, 4, 5
+MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES, MP_OP_TIES_MASKED = 0, 1, 2, 3, 4, 5, 6
 MP_NNZ_MISSING = 0xFFFFFFFF   # catalog entry without block statistics (tensor-level fallback)
 
 
@@ -89,6 +90,7 @@ def lib():
             ("mp_plan_info", [vp, vp, vp, vp, vp, vp, vp]),
             ("mp_manifest_info", [vp, vp, vp, vp, vp]),
             ("mp_manifest_lineage", [vp, vp]),
+            ("mp_manifest_threshold_reads", [vp, vp]),
         ]:
             f = getattr(L, name)
             f.restype, f.argtypes = st, args
@@ -230,6 +232,13 @@ def mp_index_hash_values(index: Handle):
     eh = np.zeros((nu // nb, nb), np.uint64)
     _check(lib().mp_index_hash_values(ctypes.c_void_p(index.ptr), bh.ctypes.data, eh.ctypes.data))
     return bh, eh
+
+
+def mp_manifest_threshold_reads(man: Handle) -> int:
+    """expert bytes read to find a TIES_MASKED threshold (0 for other operators)"""
+    v = ctypes.c_uint64()
+    _check(lib().mp_manifest_threshold_reads(ctypes.c_void_p(man.ptr), ctypes.byref(v)))
+    return v.value
 
 
 def mp_manifest_validate(fam: Family, index: Handle, plan: Handle, out, man: Handle, stream=None):

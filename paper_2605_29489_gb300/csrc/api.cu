@@ -163,8 +163,8 @@ mp_status resolve_pointers(const mp_family* f, const void*& base, ExpertPtrs& ex
 
 mp_status check_op(const mp_op* op, uint32_t K) {
   if (!op) return fail(MP_ERR_INVALID_ARG, "op is NULL");
-  if (op->kind < MP_OP_AVG || op->kind > MP_OP_DARE_TIES) return fail(MP_ERR_INVALID_ARG, "unknown operator kind");
-  if (op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES) {
+  if (op->kind < MP_OP_AVG || op->kind > MP_OP_TIES_MASKED) return fail(MP_ERR_INVALID_ARG, "unknown operator kind");
+  if (op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES || op->kind == MP_OP_TIES_MASKED) {
     if (!isfinite(op->lambda)) return fail(MP_ERR_INVALID_ARG, "lambda must be finite");
   } else {
     if (!op->alpha) return fail(MP_ERR_INVALID_ARG, "alpha is required for AVG, TA, DARE and AVG_RENORM");
@@ -174,7 +174,7 @@ mp_status check_op(const mp_op* op, uint32_t K) {
       for (uint32_t i = 0; i < K; ++i)
         if (!(op->alpha[i] > 0.0f)) return fail(MP_ERR_INVALID_ARG, "AVG_RENORM needs every alpha > 0");
   }
-  if (op->kind == MP_OP_TIES) {
+  if (op->kind == MP_OP_TIES || op->kind == MP_OP_TIES_MASKED) {
     if (!(op->density >= 0.0f && op->density <= 1.0f)) return fail(MP_ERR_INVALID_ARG, "density must be in [0, 1]");
     if (op->trim_scope > 1) return fail(MP_ERR_INVALID_ARG, "trim_scope must be 0 or 1");
   }
@@ -419,7 +419,8 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
 // table is uploaded and the error word and tau cleared on cs.
 mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t work_bytes, cudaStream_t cs,
                     mp_index_s** out, char** work) {
-  const bool ties = op && op->kind == MP_OP_TIES;
+  const bool ties = op && (op->kind == MP_OP_TIES || op->kind == MP_OP_TIES_MASKED);
+  const bool masked = op && op->kind == MP_OP_TIES_MASKED;
   const uint32_t scope = ties ? op->trim_scope : 0u;
   const uint32_t n_groups = scope == 0 ? g.n_tensors : 1u;
   const uint64_t nb = g.n_blocks, U = nb * g.K, KG = (uint64_t)g.K * n_groups;
@@ -444,6 +445,7 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
   const size_t o_tb0 = slot(((size_t)g.n_tensors + 1) * 4);
   const size_t o_norm = slot(U * 4), o_max = slot(U * 4), o_nnz = slot(U * 4), o_tau = slot(KG * 4);
   const size_t o_err = slot(16);
+  const size_t o_uh = slot(masked ? U * 256 * 4 : 0);
   const size_t o_work = slot(work_bytes);
   mp_index_s* ix = new (std::nothrow) mp_index_s();
   if (!ix) return fail(MP_ERR_OOM, "host allocation failed");
@@ -473,6 +475,7 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
   ix->d_nnz = (uint32_t*)(m + o_nnz);
   ix->d_tau = (uint32_t*)(m + o_tau);
   ix->d_err = (uint32_t*)(m + o_err);
+  ix->d_unit_hist = masked ? (uint32_t*)(m + o_uh) : nullptr;
   cudaError_t e = cudaSuccess;
   const char* what = "block table copy";
   if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_off, h_off.data(), nb * 8, cudaMemcpyHostToDevice, cs);
@@ -552,7 +555,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   Geometry g;
   mp_status st = build_geometry(family, g);
   if (st != MP_OK) return st;
-  const bool ties = op && op->kind == MP_OP_TIES;
+  const bool ties = op && (op->kind == MP_OP_TIES || op->kind == MP_OP_TIES_MASKED);
   if (op && (st = check_op(op, g.K)) != MP_OK) return st;
   const void* base;
   ExpertPtrs ex;
@@ -614,6 +617,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     p.estar = (uint32_t*)(m + o_est);
     p.rank = (unsigned long long*)(m + o_rank);
     p.tau = ix->d_tau;
+    p.unit_hist = ix->d_unit_hist;
     if ((e = cudaMemsetAsync(p.coarse, 0, KG * 256 * 8, cs)) != cudaSuccess) return bail(e, "memset");
     if ((e = cudaMemsetAsync(p.fine, 0, KG * 128 * 8, cs)) != cudaSuccess) return bail(e, "memset");
     if ((e = cudaMemcpyAsync((void*)p.kth, h_kth.data(), n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
@@ -642,6 +646,8 @@ mp_status mp_index_import(const mp_family* family, const mp_op* op, const float*
   if (st != MP_OK) return st;
   const bool ties = op && op->kind == MP_OP_TIES;
   if (op && (st = check_op(op, g.K)) != MP_OK) return st;
+  if (op && op->kind == MP_OP_TIES_MASKED)
+    return fail(MP_ERR_UNSUPPORTED, "a TIES_MASKED catalog holds per-block key histograms, which are not imported");
   if (!norm || !maxabs || !nnz) return fail(MP_ERR_INVALID_ARG, "norm, maxabs and nnz are required");
   if (ties && !tau) return fail(MP_ERR_INVALID_ARG, "a TIES catalog needs tau");
   if ((base_hash == nullptr) != (expert_hash == nullptr))
@@ -712,9 +718,9 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
   const Geometry& g = index->g;
   if ((st = check_op(op, g.K)) != MP_OK) return st;
-  if (op->kind == MP_OP_TIES &&
-      (index->op_kind != MP_OP_TIES || index->density != op->density || index->trim_scope != op->trim_scope))
-    return fail(MP_ERR_MISMATCH, "a TIES plan needs an index built with the same TIES density and trim scope");
+  if ((op->kind == MP_OP_TIES || op->kind == MP_OP_TIES_MASKED) &&
+      (index->op_kind != op->kind || index->density != op->density || index->trim_scope != op->trim_scope))
+    return fail(MP_ERR_MISMATCH, "a TIES plan needs an index built for the same TIES kind, density and trim scope");
   cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
   const uint64_t nb = g.n_blocks, U = nb * g.K;
 
@@ -780,7 +786,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   p.elem_size = g.elem_size;
   p.op_kind = op->kind;
   p.score_mode = op->score_mode;
-  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES;
+  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES || op->kind == MP_OP_TIES_MASKED;
   for (uint32_t i = 0; i < g.K; ++i) p.coef[i] = fabsf(by_lambda ? op->lambda : op->alpha[i]);
   p.blk_len = index->d_blk_len;
   p.blk_group = index->d_blk_group;
@@ -862,6 +868,9 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
         return fail(MP_ERR_INVALID_ARG, "out overlaps an expert");
   }
   cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  const bool masked = plan->op_kind == MP_OP_TIES_MASKED;
+  if (masked && !index->d_unit_hist)
+    return fail(MP_ERR_MISMATCH, "a TIES_MASKED merge needs an index built for TIES_MASKED");
 
   mp_manifest_s* mf = new (std::nothrow) mp_manifest_s();
   if (!mf) return fail(MP_ERR_OOM, "host allocation failed");
@@ -874,16 +883,24 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   mf->valid_done = nullptr;
   for (uint32_t i = 0; i <= kMaxK; ++i) mf->lineage[i] = (family->lineage_ids && i <= g.K) ? family->lineage_ids[i] : 0u;
   const size_t counters_bytes = (size_t)kCounterSlots * g.K * 8;
-  // the counters (64 slots x K), the plan summary and the error word come back in one copy
-  const size_t back_bytes = counters_bytes + 64 + 16;
+  // the counters (64 slots x K), the plan summary, the error word and the TIES_MASKED
+  // threshold reads come back in one copy
+  const size_t back_bytes = counters_bytes + 64 + 16 + 16;
   mf->h_realized = static_cast<unsigned long long*>(pin_get(back_bytes));
   if (!mf->h_realized) {
     delete mf;
     return fail(MP_ERR_OOM, "pinned host allocation failed");
   }
   auto release_pinned = [&]() { pin_put(mf->h_realized, back_bytes); };
-  // device side: what comes back, then the merge kernel's work counter
-  if ((st = dev_alloc(mf->mem, back_bytes + 16, cs)) != MP_OK) {
+  // device side: what comes back, then the merge kernel's work counter, then (TIES_MASKED)
+  // the scratch of the masked threshold
+  const uint64_t KG = (uint64_t)g.K * plan->n_groups;
+  size_t mo = 0;
+  auto mslot = [&](size_t bytes) { size_t r = mo; mo += align_up(bytes); return r; };
+  const size_t m_coarse = mslot(KG * 256 * 8), m_fine = mslot(KG * 128 * 8), m_kth = mslot(plan->n_groups * 8);
+  const size_t m_est = mslot(KG * 4), m_rank = mslot(KG * 8), m_tau = mslot(KG * 4);
+  const size_t scratch_off = align_up(back_bytes + 16);
+  if ((st = dev_alloc(mf->mem, scratch_off + (masked ? mo : 0), cs)) != MP_OK) {
     release_pinned();
     delete mf;
     return st;
@@ -904,11 +921,54 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
   if ((e = cudaStreamWaitEvent(cs, plan->done, 0)) != cudaSuccess) return bail(e, "stream wait");
   if ((e = cudaMemsetAsync(mf->mem.ptr, 0, back_bytes, cs)) != cudaSuccess) return bail(e, "memset");
+  uint32_t* masked_tau = nullptr;
+  if (masked) {
+    // TIES after masking: the threshold of the zero-completed masked deltas of this plan
+    char* sm = static_cast<char*>(mf->mem.ptr) + scratch_off;
+    std::vector<unsigned long long> kth(plan->n_groups, 0);
+    {
+      std::vector<uint64_t> gnumel(plan->n_groups, 0);
+      for (uint32_t t = 0; t < g.n_tensors; ++t) gnumel[plan->trim_scope == 0 ? t : 0] += g.t_numel[t];
+      for (uint32_t q = 0; q < plan->n_groups; ++q)
+        kth[q] = (unsigned long long)floor((double)plan->density * (double)gnumel[q]);
+    }
+    if ((e = cudaMemsetAsync(sm, 0, m_kth, cs)) != cudaSuccess) return bail(e, "memset");  // coarse + fine
+    if ((e = cudaMemcpyAsync(sm + m_kth, kth.data(), plan->n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
+      return bail(e, "k copy");
+    IndexLaunch q;
+    memset(&q, 0, sizeof(q));
+    q.dtype = g.dtype;
+    q.K = g.K;
+    q.n_blocks = g.n_blocks;
+    q.n_groups = plan->n_groups;
+    q.base = base;
+    q.experts = ex;
+    q.blk_off = index->d_blk_off;
+    q.blk_len = index->d_blk_len;
+    q.blk_group = index->d_blk_group;
+    q.norm = index->d_norm;
+    q.maxabs = index->d_maxabs;
+    q.nnz = index->d_nnz;
+    q.err = mf->d_err;
+    q.coarse = (unsigned long long*)(sm + m_coarse);
+    q.fine = (unsigned long long*)(sm + m_fine);
+    q.kth = (const unsigned long long*)(sm + m_kth);
+    q.estar = (uint32_t*)(sm + m_est);
+    q.rank = (unsigned long long*)(sm + m_rank);
+    q.tau = masked_tau = (uint32_t*)(sm + m_tau);
+    q.unit_hist = index->d_unit_hist;
+    q.mask = plan->d_mask;
+    q.thr_reads = reinterpret_cast<unsigned long long*>(static_cast<char*>(mf->mem.ptr) + counters_bytes + 80);
+    q.b_begin = 0;
+    q.b_end = g.n_blocks;
+    q.expert_origin = 0;
+    if ((e = launch_ties_masked(q, cs)) != cudaSuccess) return bail(e, "masked TIES threshold");
+  }
 
   MergeLaunch p;
   memset(&p, 0, sizeof(p));
   p.dtype = g.dtype;
-  p.op_kind = plan->op_kind;
+  p.op_kind = masked ? MP_OP_TIES : plan->op_kind;  // TIES with the plan's threshold
   p.K = g.K;
   p.n_blocks = g.n_blocks;
   p.block_elems = g.block_elems;
@@ -920,7 +980,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   p.blk_len = index->d_blk_len;
   p.blk_group = index->d_blk_group;
   p.mask = plan->d_mask;
-  p.tau = index->d_tau;
+  p.tau = masked ? masked_tau : index->d_tau;
   p.nnz = index->d_nnz;
   for (uint32_t i = 0; i < kMaxK; ++i) p.alpha[i] = plan->alpha[i];
   p.lambda = plan->lambda;
@@ -996,7 +1056,7 @@ void mp_free(void* handle) {
     if (mf->valid_done) cudaEventSynchronize(mf->valid_done), cudaEventDestroy(mf->valid_done);
     dev_free(mf->valid_mem);
     dev_free(mf->mem);
-    pin_put(mf->h_realized, (size_t)kCounterSlots * mf->K * 8 + 64 + 16);
+    pin_put(mf->h_realized, (size_t)kCounterSlots * mf->K * 8 + 64 + 16 + 16);
     mf->magic = 0;
     delete mf;
   }
@@ -1196,6 +1256,16 @@ mp_status mp_manifest_validation(const mp_manifest* man, uint64_t* checked, uint
                                      (k == 0 ? std::string("base") : "expert " + std::to_string(k - 1)) + " block " +
                                      std::to_string(b));
   }
+  return MP_OK;
+}
+
+mp_status mp_manifest_threshold_reads(const mp_manifest* man, uint64_t* bytes) {
+  mp_status st;
+  if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
+  if (!bytes) return fail(MP_ERR_INVALID_ARG, "bytes is NULL");
+  cudaError_t e;
+  if ((e = cudaEventSynchronize(man->done)) != cudaSuccess) return cuda_fail(e, "merge work");
+  *bytes = man->h_realized[(size_t)kCounterSlots * man->K + 10];
   return MP_OK;
 }
 

@@ -471,6 +471,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
           p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
           c += len - nzk;  // zero deltas have key 0
         }
+        if (p.unit_hist) p.unit_hist[(((uint64_t)(i0 + k) * p.n_blocks + b) << 8) + tid] = (uint32_t)c;
         if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + tid], c);
       }
     }
@@ -528,13 +529,16 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
       uint32_t i = i0 + k;
       uint32_t es = p.estar[(uint64_t)i * p.n_groups + grp];
       uint64_t u = (uint64_t)i * p.n_blocks + b;
-      if (es != kNoBin && p.nnz[u] != 0u && (ties_key(p.maxabs[u]) >> 7) >= es) {
+      const bool read = !p.mask || ((p.mask[b] >> i) & 1u);  // TIES_MASKED: selected blocks only
+      if (read && es != kNoBin && p.nnz[u] != 0u && (ties_key(p.maxabs[u]) >> 7) >= es) {
         estar[k] = es;
         want |= 1u << k;
       }
     }
   }
   if (want == 0u) return;  // uniform over the CTA
+  if (p.thr_reads && threadIdx.x == 0)
+    atomicAdd(p.thr_reads, (unsigned long long)__popc(want) * p.blk_len[b] * (BF16 ? 2u : 4u));
   for (uint32_t x = tid; x < (uint32_t)KG * 128u; x += 256u) (&s_fine[0][0])[x] = 0u;
   __syncthreads();
 
@@ -582,6 +586,33 @@ __global__ void ties_fine_select(const IndexLaunch p) {
   }
   // only bin 0 can fall short: its uncounted members are exact zeros, key 0
   p.tau[x] = es << 7;
+}
+
+// TIES after masking: the coarse bins of (expert i, group) summed over a window of blocks:
+// a selected block adds its catalog histogram, an unselected one adds its elements to bin 0
+// (omitted entries are zeros).  One CTA per (expert, window of kMaskWin blocks); thread e
+// owns bin e and adds its sum for each group the window touches.
+constexpr uint32_t kMaskWin = 256;
+
+__global__ void __launch_bounds__(256) ties_masked_coarse(const IndexLaunch p, uint32_t n_win) {
+  const uint32_t i = blockIdx.x / n_win;
+  const uint64_t b0 = (uint64_t)(blockIdx.x % n_win) * kMaskWin;
+  const uint64_t b1 = b0 + kMaskWin < p.n_blocks ? b0 + kMaskWin : p.n_blocks;
+  const uint32_t e = threadIdx.x;
+  const uint32_t* uh = p.unit_hist + ((uint64_t)i * p.n_blocks << 8);
+  uint32_t grp = p.blk_group[b0];
+  unsigned long long acc = 0;
+  for (uint64_t b = b0; b < b1; ++b) {
+    const uint32_t g = p.blk_group[b];
+    if (g != grp) {
+      if (acc) atomicAdd(&p.coarse[((uint64_t)i * p.n_groups + grp) * 256u + e], acc);
+      acc = 0;
+      grp = g;
+    }
+    if ((p.mask[b] >> i) & 1u) acc += uh[(b << 8) + e];
+    else if (e == 0) acc += p.blk_len[b];
+  }
+  if (acc) atomicAdd(&p.coarse[((uint64_t)i * p.n_groups + grp) * 256u + e], acc);
 }
 
 // the TIES threshold from the coarse bins of the whole family: select the bin, count
@@ -644,6 +675,16 @@ cudaError_t launch_dtype(const IndexLaunch& p, cudaStream_t st) {
 
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st) {
   return p.dtype == MP_BF16 ? launch_dtype<true>(p, st) : launch_dtype<false>(p, st);
+}
+
+cudaError_t launch_ties_masked(const IndexLaunch& p, cudaStream_t st) {
+  if (!p.unit_hist || !p.mask || p.n_blocks == 0) return cudaErrorInvalidValue;
+  const uint32_t n_win = (uint32_t)((p.n_blocks + kMaskWin - 1) / kMaskWin);
+  ties_masked_coarse<<<p.K * n_win, 256, 0, st>>>(p, n_win);
+  count_launches(1);
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) return e;
+  return launch_ties_finish(p, st);
 }
 
 cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st) {

@@ -72,6 +72,7 @@ struct mp_index_s {
   uint32_t* d_blk_tensor;  // [n_blocks] tensor of each block
   uint32_t* d_t_blk0;      // [n_tensors + 1] first block of each tensor, then n_blocks
   bool has_missing;        // some entry has nnz == kNnzMissing (imported catalogs only)
+  uint32_t* d_unit_hist;   // [K][n_blocks][256] coarse key histograms (TIES_MASKED only)
   mp::Alloc hash_mem;      // the catalog's block hashes, once computed or imported
   unsigned long long* d_base_hash;    // [n_blocks]
   unsigned long long* d_expert_hash;  // [K][n_blocks]
@@ -162,6 +163,12 @@ struct IndexLaunch {
   uint32_t* estar;             // [K][n_groups] coarse bin of tau (or 0xFFFFFFFF)
   unsigned long long* rank;    // [K][n_groups] rank of tau inside that bin
   uint32_t* tau;               // [K][n_groups]
+  // TIES after masking: the catalog keeps each unit's coarse key histogram (256 bins, zero
+  // deltas in bin 0); the fine pass then reads only the blocks the plan selected and counts
+  // the expert bytes it reads
+  uint32_t* unit_hist;         // [K][n_blocks][256] or null
+  const uint32_t* mask;        // the access mask for the fine pass, or null (every block)
+  unsigned long long* thr_reads;  // expert bytes read by the fine pass, or null
   unsigned long long* work;    // item counter of the dynamic scheduler (zeroed per launch)
   // the launch covers blocks [b_begin, b_end); expert pointers address element
   // expert_origin of the flat layout (0 for resident experts, a segment start when they
@@ -171,6 +178,10 @@ struct IndexLaunch {
 };
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
 cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st);
+// the TIES_MASKED threshold of a plan: coarse bins summed from the per-unit histograms of
+// the selected blocks (zero entries for the others), then the select, fine pass and select
+// of launch_ties_finish restricted to the selected blocks (p.mask)
+cudaError_t launch_ties_masked(const IndexLaunch& p, cudaStream_t st);
 
 // ---- plan (plan.cu) ---------------------------------------------------------------------
 struct PlanLaunch {

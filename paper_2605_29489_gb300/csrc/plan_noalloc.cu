@@ -81,9 +81,9 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   if (U > kNoAllocMaxUnits || mp::plan_scratch_bytes(U, 0) > kNoAllocScratchBytes)
     return fail_static(MP_ERR_INVALID_ARG,
                        "mp_plan_noalloc: K * n_blocks exceeds the static scratch limit of 524288 units");
-  if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_DARE_TIES)
+  if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_TIES_MASKED)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: bad op");
-  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES;
+  const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES || op->kind == MP_OP_TIES_MASKED;
   if (!by_lambda && !op->alpha)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA, DARE and AVG_RENORM");
   if (op->score_mode > 1) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: score_mode must be 0 or 1");

@@ -23,7 +23,7 @@ from paper_2605_29489_gb300 import synth  # noqa: E402
 def test_hostpool_parity_small_families(make):
     fam = make()
     base, experts = fam.host_arrays()
-    run_case(fam, base, experts, ("avg", "ties", "ties1", "dare"), FRACS, host_experts=True)
+    run_case(fam, base, experts, ("avg", "ties", "ties1", "dare", "ties_masked"), FRACS, host_experts=True)
 
 
 def test_hostpool_multi_segment_matches_oracle_and_device_path(pool):  # noqa: F811

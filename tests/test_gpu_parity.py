@@ -106,6 +106,12 @@ def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
         elif k == "dare_ties":
             out.append(("dare_ties", mp.make_op(mp.MP_OP_DARE_TIES, lam=0.8, drop_p=0.7, seed=424242),
                         oracle.Op(oracle.DARE_TIES, K, lam=0.8, drop_p=0.7, seed=424242)))
+        elif k == "ties_masked":   # App. A.1: TIES after masking (threshold of the masked deltas)
+            out.append(("ties_masked", mp.make_op(mp.MP_OP_TIES_MASKED, lam=1.0, density=0.2),
+                        oracle.Op(oracle.TIES_MASKED, K, lam=1.0, density=0.2)))
+        elif k == "ties_masked1":
+            out.append(("ties_masked1", mp.make_op(mp.MP_OP_TIES_MASKED, lam=0.7, density=0.35, trim_scope=1),
+                        oracle.Op(oracle.TIES_MASKED, K, lam=0.7, density=0.35, trim_scope=1)))
         elif k == "ties_pb":
             out.append(("ties_pb", mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, score_mode=1),
                         oracle.Op(oracle.TIES, K, lam=1.0, density=0.2, score_mode=1)))
@@ -119,7 +125,8 @@ def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=Fa
     es = fam.elem_size
     C_full = fam.K * fam.n_params * es
     for name, gop, oop in ops_for(fam.K, kinds):
-        scope = oop.trim_scope if oop.kind == oracle.TIES else 0
+        masked = oop.kind == oracle.TIES_MASKED
+        scope = oop.trim_scope if oop.kind in (oracle.TIES, oracle.TIES_MASKED) else 0
         of = oracle_family(fam, base, experts, trim_scope=scope)
         idx = mp.mp_index_blocks(mf, gop)
         norm, maxabs, nnz, tau = mp.mp_index_stats(idx)
@@ -128,7 +135,7 @@ def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=Fa
         assert np.array_equal(maxabs.view(np.uint32), o_max.view(np.uint32)), name
         assert np.array_equal(norm.view(np.uint32), o_norm.view(np.uint32)), name
         o_tau = None
-        if oop.kind == oracle.TIES:
+        if oop.kind in (oracle.TIES, oracle.TIES_MASKED):
             o_tau = oracle.ties_thresholds(of, oop.density)
             assert np.array_equal(tau, o_tau), name
         for f in fracs:
@@ -137,7 +144,7 @@ def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=Fa
             plan = mp.mp_plan(idx, gop, B)
             pi = mp.mp_plan_info(plan, idx)
             ng = of.n_groups
-            opl = oracle.plan(fam.K, bl, of.blk_group, ng, es, oop, o_norm, o_max, o_nnz, o_tau, B)
+            opl = oracle.plan(fam.K, bl, of.blk_group, ng, es, oop, o_norm, o_max, o_nnz, None if masked else o_tau, B)
             what = f"{fam.name}/{name}/f={f}"
             assert pi["chat"] == opl["chat"] <= B, what
             assert pi["n_sel"] == opl["n_sel"], what
@@ -154,9 +161,12 @@ def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=Fa
             assert mi["realized_total"] == opl["chat"], what          # Prop. 1, realized = planned
             assert mi["touched"] == int((opl["mask"] != 0).sum()), what
             assert mi["digest"] == opl["digest"], what
-            want = oracle.merge(of, oop, tau=o_tau, mask=opl["mask"])
+            m_tau = oracle.ties_masked_thresholds(of, oop.density, opl["mask"]) if masked else o_tau
+            want = oracle.merge(of, oop, tau=m_tau, mask=opl["mask"])
             got = host(fam, out)
             assert_merge_close(fam, got[covered], want[covered], what)
+            if masked:   # the threshold pass re-reads only selected blocks
+                assert 0 <= mp.mp_manifest_threshold_reads(man) <= opl["chat"], what
             if f >= 1.0:   # Eq. 5: full budget reproduces the unmasked operator
                 phi = oracle.merge(of, oop, tau=o_tau, mask=None)
                 assert_merge_close(fam, got[covered], phi[covered], what + " vs Phi")
@@ -218,8 +228,8 @@ FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 def test_parity_small_families(make):
     fam = make()
     base, experts = fam.host_arrays()
-    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb", "avg_renorm", "dare_ties"),
-             FRACS)
+    run_case(fam, base, experts, ("avg", "ta", "ties", "ties1", "dare", "ta_pb", "ties_pb", "avg_renorm", "dare_ties",
+                                  "ties_masked", "ties_masked1"), FRACS)
 
 
 @pytest.mark.parametrize("make", [fam_big_blocks, fam_max_block], ids=lambda f: f.__name__)

@@ -41,7 +41,8 @@ def check_family(fam, kinds, fracs, host_experts=False):
     mf, b, ex = upload(fam, base, experts, host_experts)
     bo, bl, _ = fam.block_table()
     for name, gop, oop in ops_for(fam.K, kinds):
-        scope = oop.trim_scope if oop.kind == oracle.TIES else 0
+        masked = oop.kind == oracle.TIES_MASKED
+        scope = oop.trim_scope if oop.kind in (oracle.TIES, oracle.TIES_MASKED) else 0
         of = oracle_family(fam, base, experts, trim_scope=scope)
         o_norm, o_max, o_nnz = oracle.index(of)
         tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
@@ -54,7 +55,8 @@ def check_family(fam, kinds, fracs, host_experts=False):
             opl = oracle.plan(fam.K, bl, of.blk_group, of.n_groups, fam.elem_size, oop, o_norm, o_max, o_nnz, tau, B)
             assert pi["digest"] == opl["digest"] and np.array_equal(pi["mask"], opl["mask"]), what
             touched = touched_elements(fam, opl["mask"])
-            want = oracle.merge(of, oop, tau=tau, mask=opl["mask"])
+            m_tau = oracle.ties_masked_thresholds(of, oop.density, opl["mask"]) if masked else tau
+            want = oracle.merge(of, oop, tau=m_tau, mask=opl["mask"])
 
             out = sentinel_like(b)
             before = host(fam, out).copy()
@@ -88,7 +90,7 @@ def dev_copy(t):
 
 @pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k32], ids=lambda f: f.__name__)
 def test_touched_only_matches_oracle_on_touched_blocks(make):
-    check_family(make(), ("avg", "ta", "ties", "dare", "avg_renorm", "dare_ties"), [0.1, 0.5, 1.0])
+    check_family(make(), ("avg", "ta", "ties", "dare", "avg_renorm", "dare_ties", "ties_masked"), [0.1, 0.5, 1.0])
 
 
 def test_touched_only_zero_budget_writes_nothing():
