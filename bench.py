@@ -52,6 +52,10 @@ def workloads():
                                      desc="Qwen2.5-0.5B shapes cut to 2 layers (profiling case), K=4, TIES density 0.2"),
         "llama-3-8b-ties": dict(make=lambda: synth.llama3_8b(), op="ties", density=0.2, budgets=[1.0, 0.5, 0.25, 0.1],
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
+        "llama-3-8b-ties-masked": dict(make=lambda: synth.llama3_8b(), op="ties_masked", density=0.2,
+                                       budgets=[1.0, 0.5, 0.25, 0.1],
+                                       desc="Llama-3-8B-shaped bf16 family, K=4, TIES applied after masking (threshold "
+                                            "of the zero-completed masked deltas, App. A.1) density 0.2"),
         "qwen2.5-1.5b-dare": dict(make=lambda: synth.qwen25_15b(), op="dare", drop_p=0.9, budgets=[0.25],
                                   desc="Qwen2.5-1.5B-shaped bf16 family, K=16, DARE p=0.9 then AVG, per-expert active sets"),
         "qwen2.5-0.5b-avg-renorm": dict(make=lambda: synth.qwen25_05b(), op="avg_renorm", budgets=[1.0, 0.5, 0.25, 0.1],
@@ -105,6 +109,9 @@ def make_ops(w, K):
     if w["op"] == "ties":
         return (mp.make_op(mp.MP_OP_TIES, lam=1.0, density=w["density"]),
                 oracle.Op(oracle.TIES, K, lam=1.0, density=w["density"]))
+    if w["op"] == "ties_masked":
+        return (mp.make_op(mp.MP_OP_TIES_MASKED, lam=1.0, density=w["density"]),
+                oracle.Op(oracle.TIES_MASKED, K, lam=1.0, density=w["density"]))
     if w["op"] == "dare":
         a = [1.0 / K] * K
         return (mp.make_op(mp.MP_OP_DARE, alpha=a, drop_p=w["drop_p"], seed=20260),
@@ -260,7 +267,8 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
         for f in budgets:
             pl = oracle.plan(fam.K, lens, groups, 1, es, oop, norm, maxabs, nnz, tau, math.floor(f * full),
                              blk_tensor=tmap)
-            oracle.merge(of, oop, tau=tau, mask=pl["mask"], nnz=nnz if tmap is not None else None)
+            m_tau = oracle.ties_masked_thresholds(of, oop.density, pl["mask"]) if oop.kind == oracle.TIES_MASKED else tau
+            oracle.merge(of, oop, tau=m_tau, mask=pl["mask"], nnz=nnz if tmap is not None else None)
         dt = time.perf_counter() - t0
         return dt, int(lens.sum())
 
@@ -408,6 +416,8 @@ def native(args, rank, world, local_rank):
                                touched_ratio=pi["chat"] / (fam.K * N * es), plan_ms=plan_ms[k], merge_ms=merge_ms[k]))
         if touched_mode:
             per_budget[-1]["touched_elements"] = int(np.asarray(blk_len)[np.asarray(pi["mask"]) != 0].sum())
+        if gop.kind == mp.MP_OP_TIES_MASKED:   # the masked threshold's second read of selected blocks
+            per_budget[-1]["threshold_read_bytes"] = mp.mp_manifest_threshold_reads(last[2 + 2 * k])
     hashes = None
     if not host_pool and not args.no_hash:
         hashes = time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream)
