@@ -93,3 +93,7 @@ def test_index_import_refuses_bad_entries_before_any_device_work():
     with pytest.raises(mp.MergePipeError) as e:
         mp.mp_index_import(fam, mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2), norm, maxabs, nnz, None, stream=0)
     assert e.value.status == -1
+    # a TIES-after-masking catalog carries per-block key histograms, which are not imported
+    with pytest.raises(mp.MergePipeError) as e:
+        mp.mp_index_import(fam, mp.make_op(mp.MP_OP_TIES_MASKED, lam=1.0, density=0.2), norm, maxabs, nnz, stream=0)
+    assert e.value.status == -7
