@@ -132,7 +132,10 @@ typedef struct mp_manifest_s mp_manifest;
  * 16-byte vectors, a per-lane fma chain, then a butterfly over lanes).  If op->kind is
  * MP_OP_TIES it also computes the trim threshold tau of each (expert, trim group): the
  * k-th largest 15-bit key bits(bf16(|delta|)) & 0x7FFF with k = floor(density * numel)
- * (k = 0 gives tau = 0x8000, nothing kept).  op may be NULL for non-TIES use.
+ * (k = 0 gives tau = 0x8000, nothing kept).  For MP_OP_TIES_MASKED it computes the same
+ * and also keeps every (expert, block)'s 256-bin histogram of the upper 8 key bits (zero
+ * deltas in bin 0; 1 KB per unit), from which each merge finds its plan's threshold.  op
+ * may be NULL for non-TIES use.
  * The family's buffers must stay valid and unchanged until the stream reaches this work.
  * Errors: MP_ERR_INVALID_ARG (bad family or op), MP_ERR_OOM, MP_ERR_CUDA; a non-finite
  * delta makes mp_index_stats (and plans built on this index) report MP_ERR_NONFINITE.
@@ -182,7 +185,8 @@ mp_status mp_index_hash_values(const mp_index* index, uint64_t* base_hash, uint6
 /*
  * mp_plan — Alg. 1 PlanGen under budget B (bytes of expert reads, Eq. 3; cost of unit
  * (i,b) = elements(b) * element size, App. A.1).
- *  candidates: units with nnz > 0 (for TIES also bf16 key of maxabs >= tau); the others
+ *  candidates: units with nnz > 0 (for TIES also bf16 key of maxabs >= tau; TIES_MASKED's
+ *              threshold depends on the plan, so it prunes nothing more); the others
  *              contribute exactly nothing and are never read;
  *  score:      |alpha_i| * norm (TIES: |lambda| * norm), fp32 (Prop. 2's utility);
  *  order:      decreasing score, ties by ascending unit id b*K + i;
