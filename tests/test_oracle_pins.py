@@ -946,3 +946,24 @@ def test_ties_masked_full_mask_merges_like_ties(tiny_family):
     a = oracle.merge(of, oracle.Op(oracle.TIES, fam.K, lam=1.0, density=0.2), tau=tau, mask=full_mask)
     b = oracle.merge(of, oracle.Op(oracle.TIES_MASKED, fam.K, lam=1.0, density=0.2), tau=tm, mask=full_mask)
     assert np.array_equal(a.view(np.uint32), b.view(np.uint32))
+
+
+def test_ties_masked_thresholds_per_expert_scope(tiny_family):
+    """trim scope 1 (one group per expert): the k-th largest masked key over the whole
+    checkpoint, brute force"""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts, trim_scope=1)
+    bo, bl, _ = fam.block_table()
+    rng = np.random.default_rng(62)
+    mask = rng.integers(0, 16, fam.n_blocks).astype(np.uint32)
+    for density in (0.1, 0.5):
+        got = oracle.ties_masked_thresholds(of, density, mask)
+        assert got.shape == (fam.K, 1)
+        for i in range(fam.K):
+            d = experts[i].astype(np.float32) - base.astype(np.float32)
+            keys = bf16_bits_torch(np.abs(d)).astype(np.int64) & 0x7FFF
+            parts = [keys[int(bo[b]):int(bo[b] + bl[b])] if (mask[b] >> i) & 1 else np.zeros(int(bl[b]), np.int64)
+                     for b in range(fam.n_blocks)]
+            allk = np.sort(np.concatenate(parts))[::-1]
+            k = int(math.floor(density * allk.size))
+            assert got[i, 0] == (oracle.TAU_NONE if k == 0 else int(allk[k - 1])), (density, i)
