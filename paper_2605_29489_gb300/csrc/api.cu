@@ -459,8 +459,15 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
   ix->n_groups = n_groups;
   ix->has_missing = false;
   ix->done = nullptr;
+  ix->order_ready = nullptr;
+  ix->order_mu = new (std::nothrow) std::mutex();
+  if (!ix->order_mu) {
+    delete ix;
+    return fail(MP_ERR_OOM, "host allocation failed");
+  }
   mp_status st;
   if ((st = dev_alloc(ix->mem, o, cs)) != MP_OK) {
+    delete ix->order_mu;
     delete ix;
     return st;
   }
@@ -523,8 +530,11 @@ void discard_index(mp_index_s* ix, cudaStream_t cs) {
   cudaStreamSynchronize(cs);
   cudaGetLastError();
   dev_free(ix->hash_mem);
+  dev_free(ix->order_mem);
   dev_free(ix->mem);
   if (ix->done) cudaEventDestroy(ix->done);
+  if (ix->order_ready) cudaEventDestroy(ix->order_ready);
+  delete ix->order_mu;
   delete ix;
 }
 
@@ -815,11 +825,39 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   put_u64(hdr, pb);
   put_u64(hdr, op->seed);
   put_u32(hdr, op->score_mode);
+  const std::vector<uint8_t> order_key = hdr;  // everything the traversal order depends on
   put_u64(hdr, budget_bytes);
   memcpy(p.hdr_prefix, hdr.data(), hdr.size());
   p.hdr_prefix_len = (uint32_t)hdr.size();
 
-  if ((e = launch_plan(p, scratch.ptr, cs)) != cudaSuccess) return bail(e, "plan kernels");
+  // the first operator planned on this index leaves its traversal order behind; later
+  // plans with the same operator start from it (the order is written once, by a launch
+  // that runs and records order_ready under the lock, and is only read afterwards)
+  mp_index_s* ixw = const_cast<mp_index_s*>(index);
+  {
+    std::lock_guard<std::mutex> lk(*ixw->order_mu);
+    bool fill = false;
+    if (!index->has_missing) {
+      if (ixw->order_mem.ptr && ixw->order_ready && ixw->order_key == order_key) {
+        if ((e = cudaStreamWaitEvent(cs, ixw->order_ready, 0)) != cudaSuccess) return bail(e, "stream wait");
+        p.cache_order_in = ixw->d_order_cache;
+        p.cache_q_in = ixw->d_order_q;
+      } else if (!ixw->order_mem.ptr && dev_alloc(ixw->order_mem, align_up(U * 4) + 16, cs) == MP_OK) {
+        ixw->d_order_cache = static_cast<uint32_t*>(ixw->order_mem.ptr);
+        ixw->d_order_q = reinterpret_cast<unsigned long long*>(static_cast<char*>(ixw->order_mem.ptr) + align_up(U * 4));
+        p.cache_order_out = ixw->d_order_cache;
+        p.cache_q_out = ixw->d_order_q;
+        fill = true;
+      }
+    }
+    if ((e = launch_plan(p, scratch.ptr, cs)) != cudaSuccess) return bail(e, "plan kernels");
+    if (fill) {
+      if ((e = cudaEventCreateWithFlags(&ixw->order_ready, cudaEventDisableTiming)) != cudaSuccess)
+        return bail(e, "event");
+      if ((e = cudaEventRecord(ixw->order_ready, cs)) != cudaSuccess) return bail(e, "event record");
+      ixw->order_key = order_key;
+    }
+  }
   if ((e = cudaFreeAsync(scratch.ptr, cs)) != cudaSuccess) return bail(e, "free scratch");
   scratch.ptr = nullptr;
   if ((e = cudaMemcpyAsync(pl->h_summary, pl->d_summary, 64, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)
@@ -1039,8 +1077,11 @@ void mp_free(void* handle) {
   if (magic == kMagicIndex) {
     mp_index_s* ix = static_cast<mp_index_s*>(handle);
     if (ix->done) cudaEventSynchronize(ix->done), cudaEventDestroy(ix->done);
+    if (ix->order_ready) cudaEventSynchronize(ix->order_ready), cudaEventDestroy(ix->order_ready);
     dev_free(ix->hash_mem);
+    dev_free(ix->order_mem);
     dev_free(ix->mem);
+    delete ix->order_mu;
     ix->magic = 0;
     delete ix;
   } else if (magic == kMagicPlan) {

@@ -6,6 +6,7 @@
 #include <stdint.h>
 
 #include <string>
+#include <mutex>
 #include <vector>
 
 #include "mergepipe.h"
@@ -73,6 +74,14 @@ struct mp_index_s {
   uint32_t* d_t_blk0;      // [n_tensors + 1] first block of each tensor, then n_blocks
   bool has_missing;        // some entry has nnz == kNnzMissing (imported catalogs only)
   uint32_t* d_unit_hist;   // [K][n_blocks][256] coarse key histograms (TIES_MASKED only)
+  // the traversal order of the first operator planned on this index, kept for later plans
+  // with the same operator (written once, then only read; guarded by order_mu on the host)
+  mp::Alloc order_mem;
+  uint32_t* d_order_cache;           // [K * n_blocks]
+  unsigned long long* d_order_q;     // candidates
+  std::vector<uint8_t> order_key;    // the operator's digest header without the budget
+  cudaEvent_t order_ready;
+  std::mutex* order_mu;
   mp::Alloc hash_mem;      // the catalog's block hashes, once computed or imported
   unsigned long long* d_base_hash;    // [n_blocks]
   unsigned long long* d_expert_hash;  // [K][n_blocks]
@@ -206,6 +215,13 @@ struct PlanLaunch {
   uint32_t n_tensors;
   const uint32_t* blk_tensor;
   const uint32_t* t_blk0;
+  // the candidates' traversal order does not depend on the budget: a plan may take it
+  // from an earlier plan of the same index and operator (cache_*_in), or leave it for
+  // later ones (cache_*_out); all null for a plan on its own
+  const uint32_t* cache_order_in;
+  const unsigned long long* cache_q_in;
+  uint32_t* cache_order_out;
+  unsigned long long* cache_q_out;
   uint64_t budget;
   uint32_t* mask;
   uint32_t* order;

@@ -286,140 +286,152 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     s.x[X_P] = kNoP;
     s.x[X_TAILMIN] = ~0ull;
   }
-  uint64_t u0, u1;
-  slice(U, u0, u1);
-  if (p.fallback) {
-    // 0a: flag the pairs holding an entry without statistics (one atomic per pair and warp)
-    for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
-      const uint64_t u = t0 + tid;
-      uint32_t pr = 0xFFFFFFFFu;
-      if (u < u1) {
-        const uint64_t b = u / p.K;
-        const uint32_t i = (uint32_t)(u % p.K);
-        if (p.nnz[(uint64_t)i * p.n_blocks + b] == kNnzMissing) pr = i * p.n_tensors + p.blk_tensor[b];
-      }
-      const uint32_t peers = __match_any_sync(0xFFFFFFFFu, pr);
-      if (pr != 0xFFFFFFFFu && lane == (uint32_t)(__ffs(peers) - 1)) atomicOr(&s.pair_flag[pr], 1u);
-    }
+  uint64_t Q = 0, q0 = 0, q1 = 0;
+  if (p.cache_q_in) {
+    // the candidates in traversal order from an earlier plan of this index and operator:
+    // phases 0 to C depend on the operator and the catalog, not on the budget
+    Q = *p.cache_q_in;
+    slice(Q, q0, q1);
+    for (uint64_t j = q0 + tid; j < q1; j += kPT) p.order[j] = p.cache_order_in[j];
     if (!grid_sync(s.x, gen, p.summary)) return;
-    // 0b: the flagged pairs' units, one warp each
-    const uint32_t n_pairs = p.K * p.n_tensors, nw = G * (kPT / 32);
-    for (uint32_t pr = c * (kPT / 32) + warp; pr < n_pairs; pr += nw)
-      if (s.pair_flag[pr]) fallback_pair(p, s, pr, lane);
-    if (!grid_sync(s.x, gen, p.summary)) return;
-  }
-  {
-    // without the fallback an entry lacking statistics cannot be planned: it is reported
-    unsigned long long cnt = 0;
-    bool miss = false;
-    for (uint64_t u = u0 + tid; u < u1; u += kPT) {
-      cnt += score_unit(p, s, u).cand ? 1ull : 0ull;
-      miss |= !p.fallback && p.nnz[(u % p.K) * p.n_blocks + u / p.K] == kNnzMissing;
-    }
-    if (__syncthreads_or(miss) && tid == 0) s.x[X_MISSING] = 1ull;
-    cnt = block_sum<unsigned long long>(cnt);
-    if (tid == 0) s.cta_a[c] = cnt;
-  }
-  if (!grid_sync(s.x, gen, p.summary)) return;
-
-  // ---- B: stable compaction into (keys_a, order) ----
-  uint64_t Q;
-  {
-    const unsigned long long before = block_sum_prefix(s.cta_a, c);
-    Q = block_sum_prefix(s.cta_a, G);
-    unsigned long long run = before;
-    for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
-      const uint64_t u = t0 + tid;
-      Unit x = u < u1 ? score_unit(p, s, u) : Unit{false, 0u};
-      uint32_t tot;
-      const uint32_t pos = block_scan<uint32_t>(x.cand ? 1u : 0u, tot);
-      if (x.cand) {
-        s.keys_a[run + pos] = x.key;
-        p.order[run + pos] = (uint32_t)u;
-      }
-      run += tot;
-    }
-  }
-  if (!grid_sync(s.x, gen, p.summary)) return;
-
-  // ---- C: stable LSD radix sort, 8-bit digits ----
-  uint32_t *kin = s.keys_a, *vin = p.order, *kout = s.keys_b, *vout = s.vals_b;
-  uint64_t q0, q1;
-  slice(Q, q0, q1);
-  for (uint32_t pass = 0; pass < 4; ++pass) {
-    const uint32_t shift = 8u * pass;
-    // C1: digit histogram of this CTA's slice
-    s_run[tid] = 0;
-    __syncthreads();
-    for (uint64_t j = q0 + tid; j < q1; j += kPT) atomicAdd(&s_run[(kin[j] >> shift) & 255u], 1u);
-    __syncthreads();
-    s.hist[(uint64_t)tid * G + c] = s_run[tid];
-    if (!grid_sync(s.x, gen, p.summary)) return;
-    // C2: per digit, exclusive prefix over the CTAs (one warp per digit) and the total
-    for (uint32_t d = c + warp * G; d < 256u; d += (kPT / 32) * G) {
-      uint32_t* h = s.hist + (uint64_t)d * G;
-      uint32_t carry = 0;
-      for (uint32_t k0 = 0; k0 < G; k0 += 32) {
-        const uint32_t v = k0 + lane < G ? h[k0 + lane] : 0u;
-        uint32_t x = v;
-#pragma unroll
-        for (int sh = 1; sh < 32; sh <<= 1) {
-          const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, sh);
-          if ((int)lane >= sh) x += y;
+  } else {
+    uint64_t u0, u1;
+    slice(U, u0, u1);
+    if (p.fallback) {
+      // 0a: flag the pairs holding an entry without statistics (one atomic per pair and warp)
+      for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
+        const uint64_t u = t0 + tid;
+        uint32_t pr = 0xFFFFFFFFu;
+        if (u < u1) {
+          const uint64_t b = u / p.K;
+          const uint32_t i = (uint32_t)(u % p.K);
+          if (p.nnz[(uint64_t)i * p.n_blocks + b] == kNnzMissing) pr = i * p.n_tensors + p.blk_tensor[b];
         }
-        if (k0 + lane < G) h[k0 + lane] = carry + x - v;
-        carry += __shfl_sync(0xFFFFFFFFu, x, 31);
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, pr);
+        if (pr != 0xFFFFFFFFu && lane == (uint32_t)(__ffs(peers) - 1)) atomicOr(&s.pair_flag[pr], 1u);
       }
-      if (lane == 0) s.tot[d] = carry;
+      if (!grid_sync(s.x, gen, p.summary)) return;
+      // 0b: the flagged pairs' units, one warp each
+      const uint32_t n_pairs = p.K * p.n_tensors, nw = G * (kPT / 32);
+      for (uint32_t pr = c * (kPT / 32) + warp; pr < n_pairs; pr += nw)
+        if (s.pair_flag[pr]) fallback_pair(p, s, pr, lane);
+      if (!grid_sync(s.x, gen, p.summary)) return;
+    }
+    {
+      // without the fallback an entry lacking statistics cannot be planned: it is reported
+      unsigned long long cnt = 0;
+      bool miss = false;
+      for (uint64_t u = u0 + tid; u < u1; u += kPT) {
+        cnt += score_unit(p, s, u).cand ? 1ull : 0ull;
+        miss |= !p.fallback && p.nnz[(u % p.K) * p.n_blocks + u / p.K] == kNnzMissing;
+      }
+      if (__syncthreads_or(miss) && tid == 0) s.x[X_MISSING] = 1ull;
+      cnt = block_sum<unsigned long long>(cnt);
+      if (tid == 0) s.cta_a[c] = cnt;
     }
     if (!grid_sync(s.x, gen, p.summary)) return;
-    // C3: digit starts; skip the pass if one digit holds every key; stable scatter
-    uint32_t total;
-    const uint32_t t_d = s.tot[tid];
-    const uint32_t start = block_scan<uint32_t>(t_d, total);
-    const bool skip = __syncthreads_or(t_d == (uint32_t)Q && Q > 0) != 0 || Q == 0;
-    if (skip) continue;  // uniform over the grid: every CTA reads the same totals
-    s_run[tid] = start + s.hist[(uint64_t)tid * G + c];
-    const uint32_t lt = (1u << lane) - 1u;
-    for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
-      for (int w = 0; w < kPT / 32; ++w) s_wcnt[w][tid] = 0;
-      __syncthreads();
-      const uint64_t j = t0 + tid;
-      const bool valid = j < q1;
-      const uint32_t key = valid ? kin[j] : 0u;
-      const uint32_t val = valid ? vin[j] : 0u;
-      const uint32_t d = valid ? ((key >> shift) & 255u) : 256u;
-      const uint32_t peers = __match_any_sync(0xFFFFFFFFu, d);
-      const uint32_t rank = __popc(peers & lt);
-      if (valid && rank == 0) s_wcnt[warp][d] = __popc(peers);
-      __syncthreads();
-      {
-        uint32_t acc = s_run[tid];
-        for (int w = 0; w < kPT / 32; ++w) {
-          const uint32_t cw = s_wcnt[w][tid];
-          s_wcnt[w][tid] = acc;
-          acc += cw;
+
+    // ---- B: stable compaction into (keys_a, order) ----
+    {
+      const unsigned long long before = block_sum_prefix(s.cta_a, c);
+      Q = block_sum_prefix(s.cta_a, G);
+      unsigned long long run = before;
+      for (uint64_t t0 = u0; t0 < u1; t0 += kPT) {
+        const uint64_t u = t0 + tid;
+        Unit x = u < u1 ? score_unit(p, s, u) : Unit{false, 0u};
+        uint32_t tot;
+        const uint32_t pos = block_scan<uint32_t>(x.cand ? 1u : 0u, tot);
+        if (x.cand) {
+          s.keys_a[run + pos] = x.key;
+          p.order[run + pos] = (uint32_t)u;
         }
-        s_run[tid] = acc;
+        run += tot;
       }
-      __syncthreads();
-      if (valid) {
-        const uint32_t pos = s_wcnt[warp][d] + rank;
-        kout[pos] = key;
-        vout[pos] = val;
-      }
-      __syncthreads();  // every warp has read its offsets before the next tile clears them
     }
     if (!grid_sync(s.x, gen, p.summary)) return;
-    uint32_t* t;
-    t = kin, kin = kout, kout = t;
-    t = vin, vin = vout, vout = t;
-  }
-  // the sorted units end in p.order, or in vals_b if an odd number of passes ran (a
-  // uniform fact: every CTA made the same skip decisions)
-  if (vin != p.order) {
-    for (uint64_t j = q0 + tid; j < q1; j += kPT) p.order[j] = vin[j];
-    if (!grid_sync(s.x, gen, p.summary)) return;
+
+    // ---- C: stable LSD radix sort, 8-bit digits ----
+    uint32_t *kin = s.keys_a, *vin = p.order, *kout = s.keys_b, *vout = s.vals_b;
+    slice(Q, q0, q1);
+    for (uint32_t pass = 0; pass < 4; ++pass) {
+      const uint32_t shift = 8u * pass;
+      // C1: digit histogram of this CTA's slice
+      s_run[tid] = 0;
+      __syncthreads();
+      for (uint64_t j = q0 + tid; j < q1; j += kPT) atomicAdd(&s_run[(kin[j] >> shift) & 255u], 1u);
+      __syncthreads();
+      s.hist[(uint64_t)tid * G + c] = s_run[tid];
+      if (!grid_sync(s.x, gen, p.summary)) return;
+      // C2: per digit, exclusive prefix over the CTAs (one warp per digit) and the total
+      for (uint32_t d = c + warp * G; d < 256u; d += (kPT / 32) * G) {
+        uint32_t* h = s.hist + (uint64_t)d * G;
+        uint32_t carry = 0;
+        for (uint32_t k0 = 0; k0 < G; k0 += 32) {
+          const uint32_t v = k0 + lane < G ? h[k0 + lane] : 0u;
+          uint32_t x = v;
+  #pragma unroll
+          for (int sh = 1; sh < 32; sh <<= 1) {
+            const uint32_t y = __shfl_up_sync(0xFFFFFFFFu, x, sh);
+            if ((int)lane >= sh) x += y;
+          }
+          if (k0 + lane < G) h[k0 + lane] = carry + x - v;
+          carry += __shfl_sync(0xFFFFFFFFu, x, 31);
+        }
+        if (lane == 0) s.tot[d] = carry;
+      }
+      if (!grid_sync(s.x, gen, p.summary)) return;
+      // C3: digit starts; skip the pass if one digit holds every key; stable scatter
+      uint32_t total;
+      const uint32_t t_d = s.tot[tid];
+      const uint32_t start = block_scan<uint32_t>(t_d, total);
+      const bool skip = __syncthreads_or(t_d == (uint32_t)Q && Q > 0) != 0 || Q == 0;
+      if (skip) continue;  // uniform over the grid: every CTA reads the same totals
+      s_run[tid] = start + s.hist[(uint64_t)tid * G + c];
+      const uint32_t lt = (1u << lane) - 1u;
+      for (uint64_t t0 = q0; t0 < q1; t0 += kPT) {
+        for (int w = 0; w < kPT / 32; ++w) s_wcnt[w][tid] = 0;
+        __syncthreads();
+        const uint64_t j = t0 + tid;
+        const bool valid = j < q1;
+        const uint32_t key = valid ? kin[j] : 0u;
+        const uint32_t val = valid ? vin[j] : 0u;
+        const uint32_t d = valid ? ((key >> shift) & 255u) : 256u;
+        const uint32_t peers = __match_any_sync(0xFFFFFFFFu, d);
+        const uint32_t rank = __popc(peers & lt);
+        if (valid && rank == 0) s_wcnt[warp][d] = __popc(peers);
+        __syncthreads();
+        {
+          uint32_t acc = s_run[tid];
+          for (int w = 0; w < kPT / 32; ++w) {
+            const uint32_t cw = s_wcnt[w][tid];
+            s_wcnt[w][tid] = acc;
+            acc += cw;
+          }
+          s_run[tid] = acc;
+        }
+        __syncthreads();
+        if (valid) {
+          const uint32_t pos = s_wcnt[warp][d] + rank;
+          kout[pos] = key;
+          vout[pos] = val;
+        }
+        __syncthreads();  // every warp has read its offsets before the next tile clears them
+      }
+      if (!grid_sync(s.x, gen, p.summary)) return;
+      uint32_t* t;
+      t = kin, kin = kout, kout = t;
+      t = vin, vin = vout, vout = t;
+    }
+    // the sorted units end in p.order, or in vals_b if an odd number of passes ran (a
+    // uniform fact: every CTA made the same skip decisions)
+    if (vin != p.order) {
+      for (uint64_t j = q0 + tid; j < q1; j += kPT) p.order[j] = vin[j];
+      if (!grid_sync(s.x, gen, p.summary)) return;
+    }
+    if (p.cache_order_out) {  // keep the order for later plans with the same operator
+      for (uint64_t j = q0 + tid; j < q1; j += kPT) p.cache_order_out[j] = p.order[j];
+      if (c == 0 && tid == 0) *p.cache_q_out = Q;
+    }
   }
   const uint32_t* order = p.order;
 
