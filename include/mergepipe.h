@@ -203,7 +203,9 @@ mp_status mp_index_hash_values(const mp_index* index, uint64_t* base_hash, uint6
  * selected units, the traversal order and a digest (FNV-1a 64 over op, theta, B, C_hat,
  * count and the sum of splitmix64(unit) over the selected units).  Budget soundness
  * (Prop. 1) holds by construction: C_hat <= B.  op must have the same kind and, for
- * TIES, the same density and trim scope as the op given to mp_index_blocks.
+ * TIES, the same density and trim scope as the op given to mp_index_blocks.  The traversal
+ * order does not depend on B: the index keeps the order of the first operator planned on
+ * it, and later plans with the same operator start from it (same result, less work).
  * Errors: MP_ERR_INVALID_ARG, MP_ERR_MISMATCH (op differs from the index's), MP_ERR_OOM,
  * MP_ERR_CUDA.
  */
