@@ -847,6 +847,8 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
         ixw->d_order_q = reinterpret_cast<unsigned long long*>(static_cast<char*>(ixw->order_mem.ptr) + align_up(U * 4));
         p.cache_order_out = ixw->d_order_cache;
         p.cache_q_out = ixw->d_order_q;
+        // an invalid count until the filling plan completes its sort
+        if ((e = cudaMemsetAsync(ixw->d_order_q, 0xFF, 8, cs)) != cudaSuccess) return bail(e, "memset");
         fill = true;
       }
     }

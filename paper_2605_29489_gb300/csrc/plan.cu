@@ -40,7 +40,7 @@ constexpr uint32_t kBarrierLimit = 1u << 24;
 enum { S_CHAT = 0, S_NSEL = 1, S_NCAND = 2, S_SETHASH = 3, S_DIGEST = 4, S_TOUCHED = 5, S_ERR = 6 };
 // scratch scalars
 enum { X_BAR_COUNT = 0, X_BAR_GEN = 1, X_P = 2, X_PBP = 3, X_TAILSUM = 4, X_DONE = 5, X_TOTAL = 6, X_MISSING = 7,
-       X_TAILMIN = 8, X_COUNT = 16 };
+       X_TAILMIN = 8, X_BADORDER = 9, X_COUNT = 16 };
 
 constexpr unsigned long long kNoP = ~0ull;
 
@@ -291,6 +291,10 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     // the candidates in traversal order from an earlier plan of this index and operator:
     // phases 0 to C depend on the operator and the catalog, not on the budget
     Q = *p.cache_q_in;
+    if (Q > U) {  // the plan that was to leave the order did not finish: report, plan nothing
+      if (c == 0 && tid == 0) s.x[X_BADORDER] = 1ull;
+      Q = 0;
+    }
     slice(Q, q0, q1);
     for (uint64_t j = q0 + tid; j < q1; j += kPT) p.order[j] = p.cache_order_in[j];
     if (!grid_sync(s.x, gen, p.summary)) return;
@@ -599,7 +603,8 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
   sum[S_CHAT] = chat;
   sum[S_NCAND] = Q;
   sum[S_DIGEST] = h;
-  sum[S_ERR] = sum[S_ERR] | (unsigned long long)*p.index_err | (s.x[X_MISSING] ? (unsigned long long)kErrMissing : 0ull);
+  sum[S_ERR] = sum[S_ERR] | (unsigned long long)*p.index_err | (s.x[X_MISSING] ? (unsigned long long)kErrMissing : 0ull) |
+               (s.x[X_BADORDER] ? (unsigned long long)kErrInternal : 0ull);
 }
 
 }  // namespace
