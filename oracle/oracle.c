@@ -488,7 +488,8 @@ int orc_plan(uint32_t K, uint64_t n_blocks, const uint32_t* blk_len, const uint3
  * Philox4x32-10 (Salmon, Moraes, Dror, Shaw, "Parallel random numbers: as easy as 1, 2,
  * 3", SC 2011): ten rounds of two 32x32->64 multiplies with multipliers 0xD2511F53 and
  * 0xCD9E8D57, the key bumped by the Weyl constants 0x9E3779B9 and 0xBB67AE85 between
- * rounds.  Pin: cuRAND's Philox4_32_10 on the GPU (an independent implementation).
+ * rounds.  Pins: cuRAND's Philox4_32_10 (an independent implementation), its host
+ * generator on the CPU and its device generator on the GPU.
  * ------------------------------------------------------------------------------------- */
 void orc_philox4x32_10(const uint32_t ctr[4], const uint32_t key[2], uint32_t out[4]) {
   uint32_t c0 = ctr[0], c1 = ctr[1], c2 = ctr[2], c3 = ctr[3];

@@ -376,6 +376,61 @@ def test_philox_word_statistics():
     assert not np.array_equal(a, b) and not np.array_equal(a, c)
 
 
+def _curand_host():
+    """cuRAND's host-side generator library (it runs on the CPU; no GPU is touched)"""
+    import ctypes
+    import ctypes.util
+    names = [os.path.join(os.environ.get("CUDA_HOME", "/usr/local/cuda"), "lib64", "libcurand.so"),
+             ctypes.util.find_library("curand")]
+    for n in names:
+        if n and (os.path.exists(n) or not os.path.isabs(n)):
+            try:
+                return ctypes.CDLL(n)
+            except OSError:
+                pass
+    pytest.skip("libcurand is not available")
+
+
+def _curand_host_philox(L, seed, offset, n_words):
+    import ctypes
+    gen = ctypes.c_void_p()
+    assert L.curandCreateGeneratorHost(ctypes.byref(gen), 161) == 0  # CURAND_RNG_PSEUDO_PHILOX4_32_10
+    try:
+        assert L.curandSetPseudoRandomGeneratorSeed(gen, ctypes.c_ulonglong(seed)) == 0
+        assert L.curandSetGeneratorOffset(gen, ctypes.c_ulonglong(offset)) == 0
+        out = np.zeros(n_words, np.uint32)
+        assert L.curandGenerate(gen, out.ctypes.data_as(ctypes.c_void_p), ctypes.c_size_t(n_words)) == 0
+    finally:
+        L.curandDestroyGenerator(gen)
+    return out
+
+
+def test_philox_matches_curand_host_generator():
+    """Philox4x32-10 against an independent implementation of the same published generator:
+    cuRAND's host generator, run on the CPU.  For seed s it emits 4-word blocks; block j
+    (j = the starting offset / 4 + the block's position) is Philox of the counter
+    (lo32(j >> 16), hi32(j >> 16), j & 0xFFFF, 0) under the key (lo32(s), hi32(s)).  That
+    reaches counter words 0-2 and both key words; word 3, which the DARE stream fixes to a
+    tag, is pinned against cuRAND's device generator in the GPU suite."""
+    L = _curand_host()
+
+    def ctr_of(j):
+        r = j >> 16
+        return [r & 0xFFFFFFFF, r >> 32, j & 0xFFFF, 0]
+
+    for seed in (0, 1, 2605, 0x0123456789ABCDEF, 0xFFFFFFFFFFFFFFFF):
+        key = [seed & 0xFFFFFFFF, seed >> 32]
+        # a run of blocks across the first change of counter word 0 (j = 65535 -> 65536)
+        j0 = 65536 - 3
+        got = _curand_host_philox(L, seed, 4 * j0, 4 * 6).reshape(-1, 4)
+        for b in range(6):
+            assert np.array_equal(oracle.philox4x32_10(ctr_of(j0 + b), key), got[b]), (seed, j0 + b)
+        # large offsets: counter words 0 and 1 both nonzero, and all ones in word 0
+        for j in ((5 << 48) + (7 << 16) + 9, (1 << 61) + 3, (0xFFFFFFFF << 16) + 11, (1 << 62) - 1):
+            got = _curand_host_philox(L, seed, 4 * j, 4)
+            assert np.array_equal(oracle.philox4x32_10(ctr_of(j), key), got), (seed, hex(j))
+
+
 # ---- Alg. 1 PlanGen ------------------------------------------------------------------------------------
 
 def _tiny_plan_case(rng, K, nb, uniform):
