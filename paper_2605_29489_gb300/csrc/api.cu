@@ -313,9 +313,17 @@ struct HostPipe {
 
   cudaError_t main_release(int b) { return cudaEventRecord(freed[b], main); }
 
-  // everything the side streams did precedes the caller stream's last wait, so the
+  // the caller's stream waits for everything the side streams were given (on the normal
+  // path it already has; after an error a gather may be the last work enqueued), so the
   // staging memory can be returned in the caller's stream order
   void finish() {
+    for (int q = 0; q < kSide && staging; ++q) {
+      if (!side[q] || !ready[0][q]) continue;
+      if (cudaEventRecord(ready[0][q], side[q]) != cudaSuccess || cudaStreamWaitEvent(main, ready[0][q], 0) != cudaSuccess) {
+        cudaGetLastError();
+        cudaStreamSynchronize(side[q]);
+      }
+    }
     if (staging) cudaFreeAsync(staging, main);
     staging = nullptr;
     for (int b = 0; b < 2; ++b) {
