@@ -269,7 +269,10 @@ mp_status mp_merge_touched(const mp_family* family, const mp_index* index, const
  *    summary[8] uint64 = {planned bytes, selected, candidates, selected-unit set hash,
  *    digest, touched blocks, error word, 0}.  The results equal mp_plan's bit for bit.
  *    This call has no tensor map, so it does not plan the tensor-level fallback: an nnz
- *    of MP_NNZ_MISSING sets bit 8 of the error word, and that entry is never read.
+ *    of MP_NNZ_MISSING sets the bit of value 8 in the error word, and that entry is never
+ *    read.  Every buffer is aligned to its element size (summary to 8 bytes); a misaligned
+ *    one returns MP_ERR_INVALID_ARG before any CUDA call.  Whether a buffer is device
+ *    memory is not checked (no pointer query is made, so the call can be captured).
  * Limit: K * n_blocks <= 524288 units; larger requests return MP_ERR_INVALID_ARG and
  * launch nothing.  The first call on a device looks up the array's device address
  * (cudaGetSymbolAddress, with that device current); make that first call before any

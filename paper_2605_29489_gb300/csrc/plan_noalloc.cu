@@ -91,6 +91,13 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: TIES needs tau and blk_group");
   if (!blk_len || !norm || !maxabs || !nnz || !index_err || !mask || !order || !summary)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: a required buffer is NULL");
+  // the kernels load every buffer by its element type: a misaligned pointer is refused
+  // here rather than met by the GPU
+  const auto misaligned = [](const void* q, uintptr_t a) { return q && reinterpret_cast<uintptr_t>(q) % a != 0; };
+  if (misaligned(blk_len, 4) || misaligned(blk_group, 4) || misaligned(norm, 4) || misaligned(maxabs, 4) ||
+      misaligned(nnz, 4) || misaligned(tau, 4) || misaligned(index_err, 4) || misaligned(mask, 4) ||
+      misaligned(order, 4) || misaligned(summary, 8))
+    return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: a buffer is not aligned to its element size");
 
   void* scratch = nullptr;
   mp_status st = scratch_for_current_device(&scratch);

@@ -97,3 +97,31 @@ def test_index_import_refuses_bad_entries_before_any_device_work():
     with pytest.raises(mp.MergePipeError) as e:
         mp.mp_index_import(fam, mp.make_op(mp.MP_OP_TIES_MASKED, lam=1.0, density=0.2), norm, maxabs, nnz, stream=0)
     assert e.value.status == -7
+
+
+def test_plan_noalloc_refuses_bad_arguments_before_any_device_work():
+    """mp_plan_noalloc checks its arguments on the host before any CUDA call: a NULL or
+    misaligned buffer, too many units or a TIES plan without thresholds is refused (the
+    addresses here are never dereferenced)"""
+    import paper_2605_29489_gb300 as mp
+
+    A = 0x100000  # an aligned address, never touched
+    op = mp.make_op(mp.MP_OP_TA, alpha=[0.5, 0.5])
+
+    def call(K=2, n_blocks=8, op=op, tau=None, blk_group=None, **bufs):
+        b = dict(blk_len=A, norm=A, maxabs=A, nnz=A, index_err=A, mask=A, order=A, summary=A)
+        b.update(bufs)
+        with pytest.raises(mp.MergePipeError) as e:
+            mp.mp_plan_noalloc(K, n_blocks, 1, mp.MP_BF16, b["blk_len"], blk_group, b["norm"], b["maxabs"],
+                               b["nnz"], tau, b["index_err"], op, 1 << 20, b["mask"], b["order"], b["summary"],
+                               stream=0)
+        assert e.value.status == -1
+        return str(e.value)
+
+    assert "aligned" in call(norm=A + 2)
+    assert "aligned" in call(order=A + 1)
+    assert "aligned" in call(summary=A + 4)  # 8-byte words
+    assert "aligned" in call(blk_group=A + 2)
+    assert "NULL" in call(mask=None)
+    assert "524288" in call(K=2, n_blocks=(1 << 18) + 1)
+    assert "tau" in call(op=mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2), blk_group=A)
