@@ -24,6 +24,11 @@ NNZ_MISSING = 0xFFFFFFFF  # catalog entry without block statistics (tensor-level
 
 _lib = None
 
+# The mutation check of the pins (tests/test_oracle_mutants.py) builds copies of oracle.c
+# with one planted mistake each and runs the pins in a child process whose oracle is
+# such a copy: the child names that library here.  Unset, the oracle is oracle.c built.
+LIBRARY_UNDER_TEST_ENV = "ORACLE_LIBRARY_UNDER_TEST"
+
 
 class _Op(ctypes.Structure):
     _fields_ = [("kind", ctypes.c_int), ("K", ctypes.c_uint32), ("alpha", ctypes.c_void_p),
@@ -40,7 +45,7 @@ class _Family(ctypes.Structure):
 def lib():
     global _lib
     if _lib is None:
-        L = ctypes.CDLL(_build.build())
+        L = ctypes.CDLL(os.environ.get(LIBRARY_UNDER_TEST_ENV) or _build.build())
         vp, u32, u64 = ctypes.c_void_p, ctypes.c_uint32, ctypes.c_uint64
         L.orc_bf16_to_f32.restype = ctypes.c_float
         L.orc_bf16_to_f32.argtypes = [ctypes.c_uint16]

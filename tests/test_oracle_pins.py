@@ -50,6 +50,22 @@ def test_bf16_rounding_matches_torch():
     assert np.array_equal(got, ref)
 
 
+def test_bf16_rounding_keeps_nan_a_nan():
+    """IEEE: a NaN converts to a NaN, also one whose payload lies only in the 16 bits that
+    bf16 drops (cutting them would leave an infinity).  The float32 bits go to the C
+    function unchanged (a Python float round trip would quiet a signalling NaN)."""
+    import ctypes
+    import struct
+
+    pats = [0x7F800001, 0xFF800001, 0x7F80FFFF, 0x7FC00000, 0x7FBFFFFF, 0xFFC00001, 0x7F801234]
+    for bits in pats:
+        x = ctypes.c_float.from_buffer_copy(struct.pack("<I", bits))
+        h = int(oracle.lib().orc_f32_to_bf16(x))
+        t = torch.from_numpy(np.array([bits], np.uint32).view(np.float32)).to(torch.bfloat16)
+        assert bool(torch.isnan(t).item())
+        assert (h & 0x7F80) == 0x7F80 and (h & 0x007F) != 0, hex(bits)   # a bf16 NaN
+
+
 def test_ties_key_is_bf16_magnitude():
     rng = np.random.default_rng(2)
     d = (rng.standard_normal(3000) * 10.0 ** rng.uniform(-8, 2, 3000)).astype(np.float32)
@@ -198,6 +214,11 @@ def test_ties_worked_example():
     assert np.array_equal(bf16_to_f32(full), np.array(g["expected_full"], np.float32))
     part = oracle.merge_block(oracle.BF16, 0, b, [experts[0], None, experts[2]], g["mask_partial"], op, tau)
     assert np.array_equal(bf16_to_f32(part), np.array(g["expected_partial"], np.float32))
+    # the omitted expert counts as zero whatever its data: the same result with it present
+    wild = to_bf16(np.full(6, 1000.0))
+    for omitted in (experts[1], wild):
+        part = oracle.merge_block(oracle.BF16, 0, b, [experts[0], omitted, experts[2]], g["mask_partial"], op, tau)
+        assert np.array_equal(bf16_to_f32(part), np.array(g["expected_partial"], np.float32))
 
 
 def test_avg_worked_example():
@@ -210,6 +231,11 @@ def test_avg_worked_example():
     assert np.array_equal(bf16_to_f32(full), np.array(g["expected_full"], np.float32))
     part = oracle.merge_block(oracle.BF16, 0, b, [experts[0], experts[1], None], g["mask_partial"], op)
     assert np.array_equal(bf16_to_f32(part), np.array(g["expected_partial"], np.float32))
+    # the omitted expert counts as zero whatever its data: the same result with it present
+    wild = to_bf16(np.full(len(base), -1000.0))
+    for omitted in (experts[2], wild):
+        part = oracle.merge_block(oracle.BF16, 0, b, [experts[0], experts[1], omitted], g["mask_partial"], op)
+        assert np.array_equal(bf16_to_f32(part), np.array(g["expected_partial"], np.float32))
 
 
 def test_ties_special_cases():
@@ -282,6 +308,27 @@ def test_full_read_ties_matches_fp64_away_from_sign_ties():
     assert safe.mean() > 0.99
     ulp = np.abs(ref) * 2.0 ** -7 + 1e-30
     assert np.all(np.abs(out - ref)[safe] <= ulp[safe])
+
+
+def test_ties_per_tensor_trim_is_separable(tiny_family):
+    """With one trim group per tensor, each tensor's trim, election and mean involve that
+    tensor alone: the whole family's TIES merge equals, tensor by tensor, the merge of that
+    tensor taken as a family of its own (its own threshold, its own element numbering)."""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    bo, bl, bt = fam.block_table()
+    dens = 0.2
+    tau = oracle.ties_thresholds(of, dens)
+    assert len(set(tau[0].tolist())) > 1            # the tensors' thresholds differ
+    op = oracle.Op(oracle.TIES, fam.K, lam=0.8, density=dens)
+    whole = oracle.merge(of, op, tau=tau)
+    for t in range(len(fam.tensors)):
+        blocks = np.nonzero(bt == t)[0]
+        lo, hi = int(bo[blocks[0]]), int(bo[blocks[-1]] + bl[blocks[-1]])
+        sub = oracle.Family(fam.dtype, bo[blocks] - lo, bl[blocks], np.zeros(len(blocks), np.uint32), 1,
+                            base[lo:hi], [e[lo:hi] for e in experts])
+        alone = oracle.merge(sub, op, tau=oracle.ties_thresholds(sub, dens))
+        assert np.array_equal(whole[lo:hi].view(np.uint32), alone.view(np.uint32)), t
 
 
 # ---- Prop. 2: additive omission bound ------------------------------------------------------------------
@@ -357,6 +404,36 @@ def test_dare_mean_over_seeds_tends_to_avg():
     # per element: mean of 400 draws of sum_i a_i * 2 * Bern(.5) * d_i; sd of the mean <= sum |a_i d_i| / sqrt(400)
     sd = sum(abs(a) * np.abs(e.astype(np.float64) - base) for a, e in zip(alpha, experts)) / math.sqrt(seeds)
     assert np.all(np.abs(acc / seeds - avg) <= 5 * sd + 1e-9)
+
+
+def test_dare_p0_never_drops_over_many_entries():
+    """p = 0 drops nothing, whatever the random word: over 2^21 + 6 entries (so every 16-bit
+    word value, 0 included, comes up many times) DARE is AVG bit for bit"""
+    rng = np.random.default_rng(21)
+    n = (1 << 20) + 3
+    base = (rng.standard_normal(n) * 0.02).astype(np.float32)
+    experts = [base + (rng.standard_normal(n) * 1e-3).astype(np.float32) for _ in range(2)]
+    alpha = [0.5, 0.5]
+    a = oracle.merge_block(oracle.F32, 77, base, experts, 0b11, oracle.Op(oracle.AVG, 2, alpha=alpha))
+    d = oracle.merge_block(oracle.F32, 77, base, experts, 0b11,
+                           oracle.Op(oracle.DARE, 2, alpha=alpha, drop_p=0.0, seed=5))
+    assert np.array_equal(a.view(np.uint32), d.view(np.uint32))
+
+
+def test_dare_drops_independently_across_blocks():
+    """App. A.1's DARE drops each entry at random: two blocks holding the same deltas at
+    different places in the checkpoint get different drop patterns (at p = 0.5 the chance
+    that 4096 independent draws agree is 2^-4096)"""
+    rng = np.random.default_rng(22)
+    E = 4096
+    b = (rng.standard_normal(E) * 0.02).astype(np.float32)
+    e = b + (rng.standard_normal(E) * 1e-2).astype(np.float32)
+    base, expert = np.concatenate([b, b]), np.concatenate([e, e])
+    fam = oracle.Family(oracle.F32, [0, E], [E, E], [0, 0], 1, base, [expert])
+    out = oracle.merge(fam, oracle.Op(oracle.DARE, 1, alpha=[1.0], drop_p=0.5, seed=3))
+    kept0, kept1 = out[:E] != b, out[E:] != b
+    assert 0.4 < kept0.mean() < 0.6 and 0.4 < kept1.mean() < 0.6
+    assert not np.array_equal(kept0, kept1)
 
 
 def test_philox_word_statistics():
@@ -509,6 +586,34 @@ def test_plan_ties_prunes_fully_trimmed_units():
     assert list(pl["mask"]) == [0b01, 0b10, 0b11]
 
 
+def test_plan_depends_on_coefficient_magnitudes_only():
+    """The utility of a unit is |coef| * ||Delta|| (Prop. 2): flipping the sign of some
+    experts' coefficients leaves the order and the selection unchanged, and scaling one
+    expert's coefficient moves its units in the order"""
+    rng = np.random.default_rng(31)
+    for trial in range(20):
+        K, nb = 3, 12
+        blk_len, norm, maxabs, nnz, alpha = _tiny_plan_case(rng, K, nb, trial % 2 == 0)
+        signs = np.where(rng.random(K) < 0.5, -1.0, 1.0).astype(np.float32)
+        signs[0] = -1.0
+        B = int(rng.integers(0, int(blk_len.sum()) * K * 2 + 1))
+        for sm in (0, 1):
+            a = oracle.plan(K, blk_len, np.zeros(nb, np.uint32), 1, 2, oracle.Op(oracle.TA, K, alpha=alpha, score_mode=sm),
+                            norm, maxabs, nnz, None, B)
+            b = oracle.plan(K, blk_len, np.zeros(nb, np.uint32), 1, 2,
+                            oracle.Op(oracle.TA, K, alpha=alpha * signs, score_mode=sm), norm, maxabs, nnz, None, B)
+            assert np.array_equal(a["order"], b["order"]) and np.array_equal(a["mask"], b["mask"])
+            assert a["chat"] == b["chat"] and a["set_hash"] == b["set_hash"]
+    # expert 1's coefficient x 4 lifts its unit above expert 0's (norms 1.0 vs 2.0, unit ids 0 and 1)
+    blk_len = np.full(1, 4, np.uint32)
+    norm = np.array([[2.0], [1.0]], np.float32)
+    nnz = np.full((2, 1), 4, np.uint32)
+    for al, want in (([1.0, 1.0], [0, 1]), ([1.0, -4.0], [1, 0])):
+        p = oracle.plan(2, blk_len, np.zeros(1, np.uint32), 1, 2, oracle.Op(oracle.TA, 2, alpha=al), norm, norm, nnz,
+                        None, 8)
+        assert p["order"].tolist() == want and p["mask"].tolist() == [1 << want[0]]
+
+
 # ---- digest ----------------------------------------------------------------------------------------------
 
 def test_fnv1a_published_vectors():
@@ -601,6 +706,32 @@ def test_avg_renorm_full_budget_equals_avg(tiny_family):
     r = oracle.merge(of, oracle.Op(oracle.AVG_RENORM, fam.K, alpha=a))
     m = oracle.merge(of, oracle.Op(oracle.AVG, fam.K, alpha=a))
     assert np.array_equal(r.view(np.uint32), m.view(np.uint32))
+
+
+def test_avg_renorm_full_budget_plan_equals_avg(tiny_family):
+    """Through the plan, as the pipeline runs it: at the full budget the mask holds every
+    unit with nnz > 0 but no unit whose delta is exactly zero (those are not candidates).
+    The renormalised AVG over that mask, told the zero deltas by the catalog's nnz (or
+    finding them in the data), still divides by the sum of all K coefficients, so it equals
+    the full-read AVG (Eq. 5).  Each expert here has its own blocks set equal to the base."""
+    fam, base, experts = tiny_family
+    bo, bl, _ = fam.block_table()
+    experts = [e.copy() for e in experts]
+    for i, e in enumerate(experts):
+        for blk in range(i, len(bl), 7 + i):
+            e[int(bo[blk]):int(bo[blk] + bl[blk])] = base[int(bo[blk]):int(bo[blk] + bl[blk])]
+    of = oracle_family(fam, base, experts)
+    norm, maxabs, nnz = oracle.index(of)
+    assert (nnz == 0).any(axis=1).all() and ((nnz == 0).sum(axis=0) < fam.K).all()
+    a = [0.25] * fam.K
+    op = oracle.Op(oracle.AVG_RENORM, fam.K, alpha=a)
+    full = fam.K * int(bl.sum()) * 4
+    pl = oracle.plan(fam.K, bl, np.zeros(len(bl), np.uint32), 1, 4, op, norm, maxabs, nnz, None, full)
+    assert pl["n_sel"] == int((nnz > 0).sum())
+    m = oracle.merge(of, oracle.Op(oracle.AVG, fam.K, alpha=a))
+    for catalog in (nnz, None):
+        r = oracle.merge(of, op, mask=pl["mask"], nnz=catalog)
+        assert np.array_equal(r.view(np.uint32), m.view(np.uint32))
 
 
 def test_avg_renorm_coefficient_drift_bound(tiny_family):
@@ -726,6 +857,18 @@ def test_fallback_worked_example():
     assert p["mask"].tolist() == [0, 0, 0, 2, 3] and p["chat"] == 24
     p = _fallback_plan(80)
     assert p["mask"].tolist() == [3] * 5 and p["chat"] == 80 and p["n_sel"] == 7
+
+
+def test_fallback_worked_example_with_unequal_coefficients():
+    """Hand-worked, the catalog above under TA with alpha = (0.25, -2): scores are |alpha_i|
+    times the norm.  (0, t0) id 0: 0.25 * 5 = 1.25; (1, t1) id 7: 2 * 6 = 12; (1, b0..b2)
+    ids 1, 3, 5: 2 each; (0, b4) id 8: 0.5; (0, b3) id 6: 0.25.  Order 7, 1, 3, 5, 0, 8, 6.
+    B = 40: 7 (16), 1, 3, 5 (40), then nothing fits: bit 1 on every block."""
+    blk_len, bt, norm, nnz = _fallback_worked_catalog()
+    op = oracle.Op(oracle.TA, 2, alpha=[0.25, -2.0])
+    p = oracle.plan(2, blk_len, bt, 2, 2, op, norm, np.ones_like(norm), nnz, None, 40, blk_tensor=bt)
+    assert p["order"].tolist() == [7, 1, 3, 5, 0, 8, 6]
+    assert p["mask"].tolist() == [2] * 5 and p["chat"] == 40 and p["n_sel"] == 4
 
 
 def test_fallback_needs_the_tensor_map():
