@@ -228,9 +228,12 @@ def profiled_traffic(workload: str):
 
 # ---- CPU oracle sample ----------------------------------------------------------------------------
 
-def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
-    """Time the oracle (index, plan per budget, merge per budget) on a bounded sample of the
-    workload's blocks.  Returns (params_merged_per_s, seconds, sample_description)."""
+def oracle_sample(w, fam, target_s: float):
+    """A bounded sample of the workload for the CPU oracle: blocks evenly spaced over the
+    family, as many as about target_s seconds of oracle work (index, then plan and merge at
+    every budget) take, regenerated on the host once.  Returns (run, description); run()
+    times one full pass of the oracle over the sample and returns (merged params/s, seconds).
+    The oracle keeps nothing between passes, so every pass does the whole work again."""
     import numpy as np
     import oracle
 
@@ -238,8 +241,9 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
     bo, bl, bt = fam.block_table()
     budgets = w["budgets"]
     miss_all = fallback_missing(fam, fam.K) if w.get("fallback") else None
+    es = fam.elem_size
 
-    def run(blocks):
+    def prepare(blocks):
         data = [fam.block_host(int(b)) for b in blocks]
         lens = np.array([bl[b] for b in blocks], np.uint32)
         offs = np.zeros(len(blocks), np.uint64)
@@ -251,38 +255,58 @@ def oracle_sample_run(w, fam, target_s: float, n_budgets_from=None):
         experts = [np.concatenate([d[1][i] for d in data]) for i in range(fam.K)]
         groups = np.zeros(len(blocks), np.uint32)
         of = oracle.Family(fam.dtype, offs, lens, groups, 1, base, experts)
-        es = fam.elem_size
-        full = fam.K * int(lens.sum()) * es
+        catalog = None
         if miss_all is not None:
-            # the catalog is imported, not computed: build it before the clock starts
+            # the catalog is imported, not computed: built before any clock starts
             norm, maxabs, nnz = oracle.index(of)
             nnz = nnz.copy()
             nnz[miss_all[:, blocks]] = oracle.NNZ_MISSING
             tmap = np.unique(bt[blocks], return_inverse=True)[1].astype(np.uint32)
+            catalog = (norm, maxabs, nnz, tmap)
+        return of, lens, groups, catalog
+
+    def timed(sample):
+        of, lens, groups, catalog = sample
+        full = fam.K * int(lens.sum()) * es
         t0 = time.perf_counter()
-        if miss_all is None:
+        if catalog is None:
             norm, maxabs, nnz = oracle.index(of)
             tmap = None
+        else:
+            norm, maxabs, nnz, tmap = catalog
         tau = oracle.ties_thresholds(of, oop.density) if oop.kind == oracle.TIES else None
         for f in budgets:
             pl = oracle.plan(fam.K, lens, groups, 1, es, oop, norm, maxabs, nnz, tau, math.floor(f * full),
                              blk_tensor=tmap)
             m_tau = oracle.ties_masked_thresholds(of, oop.density, pl["mask"]) if oop.kind == oracle.TIES_MASKED else tau
             oracle.merge(of, oop, tau=m_tau, mask=pl["mask"], nnz=nnz if tmap is not None else None)
-        dt = time.perf_counter() - t0
-        return dt, int(lens.sum())
+        return time.perf_counter() - t0
 
     nb = fam.n_blocks
     # per-block cost from an evenly spaced probe (active and inactive blocks differ in cost)
     probe = sorted(set(int(x) for x in np.linspace(0, nb - 1, min(nb, 8))))
-    dt1, p1 = run(probe)
+    dt1 = timed(prepare(probe))
     n = max(1, min(nb, int(target_s / max(dt1 / len(probe), 1e-6))))
     blocks = sorted(set(int(x) for x in np.linspace(0, nb - 1, n)))
-    dt, params = run(blocks)
+    sample = prepare(blocks)
+    params = int(sample[1].sum())
     first = "catalog imported (computed before timing)" if miss_all is not None else "oracle index"
     desc = (f"{len(blocks)} of {nb} blocks ({params} params) evenly spaced over the family, regenerated on the "
-            f"host; {first} + plan and merge at budgets {budgets} (budget relative to the sample)")
-    return len(budgets) * params / dt, dt, desc
+            f"host once; {first} + plan and merge at budgets {budgets} (budget relative to the sample)")
+
+    def run():
+        dt = timed(sample)
+        return len(budgets) * params / dt, dt
+
+    return run, desc
+
+
+def oracle_sample_run(w, fam, target_s: float):
+    """One timed pass of the oracle over a bounded sample (oracle_sample):
+    (merged params/s, seconds, sample description)"""
+    run, desc = oracle_sample(w, fam, target_s)
+    v, dt = run()
+    return v, dt, desc
 
 
 def cpu_info():
@@ -798,12 +822,14 @@ def k_sweep(args):
 def reference(args):
     W = workloads()[args.workload]
     fam = W["make"]()
-    per_step = max(0.2, min(30.0, 150.0 / max(1, args.steps + args.warmup)))
+    # about a minute of oracle work over all warm-up and timed steps, on one sample
+    per_step = max(0.2, min(20.0, 60.0 / max(1, args.steps + args.warmup)))
+    run, desc = oracle_sample(W, fam, per_step)
     for _ in range(args.warmup):
-        oracle_sample_run(W, fam, per_step)
-    vals, secs, desc = [], [], ""
+        run()
+    vals, secs = [], []
     for _ in range(args.steps):
-        v, dt, desc = oracle_sample_run(W, fam, per_step)
+        v, dt = run()
         vals.append(v)
         secs.append(dt)
     v = statistics.mean(vals)
