@@ -48,7 +48,7 @@ typedef int32_t mp_status;
 #define MP_ERR_NONFINITE (-4)   /* a delta was NaN or infinite (reported by accessors) */
 #define MP_ERR_BUDGET (-5)      /* realized reads exceeded the plan (Prop. 1 violated) */
 #define MP_ERR_TIMEOUT (-6)     /* a bounded device wait gave up (reported by accessors) */
-#define MP_ERR_UNSUPPORTED (-7) /* valid request this build does not handle */
+#define MP_ERR_UNSUPPORTED (-7) /* a valid request the library does not handle */
 #define MP_ERR_MISMATCH (-8)    /* handles that do not belong together */
 
 typedef struct CUstream_st* mp_stream;

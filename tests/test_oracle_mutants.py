@@ -10,8 +10,8 @@ live in a temporary directory.
 Left out on purpose: changes that swap one valid reading for another (the hash's key
 rotation, the digest's byte layout, which Philox word feeds which element, rounding
 p * 65536 down rather than up for the DARE threshold).  Those are
-conventions the paper leaves open; the GPU parity tests hold both sides to the one
-stated for this build.
+conventions the paper leaves open; the GPU parity tests hold both sides to the one the
+implementation states.
 """
 import concurrent.futures
 import os
