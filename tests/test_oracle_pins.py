@@ -586,6 +586,39 @@ def test_plan_ties_prunes_fully_trimmed_units():
     assert list(pl["mask"]) == [0b01, 0b10, 0b11]
 
 
+def test_plan_is_invariant_under_relabelling():
+    """Alg. 1 looks only at scores and costs: with distinct scores, relabelling the experts
+    (statistics and coefficients together) or reordering the blocks relabels the selection,
+    the traversal order and C_hat in the same way"""
+    rng = np.random.default_rng(41)
+    for trial in range(25):
+        K, nb = int(rng.integers(2, 6)), int(rng.integers(3, 30))
+        blk_len = rng.integers(1, 9, nb).astype(np.uint32)
+        norm = rng.uniform(0.1, 4.0, (K, nb)).astype(np.float32)
+        nnz = (rng.random((K, nb)) > 0.15).astype(np.uint32) * 3
+        alpha = rng.uniform(0.2, 1.0, K).astype(np.float32)
+        pe, pb = rng.permutation(K), rng.permutation(nb)      # expert i -> pe[i], block b -> pb[b]
+        norm2, nnz2 = np.empty_like(norm), np.empty_like(nnz)
+        norm2[pe[:, None], pb[None, :]] = norm
+        nnz2[pe[:, None], pb[None, :]] = nnz
+        alpha2 = np.empty_like(alpha)
+        alpha2[pe] = alpha
+        len2 = np.empty_like(blk_len)
+        len2[pb] = blk_len
+        total = int(blk_len.sum()) * K * 2
+        for B in (0, total // 5, total // 2, total):
+            a = oracle.plan(K, blk_len, np.zeros(nb, np.uint32), 1, 2, oracle.Op(oracle.TA, K, alpha=alpha),
+                            norm, norm, nnz, None, B)
+            b = oracle.plan(K, len2, np.zeros(nb, np.uint32), 1, 2, oracle.Op(oracle.TA, K, alpha=alpha2),
+                            norm2, norm2, nnz2, None, B)
+            sel_a = {(int(pb[bb]), int(pe[i])) for bb in range(nb) for i in range(K) if (a["mask"][bb] >> i) & 1}
+            sel_b = {(bb, i) for bb in range(nb) for i in range(K) if (b["mask"][bb] >> i) & 1}
+            assert sel_a == sel_b and a["chat"] == b["chat"] and a["n_cand"] == b["n_cand"]
+            order_a = [(int(pb[u // K]), int(pe[u % K])) for u in a["order"].tolist()]
+            order_b = [(u // K, u % K) for u in b["order"].tolist()]
+            assert order_a == order_b
+
+
 def test_plan_depends_on_coefficient_magnitudes_only():
     """The utility of a unit is |coef| * ||Delta|| (Prop. 2): flipping the sign of some
     experts' coefficients leaves the order and the selection unchanged, and scaling one
