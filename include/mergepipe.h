@@ -293,7 +293,9 @@ void mp_free(void* handle);
 
 /* Host copies of the index statistics, expert-major [K][n_blocks]; tau is [K][n_groups]
    (n_groups = n_tensors for trim_scope 0, 1 for trim_scope 1).  Any pointer may be NULL.
-   Waits for the index work.  Returns MP_ERR_NONFINITE if a delta was not finite. */
+   Waits for the index work.  Errors: MP_ERR_INVALID_ARG (not an index), MP_ERR_NONFINITE
+   (a delta was not finite), MP_ERR_TIMEOUT (a bounded device wait in the index kernels gave
+   up), MP_ERR_CUDA (a copy failed).  The arrays are filled before the error word is read. */
 mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint32_t* nnz, uint32_t* tau);
 
 /* Geometry of an index: number of blocks, units (K * n_blocks) and TIES trim groups. */
@@ -301,13 +303,18 @@ mp_status mp_index_shape(const mp_index* index, uint64_t* n_blocks, uint64_t* n_
 
 /* Plan summary (waits for the plan work).  mask: n_blocks words; order: the traversal
    order (unit ids of the n_candidates candidates, decreasing score).  Any pointer may be
-   NULL. */
+   NULL.  Errors: MP_ERR_INVALID_ARG (not a plan), MP_ERR_NONFINITE (the index saw a
+   non-finite delta), MP_ERR_UNSUPPORTED (a catalog entry without statistics met a plan with
+   no tensor map), MP_ERR_TIMEOUT (a bounded device wait gave up), MP_ERR_BUDGET (planned
+   bytes above the budget: never expected, Prop. 1), MP_ERR_CUDA. */
 mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t* n_selected,
                        uint64_t* n_candidates, uint64_t* digest, uint32_t* mask, uint32_t* order);
 
 /* Manifest (waits for the merge): realized expert-read bytes per expert (K words),
-   their total, touched blocks (#{b : mask_b != 0}) and the plan digest.  Returns
-   MP_ERR_BUDGET if realized reads exceed the planned bytes. */
+   their total, touched blocks (#{b : mask_b != 0}) and the plan digest.  Errors:
+   MP_ERR_INVALID_ARG (not a manifest), MP_ERR_TIMEOUT (a bounded device wait in the merge
+   gave up), MP_ERR_CUDA (the merge kernels reported another error), MP_ERR_BUDGET (realized
+   reads above the planned bytes: never expected). */
 mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_bytes_per_expert,
                            uint64_t* realized_total, uint64_t* touched_blocks, uint64_t* digest);
 
