@@ -74,6 +74,8 @@ MUTANTS = [
     ("plan_zero_blocks_are_candidates", "if (nnz[s] == 0) continue;", ""),
     ("plan_no_ties_pruning", "if (op->kind == ORC_TIES && orc_ties_key(maxabs[s])",
      "if (0 && orc_ties_key(maxabs[s])"),
+    ("plan_ties_tau_of_first_group", "orc_ties_key(maxabs[s]) < tau[(size_t)i * n_groups + blk_group[b]]",
+     "orc_ties_key(maxabs[s]) < tau[(size_t)i * n_groups]"),
     ("plan_ties_prunes_at_tau", "orc_ties_key(maxabs[s]) < tau[", "orc_ties_key(maxabs[s]) <= tau["),
     ("plan_unit_id_expert_major",
      "q[nq].unit = (uint32_t)(b * K + i);\n      q[nq].cost = (uint64_t)blk_len[b] * elem_size;",
@@ -97,6 +99,8 @@ MUTANTS = [
      "q[nq].unit = (uint32_t)(b * K + (K - 1 - i));\n        q[nq].cost = cost;"),
     ("fallback_per_byte_of_first_block", "if (op->score_mode) q[nq].score = q[nq].score / (float)cost;",
      "if (op->score_mode) q[nq].score = q[nq].score / (float)(blk_len[b] * elem_size);"),
+    ("fallback_norm_includes_missing_entries", "if (nnz[s2] != ORC_NNZ_MISSING) ss = fmaf(norm[s2], norm[s2], ss);",
+     "ss = fmaf(norm[s2], norm[s2], ss);"),
     ("fallback_without_coefficient", "q[nq].score = fabsf(coef) * sqrtf(ss);", "q[nq].score = sqrtf(ss);"),
     # Philox and DARE
     ("philox_multiplies_wrong_word", "uint64_t p0 = (uint64_t)0xD2511F53u * c0;",
@@ -137,6 +141,10 @@ MUTANTS = [
     ("ties_negative_mean_over_positive_count", "else if (P < -Nn) m = Nn / (float)cn;",
      "else if (P < -Nn) m = Nn / (float)(cp > 0 ? cp : 1);"),
     ("renorm_sums_every_coefficient", "if (((mask | known_zero) >> i) & 1u) {", "if (1) {"),
+    ("dare_ties_without_rescale", "            dh = d * sigma;\n", "            dh = d;\n"),
+    ("full_read_mask_drops_last_expert", "((1u << f->K) - 1u);", "((1u << f->K) - 1u) >> 1;"),
+    ("dare_counter_block_local_in_merge", "} else if (orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) {",
+     "} else if (orc_dare_keep(op->seed, i, k, op->drop_p)) {"),
     ("merge_known_zero_from_nonzero", "if (nnz[(size_t)i * f->n_blocks + b] == 0) known_zero |= 1u << i;",
      "if (nnz[(size_t)i * f->n_blocks + b] != 0) known_zero |= 1u << i;"),
 ]

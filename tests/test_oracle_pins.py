@@ -586,6 +586,34 @@ def test_plan_ties_prunes_fully_trimmed_units():
     assert list(pl["mask"]) == [0b01, 0b10, 0b11]
 
 
+def test_plan_ties_candidates_are_units_with_a_surviving_entry(tiny_family):
+    """TIES pruning is exact, per trim group: with one group per tensor, a unit is a
+    candidate iff some entry of it survives its own tensor's trim, i.e. the largest bf16
+    magnitude key among its deltas (computed here with torch from the data) reaches tau of
+    (its expert, its tensor).  The tensors' thresholds differ, so a unit judged against
+    another tensor's tau shows."""
+    fam, base, experts = tiny_family
+    of = oracle_family(fam, base, experts)
+    bo, bl, bt = fam.block_table()
+    norm, maxabs, nnz = oracle.index(of)
+    dens = 0.2
+    tau = oracle.ties_thresholds(of, dens)
+    assert len(set(tau[0].tolist())) > 1
+    want = set()
+    for i, e in enumerate(experts):
+        d = e.astype(np.float32) - base.astype(np.float32)
+        keys = (bf16_bits_torch(np.abs(d)) & 0x7FFF).astype(np.int64)
+        for b in range(len(bl)):
+            blk = keys[int(bo[b]):int(bo[b] + bl[b])]
+            if nnz[i, b] > 0 and blk.max() >= tau[i, bt[b]]:
+                want.add(b * fam.K + i)
+    op = oracle.Op(oracle.TIES, fam.K, lam=1.0, density=dens)
+    full = fam.K * int(bl.sum()) * 4
+    p = oracle.plan(fam.K, bl, bt, len(fam.tensors), 4, op, norm, maxabs, nnz, tau, full)
+    assert 0 < len(want) < fam.K * len(bl)
+    assert set(p["order"].tolist()) == want and p["n_cand"] == len(want) and p["n_sel"] == len(want)
+
+
 def test_plan_is_invariant_under_relabelling():
     """Alg. 1 looks only at scores and costs: with distinct scores, relabelling the experts
     (statistics and coefficients together) or reordering the blocks relabels the selection,
