@@ -61,6 +61,10 @@ MUTANTS = [
      "return orc_splitmix64(orc_block_hash_sum(bytes, len));"),
     ("hash_even_key", "const uint64_t a = k | 1u,", "const uint64_t a = k,"),
     ("hash_key_not_per_vector", "const uint64_t k = orc_splitmix64(q);", "const uint64_t k = orc_splitmix64(0);"),
+    ("index_hashes_block_major", "expert_hash[(uint64_t)i * f->n_blocks + b] = ", "expert_hash[b * f->K + i] = "),
+    ("index_hashes_length_in_elements", "const uint64_t len = (uint64_t)f->blk_len[b] * es;",
+     "const uint64_t len = (uint64_t)f->blk_len[b];"),
+    ("key_hist_accepts_nonfinite", "    if (!is_finite_f(d)) return ORC_ENONFINITE;\n    hist[", "    hist["),
     # Alg. 1 plan
     ("plan_stops_at_first_overflow", "if (chat + q[r].cost <= budget) {",
      "if (chat + q[r].cost > budget) break;\n    {"),
@@ -132,6 +136,7 @@ MUTANTS = [
     ("dare_ties_trims", "} else if (orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) {",
      "} else if (orc_ties_key(d) >= 0x3F80u) {"),
     ("renorm_ignores_known_zero", "if (((mask | known_zero) >> i) & 1u) {", "if ((mask >> i) & 1u) {"),
+    ("renorm_accepts_nonpositive_alpha", "        if (!(op->alpha[i] > 0.0f)) return ORC_EINVAL;\n", ""),
     ("renorm_not_normalised", "op->kind == ORC_AVG_RENORM ? op->alpha[i] / s_sel : op->alpha[i];",
      "op->alpha[i];"),
     ("merge_tau_of_first_group", "tau_k[i] = tau[(size_t)i * f->n_groups + f->blk_group[b]];",

@@ -135,6 +135,22 @@ def test_block_stats_rejects_nonfinite():
         assert ei.value.rc == oracle.ENONFINITE
 
 
+def test_ties_key_histogram_rejects_nonfinite():
+    """a non-finite delta has no magnitude key: the TIES threshold pass refuses it, as the
+    statistics pass does (the library reports MP_ERR_NONFINITE)"""
+    b = to_bf16(np.zeros(64))
+    for bad in [np.nan, np.inf, -np.inf]:
+        e = np.zeros(64, np.float32)
+        e[40] = bad
+        with pytest.raises(oracle.OracleError) as ei:
+            oracle.key_hist(oracle.BF16, b, to_bf16(e))
+        assert ei.value.rc == oracle.ENONFINITE
+        fam = oracle.Family(oracle.BF16, [0], [64], [0], 1, b, [to_bf16(np.zeros(64)), to_bf16(e)])
+        with pytest.raises(oracle.OracleError) as ei:
+            oracle.ties_thresholds(fam, 0.5)
+        assert ei.value.rc == oracle.ENONFINITE
+
+
 def test_index_family_layout(tiny_family):
     """per-unit statistics land at [expert, block] for every block of every tensor"""
     fam, base, experts = tiny_family
@@ -757,6 +773,20 @@ def test_avg_renorm_worked_example():
     assert out_all.tolist() == [5.25, 3.5, 5.0, 4.5]
     out_none = oracle.merge_block(oracle.F32, 0, base, [e0, e1, e2], 0, op)
     assert out_none.tolist() == base.tolist()
+
+
+def test_avg_renorm_needs_positive_coefficients():
+    """the renormalised average divides by the sum of the taking-part coefficients, which
+    needs every coefficient > 0 (else the sum can vanish or flip sign): a zero or negative
+    alpha is refused, as the library refuses it"""
+    base = np.zeros(8, np.float32)
+    ex = [np.full(8, 1.0, np.float32), np.full(8, 2.0, np.float32)]
+    for alpha in ([0.5, 0.0], [0.5, -0.5], [-1.0, 1.0]):
+        with pytest.raises(oracle.OracleError) as ei:
+            oracle.merge_block(oracle.F32, 0, base, ex, 0b11, oracle.Op(oracle.AVG_RENORM, 2, alpha=alpha))
+        assert ei.value.rc == oracle.EINVAL
+    out = oracle.merge_block(oracle.F32, 0, base, ex, 0b11, oracle.Op(oracle.AVG_RENORM, 2, alpha=[0.5, 0.5]))
+    assert out.tolist() == [1.5] * 8
 
 
 def test_avg_renorm_full_budget_equals_avg(tiny_family):
