@@ -1,5 +1,5 @@
-"""Host logic of bench.py that needs no GPU: the affine read-time model fit and the seeded
-pattern of catalog entries without statistics."""
+"""Host logic of bench.py that needs no GPU: the affine read-time model fit, the seeded
+pattern of catalog entries without statistics and the fidelity columns."""
 import math
 import os
 import sys
@@ -44,3 +44,55 @@ def test_missing_entries_pattern_is_seeded_and_pair_dominated():
     c = synth.missing_entries(fam, fam.K, pair_frac=0.0, entry_frac=0.0)
     assert c.sum() == int((bt == big).sum())     # only the forced pair
     assert 0.0 < a.mean() < 0.5
+
+
+def test_fidelity_columns_match_their_definitions():
+    """Tab. 3's fidelity columns as bench.py reports them, against the definitions written
+    out over the blocks: rel. l2 = ||M_A - M_full|| / ||M_full|| over the whole checkpoint;
+    P95 = the 95th percentile (linear interpolation) over blocks of ||d_b|| / ||M_full[b]||.
+    The family has a ragged last block in every tensor; perturbations sit in a few blocks."""
+    import torch
+
+    import bench
+
+    class Fam:
+        block_elems = 64
+        tensors = [(0, 300), (304, 130), (448, 64)]
+
+        def layout(self):
+            offs = np.array([o for o, _ in self.tensors], np.int64)
+            nums = np.array([n for _, n in self.tensors], np.int64)
+            return offs, nums, 512
+
+    fam = Fam()
+    rng = np.random.default_rng(7)
+    full = torch.from_numpy(rng.standard_normal(512).astype(np.float32))
+    budgets = [1.0, 0.5, 0.25]
+    outs = [full.clone()]
+    for scale in (1e-3, 1e-2):
+        o = full.clone()
+        idx = torch.from_numpy(rng.choice(512, 40, replace=False))
+        o[idx] += torch.from_numpy((rng.standard_normal(40) * scale).astype(np.float32))
+        outs.append(o)
+    per = [{} for _ in budgets]
+    bench.fidelity_vs_full(fam, budgets, outs, False, per)
+    F = full.double().numpy()
+    for k, out in enumerate(outs):
+        D = out.double().numpy() - F
+        num = den = 0.0
+        rel = []
+        for o, n in fam.tensors:
+            for s in range(0, n, fam.block_elems):
+                e = min(n, s + fam.block_elems)
+                d, f = D[o + s:o + e], F[o + s:o + e]
+                num += float(d @ d)
+                den += float(f @ f)
+                rel.append(math.sqrt(float(d @ d) / float(f @ f)))
+        assert math.isclose(per[k]["rel_l2_vs_full"], math.sqrt(num / den), rel_tol=1e-12)
+        assert math.isclose(per[k]["p95_block_dev_vs_full"], float(np.percentile(np.float32(rel), 95)),
+                            rel_tol=1e-6, abs_tol=1e-12)
+    assert per[0]["rel_l2_vs_full"] == 0.0 and per[0]["p95_block_dev_vs_full"] == 0.0
+    # no full-read budget in the sweep (or one shared output buffer): nothing is reported
+    per = [{}]
+    bench.fidelity_vs_full(fam, [0.5], outs[1:2], False, per)
+    assert per == [{}]
