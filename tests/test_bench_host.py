@@ -1,5 +1,6 @@
 """Host logic of bench.py that needs no GPU: the affine read-time model fit, the seeded
-pattern of catalog entries without statistics and the fidelity columns."""
+pattern of catalog entries without statistics, the fidelity columns, the agreement of the
+library's and the oracle's operator for every workload, and the clock record."""
 import math
 import os
 import sys
@@ -96,3 +97,53 @@ def test_fidelity_columns_match_their_definitions():
     per = [{}]
     bench.fidelity_vs_full(fam, [0.5], outs[1:2], False, per)
     assert per == [{}]
+
+
+def test_every_workload_gives_the_library_and_the_oracle_the_same_operator():
+    """bench.py builds each workload's operator twice, for the library and for the oracle
+    (the CPU baseline); both must describe the same merge: kind, coefficients, lambda,
+    density, trim scope, drop probability, seed and score mode"""
+    import bench
+
+    for name, w in bench.workloads().items():
+        fam = w["make"]()
+        g, o = bench.make_ops(w, fam.K)
+        c = g.c
+        assert c.kind == o.kind, name
+        if o.alpha is None:
+            assert g.alpha is None, name
+        else:
+            assert np.array_equal(g.alpha, o.alpha) and len(o.alpha) == fam.K, name
+        assert np.float32(c.lambda_) == np.float32(o.lam) and np.float32(c.density) == np.float32(o.density), name
+        assert (c.trim_scope, c.drop_p, c.seed, c.score_mode) == (o.trim_scope, o.drop_p, o.seed, o.score_mode), name
+
+
+def test_clock_sampler_summary():
+    """the clock record the bench line carries: median SM clock under load, the maximum, and
+    every throttle reason seen active in any sample (malformed lines are skipped)"""
+    import bench
+
+    class Done:
+        def terminate(self):
+            pass
+
+        def wait(self, timeout=None):
+            return 0
+
+    cs = bench.ClockSampler(0)
+    cs.proc = Done()
+    cs.lines = [
+        "0, 2070, 2070, 900.1, 0x0, Not Active, Not Active, Not Active, Not Active",
+        "0, 2055, 2070, 1390.0, 0x4, Not Active, Not Active, Not Active, Active",
+        "garbage line",
+        "0, 1980, 2070, 1400.0, 0x4, Not Active, Not Active, Not Active, Active",
+        "0, [N/A], 2070, 1400.0, 0x0, Not Active, Not Active, Not Active, Not Active",
+    ]
+    s = cs.stop()
+    assert s == {"sm_mhz": 2055.0, "sm_max_mhz": 2070.0, "reasons": ["sw_power_cap"], "samples": 3}
+    cs = bench.ClockSampler(0)
+    cs.proc = Done()
+    cs.lines = ["0, 1500, 2070, 800.0, 0x40, Active, Not Active, Active, Not Active"]
+    assert cs.stop()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
+    cs = bench.ClockSampler(0)             # nvidia-smi could not be started: no record
+    assert cs.stop() is None
