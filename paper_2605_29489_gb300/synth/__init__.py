@@ -8,8 +8,8 @@ may be partial; no block crosses a tensor).  Expert i differs from the base by
 a per-(expert, block) scale times an approximate standard normal variate:
 
 * active blocks: scale ~ lognormal(log_mu, log_sigma);
-* inactive blocks: scale = ``inactive_scale`` (1e-7, which bf16 storage mostly
-  rounds away, leaving exactly zero deltas).
+* inactive blocks: scale = ``inactive_scale`` (1e-7; bf16 storage rounds it away
+  for about 99.9 % of the elements, all but those whose base is near zero).
 
 The active set is either one set shared by all experts (a seeded choice of
 exactly floor(active_frac * n_blocks) blocks) or an independent set per expert.
