@@ -345,7 +345,10 @@ int orc_index_hashes(const orc_family* f, uint64_t* base_hash, uint64_t* expert_
  *    bit i on every block of t; it counts once in n_sel and set_hash.
  * Pins: brute force over all subsets on tiny inputs; the cardinality-knapsack optimum
  * when all costs are equal; Prop. 1 (C_hat <= B); full budget selects every candidate;
- * for the fallback, a hand-worked catalog and the known-part norm against the deltas.
+ * the order depends on |coef| only; relabelling experts or reordering blocks relabels the
+ * plan; TIES candidates per trim group against keys computed from the data; for the
+ * fallback, hand-worked catalogs (equal and unequal signed coefficients) and the
+ * known-part norm against the deltas.
  * ------------------------------------------------------------------------------------- */
 typedef struct {
   float score;
@@ -563,10 +566,13 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  *        disjoint mean without magnitude trimming: d^_i = A_i (keep_i ? delta_i * sigma : 0),
  *        then P, N, gamma, m and out as TIES
  * round = bf16 round-to-nearest-even, or none for fp32 checkpoints.
- * Pins: hand-computed TIES, AVG and renormalised-AVG examples; Eq. 5 against an fp64
- * restatement of the unmasked operator (within one bf16 ulp); Prop. 2 bound and the
- * coefficient-drift bound of App. A.1; DARE at p = 0 equals AVG and the DARE mean over
- * seeds tends to AVG; DARE-TIES at p = 0 equals TIES at density 1.
+ * Pins: hand-computed TIES, AVG and renormalised-AVG examples (an omitted expert counts as
+ * zero whatever its data); Eq. 5 against an fp64 restatement of the unmasked operator
+ * (within one bf16 ulp); per-tensor TIES trims are separable; Prop. 2 bound and the
+ * coefficient-drift bound of App. A.1; the renormalised AVG through the full-budget plan
+ * equals AVG; DARE at p = 0 equals AVG (also over 2^21 entries), drops are independent
+ * across blocks and the DARE mean over seeds tends to AVG; DARE-TIES at p = 0 equals TIES
+ * at density 1.
  * ------------------------------------------------------------------------------------- */
 int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const void* const* experts,
                     uint32_t mask, uint32_t known_zero, const orc_op* op, const uint32_t* tau_k, void* out) {
