@@ -22,7 +22,8 @@
 /* ---------------------------------------------------------------------------------------
  * Element conversion.  bf16 is the upper half of an IEEE binary32; rounding to
  * bf16 is round-to-nearest-even on the dropped 16 bits.
- * Pin: torch's CPU bfloat16 conversion on random and edge values.
+ * Pins: torch's CPU bfloat16 conversion on random and edge values; a NaN stays a NaN,
+ * also one whose payload lies only in the dropped bits.
  * ------------------------------------------------------------------------------------- */
 static uint32_t f2u(float f) {
   uint32_t u;
@@ -158,7 +159,8 @@ int orc_index(const orc_family* f, float* norm, float* maxabs, uint32_t* nnz) {
  * magnitude key with multiplicity (ties at tau are all kept); k = 0 keeps nothing.  The
  * threshold comes from the full delta (an operator parameter theta, recorded with the
  * plan), so Psi stays non-anticipatory and equals standard TIES at A = 1.
- * Pin: a full sort of the keys on random tensors; hand-computed examples.
+ * Pins: a full sort of the keys on random tensors; hand-computed examples; a non-finite
+ * delta is refused.
  * ------------------------------------------------------------------------------------- */
 int orc_key_hist(int dtype, uint64_t n, const void* base, const void* expert, uint64_t* hist) {
   if (!hist || (n > 0 && (!base || !expert))) return ORC_EINVAL;
