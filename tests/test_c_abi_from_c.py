@@ -70,6 +70,29 @@ int main(void) {
                         &op, 1000, w, w, s8, NULL) == MP_ERR_INVALID_ARG);
   CHECK(strstr(mp_last_error(), "aligned") != NULL);
 
+  /* every entry point refuses a NULL handle with MP_ERR_INVALID_ARG and a message */
+  uint64_t u64 = 0, u64b = 0;
+  uint32_t u32 = 0;
+  mp_plan_t* pl = (mp_plan_t*)1;
+  mp_manifest* man = (mp_manifest*)1;
+  CHECK(mp_plan(NULL, &op, 100, NULL, &pl) == MP_ERR_INVALID_ARG && pl == NULL);
+  CHECK(mp_merge(&f, NULL, NULL, base, NULL, &man) == MP_ERR_INVALID_ARG && man == NULL);
+  man = (mp_manifest*)1;
+  CHECK(mp_merge_touched(&f, NULL, NULL, base, NULL, &man) == MP_ERR_INVALID_ARG && man == NULL);
+  CHECK(mp_index_stats(NULL, norm, maxabs, nnz, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_index_shape(NULL, &u64, &u64b, &u32) == MP_ERR_INVALID_ARG);
+  CHECK(mp_index_hashes(&f, NULL, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_index_hash_values(NULL, &u64, &u64b) == MP_ERR_INVALID_ARG);
+  CHECK(mp_plan_info(NULL, &u64, &u64b, NULL, NULL, NULL, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_manifest_info(NULL, &u64, &u64b, NULL, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_manifest_validate(&f, NULL, NULL, base, NULL, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_manifest_validation(NULL, &u64, &u64b, NULL) == MP_ERR_INVALID_ARG);
+  CHECK(mp_manifest_threshold_reads(NULL, &u64) == MP_ERR_INVALID_ARG);
+  CHECK(mp_manifest_lineage(NULL, &u64) == MP_ERR_INVALID_ARG);
+  CHECK(strstr(mp_last_error(), "handle") != NULL);
+  CHECK(mp_plan_noalloc(3, 6, 1, MP_BF16, w, NULL, (const float*)w, (const float*)w, w, NULL, w, NULL, 1000, w, w, s8,
+                        NULL) == MP_ERR_INVALID_ARG);
+
   /* NULL is a no-op for mp_free */
   mp_free(NULL);
   printf("fails=%d\n", fails);
