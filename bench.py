@@ -845,18 +845,20 @@ def reference(args):
 
 def main():
     ap = argparse.ArgumentParser()
-    ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=100)
-    ap.add_argument("--warmup", type=int, default=5)
-    ap.add_argument("--impl", choices=["native", "reference"], default="native")
-    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads().keys()))
-    ap.add_argument("--no-e2e", action="store_true")
-    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--gpus", type=int, default=1, help="GPUs (one process each under torchrun; independent replicas)")
+    ap.add_argument("--steps", type=int, default=100, help="timed steps (one step = index, then plan + merge per budget)")
+    ap.add_argument("--warmup", type=int, default=5, help="untimed warm-up steps (at least 3)")
+    ap.add_argument("--impl", choices=["native", "reference"], default="native",
+                    help="native: the CUDA path; reference: the CPU oracle on a bounded sample")
+    ap.add_argument("--workload", default=DEFAULT_WORKLOAD, choices=sorted(workloads().keys()),
+                    help="synthetic family, operator and budgets")
+    ap.add_argument("--no-e2e", action="store_true", help="skip the end-to-end leg (host buffers, copies timed)")
+    ap.add_argument("--no-cpu-baseline", action="store_true", help="skip timing the CPU oracle")
     ap.add_argument("--no-hash", action="store_true", help="skip timing the block-hash passes")
-    ap.add_argument("--cpu-seconds", type=float, default=15.0)
+    ap.add_argument("--cpu-seconds", type=float, default=15.0, help="CPU oracle work to time for cpu_baseline")
     ap.add_argument("--k-sweep", action="store_true",
                     help="K-scaling at a fixed absolute budget (Cor. 1) instead of the workload sweep")
-    ap.add_argument("--k-list", default="4,8,16,32")
+    ap.add_argument("--k-list", default="4,8,16,32", help="expert counts of --k-sweep")
     ap.add_argument("--k-budget-experts", type=float, default=0.25,
                     help="the fixed budget of --k-sweep, in units of one expert checkpoint's bytes")
     args = ap.parse_args()
