@@ -8,6 +8,7 @@
 // draws the planner's scratch from one file-scope device array of fixed size instead of
 // allocating it.  That array exists once per GPU that loads the library and is held
 // until the process exits.
+#include <math.h>
 #include <string.h>
 
 #include <mutex>
@@ -83,9 +84,27 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
                        "mp_plan_noalloc: K * n_blocks exceeds the static scratch limit of 524288 units");
   if (!op || op->kind < MP_OP_AVG || op->kind > MP_OP_TIES_MASKED)
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: bad op");
+  // the same operator checks as mp_plan, with literal messages
   const bool by_lambda = op->kind == MP_OP_TIES || op->kind == MP_OP_DARE_TIES || op->kind == MP_OP_TIES_MASKED;
-  if (!by_lambda && !op->alpha)
-    return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA, DARE and AVG_RENORM");
+  if (by_lambda) {
+    if (!isfinite(op->lambda)) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: lambda must be finite");
+  } else {
+    if (!op->alpha)
+      return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha is required for AVG, TA, DARE and AVG_RENORM");
+    for (uint32_t i = 0; i < K; ++i)
+      if (!isfinite(op->alpha[i])) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: alpha must be finite");
+    if (op->kind == MP_OP_AVG_RENORM)
+      for (uint32_t i = 0; i < K; ++i)
+        if (!(op->alpha[i] > 0.0f))
+          return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: AVG_RENORM needs every alpha > 0");
+  }
+  if (op->kind == MP_OP_TIES || op->kind == MP_OP_TIES_MASKED) {
+    if (!(op->density >= 0.0f && op->density <= 1.0f))
+      return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: density must be in [0, 1]");
+    if (op->trim_scope > 1) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: trim_scope must be 0 or 1");
+  }
+  if ((op->kind == MP_OP_DARE || op->kind == MP_OP_DARE_TIES) && !(op->drop_p >= 0.0 && op->drop_p <= 1.0))
+    return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: drop_p must be in [0, 1]");
   if (op->score_mode > 1) return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: score_mode must be 0 or 1");
   if (op->kind == MP_OP_TIES && (!tau || !blk_group))
     return fail_static(MP_ERR_INVALID_ARG, "mp_plan_noalloc: TIES needs tau and blk_group");
@@ -111,10 +130,8 @@ extern "C" mp_status mp_plan_noalloc(uint32_t K, uint64_t n_blocks, uint32_t n_g
   p.elem_size = dtype == MP_BF16 ? 2u : 4u;
   p.op_kind = op->kind;
   p.score_mode = op->score_mode;
-  for (uint32_t i = 0; i < K; ++i) {
-    float c = by_lambda ? op->lambda : op->alpha[i];
-    p.coef[i] = c < 0.0f ? -c : c;
-  }
+  // |coef| as mp_plan takes it: fabsf also clears the sign of -0, whose score must be +0
+  for (uint32_t i = 0; i < K; ++i) p.coef[i] = fabsf(by_lambda ? op->lambda : op->alpha[i]);
   p.blk_len = blk_len;
   p.blk_group = blk_group;
   p.norm = norm;

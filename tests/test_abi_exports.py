@@ -125,3 +125,14 @@ def test_plan_noalloc_refuses_bad_arguments_before_any_device_work():
     assert "NULL" in call(mask=None)
     assert "524288" in call(K=2, n_blocks=(1 << 18) + 1)
     assert "tau" in call(op=mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2), blk_group=A)
+    # the operator checks of mp_plan, with the same refusals
+    nan = float("nan")
+    assert "alpha must be finite" in call(op=mp.make_op(mp.MP_OP_TA, alpha=[0.5, nan]))
+    assert "lambda must be finite" in call(op=mp.make_op(mp.MP_OP_TIES, lam=float("inf"), density=0.2), tau=A,
+                                           blk_group=A)
+    assert "alpha > 0" in call(op=mp.make_op(mp.MP_OP_AVG_RENORM, alpha=[0.5, 0.0]))
+    assert "alpha > 0" in call(op=mp.make_op(mp.MP_OP_AVG_RENORM, alpha=[-0.5, 0.5]))
+    assert "density" in call(op=mp.make_op(mp.MP_OP_TIES, lam=1.0, density=1.5), tau=A, blk_group=A)
+    assert "trim_scope" in call(op=mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, trim_scope=2), tau=A, blk_group=A)
+    assert "drop_p" in call(op=mp.make_op(mp.MP_OP_DARE, alpha=[0.5, 0.5], drop_p=1.5))
+    assert "drop_p" in call(op=mp.make_op(mp.MP_OP_DARE_TIES, lam=1.0, drop_p=-0.1))

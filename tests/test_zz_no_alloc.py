@@ -84,6 +84,39 @@ def test_noalloc_plan_matches_mp_plan_ties():
     _run(fam, mp.make_op(mp.MP_OP_TIES, lam=0.5, density=0.35, trim_scope=1), 1, [0.3])
 
 
+def test_noalloc_plan_with_negative_zero_coefficient_matches_mp_plan():
+    """an alpha of -0.0 scores its expert's units as +0 on both entry points (|coef| clears
+    the sign), so a zero-weight expert ranks last, not ahead of every positive score"""
+    fam = synth.custom([5000, 70001, 65536], dtype=synth.BF16, block_elems=4096, K=3, active_frac=0.5)
+    _run(fam, mp.make_op(mp.MP_OP_TA, alpha=[0.3, -0.0, 0.5]), 0, [0.1, 0.5, 1.0])
+    _run(fam, mp.make_op(mp.MP_OP_TA, alpha=[-0.0, 0.2, -0.4], score_mode=1), 0, [0.3])
+
+
+def test_noalloc_refuses_operators_that_mp_plan_refuses():
+    """a NaN alpha, an AVG_RENORM alpha <= 0 and a drop probability above 1 are refused by
+    both entry points, before anything is launched"""
+    fam = synth.custom([5000, 7001], dtype=synth.BF16, block_elems=4096, K=2, active_frac=0.5)
+    base, experts = fam.host_arrays()
+    b = torch.from_numpy(base.view(np.int16)).cuda().view(torch.bfloat16)
+    ex = [torch.from_numpy(e.view(np.int16)).cuda().view(torch.bfloat16) for e in experts]
+    offs, nums, _ = fam.layout()
+    mf = mp.family(list(zip(offs.tolist(), nums.tolist())), b, ex, fam.block_elems, fam.dtype, 0)
+    good = mp.make_op(mp.MP_OP_TA, alpha=[0.3, 0.3])
+    idx = mp.mp_index_blocks(mf, good)
+    nb, nu, ng = mp.mp_index_shape(idx)
+    t = torch.zeros(max(nu, 16), dtype=torch.int32, device="cuda")
+    summary = torch.zeros(8, dtype=torch.int64, device="cuda")
+    for bad in (mp.make_op(mp.MP_OP_TA, alpha=[float("nan"), 0.3]),
+                mp.make_op(mp.MP_OP_AVG_RENORM, alpha=[0.5, 0.0]),
+                mp.make_op(mp.MP_OP_DARE, alpha=[0.5, 0.5], drop_p=1.5)):
+        with pytest.raises(mp.MergePipeError) as e1:
+            mp.mp_plan(idx, bad, 100)
+        with pytest.raises(mp.MergePipeError) as e2:
+            mp.mp_plan_noalloc(fam.K, nb, ng, fam.dtype, t, t, t, t, t, None, t, bad, 100, t, t, summary)
+        assert e1.value.status == e2.value.status == -1
+    idx.free()
+
+
 def test_noalloc_plan_qwen_shaped_family():
     """Qwen2.5-0.5B tensor shapes cut to 2 layers, K=8, 64Ki-element blocks (20,400 units)"""
     _run(synth.qwen25_05b(layers=2), mp.make_op(mp.MP_OP_TA, alpha=[0.3] * 8), 0, [0.25, 1.0])
