@@ -117,6 +117,13 @@ __device__ __forceinline__ void f2_mul(float a0, float a1, float b0, float b1, f
       : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
+__device__ __forceinline__ void f2_add(float a0, float a1, float b0, float b1, float& d0, float& d1) {
+  asm("{\n .reg .b64 ra, rb, rd;\n mov.b64 ra, {%2, %3};\n mov.b64 rb, {%4, %5};\n add.rn.f32x2 rd, ra, rb;\n"
+      " mov.b64 {%0, %1}, rd;\n}"
+      : "=f"(d0), "=f"(d1)
+      : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
+}
+
 // (d0, d1) = (a0 * b0 + c0, a1 * b1 + c1), each a single fused rounding
 __device__ __forceinline__ void f2_fma(float a0, float a1, float b0, float b1, float c0, float c1, float& d0,
                                        float& d1) {
@@ -220,22 +227,55 @@ __device__ __forceinline__ void read_vec(const uint8_t* slot, const void* gsrc, 
   }
 }
 
+// the raw 16-byte vector at element k0 of a fill, as read_vec reads it (zeros past the chunk)
+template <bool BF16>
+__device__ __forceinline__ uint4 read_raw(const uint8_t* slot, const void* gsrc, uint64_t off, uint32_t k0,
+                                          uint32_t n, uint32_t n_tma) {
+  constexpr uint32_t V = BF16 ? 8u : 4u;
+  if (k0 + V <= n_tma) return *reinterpret_cast<const uint4*>(slot + k0 * (BF16 ? 2u : 4u));
+  uint32_t w[4] = {0u, 0u, 0u, 0u};
+#pragma unroll
+  for (uint32_t e = 0; e < V; ++e) {
+    if (k0 + e < n) {
+      if constexpr (BF16) w[e >> 1] |= (uint32_t)(static_cast<const uint16_t*>(gsrc)[off + k0 + e]) << (16u * (e & 1u));
+      else w[e] = static_cast<const uint32_t*>(gsrc)[off + k0 + e];
+    }
+  }
+  return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+// elements 2k and 2k + 1 of a raw vector as fp32 (k is a compile-time index)
+template <bool BF16, int k>
+__device__ __forceinline__ void pair_of(const uint4 r, float& a, float& b) {
+  if constexpr (BF16) {
+    const uint32_t w = k == 0 ? r.x : (k == 1 ? r.y : (k == 2 ? r.z : r.w));
+    a = __uint_as_float(w * 65536u);
+    b = __uint_as_float(w & 0xFFFF0000u);
+  } else {
+    a = __uint_as_float(k == 0 ? r.x : r.z);
+    b = __uint_as_float(k == 0 ? r.y : r.w);
+  }
+}
+
 // the tail loops are unrolled over the vector with a predicate, so that h and y stay in
 // registers (a loop bounded by navail would index them at run time, through local memory)
 template <bool BF16>
 __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t navail, const float* y) {
   constexpr uint32_t V = BF16 ? 8u : 4u;
   if constexpr (BF16) {
-    uint32_t h[8];
+    // two elements per conversion, each rounded to nearest-even: element 2k in the low half
+    uint32_t w[4];
 #pragma unroll
-    for (int e = 0; e < 8; ++e) h[e] = __bfloat16_as_ushort(__float2bfloat16_rn(y[e]));
+    for (int k = 0; k < 4; ++k) {
+      const __nv_bfloat162 h2 = __floats2bfloat162_rn(y[2 * k], y[2 * k + 1]);
+      w[k] = *reinterpret_cast<const uint32_t*>(&h2);
+    }
     if (navail >= V) {
-      uint4 w = make_uint4(h[0] | (h[1] << 16), h[2] | (h[3] << 16), h[4] | (h[5] << 16), h[6] | (h[7] << 16));
-      __stcs(reinterpret_cast<uint4*>(static_cast<char*>(ptr) + elem * 2u), w);
+      __stcs(reinterpret_cast<uint4*>(static_cast<char*>(ptr) + elem * 2u), make_uint4(w[0], w[1], w[2], w[3]));
     } else {
 #pragma unroll
       for (uint32_t e = 0; e < V; ++e)
-        if (e < navail) static_cast<uint16_t*>(ptr)[elem + e] = (uint16_t)h[e];
+        if (e < navail) static_cast<uint16_t*>(ptr)[elem + e] = (uint16_t)(w[e >> 1] >> (16u * (e & 1u)));
     }
   } else {
     if (navail >= V) {
@@ -264,6 +304,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   Smem<kSlots, SB, G>& S = *reinterpret_cast<Smem<kSlots, SB, G>*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   volatile int* abort_flag = &S.abort;
+  const uint32_t wl = wait_limit_of(p.wait_limit);
 
   if (tid == 0) {
     for (int s = 0; s < kSlots; ++s) {
@@ -288,7 +329,11 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
     auto produce = [&](uint32_t q, uint64_t off, uint32_t n, uint32_t m, uint32_t aux,
                        const char* src_row, uint32_t bytes) -> bool {
       const uint32_t s = fill % kSlots, r = fill / kSlots;
-      if (r > 0 && !mbar_wait<true>(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+      if (fill == 0 && p.stall) {  // test hook: slot 0 is never armed, so its wait runs out
+        ++fill;
+        return true;
+      }
+      if (r > 0 && !mbar_wait<true>(&S.empty[s], (r - 1) & 1u, abort_flag, wl)) return false;
       if (r > 0) fence_proxy_async_smem();
       S.meta[s].off = off;
       S.meta[s].q = q;
@@ -376,6 +421,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
       // drain: the last fill of every slot must have landed before the CTA may exit
       for (uint32_t s = 0; s < (uint32_t)kSlots && s < fill; ++s) {
         const uint32_t last = fill - 1 - ((fill - 1 + kSlots - s) % kSlots);
+        if (last == 0 && p.stall) continue;  // never armed: nothing in flight
         mbar_wait_drain(&S.full[s], (last / kSlots) & 1u);
       }
       for (uint32_t i = 0; i < p.K; ++i)
@@ -417,7 +463,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   };
   for (uint32_t fill = 0;; ++fill) {
     const uint32_t s = fill % kSlots, r = fill / kSlots;
-    if (!warp_wait<true>(&S.full[s], r & 1u, abort_flag)) {
+    if (!warp_wait<true>(&S.full[s], r & 1u, abort_flag, wl)) {
       atomicOr(p.err, kErrTimeout);
       S.abort = 1;
       break;
@@ -570,6 +616,365 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   }
 }
 
+// ---------------- TIES with at most 8 experts: whole-chunk consumers ----------------
+//
+// The same TMA ring, but a chunk (its base fill and its selected experts' fills, which sit in
+// consecutive ring slots) is published as one unit: one "full" mbarrier per chunk counts the
+// bytes of all its fills, one "empty" mbarrier per chunk counts the consumers' releases.
+// A consumer thread waits once per chunk, folds every selected expert of its vector in the
+// fixed ascending order while all of them are in shared memory, releases the chunk and only
+// then finalises: the per-element state (M_0, P, N, counts) lives for one chunk and the
+// per-fill waits, arrivals and metadata reads of the streaming kernel disappear.  The ring
+// must hold every fill of one chunk (1 + K slots), so this kernel serves K <= 8; the
+// streaming kernel above serves larger expert counts.
+constexpr uint32_t kTcSlotBytes = 4096u;
+constexpr uint32_t kTcMaxK = 8;
+
+// ring slots and CTAs per SM by expert count: K <= 4 holds two chunks of 5 fills in 11
+// slots at four CTAs per SM; K <= 8 two chunks of 9 fills in 18 slots at three
+template <int KC>
+struct TcGeo {
+  static constexpr int kSlots = KC <= 4 ? 11 : 18;
+  static constexpr int kCtasPerSm = KC <= 4 ? 4 : 3;
+  static constexpr int kConsumers = 256;
+  static constexpr int kThreads = kConsumers + 32;
+  static constexpr uint32_t kGrab = 8;
+};
+
+struct TcEntry {
+  uint64_t off;          // element offset of the chunk
+  uint32_t q;            // chunk id, or kEnd
+  uint32_t n;            // elements in the chunk
+  uint32_t m;            // the block's access mask
+  uint32_t s0;           // ring slot of the base fill; expert fill j sits in slot s0 + 1 + j (mod NS)
+  uint32_t nsel;         // selected experts
+  uint32_t fast;         // 1: every selected threshold is >= 2^-100 (no numerator needs the IEEE division)
+  float thr[kTcMaxK];    // trim thresholds (as floats) in fill order
+};
+
+template <int NS, uint32_t G>
+struct __align__(128) TcSmem {
+  uint8_t slot[NS][kTcSlotBytes];
+  TcEntry ce[NS];
+  ChunkMeta chunk[G];
+  uint32_t thr[G][kTcMaxK];  // bits threshold of (chunk of the grab, expert)
+  uint64_t full[NS];
+  uint64_t empty[NS];
+  unsigned long long realized[kMaxK];
+  float2 ntab[kTcMaxK + 1];  // {-c, RN(1/c)} for the counts c = 0..8 (entry 0: {-1, 1})
+  uint32_t nf[NS];           // producer only: fills held by the chunk of each entry
+  int abort;
+};
+
+template <bool BF16, int KC>
+__global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
+    merge_ties_chunk_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
+  constexpr int NS = TcGeo<KC>::kSlots;
+  constexpr int kConsumers = TcGeo<KC>::kConsumers;
+  constexpr uint32_t G = TcGeo<KC>::kGrab;
+  constexpr uint32_t ES = BF16 ? 2u : 4u;
+  constexpr uint32_t CH = kTcSlotBytes / ES;  // elements per chunk
+  constexpr int V = BF16 ? 8 : 4;
+  static_assert(CH == (uint32_t)(kConsumers * V), "one vector per consumer thread and chunk");
+  static_assert(NS >= 2 * (KC + 1), "the ring holds every fill of two chunks");
+  extern __shared__ __align__(128) uint8_t smem_raw[];
+  TcSmem<NS, G>& S = *reinterpret_cast<TcSmem<NS, G>*>(smem_raw);
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
+  volatile int* abort_flag = &S.abort;
+  const uint32_t wl = wait_limit_of(p.wait_limit);
+
+  if (tid == 0) {
+    for (int s = 0; s < NS; ++s) {
+      mbar_init(&S.full[s], 1);
+      mbar_init(&S.empty[s], kConsumers);  // every consumer thread arrives once per chunk
+    }
+    S.abort = 0;
+    mbar_fence_init();
+  }
+  if (tid < (uint32_t)kMaxK) S.realized[tid] = 0;
+  if (tid <= kTcMaxK) {
+    const float c = tid == 0 ? 1.0f : (float)tid;
+    S.ntab[tid] = make_float2(-c, __fdiv_rn(1.0f, c));
+  }
+  __syncthreads();
+
+  if (warp == kConsumers / 32) {
+    // ---------------- producer ----------------
+    uint32_t fill = 0;  // ring slots used so far (monotonic)
+    uint32_t seq = 0;   // chunks published
+    uint32_t head = 0;  // oldest published chunk not yet seen released
+    uint32_t used = 0;  // slots held by chunks head .. seq - 1
+    bool ok = true;
+    // lane 0: wait until entry seq % NS is free and nfill slots are free; chunks are
+    // released in order, so the oldest one is the next to free its slots
+    auto reserve = [&](uint32_t nfill) -> bool {
+      while (seq - head >= (uint32_t)NS || used + nfill > (uint32_t)NS) {
+        const uint32_t he = head % NS;
+        if (!mbar_wait<true>(&S.empty[he], (head / NS) & 1u, abort_flag, wl)) return false;
+        used -= S.nf[he];
+        ++head;
+      }
+      return true;
+    };
+    unsigned long long q_next = 0;
+    if (lane == 0) q_next = atomicAdd(work, (unsigned long long)G);
+    for (;;) {
+      const unsigned long long q0 = __shfl_sync(0xFFFFFFFFu, q_next, 0);
+      if (q0 >= n_chunks || !ok) break;
+      if (lane == 0) q_next = atomicAdd(work, (unsigned long long)G);  // used by the next grab
+      uint32_t grp = 0;
+      if (lane < G) {
+        const unsigned long long q = q0 + lane;
+        ChunkMeta cm{0, 0, 0};
+        if (q < n_chunks) {
+          const uint64_t b = p.b_begin + q / cpb;
+          const uint32_t start = (uint32_t)(q % cpb) * CH;
+          const uint32_t len = p.blk_len[b];
+          cm.off = p.blk_off[b] + start;
+          cm.m = p.mask[b];
+          cm.n = start < len ? min(CH, len - start) : 0u;
+          if (p.touched_only && cm.m == 0u) cm.n = 0u;  // left as it is: a reference to M_0
+          grp = p.blk_group[b];
+        }
+        S.chunk[lane] = cm;
+      }
+      // lane i < K: the trim thresholds of expert i for every chunk of the grab, at least the
+      // smallest subnormal (a zero delta is never kept: it would add nothing)
+#pragma unroll
+      for (uint32_t c = 0; c < G; ++c) {
+        const uint32_t g = __shfl_sync(0xFFFFFFFFu, grp, c);
+        if (lane < p.K) S.thr[c][lane] = max(ties_bits_threshold(p.tau[(uint64_t)lane * p.n_groups + g]), 1u);
+      }
+      __syncwarp();
+      if (lane == 0) {
+        const uint32_t nq = (uint32_t)min((unsigned long long)G, n_chunks - q0);
+        for (uint32_t c = 0; c < nq && ok; ++c) {
+          const ChunkMeta cm = S.chunk[c];
+          if (cm.n == 0) continue;
+          const uint32_t nsel = __popc(cm.m);
+          if (!(ok = reserve(1u + nsel))) break;
+          if (fill >= (uint32_t)NS) fence_proxy_async_smem();  // slots the consumers have read are refilled
+          const uint32_t e = seq % NS;
+          const uint32_t bytes = (cm.n * ES) & ~15u;
+          TcEntry& ce = S.ce[e];
+          ce.off = cm.off;
+          ce.q = (uint32_t)(q0 + c);
+          ce.n = cm.n;
+          ce.m = cm.m;
+          ce.s0 = fill % NS;
+          ce.nsel = nsel;
+          uint32_t fast = 1u, j = 0;
+          for (uint32_t mm = cm.m; mm; mm &= mm - 1, ++j) {
+            const uint32_t t = S.thr[c][__ffs(mm) - 1];
+            ce.thr[j] = __uint_as_float(t);
+            fast &= t >= 0x0D800000u ? 1u : 0u;  // bits of 2^-100
+          }
+          ce.fast = fast;
+          S.nf[e] = 1u + nsel;
+          // test hook: the first chunk is never armed, so the consumers' wait for it runs out
+          const bool arm = !(seq == 0 && p.stall);
+          if (arm) mbar_arrive_expect_tx(&S.full[e], (1u + nsel) * bytes);
+          if (bytes && arm)
+            tma_load_1d(S.slot[fill % NS], static_cast<const char*>(p.base) + cm.off * ES, bytes, &S.full[e]);
+          ++fill;
+          for (uint32_t mm = cm.m; mm; mm &= mm - 1) {
+            const uint32_t i = __ffs(mm) - 1;
+            if (bytes && arm)
+              tma_load_1d(S.slot[fill % NS],
+                          static_cast<const char*>(p.experts.p[i]) + (cm.off - p.expert_origin) * ES, bytes,
+                          &S.full[e]);
+            ++fill;
+            S.realized[i] += (unsigned long long)cm.n * ES;
+          }
+          used += 1u + nsel;
+          ++seq;
+        }
+      }
+      ok = __shfl_sync(0xFFFFFFFFu, ok, 0);
+      __syncwarp();
+    }
+    if (lane == 0) {
+      if (ok && (ok = reserve(0u))) {
+        const uint32_t e = seq % NS;
+        S.ce[e].q = kEnd;
+        S.nf[e] = 0u;
+        if (!(seq == 0 && p.stall)) mbar_arrive_expect_tx(&S.full[e], 0u);
+        ++seq;
+      }
+      if (!ok) {
+        atomicOr(p.err, kErrTimeout);
+        S.abort = 1;
+      }
+      // drain: the last chunk of every entry must have landed before the CTA may exit
+      for (uint32_t e = 0; e < (uint32_t)NS && e < seq; ++e) {
+        const uint32_t last = seq - 1 - ((seq - 1 + NS - e) % NS);
+        if (last == 0 && p.stall) continue;  // never armed: nothing in flight
+        mbar_wait_drain(&S.full[e], (last / NS) & 1u);
+      }
+      for (uint32_t i = 0; i < p.K; ++i)
+        if (S.realized[i])
+          atomicAdd(p.realized + (uint64_t)(blockIdx.x % kCounterSlots) * p.K + i, S.realized[i]);
+    }
+    return;
+  }
+  // ---------------- consumers: thread t owns vector t of every chunk ----------------
+  const uint32_t k0 = tid * (uint32_t)V;
+  for (uint32_t c = 0;; ++c) {
+    const uint32_t e = c % NS;
+    if (!warp_wait<true>(&S.full[e], (c / NS) & 1u, abort_flag, wl)) {
+      atomicOr(p.err, kErrTimeout);
+      S.abort = 1;
+      break;
+    }
+    const TcEntry& ce = S.ce[e];
+    if (ce.q == kEnd) break;
+    uint32_t s = ce.s0;
+    const uint32_t nsel = ce.nsel;
+    float x0[V];
+    bool in_slot;  // the thread's vector lies inside the bulk-copied bytes
+    {
+      const uint32_t n = ce.n, n_tma = ((n * ES) & ~15u) / ES;
+      in_slot = k0 + V <= n_tma;
+      read_vec<BF16>(S.slot[s], p.base, ce.off, k0, n, n_tma, x0);
+    }
+    float y[V];
+    if (nsel == 0) {  // uniform over the CTA
+      // no expert selected: the output is M_0 plus the zero the operator adds (lambda * +0)
+      const float z = __fmul_rn(p.lambda, 0.0f);
+#pragma unroll
+      for (int v = 0; v < V; ++v) y[v] = __fadd_rn(x0[v], z);
+      const uint64_t off = ce.off;
+      const uint32_t n = ce.n;
+      mbar_arrive(&S.empty[e]);
+      if (k0 < n) store_vec<BF16>(p.out, off + k0, n - k0, y);
+      continue;
+    }
+    // Per element: P and N, the sums of the kept positive and negative deltas, and both
+    // counts in one float C = 2^23 + c+ + 16 c- (exact: every value is an integer below 2^24,
+    // so the low bits of C hold c+ and c-).  A delta d is kept positive when d >= thr and kept
+    // negative when d <= -thr (thr > 0: |d| >= thr and the sign in one compare each); the
+    // keep factors k+ and k- are 1 or 0, and P = fma(k+, d, P), N = fma(k-, d, N): a factor 1
+    // adds d with the one rounding of P + d, a factor 0 adds a zero, which leaves P and N
+    // unchanged (they start at +0 and are never -0).  Two elements per packed instruction.
+    float Pp[V], Nn[V], Cc[V];
+#pragma unroll
+    for (int v = 0; v < V; ++v) {
+      Pp[v] = 0.0f;
+      Nn[v] = 0.0f;
+      Cc[v] = 8388608.0f;  // 2^23
+    }
+    // the selected experts in ascending order: fill j of the chunk sits in slot s0 + 1 + j
+#pragma unroll 1
+    for (uint32_t j = 0; j < nsel; ++j) {
+      s = s + 1 == (uint32_t)NS ? 0u : s + 1;
+      const float thr = ce.thr[j];
+      uint4 r;
+      if (in_slot) {
+        r = *reinterpret_cast<const uint4*>(S.slot[s] + k0 * ES);
+      } else {  // the ragged tail of a tensor, from global memory (expert = j-th selected)
+        const uint32_t i = __fns(ce.m, 0, (int)j + 1), n = ce.n;
+        r = read_raw<BF16>(S.slot[s], p.experts.p[i], ce.off - p.expert_origin, k0, n, ((n * ES) & ~15u) / ES);
+      }
+      // one element pair at a time, so that only the raw vector stays live
+      auto tally_pair = [&](int v, float e0, float e1) {
+        float d0, d1, t0, t1;
+        f2_sub(e0, e1, x0[v], x0[v + 1], d0, d1);
+        const float kp0 = d0 >= thr ? 1.0f : 0.0f, kp1 = d1 >= thr ? 1.0f : 0.0f;
+        const float kn0 = d0 <= -thr ? 1.0f : 0.0f, kn1 = d1 <= -thr ? 1.0f : 0.0f;
+        f2_fma(kp0, kp1, d0, d1, Pp[v], Pp[v + 1], Pp[v], Pp[v + 1]);
+        f2_fma(kn0, kn1, d0, d1, Nn[v], Nn[v + 1], Nn[v], Nn[v + 1]);
+        f2_fma(kn0, kn1, 16.0f, 16.0f, kp0, kp1, t0, t1);
+        f2_add(Cc[v], Cc[v + 1], t0, t1, Cc[v], Cc[v + 1]);
+      };
+      float e0, e1;
+      pair_of<BF16, 0>(r, e0, e1);
+      tally_pair(0, e0, e1);
+      pair_of<BF16, 1>(r, e0, e1);
+      tally_pair(2, e0, e1);
+      if constexpr (BF16) {
+        pair_of<BF16, 2>(r, e0, e1);
+        tally_pair(4, e0, e1);
+        pair_of<BF16, 3>(r, e0, e1);
+        tally_pair(6, e0, e1);
+      }
+    }
+    const uint64_t off = ce.off;
+    const uint32_t n = ce.n, fast = ce.fast;
+    mbar_arrive(&S.empty[e]);  // every read of the chunk's slots and entry is done
+    // the elected side's sum and count: the sign of P + N taken exactly as P > -N or P < -N
+    // (then that side holds at least one entry, so c >= 1); otherwise 0 / 1
+    auto num_c = [&](int v, float& num, uint32_t& cv) {
+      const bool pos = Pp[v] > -Nn[v], any = Pp[v] != -Nn[v];
+      num = any ? (pos ? Pp[v] : Nn[v]) : 0.0f;
+      const uint32_t cb = __float_as_uint(Cc[v]);
+      cv = any ? ((pos ? cb : cb >> 4) & 15u) : 0u;
+    };
+    if (fast) {  // uniform over the CTA: every nonzero numerator is >= 2^-100 in magnitude
+      // q = RN(num * y), then Markstein's correction q + RN(num - q c) * y, and the output
+      // fma(lambda, q, M_0), two elements per instruction
+#pragma unroll
+      for (int v = 0; v < V; v += 2) {
+        float a0, a1, q0, q1, r0, r1;
+        uint32_t c0, c1;
+        num_c(v, a0, c0);
+        num_c(v + 1, a1, c1);
+        const float2 t0 = S.ntab[c0], t1 = S.ntab[c1];
+        f2_mul(a0, a1, t0.y, t1.y, q0, q1);
+        f2_fma(q0, q1, t0.x, t1.x, a0, a1, r0, r1);
+        f2_fma(r0, r1, t0.y, t1.y, q0, q1, q0, q1);
+        f2_fma(p.lambda, p.lambda, q0, q1, x0[v], x0[v + 1], y[v], y[v + 1]);
+      }
+    } else {
+      // numerators 0 < |num| < 2^-100 take the IEEE division under one warp vote
+      bool exact = false;
+#pragma unroll
+      for (int v = 0; v < V; ++v) {
+        float a;
+        uint32_t cv;
+        num_c(v, a, cv);
+        const float2 t = S.ntab[cv];
+        y[v] = div_small_fast(a, -t.x, t.y);
+        exact = exact || div_small_needs_ieee(a);
+      }
+      if (__any_sync(0xFFFFFFFFu, exact)) {
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          float a;
+          uint32_t cv;
+          num_c(v, a, cv);
+          if (div_small_needs_ieee(a)) y[v] = __fdiv_rn(a, -S.ntab[cv].x);
+        }
+      }
+#pragma unroll
+      for (int v = 0; v < V; ++v) y[v] = __fmaf_rn(p.lambda, y[v], x0[v]);
+    }
+    if (k0 < n) store_vec<BF16>(p.out, off + k0, n - k0, y);
+  }
+}
+
+template <bool BF16, int KC>
+cudaError_t launch_ties_chunk(const MergeLaunch& p, cudaStream_t st) {
+  constexpr uint32_t chunk = kTcSlotBytes / (BF16 ? 2u : 4u);
+  const uint32_t cpb = (p.block_elems + chunk - 1) / chunk;
+  const uint64_t n_chunks = (p.b_end - p.b_begin) * cpb;
+  if (n_chunks == 0) return cudaSuccess;
+  if (n_chunks >= 0xFFFFFFFFull) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  const size_t smem = sizeof(TcSmem<TcGeo<KC>::kSlots, TcGeo<KC>::kGrab>);
+  auto kern = merge_ties_chunk_kernel<BF16, KC>;
+  if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
+    return e;
+  uint64_t grid = (uint64_t)sms * TcGeo<KC>::kCtasPerSm;
+  if (grid > n_chunks) grid = n_chunks;
+  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  kern<<<(unsigned)grid, TcGeo<KC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 template <bool BF16, int OPC>
 cudaError_t launch_op(const MergeLaunch& p, cudaStream_t st) {
   const uint32_t chunk = Geo<OPC>::kSlotBytes / (BF16 ? 2u : 4u);
@@ -598,7 +1003,10 @@ cudaError_t launch_dtype(const MergeLaunch& p, cudaStream_t st) {
   switch (p.op_kind) {
     case MP_OP_AVG:
     case MP_OP_TA: return launch_op<BF16, OP_ADD>(p, st);
-    case MP_OP_TIES: return launch_op<BF16, OP_TIES>(p, st);
+    case MP_OP_TIES:
+      if (p.K <= 4) return launch_ties_chunk<BF16, 4>(p, st);
+      if (p.K <= kTcMaxK) return launch_ties_chunk<BF16, 8>(p, st);
+      return launch_op<BF16, OP_TIES>(p, st);
     case MP_OP_DARE: return launch_op<BF16, OP_DARE>(p, st);
     case MP_OP_AVG_RENORM: return launch_op<BF16, OP_RENORM>(p, st);
     case MP_OP_DARE_TIES: return launch_op<BF16, OP_DTIES>(p, st);
