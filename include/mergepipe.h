@@ -364,6 +364,37 @@ const char* mp_version(void);
    all threads).  A diagnostic for counting launches per step; never resets. */
 uint64_t mp_kernel_launch_count(void);
 
+/*
+ * Test hooks for the failure paths.  The paper has no counterpart: they exist so that the
+ * error returns of this library (a run either produces its handle or leaves none, Alg. 2)
+ * can be exercised without provoking a real GPU fault.  Both settings are process-wide and
+ * are meant for tests only.
+ *
+ * mp_debug_inject_fault(kind, n): the n-th event of the kind from now on fails (n >= 1;
+ * n = 0 disarms), once, on the host, before anything is enqueued for it:
+ *   MP_FAULT_ALLOC   a device allocation of the library (handle memory, planner scratch,
+ *                    host-pool staging) fails as if the device were out of memory: the call
+ *                    returns MP_ERR_OOM and no handle;
+ *   MP_FAULT_GATHER  a host-pool gather launch (mp_index_blocks / mp_merge with experts in
+ *                    pinned host memory) is not made: the call returns MP_ERR_CUDA and no
+ *                    handle, after the work already enqueued has been joined.
+ * mp_last_error() then names the injected fault.  Returns MP_ERR_INVALID_ARG for an unknown
+ * kind.
+ *
+ * mp_debug_stall_pipeline(rounds): the index and merge kernels launched from now on never arm
+ * the first slot of each CTA's shared-memory ring (its bulk copy is not issued), so the
+ * consumers' wait for it cannot complete, and every pipeline wait (producer or consumer
+ * mbarrier) gives up after `rounds` polling rounds instead of the default 2^21.  The wait
+ * that runs out sets the handle's error word; the accessors of that handle and of the
+ * handles built from it return MP_ERR_TIMEOUT.  The waits that drain a CTA's own bulk
+ * copies before it exits keep the full limit, so no copy is in flight when a kernel
+ * returns.  rounds = 0 turns the stall off.
+ */
+#define MP_FAULT_ALLOC 1
+#define MP_FAULT_GATHER 2
+mp_status mp_debug_inject_fault(int32_t kind, uint64_t n);
+void mp_debug_stall_pipeline(uint32_t rounds);
+
 #ifdef __cplusplus
 }
 #endif

@@ -27,6 +27,7 @@ __all__ = [
     "mp_index_shape", "mp_plan_info", "mp_manifest_info", "mp_manifest_lineage", "mp_budget_from_fraction", "mp_last_error",
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "mp_index_hashes",
     "mp_index_hash_values", "mp_manifest_validate", "mp_manifest_validation", "lib",
+    "MP_FAULT_ALLOC", "MP_FAULT_GATHER", "mp_debug_inject_fault", "mp_debug_stall_pipeline",
     "library_path",
 ]
 
@@ -36,6 +37,7 @@ MP_ERR = {-1: "MP_ERR_INVALID_ARG", -2: "MP_ERR_CUDA", -3: "MP_ERR_OOM", -4: "MP
 MP_BF16, MP_F32 = 0, 1
 MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES, MP_OP_TIES_MASKED = 0, 1, 2, 3, 4, 5, 6
 MP_NNZ_MISSING = 0xFFFFFFFF   # catalog entry without block statistics (tensor-level fallback)
+MP_FAULT_ALLOC, MP_FAULT_GATHER = 1, 2  # test hooks: kinds of injected host-side failures
 
 
 class MergePipeError(RuntimeError):
@@ -99,6 +101,8 @@ def lib():
         L.mp_last_error.restype, L.mp_last_error.argtypes = ctypes.c_char_p, []
         L.mp_version.restype, L.mp_version.argtypes = ctypes.c_char_p, []
         L.mp_kernel_launch_count.restype, L.mp_kernel_launch_count.argtypes = u64, []
+        L.mp_debug_inject_fault.restype, L.mp_debug_inject_fault.argtypes = st, [ctypes.c_int32, u64]
+        L.mp_debug_stall_pipeline.restype, L.mp_debug_stall_pipeline.argtypes = None, [ctypes.c_uint32]
         _lib = L
     return _lib
 
@@ -355,6 +359,18 @@ def mp_version() -> str:
 
 def mp_kernel_launch_count() -> int:
     return int(lib().mp_kernel_launch_count())
+
+
+def mp_debug_inject_fault(kind: int, n: int) -> None:
+    """Test hook: the n-th device allocation (MP_FAULT_ALLOC) or host-pool gather launch
+    (MP_FAULT_GATHER) from now on fails once, on the host; n = 0 disarms."""
+    _check(lib().mp_debug_inject_fault(int(kind), int(n)))
+
+
+def mp_debug_stall_pipeline(rounds: int) -> None:
+    """Test hook: index and merge kernels launched from now on never arm their first ring
+    slot and give up a pipeline wait after `rounds` polling rounds (0 = off)."""
+    lib().mp_debug_stall_pipeline(int(rounds))
 
 
 def mp_plan_noalloc(K, n_blocks, n_groups, dtype, blk_len, blk_group, norm, maxabs, nnz, tau, index_err, op: Op,

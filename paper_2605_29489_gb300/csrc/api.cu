@@ -2,6 +2,7 @@
 // launch sequence of index, plan and merge.  Every device step runs in the kernels of
 // index.cu, plan.cu and merge.cu; this file only marshals arguments and memory.
 #include <float.h>
+#include <limits.h>
 #include <math.h>
 #include <string.h>
 
@@ -17,6 +18,30 @@ namespace mp {
 namespace {
 thread_local std::string g_last_error;
 thread_local const char* g_static_error = nullptr;  // set instead of g_last_error by allocation-free paths
+
+// test hooks: failures injected on the host (mp_debug_inject_fault) and device waits made to
+// run out (mp_debug_stall_pipeline); nothing faults the GPU.  g_fault_left[kind] counts down
+// to the event that fails; 0 = disarmed.
+std::atomic<int64_t> g_fault_left[MP_FAULT_GATHER + 1];
+thread_local bool g_injected = false;  // the error being reported was injected
+std::atomic<uint32_t> g_stall_rounds{0};  // mp_debug_stall_pipeline: wait rounds of stalled launches (0: off)
+
+// true when this event of the given kind is the one armed to fail (it then disarms)
+bool inject_fault(int kind) {
+  if (g_fault_left[kind].load(std::memory_order_relaxed) <= 0) return false;
+  if (g_fault_left[kind].fetch_sub(1) != 1) return false;
+  g_injected = true;
+  return true;
+}
+
+// cudaMallocAsync, or an injected out-of-memory failure
+cudaError_t malloc_async(void** p, size_t bytes, cudaStream_t st) {
+  if (inject_fault(MP_FAULT_ALLOC)) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  return cudaMallocAsync(p, bytes, st);
+}
 std::atomic<uint64_t> g_next_id{1};
 std::atomic<uint64_t> g_launches{0};
 
@@ -61,7 +86,7 @@ mp_status fail(mp_status st, const std::string& msg) {
 mp_status dev_alloc(Alloc& a, size_t bytes, cudaStream_t st) {
   a.bytes = bytes;
   a.stream = st;
-  cudaError_t e = cudaMallocAsync(&a.ptr, bytes ? bytes : 256, st);
+  cudaError_t e = malloc_async(&a.ptr, bytes ? bytes : 256, st);
   if (e != cudaSuccess) {
     a.ptr = nullptr;
     return cuda_fail(e, "cudaMallocAsync");
@@ -215,6 +240,11 @@ void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_rela
 mp_status cuda_fail(cudaError_t e, const char* what) {
   cudaGetLastError();
   g_static_error = nullptr;
+  if (g_injected) {
+    g_injected = false;
+    g_last_error = std::string(what) + ": injected fault (test hook)";
+    return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
+  }
   g_last_error = std::string(what) + ": " + cudaGetErrorString(e);
   return e == cudaErrorMemoryAllocation ? MP_ERR_OOM : MP_ERR_CUDA;
 }
@@ -238,7 +268,7 @@ mp_status alloc_hashes(mp_index_s* ix, cudaStream_t cs);
 namespace {
 
 constexpr uint64_t kSegmentElems = 32ull << 20;
-constexpr int kSide = 2;
+constexpr int kSide = 1;  // side streams of the host-pool gathers (one gather kernel saturates the link)
 
 struct Segment {
   uint64_t b0, b1, e0, e1;  // blocks [b0, b1), elements [e0, e1)
@@ -282,7 +312,7 @@ struct HostPipe {
         if ((e = cudaEventCreateWithFlags(&ready[b][q], cudaEventDisableTiming)) != cudaSuccess) return e;
       if ((e = cudaEventCreateWithFlags(&freed[b], cudaEventDisableTiming)) != cudaSuccess) return e;
     }
-    if ((e = cudaMallocAsync(&staging, 2 * (size_t)K * per_expert, main)) != cudaSuccess) {
+    if ((e = malloc_async(&staging, 2 * (size_t)K * per_expert, main)) != cudaSuccess) {
       staging = nullptr;
       return e;
     }
@@ -363,6 +393,10 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     gl.mask = nullptr;
     gl.src = p.experts;
     for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
+    if (inject_fault(MP_FAULT_GATHER)) {
+      e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
+      break;
+    }
     if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
     if ((e = hp.main_acquire(b)) != cudaSuccess) break;
     IndexLaunch ps = p;
@@ -407,6 +441,10 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
     gl.mask = p.mask;
     gl.src = p.experts;
     for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
+    if (inject_fault(MP_FAULT_GATHER)) {
+      e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
+      break;
+    }
     if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
     if ((e = hp.main_acquire(b)) != cudaSuccess) break;
     MergeLaunch ps = p;
@@ -558,6 +596,14 @@ const char* mp_version(void) { return "mergepipe-gb300 0.1 (sm_103a)"; }
 
 uint64_t mp_kernel_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
+mp_status mp_debug_inject_fault(int32_t kind, uint64_t n) {
+  if (kind != MP_FAULT_ALLOC && kind != MP_FAULT_GATHER) return fail(MP_ERR_INVALID_ARG, "unknown fault kind");
+  g_fault_left[kind].store(n > (uint64_t)INT64_MAX ? INT64_MAX : (int64_t)n, std::memory_order_relaxed);
+  return MP_OK;
+}
+
+void mp_debug_stall_pipeline(uint32_t rounds) { g_stall_rounds.store(rounds, std::memory_order_relaxed); }
+
 uint64_t mp_budget_from_fraction(const mp_family* family, double f) {
   Geometry g;
   if (build_geometry(family, g) != MP_OK) return 0;
@@ -628,6 +674,8 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   p.nnz = ix->d_nnz;
   p.err = ix->d_err;
   p.work = (unsigned long long*)(m + o_work);
+  p.wait_limit = g_stall_rounds.load(std::memory_order_relaxed);
+  p.stall = p.wait_limit ? 1u : 0u;
   if (ties) {
     p.coarse = (unsigned long long*)(m + o_coarse);
     p.fine = (unsigned long long*)(m + o_fine);
@@ -791,7 +839,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   cudaError_t e;
   if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
   const uint64_t n_pairs = index->has_missing ? (uint64_t)g.K * g.n_tensors : 0ull;
-  if ((e = cudaMallocAsync(&scratch.ptr, plan_scratch_bytes(U, n_pairs), cs)) != cudaSuccess) {
+  if ((e = malloc_async(&scratch.ptr, plan_scratch_bytes(U, n_pairs), cs)) != cudaSuccess) {
     scratch.ptr = nullptr;
     return bail(e, "plan scratch");
   }
@@ -1010,6 +1058,8 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
     q.b_begin = 0;
     q.b_end = g.n_blocks;
     q.expert_origin = 0;
+    q.wait_limit = g_stall_rounds.load(std::memory_order_relaxed);
+    q.stall = q.wait_limit ? 1u : 0u;
     if ((e = launch_ties_masked(q, cs)) != cudaSuccess) return bail(e, "masked TIES threshold");
   }
 
@@ -1050,6 +1100,8 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   p.b_end = g.n_blocks;
   p.expert_origin = 0;
   p.touched_only = touched_only ? 1u : 0u;
+  p.wait_limit = g_stall_rounds.load(std::memory_order_relaxed);
+  p.stall = p.wait_limit ? 1u : 0u;
   if (family->experts_location == 0) {
     if ((e = launch_merge(p, cs)) != cudaSuccess) return bail(e, "merge kernels");
   } else {

@@ -220,6 +220,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
   Sm& S = *reinterpret_cast<Sm*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   volatile int* abort_flag = &S.abort;
+  const uint32_t wl = wait_limit_of(p.wait_limit);
 
   if (tid == 0) {
     for (int s = 0; s < kIxSlots; ++s) {
@@ -241,7 +242,11 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
       auto produce = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, const char* src_row,
                          uint32_t bytes) -> bool {
         const uint32_t s = fill % kIxSlots, r = fill / kIxSlots;
-        if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag)) return false;
+        if (fill == 0 && p.stall) {  // test hook: slot 0 is never armed, so its wait runs out
+          ++fill;
+          return true;
+        }
+        if (r > 0 && !mbar_wait(&S.empty[s], (r - 1) & 1u, abort_flag, wl)) return false;
         if (r > 0) fence_proxy_async_smem();
         S.meta[s].off = off;
         S.meta[s].item = item;
@@ -279,6 +284,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
       }
       for (uint32_t s = 0; s < (uint32_t)kIxSlots && s < fill; ++s) {
         const uint32_t lastf = fill - 1 - ((fill - 1 + kIxSlots - s) % kIxSlots);
+        if (lastf == 0 && p.stall) continue;  // never armed: nothing in flight
         mbar_wait_drain(&S.full[s], (lastf / kIxSlots) & 1u);
       }
     }
@@ -297,7 +303,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
   uint32_t fill = 0, cphase = 0;
   bool alive = true;
   auto wait_full = [&](uint32_t f) -> bool {
-    if (!warp_wait(&S.full[f % kIxSlots], (f / kIxSlots) & 1u, abort_flag)) {
+    if (!warp_wait(&S.full[f % kIxSlots], (f / kIxSlots) & 1u, abort_flag, wl)) {
       atomicOr(p.err, kErrTimeout);
       S.abort = 1;
       return false;
@@ -407,7 +413,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
       mx[k] = 0.0f;
       nz[k] = 0u;
     }
-    if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+    if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
       atomicOr(p.err, kErrTimeout);
       S.abort = 1;
       break;
@@ -438,7 +444,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
     }
     if constexpr (TIES) {
       // every nonzero delta added 1 to exactly one bin: the histogram's total is nnz
-      if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+      if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
         break;
@@ -453,7 +459,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
         for (int s = 16; s >= 1; s >>= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, s);
         if (lane == 0) S.red_nz[k][warp] = w;
       }
-      if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+      if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
         break;
@@ -475,7 +481,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
         if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + tid], c);
       }
     }
-    if (!consumer_barrier(&S.cbar, cphase, abort_flag)) {
+    if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
       atomicOr(p.err, kErrTimeout);
       S.abort = 1;
       break;

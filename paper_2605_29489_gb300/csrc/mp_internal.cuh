@@ -184,6 +184,8 @@ struct IndexLaunch {
   // point into a staging buffer)
   uint64_t b_begin, b_end, expert_origin;
   int defer_ties_select;  // 1: leave the TIES selection to launch_ties_finish
+  uint32_t wait_limit;    // try_wait rounds of the pipeline waits (0: the default)
+  uint32_t stall;         // test hook: every CTA's first ring fill is never armed
 };
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
 cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st);
@@ -265,6 +267,8 @@ struct MergeLaunch {
   uint32_t* err;
   uint64_t b_begin, b_end, expert_origin;  // as in IndexLaunch
   uint32_t touched_only;  // 1: blocks with an empty mask are neither read nor written
+  uint32_t wait_limit;    // try_wait rounds of the pipeline waits (0: the default)
+  uint32_t stall;         // test hook: every CTA's first ring fill is never armed
 };
 cudaError_t launch_merge(const MergeLaunch& p, cudaStream_t st);
 

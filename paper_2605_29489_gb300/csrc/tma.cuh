@@ -15,6 +15,11 @@ namespace mp {
 constexpr uint32_t kSuspendHintNs = 2000;
 constexpr uint32_t kWaitLimit = 1u << 21;  // try_wait rounds before a wait gives up
 
+// the limit a kernel uses for its pipeline waits: the launch's (a test setting) or the default
+__device__ __forceinline__ uint32_t wait_limit_of(uint32_t launch_limit) {
+  return launch_limit ? launch_limit : kWaitLimit;
+}
+
 __device__ __forceinline__ uint32_t su32(const void* p) { return (uint32_t)__cvta_generic_to_shared(p); }
 
 __device__ __forceinline__ void mbar_init(uint64_t* bar, uint32_t count) {
@@ -54,10 +59,12 @@ __device__ __forceinline__ bool mbar_try_wait_sleep(uint64_t* bar, uint32_t pari
   return ok != 0;
 }
 
-// bounded wait for the phase with the given parity; false on expiry or when *abort is set
+// bounded wait for the phase with the given parity; false on expiry (after `limit` rounds)
+// or when *abort is set
 template <bool SLEEP = false>
-__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  for (uint32_t k = 0; k < kWaitLimit; ++k) {
+__device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint32_t limit = kWaitLimit) {
+  for (uint32_t k = 0; k < limit; ++k) {
     if (SLEEP ? mbar_try_wait_sleep(bar, parity) : mbar_try_wait(bar, parity)) return true;
     if ((k & 15u) == 15u && *abort) return false;
   }
@@ -89,17 +96,19 @@ __device__ __forceinline__ void tma_load_1d(void* dst, const void* src, uint32_t
 // every lane of the warp waits (each acquires the barrier); the outcome is made uniform
 // across the warp so that a give-up never splits a warp
 template <bool SLEEP = false>
-__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort) {
-  const bool ok = mbar_wait<SLEEP>(bar, parity, abort);
+__device__ __forceinline__ bool warp_wait(uint64_t* bar, uint32_t parity, volatile int* abort,
+                                          uint32_t limit = kWaitLimit) {
+  const bool ok = mbar_wait<SLEEP>(bar, parity, abort, limit);
   return __all_sync(0xFFFFFFFFu, ok);
 }
 
 // barrier over the consumer warps only (bar counts one arrival per warp), with a bounded
 // wait: a warp that has given up cannot leave the others blocked; phase counts the uses
-__device__ __forceinline__ bool consumer_barrier(uint64_t* bar, uint32_t& phase, volatile int* abort) {
+__device__ __forceinline__ bool consumer_barrier(uint64_t* bar, uint32_t& phase, volatile int* abort,
+                                                 uint32_t limit = kWaitLimit) {
   __syncwarp();
   if ((threadIdx.x & 31u) == 0) mbar_arrive(bar);
-  const bool ok = warp_wait(bar, phase & 1u, abort);
+  const bool ok = warp_wait(bar, phase & 1u, abort, limit);
   ++phase;
   return ok;
 }
