@@ -52,6 +52,10 @@ def workloads():
                                      desc="Qwen2.5-0.5B shapes cut to 2 layers (profiling case), K=4, TIES density 0.2"),
         "llama-3-8b-ties": dict(make=lambda: synth.llama3_8b(), op="ties", density=0.2, budgets=[1.0, 0.5, 0.25, 0.1],
                                 desc="Llama-3-8B-shaped bf16 family, K=4, TIES density 0.2, 64Ki-element blocks"),
+        "llama-3-8b-ties-1l": dict(make=lambda: synth.llama3_8b(layers=1), op="ties", density=0.2,
+                                   budgets=[1.0, 0.5, 0.25, 0.1],
+                                   desc="one Llama-3-8B transformer layer (no embedding or lm_head; profiling "
+                                        "case), K=4, TIES density 0.2"),
         "llama-3-8b-ties-masked": dict(make=lambda: synth.llama3_8b(), op="ties_masked", density=0.2,
                                        budgets=[1.0, 0.5, 0.25, 0.1],
                                        desc="Llama-3-8B-shaped bf16 family, K=4, TIES applied after masking (threshold "
@@ -93,7 +97,7 @@ def workloads():
     }
 
 
-DEFAULT_WORKLOAD = "qwen2.5-0.5b-ta"
+DEFAULT_WORKLOAD = "llama-3-8b-ties"
 
 
 def make_ops(w, K):
@@ -467,8 +471,13 @@ def native(args, rank, world, local_rank):
     # ---- e2e: pinned host inputs in, merged outputs back, inside the timed region ----
     e2e = None
     if not args.no_e2e and not host_pool:
-        base_h = base.cpu().pin_memory()
-        experts_h = [e.cpu().pin_memory() for e in experts]
+        def pinned_copy(t):
+            h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
+            h.copy_(t)
+            return h
+
+        base_h = pinned_copy(base)
+        experts_h = [pinned_copy(e) for e in experts]
         outs_h = [torch.empty(outs[0].shape, dtype=outs[0].dtype, pin_memory=True) for _ in budgets]
         set_bytes = (fam.K + 1) * total * es
         free_b, _ = torch.cuda.mem_get_info()
@@ -568,7 +577,7 @@ def native(args, rank, world, local_rank):
                    "step": ("catalog import" if catalog is not None else "index") + " + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
         "index_ms": idx_ms, "per_budget": per_budget, "time_model": t_model, "block_hashes": hashes,
-        "roofline": {"bound": "hbm", "kernel": "merge_tma_kernel", "achieved": achieved, "peak": peak, "unit": "GB/s",
+        "roofline": {"bound": "hbm", "kernel": merge_kernel_name(W["op"], fam.dtype), "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
                      "traffic": profiled_traffic(args.workload),
@@ -598,6 +607,13 @@ def native(args, rank, world, local_rank):
         line["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": 1, "kind": "oracle", "sample": desc,
                                 "seconds": dt, "host_cpu": model, "host_cores_available": ncpu}
     return line
+
+
+def merge_kernel_name(op: str, dtype: int) -> str:
+    """the merge kernel instance a workload's operator launches"""
+    inst = {"ta": "AVG/TA", "avg": "AVG/TA", "ties": "TIES", "ties_masked": "TIES", "dare": "DARE",
+            "avg_renorm": "AVG_RENORM", "dare_ties": "DARE_TIES"}[op]
+    return f"merge_tma_kernel<{'bf16' if dtype == 0 else 'f32'}, {inst}>"
 
 
 def time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream, reps=3):

@@ -245,10 +245,10 @@ def _qwen2_tensors(hidden, layers, n_q, n_kv, inter, vocab, head_dim=None):
     return t
 
 
-def _llama_tensors(hidden, layers, n_q, n_kv, inter, vocab):
+def _llama_tensors(hidden, layers, n_q, n_kv, inter, vocab, embeddings=True):
     hd = hidden // n_q
     kv = n_kv * hd
-    t = [("embed_tokens", vocab * hidden)]
+    t = [("embed_tokens", vocab * hidden)] if embeddings else []
     for l in range(layers):
         p = f"layers.{l}."
         t += [(p + "input_layernorm", hidden),
@@ -256,7 +256,7 @@ def _llama_tensors(hidden, layers, n_q, n_kv, inter, vocab):
               (p + "o_proj", hidden * hidden), (p + "post_attention_layernorm", hidden),
               (p + "gate_proj", inter * hidden), (p + "up_proj", inter * hidden),
               (p + "down_proj", hidden * inter)]
-    t += [("norm", hidden), ("lm_head", vocab * hidden)]
+    t += [("norm", hidden), ("lm_head", vocab * hidden)] if embeddings else [("norm", hidden)]
     return t
 
 
@@ -273,10 +273,15 @@ def qwen25_05b(seed: int = 0, K: int = 8, layers: int = 24) -> Family:
                   active_frac=0.3, log_mu=math.log(1e-3), log_sigma=1.0, seed=seed)
 
 
-def llama3_8b(seed: int = 0, K: int = 4) -> Family:
-    """Llama-3-8B shapes (hidden 4096, 32 layers, 32/8 heads, inter 14336, vocab 128256 untied), bf16"""
-    return Family("llama-3-8b", BF16, _llama_tensors(4096, 32, 32, 8, 14336, 128256), 65536, K,
-                  active_frac=0.4, log_mu=math.log(2e-4), log_sigma=1.2, seed=seed)
+def llama3_8b(seed: int = 0, K: int = 4, layers: int = 32) -> Family:
+    """Llama-3-8B shapes (hidden 4096, 32 layers, 32/8 heads, inter 14336, vocab 128256 untied), bf16.
+    With fewer layers (a profiling case) the embedding and lm_head are left out as well, so
+    that the family holds only transformer layers (218,112,000 parameters each) and a norm."""
+    if layers == 32:
+        return Family("llama-3-8b", BF16, _llama_tensors(4096, 32, 32, 8, 14336, 128256), 65536, K,
+                      active_frac=0.4, log_mu=math.log(2e-4), log_sigma=1.2, seed=seed)
+    return Family(f"llama-3-8b-{layers}l", BF16, _llama_tensors(4096, layers, 32, 8, 14336, 128256, False), 65536,
+                  K, active_frac=0.4, log_mu=math.log(2e-4), log_sigma=1.2, seed=seed)
 
 
 def qwen25_15b(seed: int = 0, K: int = 16, layers: int = 28) -> Family:
