@@ -68,3 +68,25 @@ def tensor_stats_and_tau(spec, t, density):
     numel = int(bl[blocks].sum())
     tau = np.array([oracle.tau_from_hist(hist[i], numel, density) for i in range(K)], np.uint32)
     return t, blocks, out_n, out_m, out_z, tau
+
+
+def merged_hashes(spec, blocks, cases):
+    """the oracle's merge of each given block under every budget's mask of every case,
+    hashed like the catalog's blocks.  cases: [(op_args, masks [n_budgets, len(blocks)],
+    tau [K, n_tensors] or None)], op_args = (kind, K, kwargs) of oracle.Op (trim group =
+    tensor).  Returns (blocks, [uint64 [n_budgets, len(blocks)] per case]); each block is
+    regenerated once for all cases."""
+    import oracle
+
+    fam = family(spec)
+    bo, bl, bt = fam.block_table()
+    ops = [oracle.Op(a[0], a[1], **dict(a[2])) for a, _, _ in cases]
+    outs = [np.zeros((m.shape[0], len(blocks)), np.uint64) for _, m, _ in cases]
+    for j, b in enumerate(blocks):
+        base, experts = fam.block_host(int(b))
+        for (args, masks, tau), op, out in zip(cases, ops, outs):
+            tau_k = None if tau is None else np.ascontiguousarray(tau[:, bt[b]])
+            for k in range(masks.shape[0]):
+                merged = oracle.merge_block(fam.dtype, int(bo[b]), base, experts, int(masks[k, j]), op, tau_k)
+                out[k, j] = oracle.block_hash(merged.tobytes())
+    return blocks, outs

@@ -1,8 +1,9 @@
 """Host-resident expert pool: experts in pinned host memory, base and output in HBM.
 
-The index stages each segment of the family with cudaMemcpyAsync on side streams; the
-merge gathers only the planned (block, expert) pairs over the host mapping into
-double-buffered HBM staging while the merge kernel works on the previous segment.
+The library walks the family in segments.  For each segment a gather kernel on a side
+stream reads the expert blocks over the host mapping (every block for the index, only the
+planned (block, expert) pairs for the merge) into double-buffered HBM staging, while the
+index or merge kernel works on the previous segment.
 The results must be exactly those of the oracle (and of the device-resident path)."""
 import numpy as np
 import pytest
