@@ -216,9 +216,12 @@ def merge_source_hash() -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str):
-    """dram bytes per merge launch from the committed ncu summary, if it was taken on the
-    current merge kernel source (else None)"""
+def profiled_traffic(workload: str, alg_bytes_per_launch: float):
+    """DRAM bytes per merge launch from the committed ncu summary, if it was taken on the
+    current merge kernel source (else None): either captured on this workload itself
+    (traffic_per_launch), or on a smaller case of the same kernel whose DRAM bytes per
+    algorithmic byte (traffic_ratio) scale to a full launch (traffic grows in proportion to
+    the bytes a launch moves)"""
     path = os.path.join(ROOT, "profiles", "merge_kernel_traffic.md")
     if not os.path.exists(path):
         return None
@@ -227,7 +230,10 @@ def profiled_traffic(workload: str):
     if not src or src.group(1) != merge_source_hash():
         return None
     m = re.search(rf"traffic_per_launch\[{re.escape(workload)}\]:\s*([0-9.eE+]+)", txt)
-    return float(m.group(1)) if m else None
+    if m:
+        return float(m.group(1))
+    m = re.search(rf"traffic_ratio\[{re.escape(workload)}\]:\s*([0-9.eE+]+)", txt)
+    return float(m.group(1)) * alg_bytes_per_launch if m else None
 
 
 # ---- CPU oracle sample ----------------------------------------------------------------------------
@@ -580,7 +586,7 @@ def native(args, rank, world, local_rank):
         "roofline": {"bound": "hbm", "kernel": merge_kernel_name(W["op"], fam.dtype), "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
-                     "traffic": profiled_traffic(args.workload),
+                     "traffic": profiled_traffic(args.workload, sum(alg_bytes) / len(alg_bytes)),
                      "algorithmic_bytes": ("per materialised (touched) parameter" if touched_mode else
                                            "per merged parameter") + " 2*s + s*(selected experts); summed over the "
                                           "budget sweep's launches / their summed CUDA-event time"},

@@ -641,12 +641,38 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   auto slot = [&](size_t bytes) { size_t r = o; o += align_up(bytes); return r; };
   const size_t o_work = slot(16);  // the index kernel's work counter
   size_t o_coarse = 0, o_fine = 0, o_kth = 0, o_est = 0, o_rank = 0;
+  size_t o_wfine = 0, o_wabove = 0, o_wlo = 0, o_gmiss = 0, o_miss = 0, o_wend = 0;
+  // device-resident TIES (not after masking) takes its thresholds from predicted windows
+  const bool windowed = ties && op->kind == MP_OP_TIES && family->experts_location == 0;
   if (ties) {
     o_coarse = slot(KG * 256 * 8);
     o_fine = slot(KG * 128 * 8);
     o_kth = slot(n_groups * 8);
     o_est = slot(KG * 4);
     o_rank = slot(KG * 8);
+  }
+  // the sampling CTAs' spans: up to 64 blocks of one trim group each
+  std::vector<uint32_t> h_spans;
+  size_t o_shist = 0, o_scnt = 0, o_spans = 0;
+  if (windowed) {
+    for (uint32_t q = 0; q < n_groups; ++q) {
+      const uint64_t b0 = scope == 0 ? g.t_first_block[q] : 0;
+      const uint64_t b1 = scope == 0 ? (q + 1 < g.n_tensors ? g.t_first_block[q + 1] : g.n_blocks) : g.n_blocks;
+      for (uint64_t b = b0; b < b1; b += 64) {
+        h_spans.push_back(q);
+        h_spans.push_back((uint32_t)b);
+      }
+    }
+    // zeroed together: window counts, keys above, marks, the flag, sampled bins and counts
+    o_wfine = slot(KG * 384 * 8);
+    o_wabove = slot(KG * 8);
+    o_gmiss = slot(KG * 4);
+    o_miss = slot(16);
+    o_shist = slot(KG * 256 * 8);
+    o_scnt = slot(n_groups * 8);
+    o_wend = o;
+    o_wlo = slot(KG * 4);
+    o_spans = slot(h_spans.size() * 4);
   }
   mp_index_s* ix = nullptr;
   char* m = nullptr;
@@ -688,6 +714,23 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     if ((e = cudaMemsetAsync(p.fine, 0, KG * 128 * 8, cs)) != cudaSuccess) return bail(e, "memset");
     if ((e = cudaMemcpyAsync((void*)p.kth, h_kth.data(), n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
       return bail(e, "k copy");
+  }
+  if (windowed) {
+    p.density = op->density;
+    p.grp_blk0 = ix->d_t_blk0;
+    p.wfine = (unsigned long long*)(m + o_wfine);
+    p.wabove = (unsigned long long*)(m + o_wabove);
+    p.gmiss = (uint32_t*)(m + o_gmiss);
+    p.miss = (uint32_t*)(m + o_miss);
+    p.wlo = (uint32_t*)(m + o_wlo);
+    p.shist = (unsigned long long*)(m + o_shist);
+    p.scnt = (unsigned long long*)(m + o_scnt);
+    p.samp_span = (const uint2*)(m + o_spans);
+    p.n_samp_spans = (uint32_t)(h_spans.size() / 2);
+    if ((e = cudaMemsetAsync(m + o_wfine, 0, o_wend - o_wfine, cs)) != cudaSuccess) return bail(e, "memset");
+    if ((e = cudaMemcpyAsync(m + o_spans, h_spans.data(), h_spans.size() * 4, cudaMemcpyHostToDevice, cs)) !=
+        cudaSuccess)
+      return bail(e, "span copy");
   }
   p.b_begin = 0;
   p.b_end = g.n_blocks;

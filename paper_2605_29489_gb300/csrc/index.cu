@@ -104,13 +104,24 @@ struct IxMeta {
   uint32_t pad;
 };
 
-template <int KG, int NS, uint32_t SB>
+// How the TIES catalog bins the keys of the deltas:
+//  * kBinCoarse: 256 bins of the upper 8 key bits (the two-level select: a second pass then
+//    counts the lower 7 bits inside the chosen bin);
+//  * kBinWindow: the 384 keys [L, L + 384) of a window predicted from a sample (three
+//    coarse bins at full resolution), one bin below and one above it, so that the
+//    threshold is found without a second pass whenever it lies inside the window.
+enum { kBinNone = 0, kBinCoarse = 1, kBinWindow = 2 };
+constexpr uint32_t kWinKeys = 384;           // keys of the window
+constexpr uint32_t kWinBins = kWinKeys + 2;  // + below + above
+
+template <int KG, int NS, uint32_t SB, uint32_t NB>
 struct __align__(128) IxSmem {
   uint8_t slot[NS][SB];
   IxMeta meta[NS];
   uint64_t full[NS];
   uint64_t empty[NS];
-  uint32_t hist[KG][256];
+  uint32_t hist[KG][NB];
+  int32_t wlo[KG];  // kBinWindow: L - 1 of each expert of the item's group
   float red_ss[KG][8];
   float red_mx[KG][8];
   uint32_t red_nz[KG][8];
@@ -175,6 +186,29 @@ __device__ __forceinline__ void f2_sub(float a0, float a1, float b0, float b1, f
       : "f"(a0), "f"(a1), "f"(b0), "f"(b1));
 }
 
+// TIES window bins of two deltas: a nonzero delta with key k adds 1 to bin
+// clamp(k, L - 1, L + 384) - (L - 1) of the shared histogram, i.e. bin 0 below the window,
+// bins 1..384 for the keys L..L + 383, bin 385 above it.  lo = L - 1; hist0 = the byte
+// address of bin 0 minus 4 lo.  Predicated, no branch.
+__device__ __forceinline__ void ties_win2(float d0, float d1, int32_t lo, uint32_t hist0) {
+  const __nv_bfloat162 h2 = __floats2bfloat162_rn(d0, d1);
+  const uint32_t w = *reinterpret_cast<const uint32_t*>(&h2);
+  const int32_t hi = lo + (int32_t)kWinKeys + 1;
+  const int32_t k0 = min(max((int32_t)(w & 0x7FFFu), lo), hi);
+  const int32_t k1 = min(max((int32_t)((w >> 16) & 0x7FFFu), lo), hi);
+  const uint32_t a0 = hist0 + ((uint32_t)k0 << 2), a1 = hist0 + ((uint32_t)k1 << 2);
+  asm volatile(
+      "{\n"
+      " .reg .pred p0, p1;\n"
+      " setp.ne.f32 p0, %2, 0f00000000;\n"
+      " setp.ne.f32 p1, %3, 0f00000000;\n"
+      " @p0 red.shared.add.u32 [%0], 1;\n"
+      " @p1 red.shared.add.u32 [%1], 1;\n"
+      "}\n" ::"r"(a0),
+      "r"(a1), "f"(d0), "f"(d1)
+      : "memory");
+}
+
 // TIES fine bins of two deltas: a nonzero delta whose coarse bin (key bits 7..14) is es
 // adds 1 to fine bin (key & 127) of the shared histogram at hist; predicated, no branch
 __device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint32_t hist) {
@@ -205,9 +239,11 @@ __device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint
       : "memory");
 }
 
-template <bool BF16, int KG, bool TIES>
-__global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
+template <bool BF16, int KG, int BM>
+__global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
+  constexpr bool TIES = BM != kBinNone;
+  constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;  // key bins per expert
   constexpr int kIxSlots = IxGeo<TIES>::kSlots;
   constexpr uint32_t kIxSlotBytes = IxGeo<TIES>::kSlotBytes;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
@@ -216,9 +252,11 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
   constexpr int VPT = (int)(CH / (kIxConsumers * V));
   static_assert(VPT >= 1 && CH == (uint32_t)(VPT * kIxConsumers * V), "chunk geometry");
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  using Sm = IxSmem<KG, kIxSlots, kIxSlotBytes>;
+  using Sm = IxSmem<KG, kIxSlots, kIxSlotBytes, NB>;
   Sm& S = *reinterpret_cast<Sm*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
+  // the fallback pass of the windowed catalog runs only when some threshold left its window
+  if (BM == kBinCoarse && p.miss && *p.miss == 0u) return;
   volatile int* abort_flag = &S.abort;
   const uint32_t wl = wait_limit_of(p.wait_limit);
 
@@ -231,7 +269,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
     S.abort = 0;
     mbar_fence_init();
   }
-  for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += blockDim.x) (&S.hist[0][0])[x] = 0u;
+  for (uint32_t x = tid; x < (uint32_t)KG * NB; x += blockDim.x) (&S.hist[0][0])[x] = 0u;
   __syncthreads();
 
   if (warp == kIxConsumers / 32) {
@@ -263,6 +301,12 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
         const uint64_t b = p.b_begin + it / G;
         const uint32_t i0 = (uint32_t)(it % G) * KG;
         const uint32_t kc = min((uint32_t)KG, p.K - i0);
+        if (BM == kBinCoarse && p.gmiss) {  // windowed fallback: the marked pairs' groups only
+          const uint32_t grp = p.blk_group[b];
+          bool any = false;
+          for (uint32_t k = 0; k < kc; ++k) any = any || p.gmiss[(uint64_t)(i0 + k) * p.n_groups + grp] != 0u;
+          if (!any) continue;
+        }
         const uint32_t len = p.blk_len[b];
         const uint64_t off0 = p.blk_off[b];
         const uint32_t nch = (len + CH - 1) / CH;
@@ -360,6 +404,10 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
       // a warp whose vectors all match skips them (warp-uniform, so the summation order is
       // untouched)
       if (!__all_sync(0xFFFFFFFFu, same)) {
+        // kBinWindow: L - 1 of this expert's window in the block's trim group
+        int32_t wlo_k = 0;
+        if constexpr (BM == kBinWindow)
+          wlo_k = (int32_t)__ldg(p.wlo + (uint64_t)(i0 + k) * p.n_groups + __ldg(p.blk_group + b)) - 1;
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           float xe[V];
@@ -381,7 +429,9 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
           mx[k] = fmaxf(mx[k], m[0]);
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
-            if constexpr (TIES) {
+            if constexpr (BM == kBinWindow) {
+              ties_win2(d[e], d[e + 1], wlo_k, su32(&S.hist[k][0]) - ((uint32_t)wlo_k << 2));
+            } else if constexpr (BM == kBinCoarse) {
               ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]));
             } else {
               nz[k] += d[e] != 0.0f ? 1u : 0u;
@@ -449,12 +499,18 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
         S.abort = 1;
         break;
       }
-      uint32_t hc[KG];
+      // thread t holds bin t (and, for the window bins, bin t + 256)
+      uint32_t hc[KG], hd[KG];
 #pragma unroll
       for (int k = 0; k < KG; ++k) {
         hc[k] = S.hist[k][tid];
         S.hist[k][tid] = 0u;
-        uint32_t w = hc[k];
+        hd[k] = 0u;
+        if (BM == kBinWindow && tid + 256u < NB) {
+          hd[k] = S.hist[k][tid + 256u];
+          S.hist[k][tid + 256u] = 0u;
+        }
+        uint32_t w = hc[k] + hd[k];
 #pragma unroll
         for (int s = 16; s >= 1; s >>= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, s);
         if (lane == 0) S.red_nz[k][warp] = w;
@@ -472,13 +528,21 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
         uint32_t nzk = 0;
 #pragma unroll
         for (int w = 0; w < kIxConsumers / 32; ++w) nzk += S.red_nz[k][w];
-        unsigned long long c = hc[k];
-        if (tid == 0) {
-          p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
-          c += len - nzk;  // zero deltas have key 0
+        if (tid == 0) p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
+        const uint64_t x = (uint64_t)(i0 + k) * p.n_groups + grp;
+        if constexpr (BM == kBinCoarse) {
+          unsigned long long c = hc[k];
+          if (tid == 0) c += len - nzk;  // zero deltas have key 0
+          if (p.unit_hist) p.unit_hist[(((uint64_t)(i0 + k) * p.n_blocks + b) << 8) + tid] = (uint32_t)c;
+          if (c) atomicAdd(&p.coarse[x * 256u + tid], c);
+        } else {
+          // bin 0 (below the window) only counts toward nnz; bins 1..384 are the window's
+          // keys; bin 385 is above it
+          if (tid > 0 && hc[k]) atomicAdd(&p.wfine[x * kWinKeys + tid - 1u], (unsigned long long)hc[k]);
+          const uint32_t j = tid + 256u;
+          if (j <= kWinKeys && hd[k]) atomicAdd(&p.wfine[x * kWinKeys + j - 1u], (unsigned long long)hd[k]);
+          if (j == kWinKeys + 1u && hd[k]) atomicAdd(&p.wabove[x], (unsigned long long)hd[k]);
         }
-        if (p.unit_hist) p.unit_hist[(((uint64_t)(i0 + k) * p.n_blocks + b) << 8) + tid] = (uint32_t)c;
-        if (c) atomicAdd(&p.coarse[((uint64_t)(i0 + k) * p.n_groups + grp) * 256u + tid], c);
       }
     }
     if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
@@ -494,6 +558,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<TIES>::kCtasPerSm)
 __global__ void ties_coarse_select(const IndexLaunch p) {
   uint64_t x = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (x >= (uint64_t)p.K * p.n_groups) return;
+  if (p.gmiss && p.gmiss[x] == 0u) return;  // its window already gave the threshold
   uint32_t grp = (uint32_t)(x % p.n_groups);
   unsigned long long k = p.kth[grp];
   if (k == 0) {
@@ -525,6 +590,7 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
   const uint32_t kc = min((uint32_t)KG, p.K - i0);
   const uint32_t grp = p.blk_group[b];
   const uint32_t tid = threadIdx.x;
+  if (p.miss && *p.miss == 0u) return;  // windowed thresholds: no pair needs this pass
 
   uint32_t estar[KG];
   uint32_t want = 0u;  // bit k: expert i0+k may hold keys in its bin e*
@@ -535,7 +601,8 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
       uint32_t i = i0 + k;
       uint32_t es = p.estar[(uint64_t)i * p.n_groups + grp];
       uint64_t u = (uint64_t)i * p.n_blocks + b;
-      const bool read = !p.mask || ((p.mask[b] >> i) & 1u);  // TIES_MASKED: selected blocks only
+      const bool read = (!p.mask || ((p.mask[b] >> i) & 1u)) &&  // TIES_MASKED: selected blocks only
+                        (!p.gmiss || p.gmiss[(uint64_t)i * p.n_groups + grp] != 0u);  // windowed: missed pairs only
       if (read && es != kNoBin && p.nnz[u] != 0u && (ties_key(p.maxabs[u]) >> 7) >= es) {
         estar[k] = es;
         want |= 1u << k;
@@ -576,6 +643,7 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
 __global__ void ties_fine_select(const IndexLaunch p) {
   uint64_t x = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
   if (x >= (uint64_t)p.K * p.n_groups) return;
+  if (p.gmiss && p.gmiss[x] == 0u) return;  // its window already gave the threshold
   uint32_t es = p.estar[x];
   if (es == kNoBin) {
     p.tau[x] = kTauNone;
@@ -621,6 +689,131 @@ __global__ void __launch_bounds__(256) ties_masked_coarse(const IndexLaunch p, u
   if (acc) atomicAdd(&p.coarse[((uint64_t)i * p.n_groups + grp) * 256u + e], acc);
 }
 
+// ---- TIES thresholds with a predicted window ----------------------------------------------
+//
+// The threshold of a trim group is the k-th largest key of its deltas.  A sample predicts
+// the coarse bin e (upper 8 key bits) that holds it: from every block of the group, 32
+// vectors at jittered, evenly spaced positions (every vector of a block of at most 4096
+// elements), binned like the coarse catalog — every block contributes because the scale of
+// the deltas changes from block to block; e is the bin of the k_s-th largest sampled key,
+// k_s = max(1, floor(rho * sampled elements)).  The catalog pass then counts the 384 keys
+// of the window starting at L = 128 clamp(e - 1, 0, 253) at full resolution, plus the keys
+// above it, and ties_window_finish takes the threshold from those counts.  A pair whose
+// threshold lies outside its window is marked, and the two-level select (coarse pass over
+// the marked pairs' groups, coarse select, fine pass, fine select) runs for the marked
+// pairs only; it does nothing when none is marked.  The prediction affects only which of
+// the two exact paths gives a threshold, never its value.
+constexpr uint32_t kSampleSpan = 64;  // blocks of one group per sampling CTA
+
+template <bool BF16, int KG>
+__global__ void __launch_bounds__(256) ties_sample_kernel(const IndexLaunch p) {
+  constexpr uint32_t V = BF16 ? 8u : 4u;
+  __shared__ uint32_t hist[KG][256];
+  __shared__ unsigned long long s_n;  // sampled elements
+  const uint2 span = p.samp_span[blockIdx.x];  // {group, first block}: up to kSampleSpan blocks
+  const uint32_t g = span.x, i0 = blockIdx.y * KG;
+  const uint32_t kc = min((uint32_t)KG, p.K - i0);
+  const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
+  for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += blockDim.x) (&hist[0][0])[x] = 0u;
+  if (tid == 0) s_n = 0;
+  __syncthreads();
+  const uint64_t gb1 = p.n_groups == 1 ? p.n_blocks : p.grp_blk0[g + 1];
+  const uint64_t b1 = min((uint64_t)span.y + kSampleSpan, gb1);
+  unsigned long long my_n = 0;
+  for (uint64_t b = span.y + warp; b < b1; b += 8) {
+    const uint32_t len = p.blk_len[b];
+    const uint64_t off = p.blk_off[b];
+    const uint32_t nvec = (len + V - 1) / V;
+    const bool every = len <= 4096u;
+    const uint32_t per = every ? 1u : nvec / 32u;
+    for (uint32_t v0 = lane; v0 < (every ? nvec : 32u); v0 += 32u) {
+      uint32_t v = v0;
+      if (!every) {  // a position in stretch v0 from a hash of (block, stretch)
+        uint32_t h = (uint32_t)b * 0x9E3779B1u ^ (v0 + 1u) * 0x85EBCA77u;
+        h ^= h >> 15;
+        h *= 0x2C1B3C6Du;
+        h ^= h >> 12;
+        v = v0 * per + h % per;
+      }
+      my_n += min(V, len - v * V);
+      float xb[V];
+      unpack<BF16>(load_vec_raw(p.base, BF16, off, v, len), xb);
+      for (uint32_t k = 0; k < kc; ++k) {
+        float xe[V];
+        unpack<BF16>(load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len), xe);
+#pragma unroll
+        for (uint32_t e = 0; e < V; ++e) {
+          const float d = __fsub_rn(xe[e], xb[e]);
+          if (d != 0.0f) atomicAdd(&hist[k][ties_key(d) >> 7], 1u);
+        }
+      }
+    }
+  }
+#pragma unroll
+  for (int s = 16; s >= 1; s >>= 1) my_n += __shfl_xor_sync(0xFFFFFFFFu, my_n, s);
+  if (lane == 0) atomicAdd(&s_n, my_n);
+  __syncthreads();
+  for (uint32_t x = tid; x < kc * 256u; x += blockDim.x) {
+    const uint32_t k = x >> 8, e = x & 255u;
+    if (hist[k][e]) atomicAdd(&p.shist[((uint64_t)(i0 + k) * p.n_groups + g) * 256u + e], (unsigned long long)hist[k][e]);
+  }
+  if (tid == 0 && blockIdx.y == 0) atomicAdd(&p.scnt[g], s_n);
+}
+
+// the window of each (expert, group) from its sampled coarse bins
+__global__ void ties_window_select(const IndexLaunch p) {
+  const uint64_t x = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (x >= (uint64_t)p.K * p.n_groups) return;
+  const uint32_t g = (uint32_t)(x % p.n_groups);
+  unsigned long long ks = (unsigned long long)floor((double)p.density * (double)p.scnt[g]);
+  if (ks == 0) ks = 1;
+  const unsigned long long* h = p.shist + x * 256u;
+  uint32_t e = 0;
+  unsigned long long cum = 0;
+  for (int j = 255; j >= 0; --j) {
+    cum += h[j];
+    if (cum >= ks) {
+      e = (uint32_t)j;
+      break;
+    }
+  }
+  const uint32_t lo = e == 0 ? 0u : min(e - 1u, 253u);
+  p.wlo[x] = lo << 7;
+}
+
+// the threshold of each (expert, group) from its window counts, or a mark for the
+// two-level select when it lies outside the window
+__global__ void ties_window_finish(const IndexLaunch p) {
+  const uint64_t x = (uint64_t)blockIdx.x * blockDim.x + threadIdx.x;
+  if (x >= (uint64_t)p.K * p.n_groups) return;
+  const uint32_t g = (uint32_t)(x % p.n_groups);
+  const unsigned long long k = p.kth[g];
+  if (k == 0) {
+    p.tau[x] = kTauNone;
+    return;
+  }
+  const unsigned long long above = p.wabove[x];
+  const uint32_t L = p.wlo[x];
+  if (above < k) {
+    const unsigned long long r = k - above;
+    const unsigned long long* f = p.wfine + x * kWinKeys;
+    unsigned long long cum = 0;
+    for (int j = (int)kWinKeys - 1; j >= 0; --j) {
+      cum += f[j];
+      if (cum >= r) {
+        p.tau[x] = L + (uint32_t)j;
+        return;
+      }
+    }
+    if (L == 0) {  // every uncounted delta is an exact zero, key 0
+      p.tau[x] = 0;
+      return;
+    }
+  }
+  p.gmiss[x] = 1u;
+  atomicOr(p.miss, 1u);
+}
+
 // the TIES threshold from the coarse bins of the whole family: select the bin, count
 // the lower key bits inside it (a second pass over the blocks that can reach it; experts
 // addressed with origin 0), select the threshold
@@ -637,6 +830,23 @@ cudaError_t ties_finish_t(const IndexLaunch& p, cudaStream_t st) {
   return cudaGetLastError();
 }
 
+// one persistent launch of the catalog kernel with binning mode BM
+template <bool BF16, int KG, int BM>
+cudaError_t launch_pass(const IndexLaunch& p, uint32_t G, uint64_t n_items, int sms, cudaStream_t st) {
+  constexpr bool ties = BM != kBinNone;
+  constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;
+  const size_t smem = sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>);
+  uint64_t grid = (uint64_t)sms * IxGeo<ties>::kCtasPerSm;
+  if (grid > n_items) grid = n_items;
+  cudaError_t e;
+  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  auto k = index_tma_kernel<BF16, KG, BM>;
+  if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
+  k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
 template <bool BF16, int KG>
 cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   const uint32_t G = (p.K + KG - 1) / KG;
@@ -648,24 +858,24 @@ cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  const int per_sm = ties ? IxGeo<true>::kCtasPerSm : IxGeo<false>::kCtasPerSm;
-  const size_t smem = ties ? sizeof(IxSmem<KG, IxGeo<true>::kSlots, IxGeo<true>::kSlotBytes>)
-                           : sizeof(IxSmem<KG, IxGeo<false>::kSlots, IxGeo<false>::kSlotBytes>);
-  uint64_t grid = (uint64_t)sms * per_sm;
-  if (grid > n_items) grid = n_items;
-  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
-  if (ties) {
-    auto k = index_tma_kernel<BF16, KG, true>;
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
-    k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);
-  } else {
-    auto k = index_tma_kernel<BF16, KG, false>;
-    if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
-    k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);
+  if (!ties) return launch_pass<BF16, KG, kBinNone>(p, G, n_items, sms, st);
+  if (!p.wlo) {  // the two-level select for every pair
+    if ((e = launch_pass<BF16, KG, kBinCoarse>(p, G, n_items, sms, st)) != cudaSuccess) return e;
+    if (p.defer_ties_select) return cudaSuccess;
+    return ties_finish_t<BF16, KG>(p, st);
   }
+  // predicted windows: sample, windowed catalog pass, thresholds from the windows, then the
+  // two-level select for the pairs whose threshold left its window (a no-op when none did)
+  const uint64_t nsel = (uint64_t)p.K * p.n_groups;
+  ties_sample_kernel<BF16, KG><<<dim3(p.n_samp_spans, G), 256, 0, st>>>(p);
+  ties_window_select<<<(unsigned)((nsel + 127) / 128), 128, 0, st>>>(p);
+  count_launches(2);
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_pass<BF16, KG, kBinWindow>(p, G, n_items, sms, st)) != cudaSuccess) return e;
+  ties_window_finish<<<(unsigned)((nsel + 127) / 128), 128, 0, st>>>(p);
   count_launches(1);
-  e = cudaGetLastError();
-  if (e != cudaSuccess || !ties || p.defer_ties_select) return e;
+  if ((e = cudaGetLastError()) != cudaSuccess) return e;
+  if ((e = launch_pass<BF16, KG, kBinCoarse>(p, G, n_items, sms, st)) != cudaSuccess) return e;
   return ties_finish_t<BF16, KG>(p, st);
 }
 

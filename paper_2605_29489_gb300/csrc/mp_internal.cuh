@@ -176,6 +176,21 @@ struct IndexLaunch {
   // deltas in bin 0); the fine pass then reads only the blocks the plan selected and counts
   // the expert bytes it reads
   uint32_t* unit_hist;         // [K][n_blocks][256] or null
+  // TIES with a predicted window (device-resident experts, not after masking; null
+  // otherwise): a sample of each trim group predicts the coarse bin of its threshold, the
+  // catalog pass counts the 384 keys of a window around it at full resolution, and the
+  // two-level select runs only for the (expert, group) pairs whose threshold left the window
+  float density;                  // rho
+  const uint32_t* grp_blk0;       // [n_groups + 1] first block of each trim group, then n_blocks
+  const uint2* samp_span;         // [n_samp_spans] {group, first block} of each sampling CTA
+  uint32_t n_samp_spans;
+  unsigned long long* shist;      // [K][n_groups][256] coarse bins of the sampled deltas
+  unsigned long long* scnt;       // [n_groups] sampled elements
+  uint32_t* wlo;                  // [K][n_groups] first key L of the window
+  unsigned long long* wfine;      // [K][n_groups][384] counts of the keys L .. L + 383
+  unsigned long long* wabove;     // [K][n_groups] keys above the window
+  uint32_t* gmiss;                // [K][n_groups] 1: the pair needs the two-level select
+  uint32_t* miss;                 // [1] nonzero when some pair does
   const uint32_t* mask;        // the access mask for the fine pass, or null (every block)
   unsigned long long* thr_reads;  // expert bytes read by the fine pass, or null
   unsigned long long* work;    // item counter of the dynamic scheduler (zeroed per launch)
