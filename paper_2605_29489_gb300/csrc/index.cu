@@ -101,7 +101,7 @@ struct IxMeta {
   uint32_t item;   // work item, or kIxEnd
   uint32_t n;      // elements in the chunk
   uint32_t last;   // 1 on the block's last chunk
-  uint32_t pad;
+  uint32_t s0;     // whole-chunk publication: ring slot of the base fill (experts follow)
 };
 
 // How the TIES catalog bins the keys of the deltas:
@@ -121,7 +121,7 @@ struct __align__(128) IxSmem {
   uint64_t full[NS];
   uint64_t empty[NS];
   uint32_t hist[KG][NB];
-  int32_t wlo[KG];  // kBinWindow: L - 1 of each expert of the item's group
+  uint32_t nf[NS];  // whole-chunk publication: fills held by the chunk of each entry
   float red_ss[KG][8];
   float red_mx[KG][8];
   uint32_t red_nz[KG][8];
@@ -244,7 +244,13 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
   constexpr bool TIES = BM != kBinNone;
   constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;  // key bins per expert
+  // The TIES catalog with up to 4 experts per item publishes whole chunks: the base fill and
+  // the item's expert fills of one chunk sit in consecutive ring slots under one "full"
+  // mbarrier (counting all their bytes) and one "empty" mbarrier, so that a consumer waits
+  // and releases once per chunk instead of once per fill.
+  constexpr bool CW = TIES && KG <= 4;
   constexpr int kIxSlots = IxGeo<TIES>::kSlots;
+  static_assert(!CW || kIxSlots >= 2 * (KG + 1), "two whole chunks fit the ring");
   constexpr uint32_t kIxSlotBytes = IxGeo<TIES>::kSlotBytes;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t CH = kIxSlotBytes / ES;
@@ -277,6 +283,50 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
     if (lane == 0) {
       uint32_t fill = 0;
       bool ok = true;
+      // whole-chunk publication: chunks published (seq), the oldest one not yet seen released
+      // (head) and the ring slots held by chunks head .. seq - 1 (used)
+      uint32_t seq = 0, head = 0, used = 0;
+      auto reserve = [&](uint32_t nfill) -> bool {
+        while (seq - head >= (uint32_t)kIxSlots || used + nfill > (uint32_t)kIxSlots) {
+          const uint32_t he = head % kIxSlots;
+          if (!mbar_wait(&S.empty[he], (head / kIxSlots) & 1u, abort_flag, wl)) return false;
+          used -= S.nf[he];
+          ++head;
+        }
+        return true;
+      };
+      // publishes one chunk: the base fill and kc expert fills in consecutive slots
+      auto publish = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, uint32_t i0,
+                         uint32_t kc) -> bool {
+        const uint32_t nfill = item == kIxEnd ? 0u : 1u + kc;
+        if (!reserve(nfill)) return false;
+        if (fill >= (uint32_t)kIxSlots) fence_proxy_async_smem();  // slots the consumers have read are refilled
+        const uint32_t e = seq % kIxSlots;
+        const uint32_t bytes = (n * ES) & ~15u;
+        S.meta[e].off = off;
+        S.meta[e].item = item;
+        S.meta[e].n = n;
+        S.meta[e].last = last;
+        S.meta[e].s0 = fill % kIxSlots;
+        S.nf[e] = nfill;
+        const bool arm = !(seq == 0 && p.stall);  // test hook: the first chunk is never armed
+        if (arm) mbar_arrive_expect_tx(&S.full[e], nfill * bytes);
+        if (nfill) {
+          if (bytes && arm)
+            tma_load_1d(S.slot[fill % kIxSlots], static_cast<const char*>(p.base) + off * ES, bytes, &S.full[e]);
+          ++fill;
+          for (uint32_t k = 0; k < kc; ++k) {
+            if (bytes && arm)
+              tma_load_1d(S.slot[fill % kIxSlots],
+                          static_cast<const char*>(p.experts.p[i0 + k]) + (off - p.expert_origin) * ES, bytes,
+                          &S.full[e]);
+            ++fill;
+          }
+        }
+        used += nfill;
+        ++seq;
+        return true;
+      };
       auto produce = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, const char* src_row,
                          uint32_t bytes) -> bool {
         const uint32_t s = fill % kIxSlots, r = fill / kIxSlots;
@@ -315,19 +365,26 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
           const uint64_t off = off0 + (uint64_t)c * CH;
           const uint32_t bytes = (n * ES) & ~15u;
           const uint32_t last = c + 1 == nch ? 1u : 0u;
-          ok = produce((uint32_t)it, off, n, last, static_cast<const char*>(p.base) + off * ES, bytes);
-          for (uint32_t k = 0; k < kc && ok; ++k)
-            ok = produce((uint32_t)it, off, n, last,
-                         static_cast<const char*>(p.experts.p[i0 + k]) + (off - p.expert_origin) * ES, bytes);
+          if constexpr (CW) {
+            ok = publish((uint32_t)it, off, n, last, i0, kc);
+          } else {
+            ok = produce((uint32_t)it, off, n, last, static_cast<const char*>(p.base) + off * ES, bytes);
+            for (uint32_t k = 0; k < kc && ok; ++k)
+              ok = produce((uint32_t)it, off, n, last,
+                           static_cast<const char*>(p.experts.p[i0 + k]) + (off - p.expert_origin) * ES, bytes);
+          }
         }
       }
-      if (ok) ok = produce(kIxEnd, 0, 0, 0, nullptr, 0);
+      if (ok) ok = CW ? publish(kIxEnd, 0, 0, 0, 0, 0) : produce(kIxEnd, 0, 0, 0, nullptr, 0);
       if (!ok) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
       }
-      for (uint32_t s = 0; s < (uint32_t)kIxSlots && s < fill; ++s) {
-        const uint32_t lastf = fill - 1 - ((fill - 1 + kIxSlots - s) % kIxSlots);
+      // drain: the last use of every slot (entry, when publishing whole chunks) must have
+      // landed before the CTA may exit
+      const uint32_t nuse = CW ? seq : fill;
+      for (uint32_t s = 0; s < (uint32_t)kIxSlots && s < nuse; ++s) {
+        const uint32_t lastf = nuse - 1 - ((nuse - 1 + kIxSlots - s) % kIxSlots);
         if (lastf == 0 && p.stall) continue;  // never armed: nothing in flight
         mbar_wait_drain(&S.full[s], (lastf / kIxSlots) & 1u);
       }
@@ -369,8 +426,9 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
     float xb[VPT][V];
     uint4 rb[VPT];     // the base vectors as read, for the equality test
     bool bfin = true;  // every base element finite (Inf - Inf and NaN - NaN are not zero)
+    const uint32_t s0 = mt.s0;  // whole-chunk publication: the base fill's slot
     {
-      const uint8_t* slot = S.slot[fill % kIxSlots];
+      const uint8_t* slot = S.slot[CW ? s0 : fill % kIxSlots];
 #pragma unroll
       for (int u = 0; u < VPT; ++u) {
         rb[u] = ix_read_raw<BF16>(slot, p.base, off, (tid + (uint32_t)u * kIxConsumers) * V, n, n_tma);
@@ -378,17 +436,21 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
 #pragma unroll
         for (int e = 0; e < V; ++e) bfin = bfin && fabsf(xb[u][e]) < __int_as_float(0x7F800000);
       }
-      release(fill);
-      ++fill;
+      if constexpr (!CW) {
+        release(fill);
+        ++fill;
+      }
     }
 #pragma unroll
     for (int k = 0; k < KG; ++k) {
       if ((uint32_t)k >= kc) break;
-      if (!wait_full(fill)) {
-        alive = false;
-        break;
+      if constexpr (!CW) {
+        if (!wait_full(fill)) {
+          alive = false;
+          break;
+        }
       }
-      const uint8_t* slot = S.slot[fill % kIxSlots];
+      const uint8_t* slot = S.slot[CW ? (s0 + 1u + (uint32_t)k) % kIxSlots : fill % kIxSlots];
       uint4 re[VPT];
       // the equality test pays off only for TIES, whose per-element binning it skips; for
       // the other operators the comparison and vote cost more than the arithmetic they save
@@ -440,6 +502,12 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
           }
         }
       }
+      if constexpr (!CW) {
+        release(fill);
+        ++fill;
+      }
+    }
+    if constexpr (CW) {  // every read of the chunk's slots and entry is done
       release(fill);
       ++fill;
     }
