@@ -288,6 +288,26 @@ __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t nav
   }
 }
 
+// DARE keep words of the vector at flat element j0 for expert i: element j keeps its delta
+// iff 16-bit word j mod 8 of the Philox4x32-10 output for counter j / 8 is >= T.  A bf16
+// vector is exactly the 8 words of one call (chunk and tensor offsets are multiples of 8
+// elements); an fp32 vector is half of one.  Word j mod 8 of element j is returned in the
+// upper half of a 32-bit register: the upper word as it stands, the lower one moved up by a
+// multiply (FMA pipe; the ALU pipe is the busy one); it is kept iff that register >= T << 16.
+template <bool BF16>
+__device__ __forceinline__ void dare_keep_words(const MergeLaunch& p, uint32_t i, uint64_t j0,
+                                                uint32_t (&kw)[BF16 ? 8 : 4]) {
+  constexpr int V = BF16 ? 8 : 4;
+  const uint64_t g = j0 >> 3;
+  const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
+  const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
+#pragma unroll
+  for (int e = 0; e < V; ++e) {
+    const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
+    kw[e] = (e & 1) ? wd : wd * 65536u;
+  }
+}
+
 template <bool BF16, int OPC>
 __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
     merge_tma_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
@@ -438,23 +458,8 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   uint32_t n = 0, n_tma = 0, remaining = 0;
   uint32_t m_chunk = 0, m_rest = 0;  // the chunk's access mask; its experts still to come
   float s_sel = 0.0f;  // renormalised AVG: sum of the counted experts' alpha (ascending)
-  // DARE keep decisions of the vector's elements: element j keeps its delta iff 16-bit
-  // word j mod 8 of the Philox output for counter j / 8 is >= T.  A bf16 vector is exactly
-  // the 8 words of one call (chunk and tensor offsets are multiples of 8 elements); an
-  // fp32 vector is half of one.
-  // word j mod 8 of element j, in the upper half of a 32-bit register: the upper word as it
-  // stands, the lower one moved up by a multiply (FMA pipe; the ALU pipe is the busy one);
-  // it is kept iff that register >= T << 16
-  auto dare_words = [&](uint32_t i, uint64_t j0, uint32_t (&kw)[V]) {
-    const uint64_t g = j0 >> 3;
-    const Philox4 r = philox4x32_10_rk((uint32_t)g, (uint32_t)(g >> 32), i, 0x44415245u, p.dare_rk);
-    const uint32_t e0 = (uint32_t)(j0 & 7u);  // 0 for bf16; 0 or 4 for fp32
-#pragma unroll
-    for (int e = 0; e < V; ++e) {
-      const uint32_t wd = BF16 ? r.w[e >> 1] : (e0 ? r.w[2 + (e >> 1)] : r.w[e >> 1]);
-      kw[e] = (e & 1) ? wd : wd * 65536u;
-    }
-  };
+  // DARE keep decisions of the vector's elements (dare_keep_words)
+  auto dare_words = [&](uint32_t i, uint64_t j0, uint32_t (&kw)[V]) { dare_keep_words<BF16>(p, i, j0, kw); };
   auto dare_kept = [&](uint32_t i, uint64_t j0, bool (&kept)[V]) {
     uint32_t kw[V];
     dare_words(i, j0, kw);
@@ -616,25 +621,28 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
   }
 }
 
-// ---------------- TIES with at most 8 experts: whole-chunk consumers ----------------
+// ---------------- TIES (at most 8 experts) and DARE (at most 16): whole-chunk consumers ----------------
 //
 // The same TMA ring, but a chunk (its base fill and its selected experts' fills, which sit in
 // consecutive ring slots) is published as one unit: one "full" mbarrier per chunk counts the
 // bytes of all its fills, one "empty" mbarrier per chunk counts the consumers' releases.
 // A consumer thread waits once per chunk, folds every selected expert of its vector in the
 // fixed ascending order while all of them are in shared memory, releases the chunk and only
-// then finalises: the per-element state (M_0, P, N, counts) lives for one chunk and the
-// per-fill waits, arrivals and metadata reads of the streaming kernel disappear.  The ring
-// must hold every fill of one chunk (1 + K slots), so this kernel serves K <= 8; the
-// streaming kernel above serves larger expert counts.
+// then finalises: the per-element state (M_0 and P, N, counts for TIES, the accumulator for
+// DARE) lives for one chunk and the per-fill waits, arrivals and metadata reads of the
+// streaming kernel disappear.  The ring must hold every fill of one chunk (1 + K slots), so
+// this kernel serves TIES with K <= 8 and DARE with K <= 16; the streaming kernel above
+// serves the other operators and larger expert counts.
 constexpr uint32_t kTcSlotBytes = 4096u;
-constexpr uint32_t kTcMaxK = 8;
+constexpr uint32_t kTcMaxK = 16;
 
 // ring slots and CTAs per SM by expert count: K <= 4 holds two chunks of 5 fills in 11
-// slots at four CTAs per SM; K <= 8 two chunks of 9 fills in 18 slots at three
+// slots at four CTAs per SM; K <= 8 two chunks of 9 fills in 18 slots at three; K <= 16
+// (DARE) one chunk of 17 fills, or several of the usual few selected experts, in 17 slots
+// at three
 template <int KC>
 struct TcGeo {
-  static constexpr int kSlots = KC <= 4 ? 11 : 18;
+  static constexpr int kSlots = KC <= 4 ? 11 : (KC <= 8 ? 18 : 17);
   static constexpr int kCtasPerSm = KC <= 4 ? 4 : 3;
   static constexpr int kConsumers = 256;
   static constexpr int kThreads = kConsumers + 32;
@@ -649,7 +657,8 @@ struct TcEntry {
   uint32_t s0;           // ring slot of the base fill; expert fill j sits in slot s0 + 1 + j (mod NS)
   uint32_t nsel;         // selected experts
   uint32_t fast;         // 1: every selected threshold is >= 2^-100 (no numerator needs the IEEE division)
-  float thr[kTcMaxK];    // trim thresholds (as floats) in fill order
+  float thr[kTcMaxK];    // TIES: trim thresholds (as floats) in fill order
+  uint8_t ex[kTcMaxK];   // the selected experts in fill order
 };
 
 template <int NS, uint32_t G>
@@ -661,14 +670,15 @@ struct __align__(128) TcSmem {
   uint64_t full[NS];
   uint64_t empty[NS];
   unsigned long long realized[kMaxK];
-  float2 ntab[kTcMaxK + 1];  // {-c, RN(1/c)} for the counts c = 0..8 (entry 0: {-1, 1})
+  float2 ntab[9];             // {-c, RN(1/c)} for the TIES counts c = 0..8 (entry 0: {-1, 1})
   uint32_t nf[NS];           // producer only: fills held by the chunk of each entry
   int abort;
 };
 
-template <bool BF16, int KC>
+template <bool BF16, int OPC, int KC>
 __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
-    merge_ties_chunk_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
+    merge_chunk_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
+  static_assert(OPC == OP_TIES || OPC == OP_DARE, "whole-chunk consumers: TIES or DARE");
   constexpr int NS = TcGeo<KC>::kSlots;
   constexpr int kConsumers = TcGeo<KC>::kConsumers;
   constexpr uint32_t G = TcGeo<KC>::kGrab;
@@ -676,7 +686,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
   constexpr uint32_t CH = kTcSlotBytes / ES;  // elements per chunk
   constexpr int V = BF16 ? 8 : 4;
   static_assert(CH == (uint32_t)(kConsumers * V), "one vector per consumer thread and chunk");
-  static_assert(NS >= 2 * (KC + 1), "the ring holds every fill of two chunks");
+  static_assert(NS >= KC + 1, "the ring holds every fill of a chunk");
   extern __shared__ __align__(128) uint8_t smem_raw[];
   TcSmem<NS, G>& S = *reinterpret_cast<TcSmem<NS, G>*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
@@ -692,7 +702,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
     mbar_fence_init();
   }
   if (tid < (uint32_t)kMaxK) S.realized[tid] = 0;
-  if (tid <= kTcMaxK) {
+  if (tid <= 8u) {
     const float c = tid == 0 ? 1.0f : (float)tid;
     S.ntab[tid] = make_float2(-c, __fdiv_rn(1.0f, c));
   }
@@ -734,16 +744,18 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
           cm.m = p.mask[b];
           cm.n = start < len ? min(CH, len - start) : 0u;
           if (p.touched_only && cm.m == 0u) cm.n = 0u;  // left as it is: a reference to M_0
-          grp = p.blk_group[b];
+          if (OPC == OP_TIES) grp = p.blk_group[b];
         }
         S.chunk[lane] = cm;
       }
-      // lane i < K: the trim thresholds of expert i for every chunk of the grab, at least the
-      // smallest subnormal (a zero delta is never kept: it would add nothing)
+      if constexpr (OPC == OP_TIES) {
+        // lane i < K: the trim thresholds of expert i for every chunk of the grab, at least the
+        // smallest subnormal (a zero delta is never kept: it would add nothing)
 #pragma unroll
-      for (uint32_t c = 0; c < G; ++c) {
-        const uint32_t g = __shfl_sync(0xFFFFFFFFu, grp, c);
-        if (lane < p.K) S.thr[c][lane] = max(ties_bits_threshold(p.tau[(uint64_t)lane * p.n_groups + g]), 1u);
+        for (uint32_t c = 0; c < G; ++c) {
+          const uint32_t g = __shfl_sync(0xFFFFFFFFu, grp, c);
+          if (lane < p.K) S.thr[c][lane] = max(ties_bits_threshold(p.tau[(uint64_t)lane * p.n_groups + g]), 1u);
+        }
       }
       __syncwarp();
       if (lane == 0) {
@@ -765,9 +777,13 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
           ce.nsel = nsel;
           uint32_t fast = 1u, j = 0;
           for (uint32_t mm = cm.m; mm; mm &= mm - 1, ++j) {
-            const uint32_t t = S.thr[c][__ffs(mm) - 1];
-            ce.thr[j] = __uint_as_float(t);
-            fast &= t >= 0x0D800000u ? 1u : 0u;  // bits of 2^-100
+            const uint32_t i = __ffs(mm) - 1;
+            ce.ex[j] = (uint8_t)i;
+            if constexpr (OPC == OP_TIES) {
+              const uint32_t t = S.thr[c][i];
+              ce.thr[j] = __uint_as_float(t);
+              fast &= t >= 0x0D800000u ? 1u : 0u;  // bits of 2^-100
+            }
           }
           ce.fast = fast;
           S.nf[e] = 1u + nsel;
@@ -839,13 +855,62 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
     }
     float y[V];
     if (nsel == 0) {  // uniform over the CTA
-      // no expert selected: the output is M_0 plus the zero the operator adds (lambda * +0)
-      const float z = __fmul_rn(p.lambda, 0.0f);
+      // no expert selected: the output is M_0 plus the zero the operator adds (lambda * +0
+      // for TIES, +0 for DARE)
+      const float z = OPC == OP_TIES ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
 #pragma unroll
       for (int v = 0; v < V; ++v) y[v] = __fadd_rn(x0[v], z);
       const uint64_t off = ce.off;
       const uint32_t n = ce.n;
       mbar_arrive(&S.empty[e]);
+      if (k0 < n) store_vec<BF16>(p.out, off + k0, n - k0, y);
+      continue;
+    }
+    if constexpr (OPC == OP_DARE) {
+      // acc = fma(alpha_i, v_i, acc) over the selected experts in ascending order, with
+      // v_i = delta_i * sigma where expert i's keep word passes and +0 where it is dropped
+      float acc[V];
+#pragma unroll
+      for (int v = 0; v < V; ++v) acc[v] = 0.0f;
+#pragma unroll 1
+      for (uint32_t j = 0; j < nsel; ++j) {
+        s = s + 1 == (uint32_t)NS ? 0u : s + 1;
+        const uint32_t i = ce.ex[j];
+        const float a = p.alpha[i];
+        uint4 r;
+        if (in_slot) {
+          r = *reinterpret_cast<const uint4*>(S.slot[s] + k0 * ES);
+        } else {  // the ragged tail of a tensor, from global memory
+          const uint32_t n = ce.n;
+          r = read_raw<BF16>(S.slot[s], p.experts.p[i], ce.off - p.expert_origin, k0, n, ((n * ES) & ~15u) / ES);
+        }
+        uint32_t kw[V];
+        dare_keep_words<BF16>(p, i, ce.off + k0, kw);
+        auto fold_pair = [&](int v, float e0, float e1) {
+          float d0, d1, s0, s1;
+          f2_sub(e0, e1, x0[v], x0[v + 1], d0, d1);
+          f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
+          d0 = kw[v] >= p.dare_T16 ? s0 : 0.0f;
+          d1 = kw[v + 1] >= p.dare_T16 ? s1 : 0.0f;
+          f2_fma(a, a, d0, d1, acc[v], acc[v + 1], acc[v], acc[v + 1]);
+        };
+        float e0, e1;
+        pair_of<BF16, 0>(r, e0, e1);
+        fold_pair(0, e0, e1);
+        pair_of<BF16, 1>(r, e0, e1);
+        fold_pair(2, e0, e1);
+        if constexpr (BF16) {
+          pair_of<BF16, 2>(r, e0, e1);
+          fold_pair(4, e0, e1);
+          pair_of<BF16, 3>(r, e0, e1);
+          fold_pair(6, e0, e1);
+        }
+      }
+      const uint64_t off = ce.off;
+      const uint32_t n = ce.n;
+      mbar_arrive(&S.empty[e]);  // every read of the chunk's slots and entry is done
+#pragma unroll
+      for (int v = 0; v < V; v += 2) f2_add(x0[v], x0[v + 1], acc[v], acc[v + 1], y[v], y[v + 1]);
       if (k0 < n) store_vec<BF16>(p.out, off + k0, n - k0, y);
       continue;
     }
@@ -952,8 +1017,8 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
   }
 }
 
-template <bool BF16, int KC>
-cudaError_t launch_ties_chunk(const MergeLaunch& p, cudaStream_t st) {
+template <bool BF16, int OPC, int KC>
+cudaError_t launch_chunk(const MergeLaunch& p, cudaStream_t st) {
   constexpr uint32_t chunk = kTcSlotBytes / (BF16 ? 2u : 4u);
   const uint32_t cpb = (p.block_elems + chunk - 1) / chunk;
   const uint64_t n_chunks = (p.b_end - p.b_begin) * cpb;
@@ -964,7 +1029,7 @@ cudaError_t launch_ties_chunk(const MergeLaunch& p, cudaStream_t st) {
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
   const size_t smem = sizeof(TcSmem<TcGeo<KC>::kSlots, TcGeo<KC>::kGrab>);
-  auto kern = merge_ties_chunk_kernel<BF16, KC>;
+  auto kern = merge_chunk_kernel<BF16, OPC, KC>;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
     return e;
   uint64_t grid = (uint64_t)sms * TcGeo<KC>::kCtasPerSm;
@@ -1004,10 +1069,14 @@ cudaError_t launch_dtype(const MergeLaunch& p, cudaStream_t st) {
     case MP_OP_AVG:
     case MP_OP_TA: return launch_op<BF16, OP_ADD>(p, st);
     case MP_OP_TIES:
-      if (p.K <= 4) return launch_ties_chunk<BF16, 4>(p, st);
-      if (p.K <= kTcMaxK) return launch_ties_chunk<BF16, 8>(p, st);
+      if (p.K <= 4) return launch_chunk<BF16, OP_TIES, 4>(p, st);
+      if (p.K <= 8) return launch_chunk<BF16, OP_TIES, 8>(p, st);
       return launch_op<BF16, OP_TIES>(p, st);
-    case MP_OP_DARE: return launch_op<BF16, OP_DARE>(p, st);
+    case MP_OP_DARE:
+      if (p.K <= 4) return launch_chunk<BF16, OP_DARE, 4>(p, st);
+      if (p.K <= 8) return launch_chunk<BF16, OP_DARE, 8>(p, st);
+      if (p.K <= 16) return launch_chunk<BF16, OP_DARE, 16>(p, st);
+      return launch_op<BF16, OP_DARE>(p, st);
     case MP_OP_AVG_RENORM: return launch_op<BF16, OP_RENORM>(p, st);
     case MP_OP_DARE_TIES: return launch_op<BF16, OP_DTIES>(p, st);
     default: return cudaErrorInvalidValue;
