@@ -637,13 +637,13 @@ constexpr uint32_t kTcSlotBytes = 4096u;
 constexpr uint32_t kTcMaxK = 16;
 
 // ring slots and CTAs per SM by expert count: K <= 4 holds two chunks of 5 fills in 11
-// slots at four CTAs per SM; K <= 8 two chunks of 9 fills in 18 slots at three; K <= 16
-// (DARE) one chunk of 17 fills, or several of the usual few selected experts, in 17 slots
-// at three
-template <int KC>
+// slots at four CTAs per SM (three for DARE-TIES, whose state needs more registers); K <= 8
+// two chunks of 9 fills in 18 slots at three; K <= 16 one chunk of 17 fills, or several of
+// the usual few selected experts, in 17 slots at three
+template <int OPC, int KC>
 struct TcGeo {
   static constexpr int kSlots = KC <= 4 ? 11 : (KC <= 8 ? 18 : 17);
-  static constexpr int kCtasPerSm = KC <= 4 ? 4 : 3;
+  static constexpr int kCtasPerSm = KC <= 4 && OPC != OP_DTIES ? 4 : 3;
   static constexpr int kConsumers = 256;
   static constexpr int kThreads = kConsumers + 32;
   static constexpr uint32_t kGrab = 8;
@@ -670,18 +670,20 @@ struct __align__(128) TcSmem {
   uint64_t full[NS];
   uint64_t empty[NS];
   unsigned long long realized[kMaxK];
-  float2 ntab[9];             // {-c, RN(1/c)} for the TIES counts c = 0..8 (entry 0: {-1, 1})
+  float2 ntab[kTcMaxK + 1];  // {-c, RN(1/c)} for the counts c = 0..16 (entry 0: {-1, 1})
   uint32_t nf[NS];           // producer only: fills held by the chunk of each entry
   int abort;
 };
 
 template <bool BF16, int OPC, int KC>
-__global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
+__global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCtasPerSm)
     merge_chunk_kernel(const MergeLaunch p, uint32_t cpb, uint64_t n_chunks, unsigned long long* work) {
-  static_assert(OPC == OP_TIES || OPC == OP_DARE, "whole-chunk consumers: TIES or DARE");
-  constexpr int NS = TcGeo<KC>::kSlots;
-  constexpr int kConsumers = TcGeo<KC>::kConsumers;
-  constexpr uint32_t G = TcGeo<KC>::kGrab;
+  static_assert(OPC == OP_TIES || OPC == OP_DARE || OPC == OP_DTIES, "whole-chunk consumers: TIES, DARE, DARE-TIES");
+  // the packed counts C = 2^23 + c+ + 2^CB c-: CB = 4 bits for up to 8 experts, 5 for 16
+  constexpr uint32_t CB = KC <= 8 ? 4u : 5u;
+  constexpr int NS = TcGeo<OPC, KC>::kSlots;
+  constexpr int kConsumers = TcGeo<OPC, KC>::kConsumers;
+  constexpr uint32_t G = TcGeo<OPC, KC>::kGrab;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t CH = kTcSlotBytes / ES;  // elements per chunk
   constexpr int V = BF16 ? 8 : 4;
@@ -702,7 +704,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
     mbar_fence_init();
   }
   if (tid < (uint32_t)kMaxK) S.realized[tid] = 0;
-  if (tid <= 8u) {
+  if (tid <= kTcMaxK) {
     const float c = tid == 0 ? 1.0f : (float)tid;
     S.ntab[tid] = make_float2(-c, __fdiv_rn(1.0f, c));
   }
@@ -785,7 +787,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
               fast &= t >= 0x0D800000u ? 1u : 0u;  // bits of 2^-100
             }
           }
-          ce.fast = fast;
+          ce.fast = OPC == OP_TIES ? fast : 0u;  // DARE-TIES: rescaled deltas may be tiny
           S.nf[e] = 1u + nsel;
           // test hook: the first chunk is never armed, so the consumers' wait for it runs out
           const bool arm = !(seq == 0 && p.stall);
@@ -857,7 +859,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
     if (nsel == 0) {  // uniform over the CTA
       // no expert selected: the output is M_0 plus the zero the operator adds (lambda * +0
       // for TIES, +0 for DARE)
-      const float z = OPC == OP_TIES ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
+      const float z = kTiesLike<OPC> ? __fmul_rn(p.lambda, 0.0f) : 0.0f;
 #pragma unroll
       for (int v = 0; v < V; ++v) y[v] = __fadd_rn(x0[v], z);
       const uint64_t off = ce.off;
@@ -915,8 +917,9 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
       continue;
     }
     // Per element: P and N, the sums of the kept positive and negative deltas, and both
-    // counts in one float C = 2^23 + c+ + 16 c- (exact: every value is an integer below 2^24,
-    // so the low bits of C hold c+ and c-).  A delta d is kept positive when d >= thr and kept
+    // counts in one float C = 2^23 + c+ + 2^CB c- (exact: every value is an integer below
+    // 2^24, so the low bits of C hold c+ and c-).  DARE-TIES keeps, instead, every nonzero
+    // rescaled delta s = d sigma whose keep word passes (no magnitude trim).  A delta d is kept positive when d >= thr and kept
     // negative when d <= -thr (thr > 0: |d| >= thr and the sign in one compare each); the
     // keep factors k+ and k- are 1 or 0, and P = fma(k+, d, P), N = fma(k-, d, N): a factor 1
     // adds d with the one rounding of P + d, a factor 0 adds a zero, which leaves P and N
@@ -932,7 +935,9 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
 #pragma unroll 1
     for (uint32_t j = 0; j < nsel; ++j) {
       s = s + 1 == (uint32_t)NS ? 0u : s + 1;
-      const float thr = ce.thr[j];
+      const float thr = OPC == OP_TIES ? ce.thr[j] : 0.0f;
+      uint32_t kw[V];
+      if constexpr (OPC == OP_DTIES) dare_keep_words<BF16>(p, ce.ex[j], ce.off + k0, kw);
       uint4 r;
       if (in_slot) {
         r = *reinterpret_cast<const uint4*>(S.slot[s] + k0 * ES);
@@ -942,13 +947,24 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
       }
       // one element pair at a time, so that only the raw vector stays live
       auto tally_pair = [&](int v, float e0, float e1) {
-        float d0, d1, t0, t1;
+        float d0, d1, t0, t1, kp0, kp1, kn0, kn1;
         f2_sub(e0, e1, x0[v], x0[v + 1], d0, d1);
-        const float kp0 = d0 >= thr ? 1.0f : 0.0f, kp1 = d1 >= thr ? 1.0f : 0.0f;
-        const float kn0 = d0 <= -thr ? 1.0f : 0.0f, kn1 = d1 <= -thr ? 1.0f : 0.0f;
+        if constexpr (OPC == OP_DTIES) {
+          f2_mul(d0, d1, p.sigma, p.sigma, d0, d1);
+          const bool k0w = kw[v] >= p.dare_T16, k1w = kw[v + 1] >= p.dare_T16;
+          kp0 = k0w && d0 > 0.0f ? 1.0f : 0.0f;
+          kp1 = k1w && d1 > 0.0f ? 1.0f : 0.0f;
+          kn0 = k0w && d0 < 0.0f ? 1.0f : 0.0f;
+          kn1 = k1w && d1 < 0.0f ? 1.0f : 0.0f;
+        } else {
+          kp0 = d0 >= thr ? 1.0f : 0.0f;
+          kp1 = d1 >= thr ? 1.0f : 0.0f;
+          kn0 = d0 <= -thr ? 1.0f : 0.0f;
+          kn1 = d1 <= -thr ? 1.0f : 0.0f;
+        }
         f2_fma(kp0, kp1, d0, d1, Pp[v], Pp[v + 1], Pp[v], Pp[v + 1]);
         f2_fma(kn0, kn1, d0, d1, Nn[v], Nn[v + 1], Nn[v], Nn[v + 1]);
-        f2_fma(kn0, kn1, 16.0f, 16.0f, kp0, kp1, t0, t1);
+        f2_fma(kn0, kn1, (float)(1u << CB), (float)(1u << CB), kp0, kp1, t0, t1);
         f2_add(Cc[v], Cc[v + 1], t0, t1, Cc[v], Cc[v + 1]);
       };
       float e0, e1;
@@ -972,7 +988,7 @@ __global__ void __launch_bounds__(TcGeo<KC>::kThreads, TcGeo<KC>::kCtasPerSm)
       const bool pos = Pp[v] > -Nn[v], any = Pp[v] != -Nn[v];
       num = any ? (pos ? Pp[v] : Nn[v]) : 0.0f;
       const uint32_t cb = __float_as_uint(Cc[v]);
-      cv = any ? ((pos ? cb : cb >> 4) & 15u) : 0u;
+      cv = any ? ((pos ? cb : cb >> CB) & ((1u << CB) - 1u)) : 0u;
     };
     if (fast) {  // uniform over the CTA: every nonzero numerator is >= 2^-100 in magnitude
       // q = RN(num * y), then Markstein's correction q + RN(num - q c) * y, and the output
@@ -1028,14 +1044,14 @@ cudaError_t launch_chunk(const MergeLaunch& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  const size_t smem = sizeof(TcSmem<TcGeo<KC>::kSlots, TcGeo<KC>::kGrab>);
+  const size_t smem = sizeof(TcSmem<TcGeo<OPC, KC>::kSlots, TcGeo<OPC, KC>::kGrab>);
   auto kern = merge_chunk_kernel<BF16, OPC, KC>;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
     return e;
-  uint64_t grid = (uint64_t)sms * TcGeo<KC>::kCtasPerSm;
+  uint64_t grid = (uint64_t)sms * TcGeo<OPC, KC>::kCtasPerSm;
   if (grid > n_chunks) grid = n_chunks;
   if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
-  kern<<<(unsigned)grid, TcGeo<KC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
+  kern<<<(unsigned)grid, TcGeo<OPC, KC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
   count_launches(1);
   return cudaGetLastError();
 }
@@ -1078,7 +1094,11 @@ cudaError_t launch_dtype(const MergeLaunch& p, cudaStream_t st) {
       if (p.K <= 16) return launch_chunk<BF16, OP_DARE, 16>(p, st);
       return launch_op<BF16, OP_DARE>(p, st);
     case MP_OP_AVG_RENORM: return launch_op<BF16, OP_RENORM>(p, st);
-    case MP_OP_DARE_TIES: return launch_op<BF16, OP_DTIES>(p, st);
+    case MP_OP_DARE_TIES:
+      if (p.K <= 4) return launch_chunk<BF16, OP_DTIES, 4>(p, st);
+      if (p.K <= 8) return launch_chunk<BF16, OP_DTIES, 8>(p, st);
+      if (p.K <= 16) return launch_chunk<BF16, OP_DTIES, 16>(p, st);
+      return launch_op<BF16, OP_DTIES>(p, st);
     default: return cudaErrorInvalidValue;
   }
 }

@@ -192,6 +192,18 @@ def fam_k9():
                         per_expert_active=True, name="k9")
 
 
+def fam_k7():
+    # K = 7: the whole-chunk merges for up to 8 experts (bf16)
+    return synth.custom([30000, 8191, 65536 + 8], dtype=synth.BF16, block_elems=4096, K=7, active_frac=0.6,
+                        per_expert_active=True, name="k7")
+
+
+def fam_k16():
+    # K = 16 with most blocks active for every expert: chunks of 17 fills fill the 17-slot ring
+    return synth.custom([40000, 4097, 24576], dtype=synth.BF16, block_elems=4096, K=16, active_frac=0.9,
+                        name="k16")
+
+
 def fam_k17():
     return synth.custom([20000, 7777, 40000], dtype=synth.BF16, block_elems=2048, K=17, active_frac=0.3,
                         per_expert_active=True, name="k17")
@@ -223,7 +235,7 @@ def fam_max_block():
 FRACS = [0.0, 0.1, 0.25, 0.5, 0.9, 1.0, 1000.0]
 
 
-@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k9, fam_k17, fam_k32, fam_k1],
+@pytest.mark.parametrize("make", [fam_ragged_bf16, fam_ragged_f32, fam_k7, fam_k9, fam_k16, fam_k17, fam_k32, fam_k1],
                          ids=lambda f: f.__name__)
 def test_parity_small_families(make):
     fam = make()
