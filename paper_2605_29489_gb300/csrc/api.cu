@@ -378,9 +378,11 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     const int b = (int)(s & 1);
     const Segment& g = segs[s];
     if ((e = hp.side_acquire(b)) != cudaSuccess) break;
-    // every expert block of the segment, read over the host mapping by a copy kernel: on
-    // GB300 this reaches the host link's rate where 64 MiB cudaMemcpyAsync copies on two
-    // side streams reached about 60 % of it
+    // every expert block of the segment, read over the host mapping by a copy kernel.  It
+    // moves bytes at the host link's rate, as large contiguous cudaMemcpyAsync copies do,
+    // and it gathers any selection of blocks in one launch per segment, where copies would
+    // take one call per run of consecutive selected blocks (the merge below gathers only
+    // the planned blocks)
     GatherLaunch gl;
     memset(&gl, 0, sizeof(gl));
     gl.K = p.K;

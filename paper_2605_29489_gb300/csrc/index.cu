@@ -49,13 +49,14 @@ __device__ __forceinline__ uint4 load_vec_raw(const void* base_ptr, bool bf16, u
 template <bool BF16>
 __device__ __forceinline__ void unpack(const uint4 r, float (&x)[BF16 ? 8 : 4]) {
   if constexpr (BF16) {
-    x[0] = __uint_as_float(r.x << 16);
+    // the lower element moved up by a multiply (FMA pipe), the upper one by a mask (ALU)
+    x[0] = __uint_as_float(r.x * 65536u);
     x[1] = __uint_as_float(r.x & 0xFFFF0000u);
-    x[2] = __uint_as_float(r.y << 16);
+    x[2] = __uint_as_float(r.y * 65536u);
     x[3] = __uint_as_float(r.y & 0xFFFF0000u);
-    x[4] = __uint_as_float(r.z << 16);
+    x[4] = __uint_as_float(r.z * 65536u);
     x[5] = __uint_as_float(r.z & 0xFFFF0000u);
-    x[6] = __uint_as_float(r.w << 16);
+    x[6] = __uint_as_float(r.w * 65536u);
     x[7] = __uint_as_float(r.w & 0xFFFF0000u);
   } else {
     x[0] = __uint_as_float(r.x);
@@ -102,6 +103,7 @@ struct IxMeta {
   uint32_t n;      // elements in the chunk
   uint32_t last;   // 1 on the block's last chunk
   uint32_t s0;     // whole-chunk publication: ring slot of the base fill (experts follow)
+  int32_t wlo[4];  // whole-chunk publication, window bins: L - 1 of the item's experts' windows
 };
 
 // How the TIES catalog bins the keys of the deltas:
@@ -196,7 +198,10 @@ __device__ __forceinline__ void ties_win2(float d0, float d1, int32_t lo, uint32
   const int32_t hi = lo + (int32_t)kWinKeys + 1;
   const int32_t k0 = min(max((int32_t)(w & 0x7FFFu), lo), hi);
   const int32_t k1 = min(max((int32_t)((w >> 16) & 0x7FFFu), lo), hi);
-  const uint32_t a0 = hist0 + ((uint32_t)k0 << 2), a1 = hist0 + ((uint32_t)k1 << 2);
+  // byte addresses by multiply-add (FMA pipe; the ALU pipe carries the clamps)
+  uint32_t a0, a1;
+  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a0) : "r"((uint32_t)k0), "r"(hist0));
+  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a1) : "r"((uint32_t)k1), "r"(hist0));
   asm volatile(
       "{\n"
       " .reg .pred p0, p1;\n"
@@ -296,6 +301,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
         return true;
       };
       // publishes one chunk: the base fill and kc expert fills in consecutive slots
+      int32_t item_wlo[4] = {0, 0, 0, 0};  // window bins: L - 1 of the current item's experts
       auto publish = [&](uint32_t item, uint64_t off, uint32_t n, uint32_t last, uint32_t i0,
                          uint32_t kc) -> bool {
         const uint32_t nfill = item == kIxEnd ? 0u : 1u + kc;
@@ -308,6 +314,10 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
         S.meta[e].n = n;
         S.meta[e].last = last;
         S.meta[e].s0 = fill % kIxSlots;
+        if constexpr (BM == kBinWindow) {
+#pragma unroll
+          for (int k = 0; k < 4; ++k) S.meta[e].wlo[k] = item_wlo[k];
+        }
         S.nf[e] = nfill;
         const bool arm = !(seq == 0 && p.stall);  // test hook: the first chunk is never armed
         if (arm) mbar_arrive_expect_tx(&S.full[e], nfill * bytes);
@@ -360,6 +370,12 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
         const uint32_t len = p.blk_len[b];
         const uint64_t off0 = p.blk_off[b];
         const uint32_t nch = (len + CH - 1) / CH;
+        if constexpr (CW && BM == kBinWindow) {
+          const uint32_t grp = p.blk_group[b];
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+            item_wlo[k] = (uint32_t)k < kc ? (int32_t)p.wlo[(uint64_t)(i0 + k) * p.n_groups + grp] - 1 : 0;
+        }
         for (uint32_t c = 0; c < nch && ok; ++c) {
           const uint32_t n = min(CH, len - c * CH);
           const uint64_t off = off0 + (uint64_t)c * CH;
@@ -468,8 +484,10 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
       if (!__all_sync(0xFFFFFFFFu, same)) {
         // kBinWindow: L - 1 of this expert's window in the block's trim group
         int32_t wlo_k = 0;
-        if constexpr (BM == kBinWindow)
-          wlo_k = (int32_t)__ldg(p.wlo + (uint64_t)(i0 + k) * p.n_groups + __ldg(p.blk_group + b)) - 1;
+        if constexpr (BM == kBinWindow) {
+          if constexpr (CW) wlo_k = mt.wlo[k < 4 ? k : 0];
+          else wlo_k = (int32_t)__ldg(p.wlo + (uint64_t)(i0 + k) * p.n_groups + __ldg(p.blk_group + b)) - 1;
+        }
 #pragma unroll
         for (int u = 0; u < VPT; ++u) {
           float xe[V];
