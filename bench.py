@@ -583,7 +583,7 @@ def native(args, rank, world, local_rank):
                    "step": ("catalog import" if catalog is not None else "index") + " + (plan + merge) per budget"},
         "accessed_expert_gbs": sum(pb["planned_bytes"] for pb in per_budget) / merge_total_s / 1e9,
         "index_ms": idx_ms, "per_budget": per_budget, "time_model": t_model, "block_hashes": hashes,
-        "roofline": {"bound": "hbm", "kernel": merge_kernel_name(W["op"], fam.dtype), "achieved": achieved, "peak": peak, "unit": "GB/s",
+        "roofline": {"bound": "hbm", "kernel": merge_kernel_name(W["op"], fam.dtype, fam.K), "achieved": achieved, "peak": peak, "unit": "GB/s",
                      "frac": achieved / peak, "peak_kind": peak_kind,
                      "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
                      "traffic": profiled_traffic(args.workload, sum(alg_bytes) / len(alg_bytes)),
@@ -615,11 +615,14 @@ def native(args, rank, world, local_rank):
     return line
 
 
-def merge_kernel_name(op: str, dtype: int) -> str:
-    """the merge kernel instance a workload's operator launches"""
+def merge_kernel_name(op: str, dtype: int, K: int) -> str:
+    """the merge kernel instance a workload's operator launches: whole-chunk consumers for
+    TIES with up to 8 experts and DARE / DARE-TIES with up to 16, streaming consumers
+    otherwise"""
     inst = {"ta": "AVG/TA", "avg": "AVG/TA", "ties": "TIES", "ties_masked": "TIES", "dare": "DARE",
             "avg_renorm": "AVG_RENORM", "dare_ties": "DARE_TIES"}[op]
-    return f"merge_tma_kernel<{'bf16' if dtype == 0 else 'f32'}, {inst}>"
+    chunk = (inst == "TIES" and K <= 8) or (inst in ("DARE", "DARE_TIES") and K <= 16)
+    return f"{'merge_chunk_kernel' if chunk else 'merge_tma_kernel'}<{'bf16' if dtype == 0 else 'f32'}, {inst}>"
 
 
 def time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream, reps=3):
