@@ -670,59 +670,64 @@ template <bool BF16, int KG>
 __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
   constexpr int V = BF16 ? 8 : 4;
   __shared__ uint32_t s_fine[KG][128];
-  const uint32_t G = (p.K + KG - 1) / KG;
-  const uint64_t b = blockIdx.x / G;
-  const uint32_t i0 = (blockIdx.x % G) * KG;
-  const uint32_t kc = min((uint32_t)KG, p.K - i0);
-  const uint32_t grp = p.blk_group[b];
-  const uint32_t tid = threadIdx.x;
   if (p.miss && *p.miss == 0u) return;  // windowed thresholds: no pair needs this pass
+  const uint32_t G = (p.K + KG - 1) / KG;
+  const uint64_t n_items = p.n_blocks * G;
+  const uint32_t tid = threadIdx.x;
+  // items (block, group of KG experts) in a grid-stride loop: a grid of resident CTAs
+  for (uint64_t it = blockIdx.x; it < n_items; it += gridDim.x) {
+    const uint64_t b = it / G;
+    const uint32_t i0 = (uint32_t)(it % G) * KG;
+    const uint32_t kc = min((uint32_t)KG, p.K - i0);
+    const uint32_t grp = p.blk_group[b];
 
-  uint32_t estar[KG];
-  uint32_t want = 0u;  // bit k: expert i0+k may hold keys in its bin e*
-#pragma unroll
-  for (int k = 0; k < KG; ++k) {
-    estar[k] = kNoBin;
-    if ((uint32_t)k < kc) {
-      uint32_t i = i0 + k;
-      uint32_t es = p.estar[(uint64_t)i * p.n_groups + grp];
-      uint64_t u = (uint64_t)i * p.n_blocks + b;
-      const bool read = (!p.mask || ((p.mask[b] >> i) & 1u)) &&  // TIES_MASKED: selected blocks only
-                        (!p.gmiss || p.gmiss[(uint64_t)i * p.n_groups + grp] != 0u);  // windowed: missed pairs only
-      if (read && es != kNoBin && p.nnz[u] != 0u && (ties_key(p.maxabs[u]) >> 7) >= es) {
-        estar[k] = es;
-        want |= 1u << k;
-      }
-    }
-  }
-  if (want == 0u) return;  // uniform over the CTA
-  if (p.thr_reads && threadIdx.x == 0)
-    atomicAdd(p.thr_reads, (unsigned long long)__popc(want) * p.blk_len[b] * (BF16 ? 2u : 4u));
-  for (uint32_t x = tid; x < (uint32_t)KG * 128u; x += 256u) (&s_fine[0][0])[x] = 0u;
-  __syncthreads();
-
-  const uint64_t off = p.blk_off[b];
-  const uint32_t len = p.blk_len[b];
-  const uint32_t nvec = (len + V - 1) / V;
-  for (uint32_t v = tid; v < nvec; v += kLanes) {
-    float xb[V];
-    unpack<BF16>(load_vec_raw(p.base, BF16, off, v, len), xb);
+    uint32_t estar[KG];
+    uint32_t want = 0u;  // bit k: expert i0+k may hold keys in its bin e*
 #pragma unroll
     for (int k = 0; k < KG; ++k) {
-      if (!((want >> k) & 1u)) continue;
-      float xe[V];
-      unpack<BF16>(load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len), xe);
-#pragma unroll
-      for (int e = 0; e < V; e += 2)
-        ties_fine2(__fsub_rn(xe[e], xb[e]), __fsub_rn(xe[e + 1], xb[e + 1]), estar[k], su32(&s_fine[k][0]));
+      estar[k] = kNoBin;
+      if ((uint32_t)k < kc) {
+        uint32_t i = i0 + k;
+        uint32_t es = p.estar[(uint64_t)i * p.n_groups + grp];
+        uint64_t u = (uint64_t)i * p.n_blocks + b;
+        const bool read = (!p.mask || ((p.mask[b] >> i) & 1u)) &&  // TIES_MASKED: selected blocks only
+                          (!p.gmiss || p.gmiss[(uint64_t)i * p.n_groups + grp] != 0u);  // windowed: missed pairs only
+        if (read && es != kNoBin && p.nnz[u] != 0u && (ties_key(p.maxabs[u]) >> 7) >= es) {
+          estar[k] = es;
+          want |= 1u << k;
+        }
+      }
     }
-  }
-  __syncthreads();
-  for (uint32_t x = tid; x < (uint32_t)KG * 128u; x += 256u) {
-    uint32_t k = x >> 7, m = x & 127u;
-    if (!((want >> k) & 1u)) continue;
-    uint32_t c = s_fine[k][m];
-    if (c) atomicAdd(&p.fine[((uint64_t)(i0 + k) * p.n_groups + grp) * 128u + m], (unsigned long long)c);
+    if (want == 0u) continue;  // uniform over the CTA
+    if (p.thr_reads && threadIdx.x == 0)
+      atomicAdd(p.thr_reads, (unsigned long long)__popc(want) * p.blk_len[b] * (BF16 ? 2u : 4u));
+    for (uint32_t x = tid; x < (uint32_t)KG * 128u; x += 256u) (&s_fine[0][0])[x] = 0u;
+    __syncthreads();
+
+    const uint64_t off = p.blk_off[b];
+    const uint32_t len = p.blk_len[b];
+    const uint32_t nvec = (len + V - 1) / V;
+    for (uint32_t v = tid; v < nvec; v += kLanes) {
+      float xb[V];
+      unpack<BF16>(load_vec_raw(p.base, BF16, off, v, len), xb);
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        if (!((want >> k) & 1u)) continue;
+        float xe[V];
+        unpack<BF16>(load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len), xe);
+#pragma unroll
+        for (int e = 0; e < V; e += 2)
+          ties_fine2(__fsub_rn(xe[e], xb[e]), __fsub_rn(xe[e + 1], xb[e + 1]), estar[k], su32(&s_fine[k][0]));
+      }
+    }
+    __syncthreads();
+    for (uint32_t x = tid; x < (uint32_t)KG * 128u; x += 256u) {
+      uint32_t k = x >> 7, m = x & 127u;
+      if (!((want >> k) & 1u)) continue;
+      uint32_t c = s_fine[k][m];
+      if (c) atomicAdd(&p.fine[((uint64_t)(i0 + k) * p.n_groups + grp) * 128u + m], (unsigned long long)c);
+    }
+    __syncthreads();  // the next item clears s_fine
   }
 }
 
@@ -908,7 +913,16 @@ cudaError_t ties_finish_t(const IndexLaunch& p, cudaStream_t st) {
   const uint32_t G = (p.K + KG - 1) / KG;
   const uint64_t nsel = (uint64_t)p.K * p.n_groups;
   const unsigned sgrid = (unsigned)((nsel + 127) / 128);
-  const uint64_t fgrid = p.n_blocks * G;
+  int dev = 0, sms = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  int per_sm = 0;  // resident CTAs of 256 threads; items by grid stride
+  if ((e = cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, ties_fine_kernel<BF16, KG>, 256, 0)) != cudaSuccess)
+    return e;
+  uint64_t fgrid = (uint64_t)sms * (per_sm > 0 ? per_sm : 1);
+  if (fgrid > p.n_blocks * G) fgrid = p.n_blocks * G;
+  if (fgrid == 0) fgrid = 1;
   ties_coarse_select<<<sgrid, 128, 0, st>>>(p);
   ties_fine_kernel<BF16, KG><<<(unsigned)fgrid, 256, 0, st>>>(p);
   ties_fine_select<<<sgrid, 128, 0, st>>>(p);

@@ -136,3 +136,17 @@ def test_plan_noalloc_refuses_bad_arguments_before_any_device_work():
     assert "trim_scope" in call(op=mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, trim_scope=2), tau=A, blk_group=A)
     assert "drop_p" in call(op=mp.make_op(mp.MP_OP_DARE, alpha=[0.5, 0.5], drop_p=1.5))
     assert "drop_p" in call(op=mp.make_op(mp.MP_OP_DARE_TIES, lam=1.0, drop_p=-0.1))
+
+
+def test_fault_injection_hook_arms_and_refuses_unknown_kinds_without_gpu():
+    """the host-side fault hook is plain host state: arming and disarming the two kinds
+    succeeds, an unknown kind is refused (no CUDA call is made)"""
+    import paper_2605_29489_gb300 as mp
+
+    for kind in (mp.MP_FAULT_ALLOC, mp.MP_FAULT_GATHER):
+        mp.mp_debug_inject_fault(kind, 3)
+        mp.mp_debug_inject_fault(kind, 0)
+    with pytest.raises(mp.MergePipeError) as e:
+        mp.mp_debug_inject_fault(0, 1)
+    assert e.value.status == -1
+    mp.mp_debug_stall_pipeline(0)
