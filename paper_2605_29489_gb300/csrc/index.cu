@@ -189,19 +189,24 @@ __device__ __forceinline__ void f2_sub(float a0, float a1, float b0, float b1, f
 }
 
 // TIES window bins of two deltas: a nonzero delta with key k adds 1 to bin
-// clamp(k, L - 1, L + 384) - (L - 1) of the shared histogram, i.e. bin 0 below the window,
-// bins 1..384 for the keys L..L + 383, bin 385 above it.  lo = L - 1; hist0 = the byte
-// address of bin 0 minus 4 lo.  Predicated, no branch.
+// clamp(k - lo, 0, 385) of the shared histogram at hist0, with lo = L - 1: bin 0 below the
+// window, bins 1..384 for the keys L..L + 383, bin 385 above it.  Both keys at once in
+// 16-bit lanes: one add and one clamp at zero and 385 (k - lo lies in [-32383, 32768]; it
+// wraps only for the NaN key 0x7FFF at lo = -1, whose bin the clamp still keeps in range and
+// whose NaN the statistics report).  Predicated, no branch.
 __device__ __forceinline__ void ties_win2(float d0, float d1, int32_t lo, uint32_t hist0) {
   const __nv_bfloat162 h2 = __floats2bfloat162_rn(d0, d1);
-  const uint32_t w = *reinterpret_cast<const uint32_t*>(&h2);
-  const int32_t hi = lo + (int32_t)kWinKeys + 1;
-  const int32_t k0 = min(max((int32_t)(w & 0x7FFFu), lo), hi);
-  const int32_t k1 = min(max((int32_t)((w >> 16) & 0x7FFFu), lo), hi);
-  // byte addresses by multiply-add (FMA pipe; the ALU pipe carries the clamps)
+  const uint32_t w = *reinterpret_cast<const uint32_t*>(&h2) & 0x7FFF7FFFu;
+  static_assert(kWinKeys + 1u == 0x181u, "the clamp bound is the above-window bin");
+  const uint32_t nlo2 = ((uint32_t)(-lo) & 0xFFFFu) * 0x00010001u;
+  uint32_t kk;
+  asm("{\n .reg .b32 t;\n add.s16x2 t, %1, %2;\n min.s16x2.relu %0, t, %3;\n}"
+      : "=r"(kk)
+      : "r"(w), "r"(nlo2), "r"(0x01810181u));
+  // byte addresses by multiply-add (FMA pipe; the ALU pipe carries the rest)
   uint32_t a0, a1;
-  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a0) : "r"((uint32_t)k0), "r"(hist0));
-  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a1) : "r"((uint32_t)k1), "r"(hist0));
+  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a0) : "r"(kk & 0xFFFFu), "r"(hist0));
+  asm("mad.lo.u32 %0, %1, 4, %2;" : "=r"(a1) : "r"(kk >> 16), "r"(hist0));
   asm volatile(
       "{\n"
       " .reg .pred p0, p1;\n"
@@ -510,7 +515,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
 #pragma unroll
           for (int e = 0; e < V; e += 2) {
             if constexpr (BM == kBinWindow) {
-              ties_win2(d[e], d[e + 1], wlo_k, su32(&S.hist[k][0]) - ((uint32_t)wlo_k << 2));
+              ties_win2(d[e], d[e + 1], wlo_k, su32(&S.hist[k][0]));
             } else if constexpr (BM == kBinCoarse) {
               ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]));
             } else {
@@ -827,11 +832,19 @@ __global__ void __launch_bounds__(256) ties_sample_kernel(const IndexLaunch p) {
         v = v0 * per + h % per;
       }
       my_n += min(V, len - v * V);
+      // every checkpoint's vector in flight at once: one memory round trip per position
+      const uint4 rb = load_vec_raw(p.base, BF16, off, v, len);
+      uint4 re[KG];
+#pragma unroll
+      for (int k = 0; k < KG; ++k)
+        if ((uint32_t)k < kc) re[k] = load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len);
       float xb[V];
-      unpack<BF16>(load_vec_raw(p.base, BF16, off, v, len), xb);
-      for (uint32_t k = 0; k < kc; ++k) {
+      unpack<BF16>(rb, xb);
+#pragma unroll
+      for (int k = 0; k < KG; ++k) {
+        if ((uint32_t)k >= kc) break;
         float xe[V];
-        unpack<BF16>(load_vec_raw(p.experts.p[i0 + k], BF16, off, v, len), xe);
+        unpack<BF16>(re[k], xe);
 #pragma unroll
         for (uint32_t e = 0; e < V; ++e) {
           const float d = __fsub_rn(xe[e], xb[e]);

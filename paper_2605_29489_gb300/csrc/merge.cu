@@ -649,6 +649,7 @@ struct TcGeo {
   static constexpr uint32_t kGrab = 8;
 };
 
+template <int KC>
 struct TcEntry {
   uint64_t off;          // element offset of the chunk
   uint32_t q;            // chunk id, or kEnd
@@ -657,19 +658,20 @@ struct TcEntry {
   uint32_t s0;           // ring slot of the base fill; expert fill j sits in slot s0 + 1 + j (mod NS)
   uint32_t nsel;         // selected experts
   uint32_t fast;         // 1: every selected threshold is >= 2^-100 (no numerator needs the IEEE division)
-  float thr[kTcMaxK];    // TIES: trim thresholds (as floats) in fill order
-  uint8_t ex[kTcMaxK];   // the selected experts in fill order
+  float thr[KC];         // TIES: trim thresholds (as floats) in fill order
+  uint8_t ex[KC];        // the selected experts in fill order
 };
 
-template <int NS, uint32_t G>
+// sized by the expert count KC so that three CTAs of 18 slots fit one SM's 228 KB
+template <int NS, uint32_t G, int KC>
 struct __align__(128) TcSmem {
   uint8_t slot[NS][kTcSlotBytes];
-  TcEntry ce[NS];
+  TcEntry<KC> ce[NS];
   ChunkMeta chunk[G];
-  uint32_t thr[G][kTcMaxK];  // bits threshold of (chunk of the grab, expert)
+  uint32_t thr[G][KC];  // bits threshold of (chunk of the grab, expert)
   uint64_t full[NS];
   uint64_t empty[NS];
-  unsigned long long realized[kMaxK];
+  unsigned long long realized[KC];
   float2 ntab[kTcMaxK + 1];  // {-c, RN(1/c)} for the counts c = 0..16 (entry 0: {-1, 1})
   uint32_t nf[NS];           // producer only: fills held by the chunk of each entry
   int abort;
@@ -690,7 +692,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
   static_assert(CH == (uint32_t)(kConsumers * V), "one vector per consumer thread and chunk");
   static_assert(NS >= KC + 1, "the ring holds every fill of a chunk");
   extern __shared__ __align__(128) uint8_t smem_raw[];
-  TcSmem<NS, G>& S = *reinterpret_cast<TcSmem<NS, G>*>(smem_raw);
+  TcSmem<NS, G, KC>& S = *reinterpret_cast<TcSmem<NS, G, KC>*>(smem_raw);
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   volatile int* abort_flag = &S.abort;
   const uint32_t wl = wait_limit_of(p.wait_limit);
@@ -703,7 +705,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
     S.abort = 0;
     mbar_fence_init();
   }
-  if (tid < (uint32_t)kMaxK) S.realized[tid] = 0;
+  if (tid < (uint32_t)KC) S.realized[tid] = 0;
   if (tid <= kTcMaxK) {
     const float c = tid == 0 ? 1.0f : (float)tid;
     S.ntab[tid] = make_float2(-c, __fdiv_rn(1.0f, c));
@@ -770,7 +772,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
           if (fill >= (uint32_t)NS) fence_proxy_async_smem();  // slots the consumers have read are refilled
           const uint32_t e = seq % NS;
           const uint32_t bytes = (cm.n * ES) & ~15u;
-          TcEntry& ce = S.ce[e];
+          TcEntry<KC>& ce = S.ce[e];
           ce.off = cm.off;
           ce.q = (uint32_t)(q0 + c);
           ce.n = cm.n;
@@ -844,7 +846,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
       S.abort = 1;
       break;
     }
-    const TcEntry& ce = S.ce[e];
+    const TcEntry<KC>& ce = S.ce[e];
     if (ce.q == kEnd) break;
     uint32_t s = ce.s0;
     const uint32_t nsel = ce.nsel;
@@ -1044,7 +1046,11 @@ cudaError_t launch_chunk(const MergeLaunch& p, cudaStream_t st) {
   cudaError_t e;
   if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
   if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
-  const size_t smem = sizeof(TcSmem<TcGeo<OPC, KC>::kSlots, TcGeo<OPC, KC>::kGrab>);
+  using Smem = TcSmem<TcGeo<OPC, KC>::kSlots, TcGeo<OPC, KC>::kGrab, KC>;
+  // every CTA also holds 1 KB of the SM's 228 KB for the system
+  static_assert(TcGeo<OPC, KC>::kCtasPerSm * (sizeof(Smem) + 1024) <= 228u * 1024u,
+                "the CTAs per SM that the grid assumes fit one SM's shared memory");
+  const size_t smem = sizeof(Smem);
   auto kern = merge_chunk_kernel<BF16, OPC, KC>;
   if ((e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess)
     return e;
