@@ -452,6 +452,7 @@ def native(args, rank, world, local_rank):
             per_budget[-1]["touched_elements"] = int(np.asarray(blk_len)[np.asarray(pi["mask"]) != 0].sum())
         if gop.kind == mp.MP_OP_TIES_MASKED:   # the masked threshold's second read of selected blocks
             per_budget[-1]["threshold_read_bytes"] = mp.mp_manifest_threshold_reads(last[2 + 2 * k])
+    timeline = host_timeline(mp, step, mf, budgets, args.trace_out) if host_pool else None
     hashes = None
     if not host_pool and not args.no_hash:
         hashes = time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream)
@@ -597,6 +598,7 @@ def native(args, rank, world, local_rank):
                                            "per merged parameter") + " 2*s + s*(selected experts); summed over the "
                                           "budget sweep's launches / their summed CUDA-event time"},
         "gpu_launches": launches,
+        "host_timeline": timeline,
         "host_link": None if link is None else dict(
             h2d_gbs_measured=link, gathered_bytes=[pb["planned_bytes"] for pb in per_budget],
             gathered_gbs=[pb["planned_bytes"] / (pb["merge_ms"] / 1e3) / 1e9 for pb in per_budget],
@@ -629,6 +631,60 @@ def merge_kernel_name(op: str, dtype: int, K: int) -> str:
             "avg_renorm": "AVG_RENORM", "dare_ties": "DARE_TIES"}[op]
     chunk = (inst == "TIES" and K <= 8) or (inst in ("DARE", "DARE_TIES") and K <= 16)
     return f"{'merge_chunk_kernel' if chunk else 'merge_tma_kernel'}<{'bf16' if dtype == 0 else 'f32'}, {inst}>"
+
+
+def _union_ms(iv):
+    """total length of a union of intervals [(t0, t1), ...]"""
+    tot, end = 0.0, None
+    for a, b in sorted(iv):
+        if end is None or a > end:
+            tot += b - a
+            end = b
+        elif b > end:
+            tot += b - end
+            end = b
+    return tot
+
+
+def _overlap_ms(a, b, iv):
+    """length of [a, b] covered by the union of the intervals iv"""
+    return _union_ms([(max(a, x), min(b, y)) for x, y in iv if min(b, y) > max(a, x)])
+
+
+def host_timeline(mp, step, mf, budgets, trace_out=None):
+    """One more step, untimed, with the device-time trace on: per call (the index, each
+    budget's merge), the wall time, how busy the gather stream kept the host link, and how
+    much of the segment kernels' time ran while a gather was in flight."""
+    import torch
+    torch.cuda.synchronize()
+    mp.mp_trace_start(1 << 16)
+    hs = step(mf)
+    torch.cuda.synchronize()
+    ranges = mp.mp_trace_stop()
+    for h in hs:
+        h.free()
+    if trace_out:
+        with open(trace_out, "w") as fo:
+            fo.write("kind,segment,stream,t0_ms,t1_ms\n")
+            for r in ranges:
+                fo.write(f"{r['kind']},{r['segment']},{r['stream']},{r['t0_ms']:.4f},{r['t1_ms']:.4f}\n")
+    calls = []   # ranges in enqueue order: a segment range belongs to the call begun before it
+    for r in ranges:
+        if r["kind"] in (mp.MP_TRACE_INDEX, mp.MP_TRACE_MERGE):
+            calls.append({"call": r, "g": [], "k": []})
+        elif r["kind"] == mp.MP_TRACE_GATHER and calls:
+            calls[-1]["g"].append((r["t0_ms"], r["t1_ms"]))
+        elif r["kind"] == mp.MP_TRACE_SEGMENT and calls:
+            calls[-1]["k"].append((r["t0_ms"], r["t1_ms"]))
+    out = []
+    for c, name in zip(calls, ["index"] + [f"merge f={f}" for f in budgets]):
+        wall = c["call"]["t1_ms"] - c["call"]["t0_ms"]
+        kern = sum(b - a for a, b in c["k"])
+        under = sum(_overlap_ms(a, b, c["g"]) for a, b in c["k"])
+        out.append(dict(call=name, segments=len(c["g"]), wall_ms=wall, gather_busy_ms=_union_ms(c["g"]),
+                        gather_busy_frac=_union_ms(c["g"]) / wall if wall > 0 else None, kernel_ms=kern,
+                        kernel_under_gather_frac=under / kern if kern > 0 else None))
+    return out
 
 
 def time_hashes(mp, fam, mf, last, outs, shared_out, per_budget, stream, reps=3):
@@ -890,6 +946,8 @@ def main():
     ap.add_argument("--k-sweep", action="store_true",
                     help="K-scaling at a fixed absolute budget (Cor. 1) instead of the workload sweep")
     ap.add_argument("--k-list", default="4,8,16,32", help="expert counts of --k-sweep")
+    ap.add_argument("--trace-out", default=None,
+                    help="host-pool workloads: write the traced step's device-time ranges to this CSV")
     ap.add_argument("--k-budget-experts", type=float, default=0.25,
                     help="the fixed budget of --k-sweep, in units of one expert checkpoint's bytes")
     args = ap.parse_args()

@@ -364,6 +364,41 @@ const char* mp_version(void);
    all threads).  A diagnostic for counting launches per step; never resets. */
 uint64_t mp_kernel_launch_count(void);
 
+/* Device-time trace of the calls (tracing for the phase timings of Tab. 4 and the
+ * gather/merge overlap of a host-resident pool, Sec. 3 "Executor").
+ *
+ * mp_trace_start(capacity): from now on every call records the device time of its work
+ * as ranges of two CUDA events, on the stream that runs it, until capacity ranges are
+ * held: one range per mp_index_blocks (MP_TRACE_INDEX), mp_plan (MP_TRACE_PLAN) and
+ * mp_merge / mp_merge_touched (MP_TRACE_MERGE) on the caller's stream, and, for experts in
+ * pinned host memory, one range per segment for its gather on the side stream
+ * (MP_TRACE_GATHER) and for its kernels on the caller's stream (MP_TRACE_SEGMENT).  A
+ * start while a trace is held discards it.  Returns MP_ERR_INVALID_ARG for capacity 0 or
+ * above 2^20, MP_ERR_CUDA if the events cannot be created.
+ * mp_trace_stop(n_ranges): stops recording, waits for the recorded events and returns the
+ * number of ranges held (ranges beyond the capacity are dropped, not recorded).
+ * mp_trace_read(out, n): copies the first n ranges (n <= the count mp_trace_stop gave) in
+ * the order they were enqueued; times are in ms from the earliest start among them.
+ * Process-wide; the host-side NVTX ranges of the calls (one per entry point, named after
+ * it) are always emitted and cost nothing without a tool attached.
+ */
+#define MP_TRACE_INDEX 1
+#define MP_TRACE_PLAN 2
+#define MP_TRACE_MERGE 3
+#define MP_TRACE_GATHER 4
+#define MP_TRACE_SEGMENT 5
+typedef struct mp_trace_range {
+  uint32_t kind;     /* MP_TRACE_* */
+  uint32_t segment;  /* host-pool segment (GATHER, SEGMENT), else 0 */
+  uint32_t stream;   /* 0: the caller's stream; 1: the host-pool gather stream */
+  uint32_t reserved;
+  double t0_ms;      /* start of the range's device work */
+  double t1_ms;      /* end of the range's device work */
+} mp_trace_range;
+mp_status mp_trace_start(uint32_t capacity);
+mp_status mp_trace_stop(uint64_t* n_ranges);
+mp_status mp_trace_read(mp_trace_range* out, uint64_t n);
+
 /*
  * Test hooks for the failure paths.  The paper has no counterpart: they exist so that the
  * error returns of this library (a run either produces its handle or leaves none, Alg. 2)

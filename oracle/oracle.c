@@ -550,8 +550,9 @@ int orc_dare_keep(uint64_t seed, uint32_t expert, uint64_t j, double p) {
  * fp32 operations (reading; the paper fixes none): experts in ascending index.
  *  AVG / TA (zero-completed tuple):  acc = sum_i fma(alpha_i, A_i delta_i, acc);
  *                                    out = round(M_0 + acc)
- *  DARE: v_i = keep_i ? delta_i * sigma : 0, sigma = fp32(1/(1-p));
- *        acc = sum_i fma(alpha_i, A_i v_i, acc); out = round(M_0 + acc)
+ *  DARE: v_i = delta_i * sigma for a kept entry, sigma = fp32(1/(1-p)); a dropped entry is
+ *        omitted from the sum, as an unselected one is (its zero is never added);
+ *        acc = sum over the kept selected i of fma(alpha_i, v_i, acc); out = round(M_0 + acc)
  *  TIES: d^_i = A_i delta_i if key(delta_i) >= tau_i else 0;  P = sum of the d^_i > 0,
  *        N = sum of the d^_i < 0 (each an ascending fp32 chain from +0), c+ and c- their
  *        counts;  gamma = sign(P + N), taken exactly as P > -N, P < -N or P = -N (the
@@ -633,7 +634,10 @@ int orc_merge_block(int dtype, uint64_t n, uint64_t j0, const void* base, const 
       for (uint32_t i = 0; i < K; ++i) {
         if (!((mask >> i) & 1u)) continue; /* omitted: zero entry, never read */
         float d = load_elem(dtype, experts[i], k) - x0;
-        if (op->kind == ORC_DARE) d = orc_dare_keep(op->seed, i, j0 + k, op->drop_p) ? d * sigma : 0.0f;
+        if (op->kind == ORC_DARE) {
+          if (!orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) continue; /* dropped: omitted */
+          d = d * sigma;
+        }
         const float coef = op->kind == ORC_AVG_RENORM ? op->alpha[i] / s_sel : op->alpha[i];
         acc = fmaf(coef, d, acc);
       }

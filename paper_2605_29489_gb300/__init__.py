@@ -28,7 +28,8 @@ __all__ = [
     "mp_version", "mp_kernel_launch_count", "mp_plan_noalloc", "mp_index_import", "MP_NNZ_MISSING", "mp_index_hashes",
     "mp_index_hash_values", "mp_manifest_validate", "mp_manifest_validation", "lib",
     "MP_FAULT_ALLOC", "MP_FAULT_GATHER", "mp_debug_inject_fault", "mp_debug_stall_pipeline",
-    "library_path",
+    "MP_TRACE_INDEX", "MP_TRACE_PLAN", "MP_TRACE_MERGE", "MP_TRACE_GATHER", "MP_TRACE_SEGMENT",
+    "mp_trace_start", "mp_trace_stop", "library_path",
 ]
 
 MP_OK = 0
@@ -38,6 +39,8 @@ MP_BF16, MP_F32 = 0, 1
 MP_OP_AVG, MP_OP_TA, MP_OP_TIES, MP_OP_DARE, MP_OP_AVG_RENORM, MP_OP_DARE_TIES, MP_OP_TIES_MASKED = 0, 1, 2, 3, 4, 5, 6
 MP_NNZ_MISSING = 0xFFFFFFFF   # catalog entry without block statistics (tensor-level fallback)
 MP_FAULT_ALLOC, MP_FAULT_GATHER = 1, 2  # test hooks: kinds of injected host-side failures
+# kinds of traced device-time ranges (mp_trace_start)
+MP_TRACE_INDEX, MP_TRACE_PLAN, MP_TRACE_MERGE, MP_TRACE_GATHER, MP_TRACE_SEGMENT = 1, 2, 3, 4, 5
 
 
 class MergePipeError(RuntimeError):
@@ -55,6 +58,11 @@ class _Family(ctypes.Structure):
                 ("block_elems", ctypes.c_uint32), ("base", ctypes.c_void_p), ("K", ctypes.c_uint32),
                 ("experts", ctypes.POINTER(ctypes.c_void_p)), ("experts_location", ctypes.c_uint32),
                 ("lineage_ids", ctypes.POINTER(ctypes.c_uint64))]
+
+
+class _TraceRange(ctypes.Structure):
+    _fields_ = [("kind", ctypes.c_uint32), ("segment", ctypes.c_uint32), ("stream", ctypes.c_uint32),
+                ("reserved", ctypes.c_uint32), ("t0_ms", ctypes.c_double), ("t1_ms", ctypes.c_double)]
 
 
 class _Op(ctypes.Structure):
@@ -103,6 +111,9 @@ def lib():
         L.mp_kernel_launch_count.restype, L.mp_kernel_launch_count.argtypes = u64, []
         L.mp_debug_inject_fault.restype, L.mp_debug_inject_fault.argtypes = st, [ctypes.c_int32, u64]
         L.mp_debug_stall_pipeline.restype, L.mp_debug_stall_pipeline.argtypes = None, [ctypes.c_uint32]
+        L.mp_trace_start.restype, L.mp_trace_start.argtypes = st, [ctypes.c_uint32]
+        L.mp_trace_stop.restype, L.mp_trace_stop.argtypes = st, [ctypes.POINTER(u64)]
+        L.mp_trace_read.restype, L.mp_trace_read.argtypes = st, [ctypes.POINTER(_TraceRange), u64]
         _lib = L
     return _lib
 
@@ -371,6 +382,22 @@ def mp_debug_stall_pipeline(rounds: int) -> None:
     """Test hook: index and merge kernels launched from now on never arm their first ring
     slot and give up a pipeline wait after `rounds` polling rounds (0 = off)."""
     lib().mp_debug_stall_pipeline(int(rounds))
+
+
+def mp_trace_start(capacity: int = 4096) -> None:
+    """Record the device time of the calls from now on (at most `capacity` ranges)."""
+    _check(lib().mp_trace_start(int(capacity)))
+
+
+def mp_trace_stop() -> list:
+    """Stop recording; the ranges as dicts (kind, segment, stream, t0_ms, t1_ms) in the
+    order they were enqueued, times in ms from the earliest start."""
+    n = ctypes.c_uint64(0)
+    _check(lib().mp_trace_stop(ctypes.byref(n)))
+    arr = (_TraceRange * max(1, n.value))()
+    _check(lib().mp_trace_read(arr, n.value))
+    return [{"kind": r.kind, "segment": r.segment, "stream": r.stream, "t0_ms": r.t0_ms, "t1_ms": r.t1_ms}
+            for r in arr[:n.value]]
 
 
 def mp_plan_noalloc(K, n_blocks, n_groups, dtype, blk_len, blk_group, norm, maxabs, nnz, tau, index_err, op: Op,

@@ -399,7 +399,10 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
       e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
       break;
     }
-    if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
+    const int tg = trace_begin(MP_TRACE_GATHER, (uint32_t)s, 1, hp.side[0]);
+    e = launch_gather(gl, hp.side[0]);
+    trace_end(tg, hp.side[0]);
+    if (e != cudaSuccess) break;
     if ((e = hp.main_acquire(b)) != cudaSuccess) break;
     IndexLaunch ps = p;
     ps.b_begin = g.b0;
@@ -407,7 +410,10 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     ps.expert_origin = g.e0;
     ps.defer_ties_select = 1;
     for (uint32_t i = 0; i < p.K; ++i) ps.experts.p[i] = hp.buf(b, i);
-    if ((e = launch_index(ps, cs)) != cudaSuccess) break;
+    const int tk = trace_begin(MP_TRACE_SEGMENT, (uint32_t)s, 0, cs);
+    e = launch_index(ps, cs);
+    trace_end(tk, cs);
+    if (e != cudaSuccess) break;
     e = hp.main_release(b);
   }
   if (e == cudaSuccess && p.coarse) {
@@ -447,14 +453,20 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
       e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
       break;
     }
-    if ((e = launch_gather(gl, hp.side[0])) != cudaSuccess) break;
+    const int tg = trace_begin(MP_TRACE_GATHER, (uint32_t)s, 1, hp.side[0]);
+    e = launch_gather(gl, hp.side[0]);
+    trace_end(tg, hp.side[0]);
+    if (e != cudaSuccess) break;
     if ((e = hp.main_acquire(b)) != cudaSuccess) break;
     MergeLaunch ps = p;
     ps.b_begin = g.b0;
     ps.b_end = g.b1;
     ps.expert_origin = g.e0;
     ps.experts = gl.dst;
-    if ((e = launch_merge(ps, cs)) != cudaSuccess) break;
+    const int tk = trace_begin(MP_TRACE_SEGMENT, (uint32_t)s, 0, cs);
+    e = launch_merge(ps, cs);
+    trace_end(tk, cs);
+    if (e != cudaSuccess) break;
     e = hp.main_release(b);
   }
   hp.finish();
@@ -616,6 +628,7 @@ uint64_t mp_budget_from_fraction(const mp_family* family, double f) {
 }
 
 mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream stream, mp_index** out) {
+  NvtxScope nv("mp_index_blocks");
   if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
   Geometry g;
@@ -627,6 +640,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   ExpertPtrs ex;
   if ((st = resolve_pointers(family, base, ex)) != MP_OK) return st;
   cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  TraceScope tr(MP_TRACE_INDEX, cs);
 
   const uint32_t scope = ties ? op->trim_scope : 0u;
   const uint32_t n_groups = scope == 0 ? g.n_tensors : 1u;
@@ -823,6 +837,7 @@ mp_status mp_index_import(const mp_family* family, const mp_op* op, const float*
 }
 
 mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes, mp_stream stream, mp_plan_t** out) {
+  NvtxScope nv("mp_plan");
   if (!out) return fail(MP_ERR_INVALID_ARG, "out is NULL");
   *out = nullptr;
   mp_status st;
@@ -833,6 +848,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
       (index->op_kind != op->kind || index->density != op->density || index->trim_scope != op->trim_scope))
     return fail(MP_ERR_MISMATCH, "a TIES plan needs an index built for the same TIES kind, density and trim scope");
   cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  TraceScope tr(MP_TRACE_PLAN, cs);
   const uint64_t nb = g.n_blocks, U = nb * g.K;
 
   mp_plan_s* pl = new (std::nothrow) mp_plan_s();
@@ -979,6 +995,7 @@ namespace {
 // unwritten (and then out may be the base itself)
 mp_status merge_common(const mp_family* family, const mp_index* index, const mp_plan_t* plan, void* out_buf,
                        mp_stream stream, mp_manifest** man_out, bool touched_only) {
+  NvtxScope nv(touched_only ? "mp_merge_touched" : "mp_merge");
   if (!man_out) return fail(MP_ERR_INVALID_ARG, "manifest out is NULL");
   *man_out = nullptr;
   mp_status st;
@@ -1009,6 +1026,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
         return fail(MP_ERR_INVALID_ARG, "out overlaps an expert");
   }
   cudaStream_t cs = reinterpret_cast<cudaStream_t>(stream);
+  TraceScope tr(MP_TRACE_MERGE, cs);
   const bool masked = plan->op_kind == MP_OP_TIES_MASKED;
   if (masked && !index->d_unit_hist)
     return fail(MP_ERR_MISMATCH, "a TIES_MASKED merge needs an index built for TIES_MASKED");

@@ -89,10 +89,10 @@ constexpr uint32_t kIxEnd = 0xFFFFFFFFu;
 // slots.  The TIES catalog also bins every delta, which makes it bound by instruction
 // latency: four CTAs per SM (more warps to hide it; the state fits 56 registers) with twelve
 // 4 KiB slots (one vector per consumer thread and fill).  With eight experts per item the
-// histograms make a CTA too large for four per SM, and three run.
-template <bool TIES>
+// histograms make a CTA too large for four per SM: three run, with the registers of three.
+template <bool TIES, int KG = 1>
 struct IxGeo {
-  static constexpr int kCtasPerSm = TIES ? 4 : 2;
+  static constexpr int kCtasPerSm = TIES ? (KG > 4 ? 3 : 4) : 2;
   static constexpr uint32_t kSlotBytes = TIES ? 4096u : 8192u;
   static constexpr int kSlots = 12;
 };
@@ -118,11 +118,11 @@ constexpr uint32_t kWinBins = kWinKeys + 2;  // + below + above
 
 template <int KG, int NS, uint32_t SB, uint32_t NB>
 struct __align__(128) IxSmem {
-  uint8_t slot[NS][SB];
+  uint32_t hist[KG][NB];  // first: its byte addresses stay below 2^16 (ties_win2k packs two)
+  alignas(128) uint8_t slot[NS][SB];
   IxMeta meta[NS];
   uint64_t full[NS];
   uint64_t empty[NS];
-  uint32_t hist[KG][NB];
   uint32_t nf[NS];  // whole-chunk publication: fills held by the chunk of each entry
   float red_ss[KG][8];
   float red_mx[KG][8];
@@ -219,6 +219,46 @@ __device__ __forceinline__ void ties_win2(float d0, float d1, int32_t lo, uint32
       : "memory");
 }
 
+// The same bins for deltas of two bf16 checkpoints, where key 0 holds exactly the zero
+// deltas (the difference of two distinct bf16 values is at least the smallest bf16
+// subnormal, whose key is 1).  Every delta adds 1 to its bin, zeros included: a zero has
+// key 0 and lands below the window, in bin 0, which no threshold reads (with the window at
+// the bottom, L = 0 and lo = -1, it lands in key 0's bin, where it can only decide a
+// threshold of key 0, the one that an uncounted zero gives too).  The nonzero deltas are
+// counted from the returned key word instead (nz_halves).  Both byte addresses come from one
+// multiply-add in 16-bit lanes: h2 = the histogram's byte address in both lanes, which the
+// caller keeps below 2^16 - 4 * 385.  No predicate and no branch.
+__device__ __forceinline__ uint32_t ties_win2k(float d0, float d1, int32_t lo, uint32_t h2) {
+  const __nv_bfloat162 hb = __floats2bfloat162_rn(d0, d1);
+  const uint32_t w = *reinterpret_cast<const uint32_t*>(&hb) & 0x7FFF7FFFu;
+  const uint32_t nlo2 = ((uint32_t)(-lo) & 0xFFFFu) * 0x00010001u;
+  uint32_t kk;
+  asm("{\n .reg .b32 t;\n add.s16x2 t, %1, %2;\n min.s16x2.relu %0, t, %3;\n}"
+      : "=r"(kk)
+      : "r"(w), "r"(nlo2), "r"(0x01810181u));
+  const uint32_t a2 = kk * 4u + h2;  // lanes: h + 4 b0 and h + 4 b1 (no carry between them)
+  asm volatile(
+      "{\n"
+      " .reg .b32 a0, a1;\n"
+      " and.b32 a0, %0, 65535;\n"
+      " shr.u32 a1, %0, 16;\n"
+      " red.shared.add.u32 [a0], 1;\n"
+      " red.shared.add.u32 [a1], 1;\n"
+      "}\n" ::"r"(a2)
+      : "memory");
+  return w;
+}
+
+// number of nonzero keys among the four key words of a vector, in two 16-bit lanes
+__device__ __forceinline__ uint32_t nz_halves(uint32_t w0, uint32_t w1, uint32_t w2, uint32_t w3) {
+  uint32_t m0, m1, m2, m3;
+  asm("min.u16x2 %0, %1, %2;" : "=r"(m0) : "r"(w0), "r"(0x00010001u));
+  asm("min.u16x2 %0, %1, %2;" : "=r"(m1) : "r"(w1), "r"(0x00010001u));
+  asm("min.u16x2 %0, %1, %2;" : "=r"(m2) : "r"(w2), "r"(0x00010001u));
+  asm("min.u16x2 %0, %1, %2;" : "=r"(m3) : "r"(w3), "r"(0x00010001u));
+  return m0 + m1 + m2 + m3;
+}
+
 // TIES fine bins of two deltas: a nonzero delta whose coarse bin (key bits 7..14) is es
 // adds 1 to fine bin (key & 127) of the shared histogram at hist; predicated, no branch
 __device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint32_t hist) {
@@ -250,7 +290,7 @@ __device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint
 }
 
 template <bool BF16, int KG, int BM>
-__global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
+__global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone, KG>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
   constexpr bool TIES = BM != kBinNone;
   constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;  // key bins per expert
@@ -259,6 +299,9 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
   // mbarrier (counting all their bytes) and one "empty" mbarrier, so that a consumer waits
   // and releases once per chunk instead of once per fill.
   constexpr bool CW = TIES && KG <= 4;
+  // window bins of bf16 deltas: the nonzero count comes from the keys (ties_win2k,
+  // nz_halves) and the zeros share the below-window bin
+  constexpr bool KNZ = BM == kBinWindow && BF16;
   constexpr int kIxSlots = IxGeo<TIES>::kSlots;
   static_assert(!CW || kIxSlots >= 2 * (KG + 1), "two whole chunks fit the ring");
   constexpr uint32_t kIxSlotBytes = IxGeo<TIES>::kSlotBytes;
@@ -273,6 +316,12 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   // the fallback pass of the windowed catalog runs only when some threshold left its window
   if (BM == kBinCoarse && p.miss && *p.miss == 0u) return;
+  if constexpr (KNZ) {  // the packed bin addresses need the histogram below 2^16 - 4 * 385
+    if (su32(&S.hist[KG - 1][NB - 1]) >= 65536u - 4u * (kWinKeys + 1u)) {
+      if (threadIdx.x == 0) atomicOr(p.err, kErrInternal);
+      return;
+    }
+  }
   volatile int* abort_flag = &S.abort;
   const uint32_t wl = wait_limit_of(p.wait_limit);
 
@@ -512,15 +561,23 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
 #pragma unroll
             for (int e = 0; e < w; ++e) m[e] = fmaxf(m[e], m[e + w]);
           mx[k] = fmaxf(mx[k], m[0]);
+          if constexpr (KNZ) {
+            const uint32_t h2 = su32(&S.hist[k][0]) * 0x00010001u;
+            uint32_t wk[V / 2];
 #pragma unroll
-          for (int e = 0; e < V; e += 2) {
-            if constexpr (BM == kBinWindow) {
-              ties_win2(d[e], d[e + 1], wlo_k, su32(&S.hist[k][0]));
-            } else if constexpr (BM == kBinCoarse) {
-              ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]));
-            } else {
-              nz[k] += d[e] != 0.0f ? 1u : 0u;
-              nz[k] += d[e + 1] != 0.0f ? 1u : 0u;
+            for (int e = 0; e < V; e += 2) wk[e / 2] = ties_win2k(d[e], d[e + 1], wlo_k, h2);
+            nz[k] += nz_halves(wk[0], wk[1], wk[2], wk[3]);
+          } else {
+#pragma unroll
+            for (int e = 0; e < V; e += 2) {
+              if constexpr (BM == kBinWindow) {
+                ties_win2(d[e], d[e + 1], wlo_k, su32(&S.hist[k][0]));
+              } else if constexpr (BM == kBinCoarse) {
+                ties_bin2(d[e], d[e + 1], su32(&S.hist[k][0]));
+              } else {
+                nz[k] += d[e] != 0.0f ? 1u : 0u;
+                nz[k] += d[e + 1] != 0.0f ? 1u : 0u;
+              }
             }
           }
         }
@@ -539,6 +596,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
     // end of the block: the canonical combine, then the statistics (and TIES bins)
 #pragma unroll
     for (int k = 0; k < KG; ++k) {
+      if constexpr (KNZ) nz[k] = (nz[k] & 0xFFFFu) + (nz[k] >> 16);  // the two 16-bit lanes
 #pragma unroll
       for (int s = 16; s >= 1; s >>= 1) {
         ss[k] = __fadd_rn(ss[k], __shfl_xor_sync(0xFFFFFFFFu, ss[k], s));
@@ -576,7 +634,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
           const uint64_t u = (uint64_t)(i0 + k) * p.n_blocks + b;
           p.norm[u] = __fsqrt_rn(a);
           p.maxabs[u] = m;
-          if constexpr (!TIES) p.nnz[u] = c;
+          if constexpr (!TIES || KNZ) p.nnz[u] = c;
           // a NaN delta makes the sum of squares NaN; an infinite one makes max |delta| infinite
           if (isnan(a) || isinf(m)) bad = 1u;
         }
@@ -584,7 +642,8 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
       if (lane == 0 && bad) atomicOr(p.err, kErrNonfinite);
     }
     if constexpr (TIES) {
-      // every nonzero delta added 1 to exactly one bin: the histogram's total is nnz
+      // every nonzero delta added 1 to exactly one bin: the histogram's total is nnz (not
+      // for KNZ, whose nonzero deltas were counted by key and whose bin 0 holds the zeros too)
       if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
         atomicOr(p.err, kErrTimeout);
         S.abort = 1;
@@ -601,15 +660,19 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
           hd[k] = S.hist[k][tid + 256u];
           S.hist[k][tid + 256u] = 0u;
         }
-        uint32_t w = hc[k] + hd[k];
+        if constexpr (!KNZ) {
+          uint32_t w = hc[k] + hd[k];
 #pragma unroll
-        for (int s = 16; s >= 1; s >>= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, s);
-        if (lane == 0) S.red_nz[k][warp] = w;
+          for (int s = 16; s >= 1; s >>= 1) w += __shfl_xor_sync(0xFFFFFFFFu, w, s);
+          if (lane == 0) S.red_nz[k][warp] = w;
+        }
       }
-      if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
-        atomicOr(p.err, kErrTimeout);
-        S.abort = 1;
-        break;
+      if constexpr (!KNZ) {
+        if (!consumer_barrier(&S.cbar, cphase, abort_flag, wl)) {
+          atomicOr(p.err, kErrTimeout);
+          S.abort = 1;
+          break;
+        }
       }
       const uint32_t grp = p.blk_group[b];
       const uint32_t len = p.blk_len[b];
@@ -617,9 +680,11 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone>::kCtasPerSm)
       for (int k = 0; k < KG; ++k) {
         if ((uint32_t)k >= kc) break;
         uint32_t nzk = 0;
+        if constexpr (!KNZ) {
 #pragma unroll
-        for (int w = 0; w < kIxConsumers / 32; ++w) nzk += S.red_nz[k][w];
-        if (tid == 0) p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
+          for (int w = 0; w < kIxConsumers / 32; ++w) nzk += S.red_nz[k][w];
+          if (tid == 0) p.nnz[(uint64_t)(i0 + k) * p.n_blocks + b] = nzk;
+        }
         const uint64_t x = (uint64_t)(i0 + k) * p.n_groups + grp;
         if constexpr (BM == kBinCoarse) {
           unsigned long long c = hc[k];
@@ -949,7 +1014,11 @@ cudaError_t launch_pass(const IndexLaunch& p, uint32_t G, uint64_t n_items, int 
   constexpr bool ties = BM != kBinNone;
   constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;
   const size_t smem = sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>);
-  uint64_t grid = (uint64_t)sms * IxGeo<ties>::kCtasPerSm;
+  static_assert(IxGeo<ties, KG>::kCtasPerSm *
+                        (sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>) + 1024) <=
+                    228u * 1024u,
+                "the CTAs per SM that the grid assumes fit one SM's shared memory");
+  uint64_t grid = (uint64_t)sms * IxGeo<ties, KG>::kCtasPerSm;
   if (grid > n_items) grid = n_items;
   cudaError_t e;
   if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;

@@ -549,13 +549,14 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
           for (int e = 0; e < V; e += 2) {
             float d0, d1;
             f2_sub(xe[e], xe[e + 1], x0[u][e], x0[u][e + 1], d0, d1);
-            if constexpr (OPC == OP_DARE) {
+            if constexpr (OPC == OP_DARE) {  // a dropped entry is omitted from the sum
               float s0, s1;
               f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
-              d0 = kept[e] ? s0 : 0.0f;
-              d1 = kept[e + 1] ? s1 : 0.0f;
+              if (kept[e]) acc[u][e] = __fmaf_rn(a, s0, acc[u][e]);
+              if (kept[e + 1]) acc[u][e + 1] = __fmaf_rn(a, s1, acc[u][e + 1]);
+            } else {
+              f2_fma(a, a, d0, d1, acc[u][e], acc[u][e + 1], acc[u][e], acc[u][e + 1]);
             }
-            f2_fma(a, a, d0, d1, acc[u][e], acc[u][e + 1], acc[u][e], acc[u][e + 1]);
           }
         }
       }
@@ -871,8 +872,8 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
       continue;
     }
     if constexpr (OPC == OP_DARE) {
-      // acc = fma(alpha_i, v_i, acc) over the selected experts in ascending order, with
-      // v_i = delta_i * sigma where expert i's keep word passes and +0 where it is dropped
+      // acc = fma(alpha_i, v_i, acc) over the selected experts whose keep word passes, in
+      // ascending order, with v_i = delta_i * sigma (a dropped entry is omitted)
       float acc[V];
 #pragma unroll
       for (int v = 0; v < V; ++v) acc[v] = 0.0f;
@@ -894,9 +895,9 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
           float d0, d1, s0, s1;
           f2_sub(e0, e1, x0[v], x0[v + 1], d0, d1);
           f2_mul(d0, d1, p.sigma, p.sigma, s0, s1);
-          d0 = kw[v] >= p.dare_T16 ? s0 : 0.0f;
-          d1 = kw[v + 1] >= p.dare_T16 ? s1 : 0.0f;
-          f2_fma(a, a, d0, d1, acc[v], acc[v + 1], acc[v], acc[v + 1]);
+          // a dropped entry is omitted from the sum, as an unselected one is
+          if (kw[v] >= p.dare_T16) acc[v] = __fmaf_rn(a, s0, acc[v]);
+          if (kw[v + 1] >= p.dare_T16) acc[v + 1] = __fmaf_rn(a, s1, acc[v + 1]);
         };
         float e0, e1;
         pair_of<BF16, 0>(r, e0, e1);
@@ -953,11 +954,12 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
         f2_sub(e0, e1, x0[v], x0[v + 1], d0, d1);
         if constexpr (OPC == OP_DTIES) {
           f2_mul(d0, d1, p.sigma, p.sigma, d0, d1);
-          const bool k0w = kw[v] >= p.dare_T16, k1w = kw[v + 1] >= p.dare_T16;
-          kp0 = k0w && d0 > 0.0f ? 1.0f : 0.0f;
-          kp1 = k1w && d1 > 0.0f ? 1.0f : 0.0f;
-          kn0 = k0w && d0 < 0.0f ? 1.0f : 0.0f;
-          kn1 = k1w && d1 < 0.0f ? 1.0f : 0.0f;
+          // keep factors as 1.0 / 0.0 straight from compares joined with the keep test
+          asm("{\n .reg .pred q;\n setp.ge.u32 q, %4, %5;\n set.gt.and.f32.f32 %0, %6, 0f00000000, q;\n"
+              " set.lt.and.f32.f32 %1, %6, 0f00000000, q;\n setp.ge.u32 q, %7, %5;\n"
+              " set.gt.and.f32.f32 %2, %8, 0f00000000, q;\n set.lt.and.f32.f32 %3, %8, 0f00000000, q;\n}"
+              : "=f"(kp0), "=f"(kn0), "=f"(kp1), "=f"(kn1)
+              : "r"(kw[v]), "r"(p.dare_T16), "f"(d0), "r"(kw[v + 1]), "f"(d1));
         } else {
           kp0 = d0 >= thr ? 1.0f : 0.0f;
           kp1 = d1 >= thr ? 1.0f : 0.0f;

@@ -150,6 +150,23 @@ void set_error(const std::string& msg);
 void set_static_error(const char* msg);
 mp_status cuda_fail(cudaError_t e, const char* what);
 
+// device-time ranges of the calls (trace.cu): trace_begin records the start of a range on
+// st and returns its ticket, or -1 while no trace is recording (or it is full); trace_end
+// records the end on the stream that ran the range's work
+int trace_begin(uint32_t kind, uint32_t segment, uint32_t stream_kind, cudaStream_t st);
+void trace_end(int ticket, cudaStream_t st);
+struct TraceScope {
+  int ticket;
+  cudaStream_t st;
+  TraceScope(uint32_t kind, cudaStream_t s) : ticket(trace_begin(kind, 0, 0, s)), st(s) {}
+  ~TraceScope() { trace_end(ticket, st); }
+};
+// host-side NVTX range of an entry point, for the lifetime of the object
+struct NvtxScope {
+  explicit NvtxScope(const char* name);
+  ~NvtxScope();
+};
+
 // ---- index (index.cu) -------------------------------------------------------------------
 struct IndexLaunch {
   mp_dtype dtype;

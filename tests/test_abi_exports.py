@@ -150,3 +150,18 @@ def test_fault_injection_hook_arms_and_refuses_unknown_kinds_without_gpu():
         mp.mp_debug_inject_fault(0, 1)
     assert e.value.status == -1
     mp.mp_debug_stall_pipeline(0)
+
+
+def test_trace_refuses_bad_arguments_and_stops_empty_without_gpu():
+    """the trace API checks its arguments on the host: capacity 0 or above 2^20 is refused,
+    and a stop without a start holds no ranges (neither makes a CUDA call)"""
+    import paper_2605_29489_gb300 as mp
+
+    for cap in (0, (1 << 20) + 1):
+        with pytest.raises(mp.MergePipeError) as e:
+            mp.mp_trace_start(cap)
+        assert e.value.status == -1
+    assert mp.mp_trace_stop() == []
+    with pytest.raises(mp.MergePipeError) as e:
+        mp._check(mp.lib().mp_trace_read(None, 1))
+    assert e.value.status == -1

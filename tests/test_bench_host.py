@@ -147,3 +147,16 @@ def test_clock_sampler_summary():
     assert cs.stop()["reasons"] == ["hw_slowdown", "sw_thermal_slowdown"]
     cs = bench.ClockSampler(0)             # nvidia-smi could not be started: no record
     assert cs.stop() is None
+
+
+def test_interval_union_and_overlap_of_the_host_timeline():
+    """the timeline's busy time is the length of a union of intervals (overlaps counted
+    once, gaps not at all), and a kernel's time under gathers is its intersection with it"""
+    import bench
+
+    iv = [(0.0, 2.0), (1.0, 3.0), (5.0, 6.0), (5.5, 5.7), (8.0, 8.0)]
+    assert bench._union_ms(iv) == 4.0
+    assert bench._union_ms([]) == 0.0
+    assert bench._overlap_ms(2.5, 5.5, iv) == 1.0   # [2.5, 3] and [5, 5.5]
+    assert bench._overlap_ms(3.0, 5.0, iv) == 0.0
+    assert bench._overlap_ms(-1.0, 10.0, iv) == bench._union_ms(iv)
