@@ -509,8 +509,12 @@ def native(args, rank, world, local_rank):
         h2d_stream = torch.cuda.Stream() if n_sets > 1 else stream
 
         # each budget's output goes back on a copy stream while the next budget is planned and
-        # merged (separate output buffers); with a shared output buffer the copies stay in order
+        # merged (separate output buffers); with a shared output buffer the copies stay in order.
+        # A budget's merge waits only for the previous step's copy of its own output buffer.
         copy_stream = torch.cuda.Stream() if not shared_out else stream
+        out_copied = [E() for _ in Bs]  # the previous step's copy of output k has read it
+        for ev in out_copied:
+            ev.record(copy_stream)
 
         def issue_inputs(j):
             h2d_stream.wait_event(in_free[j])
@@ -526,14 +530,15 @@ def native(args, rank, world, local_rank):
             hs = []
             idx = make_index(mf_d)
             hs.append(idx)
-            stream.wait_stream(copy_stream)  # the previous step's copies have read the outputs
             for k, B in enumerate(Bs):
                 plan = mp.mp_plan(idx, gop, B, stream)
                 out = outs[0 if shared_out else k]
+                stream.wait_event(out_copied[0 if shared_out else k])
                 man = mp.mp_merge(mf_d, idx, plan, out, stream)
                 copy_stream.wait_stream(stream)
                 with torch.cuda.stream(copy_stream):
                     outs_h[k].copy_(out, non_blocking=True)
+                out_copied[0 if shared_out else k].record(copy_stream)
                 hs += [plan, man]
             in_free[j].record(stream)
             return hs

@@ -368,12 +368,17 @@ struct HostPipe {
 
 }  // namespace
 
-cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs) {
+// One walk over the segments: every expert block of a segment is brought into HBM staging by
+// the gather kernel (on a side stream, one segment ahead), then `stage` enqueues the
+// segment's catalog kernels on the caller's stream.  gate: when set, the gathers copy
+// nothing unless *gate != 0 (the fallback walk of the windowed TIES catalog).
+template <typename Stage>
+cudaError_t walk_segments(const IndexLaunch& p, const mp_index_s* ix, cudaStream_t cs, const uint32_t* gate,
+                          Stage stage) {
   uint64_t span = 0;
   const std::vector<Segment> segs = make_segments(ix->h_blk_off, ix->h_blk_len, span);
-  const uint32_t es = ix->g.elem_size;
   HostPipe hp;
-  cudaError_t e = hp.init(cs, p.K, span, es);
+  cudaError_t e = hp.init(cs, p.K, span, ix->g.elem_size);
   for (size_t s = 0; s < segs.size() && e == cudaSuccess; ++s) {
     const int b = (int)(s & 1);
     const Segment& g = segs[s];
@@ -386,7 +391,7 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     GatherLaunch gl;
     memset(&gl, 0, sizeof(gl));
     gl.K = p.K;
-    gl.elem_size = es;
+    gl.elem_size = ix->g.elem_size;
     gl.b_begin = g.b0;
     gl.b_end = g.b1;
     gl.origin = g.e0;
@@ -394,6 +399,7 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     gl.blk_len = p.blk_len;
     gl.mask = nullptr;
     gl.src = p.experts;
+    gl.gate = gate;
     for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
     if (inject_fault(MP_FAULT_GATHER)) {
       e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
@@ -411,19 +417,43 @@ cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs
     ps.defer_ties_select = 1;
     for (uint32_t i = 0; i < p.K; ++i) ps.experts.p[i] = hp.buf(b, i);
     const int tk = trace_begin(MP_TRACE_SEGMENT, (uint32_t)s, 0, cs);
-    e = launch_index(ps, cs);
+    e = stage(ps);
     trace_end(tk, cs);
     if (e != cudaSuccess) break;
     e = hp.main_release(b);
   }
-  if (e == cudaSuccess && p.coarse) {
-    // the second level of the TIES select reads the host experts directly (fewer blocks)
+  hp.finish();
+  return e;
+}
+
+cudaError_t index_host_pool(IndexLaunch p, const mp_index_s* ix, cudaStream_t cs) {
+  cudaError_t e;
+  if (p.wlo) {
+    // the windowed TIES catalog: the sample reads the host experts in place (32 vectors per
+    // block), one walk counts every pair's window, the finish marks the pairs whose threshold
+    // left it; a second walk, whose gathers and kernels do nothing unless some pair was
+    // marked, bins the marked groups coarsely for the two-level select
+    if ((e = launch_ties_window_begin(p, cs)) != cudaSuccess) return e;
+    if ((e = walk_segments(p, ix, cs, nullptr, [&](const IndexLaunch& ps) { return launch_index_pass(ps, true, cs); })) !=
+        cudaSuccess)
+      return e;
+    if ((e = launch_ties_window_end(p, cs)) != cudaSuccess) return e;
+    if ((e = walk_segments(p, ix, cs, p.miss, [&](const IndexLaunch& ps) { return launch_index_pass(ps, false, cs); })) !=
+        cudaSuccess)
+      return e;
+  } else {
+    if ((e = walk_segments(p, ix, cs, nullptr, [&](const IndexLaunch& ps) { return launch_index(ps, cs); })) !=
+        cudaSuccess)
+      return e;
+  }
+  if (p.coarse) {
+    // the second level of the TIES select reads the host experts directly (fewer blocks; in
+    // the windowed catalog only for the marked pairs)
     p.b_begin = 0;
     p.b_end = p.n_blocks;
     p.expert_origin = 0;
     e = launch_ties_finish(p, cs);
   }
-  hp.finish();
   return e;
 }
 
@@ -659,7 +689,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   size_t o_coarse = 0, o_fine = 0, o_kth = 0, o_est = 0, o_rank = 0;
   size_t o_wfine = 0, o_wabove = 0, o_wlo = 0, o_gmiss = 0, o_miss = 0, o_wend = 0;
   // device-resident TIES (not after masking) takes its thresholds from predicted windows
-  const bool windowed = ties && op->kind == MP_OP_TIES && family->experts_location == 0;
+  const bool windowed = ties && op->kind == MP_OP_TIES;
   if (ties) {
     o_coarse = slot(KG * 256 * 8);
     o_fine = slot(KG * 128 * 8);

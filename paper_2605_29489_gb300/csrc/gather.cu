@@ -17,6 +17,7 @@ constexpr int kUnroll = 4;
 __global__ void __launch_bounds__(kThreads) gather_kernel(const GatherLaunch g) {
   const uint64_t b = g.b_begin + blockIdx.x;
   if (b >= g.b_end) return;
+  if (g.gate && *g.gate == 0u) return;  // a gated launch with nothing to bring in
   const uint32_t all = g.K >= 32 ? 0xFFFFFFFFu : ((1u << g.K) - 1u);
   const uint32_t m = g.mask ? g.mask[b] : all;
   if (m == 0u) return;

@@ -1061,6 +1061,31 @@ cudaError_t launch_t(const IndexLaunch& p, cudaStream_t st) {
   return ties_finish_t<BF16, KG>(p, st);
 }
 
+template <bool BF16, int KG>
+cudaError_t window_begin_t(const IndexLaunch& p, cudaStream_t st) {
+  const uint32_t G = (p.K + KG - 1) / KG;
+  const uint64_t nsel = (uint64_t)p.K * p.n_groups;
+  if (p.n_samp_spans == 0 || nsel == 0) return cudaSuccess;
+  ties_sample_kernel<BF16, KG><<<dim3(p.n_samp_spans, G), 256, 0, st>>>(p);
+  ties_window_select<<<(unsigned)((nsel + 127) / 128), 128, 0, st>>>(p);
+  count_launches(2);
+  return cudaGetLastError();
+}
+
+template <bool BF16, int KG>
+cudaError_t pass_t(const IndexLaunch& p, bool window, cudaStream_t st) {
+  const uint32_t G = (p.K + KG - 1) / KG;
+  const uint64_t n_items = (p.b_end - p.b_begin) * G;
+  if (n_items == 0) return cudaSuccess;
+  if (n_items > 0x7FFFFFFFull) return cudaErrorInvalidValue;
+  int dev = 0, sms = 0;
+  cudaError_t e;
+  if ((e = cudaGetDevice(&dev)) != cudaSuccess) return e;
+  if ((e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev)) != cudaSuccess) return e;
+  return window ? launch_pass<BF16, KG, kBinWindow>(p, G, n_items, sms, st)
+                : launch_pass<BF16, KG, kBinCoarse>(p, G, n_items, sms, st);
+}
+
 template <bool BF16>
 cudaError_t launch_dtype(const IndexLaunch& p, cudaStream_t st) {
   if (p.K <= 1) return launch_t<BF16, 1>(p, st);
@@ -1073,6 +1098,33 @@ cudaError_t launch_dtype(const IndexLaunch& p, cudaStream_t st) {
 
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st) {
   return p.dtype == MP_BF16 ? launch_dtype<true>(p, st) : launch_dtype<false>(p, st);
+}
+
+cudaError_t launch_ties_window_begin(const IndexLaunch& p, cudaStream_t st) {
+  if (!p.wlo || !p.coarse) return cudaErrorInvalidValue;
+  const bool bf = p.dtype == MP_BF16;
+  if (p.K <= 1) return bf ? window_begin_t<true, 1>(p, st) : window_begin_t<false, 1>(p, st);
+  if (p.K <= 2) return bf ? window_begin_t<true, 2>(p, st) : window_begin_t<false, 2>(p, st);
+  if (p.K <= 4) return bf ? window_begin_t<true, 4>(p, st) : window_begin_t<false, 4>(p, st);
+  return bf ? window_begin_t<true, 8>(p, st) : window_begin_t<false, 8>(p, st);
+}
+
+cudaError_t launch_index_pass(const IndexLaunch& p, bool window, cudaStream_t st) {
+  if (!p.wlo || !p.coarse) return cudaErrorInvalidValue;
+  const bool bf = p.dtype == MP_BF16;
+  if (p.K <= 1) return bf ? pass_t<true, 1>(p, window, st) : pass_t<false, 1>(p, window, st);
+  if (p.K <= 2) return bf ? pass_t<true, 2>(p, window, st) : pass_t<false, 2>(p, window, st);
+  if (p.K <= 4) return bf ? pass_t<true, 4>(p, window, st) : pass_t<false, 4>(p, window, st);
+  return bf ? pass_t<true, 8>(p, window, st) : pass_t<false, 8>(p, window, st);
+}
+
+cudaError_t launch_ties_window_end(const IndexLaunch& p, cudaStream_t st) {
+  if (!p.wlo || !p.coarse) return cudaErrorInvalidValue;
+  const uint64_t nsel = (uint64_t)p.K * p.n_groups;
+  if (nsel == 0) return cudaSuccess;
+  ties_window_finish<<<(unsigned)((nsel + 127) / 128), 128, 0, st>>>(p);
+  count_launches(1);
+  return cudaGetLastError();
 }
 
 cudaError_t launch_ties_masked(const IndexLaunch& p, cudaStream_t st) {

@@ -221,6 +221,14 @@ struct IndexLaunch {
 };
 cudaError_t launch_index(const IndexLaunch& p, cudaStream_t st);
 cudaError_t launch_ties_finish(const IndexLaunch& p, cudaStream_t st);
+// the windowed TIES catalog in stages, for a host-resident pool walked in segments: the
+// sample and window select over the whole family (experts read in place over the host
+// mapping); one pass over blocks [b_begin, b_end) of staged experts with window bins, or with
+// coarse bins for the pairs the window finish marked (a launch that returns at once when
+// none is); the window finish
+cudaError_t launch_ties_window_begin(const IndexLaunch& p, cudaStream_t st);
+cudaError_t launch_index_pass(const IndexLaunch& p, bool window, cudaStream_t st);
+cudaError_t launch_ties_window_end(const IndexLaunch& p, cudaStream_t st);
 // the TIES_MASKED threshold of a plan: coarse bins summed from the per-unit histograms of
 // the selected blocks (zero entries for the others), then the select, fine pass and select
 // of launch_ties_finish restricted to the selected blocks (p.mask)
@@ -318,6 +326,7 @@ struct GatherLaunch {
   ExpertPtrs src;         // device views of the host experts
   ExpertPtrs dst;         // staging buffers
   unsigned long long* gathered;  // bytes copied, accumulated (may be NULL)
+  const uint32_t* gate;          // when set, the launch copies nothing unless *gate != 0
 };
 cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st);
 

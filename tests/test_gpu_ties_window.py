@@ -49,13 +49,16 @@ def _with_deltas(fam, scale_of_block, seed):
     return base, experts
 
 
-def test_sample_that_misses_the_threshold_falls_back_to_the_two_level_select():
+@pytest.mark.parametrize("host_experts", [False, True], ids=["device", "host_pool"])
+def test_sample_that_misses_the_threshold_falls_back_to_the_two_level_select(host_experts):
     """The sample reads 32 vectors of every block longer than 4096 elements and every vector
     of a shorter one, so short blocks weigh far more in it.  Here the short blocks (a
     tensor's tail, small tensors) carry deltas about 10^4 times larger than the full
     blocks: the sample predicts a window among the large keys while the threshold lies
     among the small ones — for tensor 0 with per-tensor trim groups, and for the single
-    group of trim scope 1.  The two-level select must give the oracle's thresholds."""
+    group of trim scope 1.  The two-level select must give the oracle's thresholds — also
+    with the experts in pinned host memory, where the sample reads them in place and the
+    fallback walk's gathers run only because a pair was marked."""
     E = 65536
     shapes = [2 * E + 4000, 16 * E] + [4096] * 20 + [70001]
     fam = synth.custom(shapes, dtype=synth.BF16, block_elems=E, K=3, active_frac=0.5, name="window-miss")
@@ -70,9 +73,9 @@ def test_sample_that_misses_the_threshold_falls_back_to_the_two_level_select():
         return 1e-3 * (1 + i)
 
     base, experts = _with_deltas(fam, scale, seed=11)
-    run_case(fam, base, experts, ("ties", "ties1"), [1.0, 0.5, 0.25])
+    run_case(fam, base, experts, ("ties", "ties1"), [1.0, 0.5, 0.25], host_experts=host_experts)
     # the threshold of tensor 0 lies among its small deltas, far below the sampled ones
-    mf, _, _ = upload(fam, base, experts)
+    mf, _, _ = upload(fam, base, experts, host_experts)
     idx = mp.mp_index_blocks(mf, mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2))
     tau = mp.mp_index_stats(idx)[3]
     key_mid = int(_bf16_bits(np.float32([1e-2]))[0]) & 0x7FFF
@@ -80,14 +83,15 @@ def test_sample_that_misses_the_threshold_falls_back_to_the_two_level_select():
     idx.free()
 
 
+@pytest.mark.parametrize("host_experts", [False, True], ids=["device", "host_pool"])
 @pytest.mark.parametrize("density", [0.5, 0.9, 1.0])
-def test_threshold_at_the_key_of_an_exact_zero(density):
+def test_threshold_at_the_key_of_an_exact_zero(density, host_experts):
     """nine blocks in ten have no delta at all: from density 0.5 on, the k-th largest key
     is the key 0 of an exact zero, reached through the window at the bottom of the keys"""
     fam = synth.custom([64 * E, 5 * E + 3], dtype=synth.BF16, block_elems=E, K=3, active_frac=0.5,
                        name="window-zero")
     base, experts = _with_deltas(fam, lambda i, b: 1e-2 if b % 10 == 3 else 0.0, seed=12)
-    mf, _, _ = upload(fam, base, experts)
+    mf, _, _ = upload(fam, base, experts, host_experts)
     gop = mp.make_op(mp.MP_OP_TIES, lam=1.0, density=density)
     idx = mp.mp_index_blocks(mf, gop)
     tau = mp.mp_index_stats(idx)[3]
