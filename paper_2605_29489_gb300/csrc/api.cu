@@ -45,14 +45,18 @@ cudaError_t malloc_async(void** p, size_t bytes, cudaStream_t st) {
 std::atomic<uint64_t> g_next_id{1};
 std::atomic<uint64_t> g_launches{0};
 
-// pinned host slots for the small results copied back per handle, in two size classes
-// (256 bytes: plan summaries; 32 KiB: manifest counters), recycled through free lists
+// pinned host slots for the small results copied back per handle and the tables a call
+// uploads, in three size classes (256 bytes: plan summaries; 32 KiB: manifest counters and
+// small tables; 8 MiB: block tables), recycled through free lists.  Kernels read and write
+// them through the host mapping, so no copy engine is involved.
 std::mutex g_pin_mu;
-std::vector<void*> g_pin_free[2];
-constexpr size_t kPinSlot[2] = {256, 32768};
-constexpr size_t kPinChunk = 1 << 20;
+std::vector<void*> g_pin_free[3];
+constexpr size_t kPinSlot[3] = {256, 32768, 8u << 20};
+constexpr size_t kPinChunk[3] = {1u << 20, 1u << 20, 8u << 20};
 
-int pin_class(size_t bytes) { return bytes <= kPinSlot[0] ? 0 : (bytes <= kPinSlot[1] ? 1 : -1); }
+int pin_class(size_t bytes) {
+  return bytes <= kPinSlot[0] ? 0 : (bytes <= kPinSlot[1] ? 1 : (bytes <= kPinSlot[2] ? 2 : -1));
+}
 
 void* pin_get(size_t bytes) {
   int c = pin_class(bytes);
@@ -60,8 +64,12 @@ void* pin_get(size_t bytes) {
   std::lock_guard<std::mutex> lk(g_pin_mu);
   if (g_pin_free[c].empty()) {
     void* chunk = nullptr;
-    if (cudaHostAlloc(&chunk, kPinChunk, cudaHostAllocDefault) != cudaSuccess) return nullptr;
-    for (size_t k = 0; k < kPinChunk / kPinSlot[c]; ++k) g_pin_free[c].push_back(static_cast<char*>(chunk) + kPinSlot[c] * k);
+    if (cudaHostAlloc(&chunk, kPinChunk[c], cudaHostAllocDefault) != cudaSuccess) {
+      cudaGetLastError();
+      return nullptr;
+    }
+    for (size_t k = 0; k < kPinChunk[c] / kPinSlot[c]; ++k)
+      g_pin_free[c].push_back(static_cast<char*>(chunk) + kPinSlot[c] * k);
   }
   void* p = g_pin_free[c].back();
   g_pin_free[c].pop_back();
@@ -76,6 +84,23 @@ void pin_put(void* p, size_t bytes) {
 }
 
 size_t align_up(size_t v) { return (v + 255) & ~(size_t)255; }
+
+// Host data into the index's device memory by kernel: staged in a pinned slot that the handle
+// keeps until mp_free, read by launch_copy over the host mapping.  Data larger than the
+// largest slot goes by cudaMemcpyAsync.
+cudaError_t upload(mp_index_s* ix, void* dst, const void* src, size_t bytes, cudaStream_t cs) {
+  if (bytes == 0) return cudaSuccess;
+  void* h = pin_get(bytes);
+  if (!h) return cudaMemcpyAsync(dst, src, bytes, cudaMemcpyHostToDevice, cs);
+  memcpy(h, src, bytes);
+  ix->pinned.push_back({h, bytes});
+  return launch_copy(dst, h, bytes, cs);
+}
+
+void release_pinned(mp_index_s* ix) {
+  for (auto& q : ix->pinned) pin_put(q.first, q.second);
+  ix->pinned.clear();
+}
 
 mp_status fail(mp_status st, const std::string& msg) {
   g_static_error = nullptr;
@@ -575,14 +600,19 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
   ix->d_unit_hist = masked ? (uint32_t*)(m + o_uh) : nullptr;
   cudaError_t e = cudaSuccess;
   const char* what = "block table copy";
-  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_off, h_off.data(), nb * 8, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_len, h_len.data(), nb * 4, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_group, h_grp.data(), nb * 4, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) e = cudaMemcpyAsync(ix->d_blk_tensor, h_tens.data(), nb * 4, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess)
-    e = cudaMemcpyAsync(ix->d_t_blk0, h_tb0.data(), ((size_t)g.n_tensors + 1) * 4, cudaMemcpyHostToDevice, cs);
-  if (e == cudaSuccess) what = "memset", e = cudaMemsetAsync(ix->d_err, 0, 16, cs);
-  if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_tau, 0, KG * 4, cs);
+  {
+    // the five table arrays are consecutive in the allocation: one staged upload
+    const size_t t_end = o_tb0 + ((size_t)g.n_tensors + 1) * 4;
+    std::vector<char> tab(t_end, 0);
+    memcpy(tab.data() + o_off, h_off.data(), nb * 8);
+    memcpy(tab.data() + o_len, h_len.data(), nb * 4);
+    memcpy(tab.data() + o_grp, h_grp.data(), nb * 4);
+    memcpy(tab.data() + o_tens, h_tens.data(), nb * 4);
+    memcpy(tab.data() + o_tb0, h_tb0.data(), ((size_t)g.n_tensors + 1) * 4);
+    e = upload(ix, m, tab.data(), t_end, cs);
+  }
+  if (e == cudaSuccess) what = "fill", e = launch_fill(ix->d_err, 0, 16, cs);
+  if (e == cudaSuccess) e = launch_fill(ix->d_tau, 0, KG * 4, cs);
   if (e != cudaSuccess) {
     mp_status r = cuda_fail(e, what);
     discard_index(ix, cs);
@@ -619,6 +649,7 @@ mp_status alloc_hashes(mp_index_s* ix, cudaStream_t cs) {
 void discard_index(mp_index_s* ix, cudaStream_t cs) {
   cudaStreamSynchronize(cs);
   cudaGetLastError();
+  release_pinned(ix);
   dev_free(ix->hash_mem);
   dev_free(ix->order_mem);
   dev_free(ix->mem);
@@ -756,10 +787,9 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     p.rank = (unsigned long long*)(m + o_rank);
     p.tau = ix->d_tau;
     p.unit_hist = ix->d_unit_hist;
-    if ((e = cudaMemsetAsync(p.coarse, 0, KG * 256 * 8, cs)) != cudaSuccess) return bail(e, "memset");
-    if ((e = cudaMemsetAsync(p.fine, 0, KG * 128 * 8, cs)) != cudaSuccess) return bail(e, "memset");
-    if ((e = cudaMemcpyAsync((void*)p.kth, h_kth.data(), n_groups * 8, cudaMemcpyHostToDevice, cs)) != cudaSuccess)
-      return bail(e, "k copy");
+    if ((e = launch_fill(p.coarse, 0, KG * 256 * 8, cs)) != cudaSuccess) return bail(e, "fill");
+    if ((e = launch_fill(p.fine, 0, KG * 128 * 8, cs)) != cudaSuccess) return bail(e, "fill");
+    if ((e = upload(ix, (void*)p.kth, h_kth.data(), n_groups * 8, cs)) != cudaSuccess) return bail(e, "k copy");
   }
   if (windowed) {
     p.density = op->density;
@@ -773,9 +803,8 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
     p.scnt = (unsigned long long*)(m + o_scnt);
     p.samp_span = (const uint2*)(m + o_spans);
     p.n_samp_spans = (uint32_t)(h_spans.size() / 2);
-    if ((e = cudaMemsetAsync(m + o_wfine, 0, o_wend - o_wfine, cs)) != cudaSuccess) return bail(e, "memset");
-    if ((e = cudaMemcpyAsync(m + o_spans, h_spans.data(), h_spans.size() * 4, cudaMemcpyHostToDevice, cs)) !=
-        cudaSuccess)
+    if ((e = launch_fill(m + o_wfine, 0, o_wend - o_wfine, cs)) != cudaSuccess) return bail(e, "fill");
+    if ((e = upload(ix, m + o_spans, h_spans.data(), h_spans.size() * 4, cs)) != cudaSuccess)
       return bail(e, "span copy");
   }
   p.b_begin = 0;
@@ -995,7 +1024,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
         p.cache_order_out = ixw->d_order_cache;
         p.cache_q_out = ixw->d_order_q;
         // an invalid count until the filling plan completes its sort
-        if ((e = cudaMemsetAsync(ixw->d_order_q, 0xFF, 8, cs)) != cudaSuccess) return bail(e, "memset");
+        if ((e = launch_fill(ixw->d_order_q, 0xFF, 8, cs)) != cudaSuccess) return bail(e, "fill");
         fill = true;
       }
     }
@@ -1009,7 +1038,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   }
   if ((e = cudaFreeAsync(scratch.ptr, cs)) != cudaSuccess) return bail(e, "free scratch");
   scratch.ptr = nullptr;
-  if ((e = cudaMemcpyAsync(pl->h_summary, pl->d_summary, 64, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)
+  if ((e = launch_copy(pl->h_summary, pl->d_summary, 64, cs)) != cudaSuccess)
     return bail(e, "summary copy");
   if ((e = cudaEventCreateWithFlags(&pl->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
   if ((e = cudaEventRecord(pl->done, cs)) != cudaSuccess) return bail(e, "event record");
@@ -1109,7 +1138,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   cudaError_t e;
   if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
   if ((e = cudaStreamWaitEvent(cs, plan->done, 0)) != cudaSuccess) return bail(e, "stream wait");
-  if ((e = cudaMemsetAsync(mf->mem.ptr, 0, back_bytes, cs)) != cudaSuccess) return bail(e, "memset");
+  if ((e = launch_fill(mf->mem.ptr, 0, back_bytes, cs)) != cudaSuccess) return bail(e, "fill");
   uint32_t* masked_tau = nullptr;
   if (masked) {
     // TIES after masking: the threshold of the zero-completed masked deltas of this plan
@@ -1202,9 +1231,9 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
       return bail(cudaErrorInvalidValue, "an index of a host-resident pool is needed for a host-pool merge");
     if ((e = merge_host_pool(p, index, cs)) != cudaSuccess) return bail(e, "merge (host pool)");
   }
-  if ((e = cudaMemcpyAsync(d_sum_copy, plan->d_summary, 64, cudaMemcpyDeviceToDevice, cs)) != cudaSuccess)
+  if ((e = launch_copy(d_sum_copy, plan->d_summary, 64, cs)) != cudaSuccess)
     return bail(e, "summary copy");
-  if ((e = cudaMemcpyAsync(mf->h_realized, mf->mem.ptr, back_bytes, cudaMemcpyDeviceToHost, cs)) != cudaSuccess)
+  if ((e = launch_copy(mf->h_realized, mf->mem.ptr, back_bytes, cs)) != cudaSuccess)
     return bail(e, "manifest copy");
   if ((e = cudaEventCreateWithFlags(&mf->done, cudaEventDisableTiming)) != cudaSuccess) return bail(e, "event");
   if ((e = cudaEventRecord(mf->done, cs)) != cudaSuccess) return bail(e, "event record");
@@ -1236,6 +1265,7 @@ void mp_free(void* handle) {
     dev_free(ix->hash_mem);
     dev_free(ix->order_mem);
     dev_free(ix->mem);
+    release_pinned(ix);
     delete ix->order_mu;
     ix->magic = 0;
     delete ix;

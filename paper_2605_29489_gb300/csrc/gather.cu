@@ -6,6 +6,12 @@
 // needs no host synchronisation; unselected expert blocks are never touched (the realized
 // reads stay within the plan, Prop. 1).  One CTA per block; four 16-byte loads in flight
 // per thread.
+//
+// The small copies and fills of the calls (block tables in, summaries and manifests out,
+// zeroed counters) are kernels here too: a copy engine serves its direction in order, so a
+// small cudaMemcpyAsync queued behind a caller's multi-gigabyte transfer on another stream
+// would wait for all of it.  A host buffer these kernels read or write is pinned memory,
+// which the device reaches through its host mapping.
 #include "mp_internal.cuh"
 
 namespace mp {
@@ -47,7 +53,52 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const GatherLaunch g) 
   if (threadIdx.x == 0 && g.gathered) atomicAdd(g.gathered, copied);
 }
 
+// small copies and fills on the caller's stream, by kernel: 16-byte vectors where both
+// addresses allow, bytes at the ends
+__global__ void __launch_bounds__(kThreads) copy_kernel(char* dst, const char* src, size_t bytes) {
+  const size_t tid = (size_t)blockIdx.x * kThreads + threadIdx.x, nt = (size_t)gridDim.x * kThreads;
+  if (((reinterpret_cast<uintptr_t>(dst) | reinterpret_cast<uintptr_t>(src)) & 15u) == 0) {
+    const size_t nv = bytes / 16u;
+    for (size_t v = tid; v < nv; v += nt) reinterpret_cast<uint4*>(dst)[v] = reinterpret_cast<const uint4*>(src)[v];
+    for (size_t i = nv * 16u + tid; i < bytes; i += nt) dst[i] = src[i];
+  } else {
+    for (size_t i = tid; i < bytes; i += nt) dst[i] = src[i];
+  }
+}
+
+__global__ void __launch_bounds__(kThreads) fill_kernel(char* dst, uint32_t v, size_t bytes) {
+  const size_t tid = (size_t)blockIdx.x * kThreads + threadIdx.x, nt = (size_t)gridDim.x * kThreads;
+  const uint32_t w = (v & 0xFFu) * 0x01010101u;
+  if ((reinterpret_cast<uintptr_t>(dst) & 15u) == 0) {
+    const size_t nv = bytes / 16u;
+    for (size_t k = tid; k < nv; k += nt) reinterpret_cast<uint4*>(dst)[k] = make_uint4(w, w, w, w);
+    for (size_t i = nv * 16u + tid; i < bytes; i += nt) dst[i] = (char)v;
+  } else {
+    for (size_t i = tid; i < bytes; i += nt) dst[i] = (char)v;
+  }
+}
+
+unsigned small_grid(size_t bytes) {
+  const size_t per = (size_t)kThreads * 16u * 4u;  // four vectors per thread
+  const size_t g = (bytes + per - 1) / per;
+  return (unsigned)(g < 1 ? 1 : (g > 1024 ? 1024 : g));
+}
+
 }  // namespace
+
+cudaError_t launch_copy(void* dst, const void* src, size_t bytes, cudaStream_t st) {
+  if (bytes == 0) return cudaSuccess;
+  copy_kernel<<<small_grid(bytes), kThreads, 0, st>>>(static_cast<char*>(dst), static_cast<const char*>(src), bytes);
+  count_launches(1);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_fill(void* dst, uint32_t byte_value, size_t bytes, cudaStream_t st) {
+  if (bytes == 0) return cudaSuccess;
+  fill_kernel<<<small_grid(bytes), kThreads, 0, st>>>(static_cast<char*>(dst), byte_value, bytes);
+  count_launches(1);
+  return cudaGetLastError();
+}
 
 cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st) {
   const uint64_t nb = g.b_end - g.b_begin;

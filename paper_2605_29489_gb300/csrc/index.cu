@@ -1021,7 +1021,7 @@ cudaError_t launch_pass(const IndexLaunch& p, uint32_t G, uint64_t n_items, int 
   uint64_t grid = (uint64_t)sms * IxGeo<ties, KG>::kCtasPerSm;
   if (grid > n_items) grid = n_items;
   cudaError_t e;
-  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if ((e = launch_fill(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
   auto k = index_tma_kernel<BF16, KG, BM>;
   if ((e = cudaFuncSetAttribute(k, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem)) != cudaSuccess) return e;
   k<<<(unsigned)grid, kIxThreads, smem, st>>>(p, G, n_items, p.work);

@@ -1058,7 +1058,7 @@ cudaError_t launch_chunk(const MergeLaunch& p, cudaStream_t st) {
     return e;
   uint64_t grid = (uint64_t)sms * TcGeo<OPC, KC>::kCtasPerSm;
   if (grid > n_chunks) grid = n_chunks;
-  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if ((e = launch_fill(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
   kern<<<(unsigned)grid, TcGeo<OPC, KC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
   count_launches(1);
   return cudaGetLastError();
@@ -1081,7 +1081,7 @@ cudaError_t launch_op(const MergeLaunch& p, cudaStream_t st) {
     return e;
   uint64_t grid = (uint64_t)sms * Geo<OPC>::kCtasPerSm;
   if (grid > n_chunks) grid = n_chunks;
-  if ((e = cudaMemsetAsync(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if ((e = launch_fill(p.work, 0, sizeof(unsigned long long), st)) != cudaSuccess) return e;
   merge_tma_kernel<BF16, OPC><<<(unsigned)grid, Geo<OPC>::kThreads, smem, st>>>(p, cpb, n_chunks, p.work);
   count_launches(1);
   return cudaGetLastError();

@@ -7,6 +7,7 @@
 
 #include <string>
 #include <mutex>
+#include <utility>
 #include <vector>
 
 #include "mergepipe.h"
@@ -91,6 +92,7 @@ struct mp_index_s {
   uint32_t* d_tau;         // [K][n_groups] (TIES only)
   uint32_t* d_err;         // error word
   cudaEvent_t done;
+  std::vector<std::pair<void*, size_t>> pinned;  // pinned staging of the uploads (released by mp_free)
   std::vector<uint64_t> h_blk_off;  // host copy of the block table (segments of a host pool)
   std::vector<uint32_t> h_blk_len;
 };
@@ -329,6 +331,9 @@ struct GatherLaunch {
   const uint32_t* gate;          // when set, the launch copies nothing unless *gate != 0
 };
 cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st);
+// copies and fills by kernel on st (no copy engine); host buffers must be pinned memory
+cudaError_t launch_copy(void* dst, const void* src, size_t bytes, cudaStream_t st);
+cudaError_t launch_fill(void* dst, uint32_t byte_value, size_t bytes, cudaStream_t st);
 
 // ---- block content hashes (hash.cu) --------------------------------------------------------
 // catalog mode (validate = 0): hash every block of the base and of each expert into

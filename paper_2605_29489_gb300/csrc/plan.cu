@@ -630,9 +630,9 @@ cudaError_t launch_plan(const PlanLaunch& p, void* scratch, cudaStream_t st) {
   if (grid > cap) grid = cap;
   if (grid > kMaxGrid) grid = kMaxGrid;
   if (grid < 1) grid = 1;
-  if ((e = cudaMemsetAsync(s.x, 0, X_COUNT * sizeof(unsigned long long), st)) != cudaSuccess) return e;
-  if (n_pairs && (e = cudaMemsetAsync(s.pair_flag, 0, n_pairs * 4, st)) != cudaSuccess) return e;
-  if (n_pairs && (e = cudaMemsetAsync(s.sel_bits, 0, (size_t)p.n_tensors * 4, st)) != cudaSuccess) return e;
+  if ((e = launch_fill(s.x, 0, X_COUNT * sizeof(unsigned long long), st)) != cudaSuccess) return e;
+  if (n_pairs && (e = launch_fill(s.pair_flag, 0, n_pairs * 4, st)) != cudaSuccess) return e;
+  if (n_pairs && (e = launch_fill(s.sel_bits, 0, (size_t)p.n_tensors * 4, st)) != cudaSuccess) return e;
   PlanLaunch pc = p;
   void* args[] = {&pc, &s};
   if ((e = cudaLaunchCooperativeKernel((const void*)plan_kernel, dim3((unsigned)grid), dim3(kPT), args, 0, st)) !=
