@@ -93,6 +93,14 @@ int main(void) {
   CHECK(mp_plan_noalloc(3, 6, 1, MP_BF16, w, NULL, (const float*)w, (const float*)w, w, NULL, w, NULL, 1000, w, w, s8,
                         NULL) == MP_ERR_INVALID_ARG);
 
+  /* the trace API checks its arguments on the host; a stop without a start holds nothing */
+  CHECK(mp_trace_start(0) == MP_ERR_INVALID_ARG);
+  CHECK(mp_trace_start((1u << 20) + 1u) == MP_ERR_INVALID_ARG);
+  u64 = 7;
+  CHECK(mp_trace_stop(&u64) == MP_OK && u64 == 0);
+  CHECK(mp_trace_read(NULL, 1) == MP_ERR_INVALID_ARG);
+  CHECK(mp_trace_read(NULL, 0) == MP_OK);
+
   /* NULL is a no-op for mp_free */
   mp_free(NULL);
   printf("fails=%d\n", fails);
