@@ -34,6 +34,8 @@
 // (bounded) for its own copies in flight and returns.
 #include <cuda_bf16.h>
 
+#include <type_traits>
+
 #include "mp_internal.cuh"
 #include "philox.cuh"
 #include "small_div.cuh"
@@ -994,23 +996,41 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
       const uint32_t cb = __float_as_uint(Cc[v]);
       cv = any ? ((pos ? cb : cb >> CB) & ((1u << CB) - 1u)) : 0u;
     };
-    if (fast) {  // uniform over the CTA: every nonzero numerator is >= 2^-100 in magnitude
-      // q = RN(num * y), then Markstein's correction q + RN(num - q c) * y, and the output
-      // fma(lambda, q, M_0), two elements per instruction
+    // q = RN(num * y), then Markstein's correction q + RN(num - q c) * y, and the output
+    // fma(lambda, q, M_0), two elements per instruction; `checked` also notes the numerators
+    // 0 < |num| < 2^-100, which then take the IEEE division under one warp vote
+    auto finalise = [&](auto checked) {
+      bool exact = false;
 #pragma unroll
       for (int v = 0; v < V; v += 2) {
         float a0, a1, q0, q1, r0, r1;
         uint32_t c0, c1;
         num_c(v, a0, c0);
         num_c(v + 1, a1, c1);
+        if constexpr (decltype(checked)::value)
+          exact = exact || div_small_needs_ieee(a0) || div_small_needs_ieee(a1);
         const float2 t0 = S.ntab[c0], t1 = S.ntab[c1];
         f2_mul(a0, a1, t0.y, t1.y, q0, q1);
         f2_fma(q0, q1, t0.x, t1.x, a0, a1, r0, r1);
         f2_fma(r0, r1, t0.y, t1.y, q0, q1, q0, q1);
         f2_fma(p.lambda, p.lambda, q0, q1, x0[v], x0[v + 1], y[v], y[v + 1]);
       }
+      if (decltype(checked)::value && __any_sync(0xFFFFFFFFu, exact)) {
+#pragma unroll
+        for (int v = 0; v < V; ++v) {
+          float a;
+          uint32_t cv;
+          num_c(v, a, cv);
+          if (div_small_needs_ieee(a)) y[v] = __fmaf_rn(p.lambda, __fdiv_rn(a, -S.ntab[cv].x), x0[v]);
+        }
+      }
+    };
+    if constexpr (OPC == OP_DTIES) {
+      finalise(std::true_type{});  // rescaled deltas may be tiny: always checked
+    } else if (fast) {             // uniform over the CTA: every nonzero numerator >= 2^-100
+      finalise(std::false_type{});
     } else {
-      // numerators 0 < |num| < 2^-100 take the IEEE division under one warp vote
+      // TIES chunks with a threshold below 2^-100 (rare): one element at a time
       bool exact = false;
 #pragma unroll
       for (int v = 0; v < V; ++v) {
