@@ -477,7 +477,23 @@ def native(args, rank, world, local_rank):
 
     # ---- e2e: pinned host inputs in, merged outputs back, inside the timed region ----
     e2e = None
+    # the end-to-end leg pins the inputs and the outputs in host memory on every rank: it runs
+    # only where each rank's share of the host's available memory holds them (with one output
+    # buffer shared by the budgets if four do not fit); the decision is the same on every rank
+    out_bufs = len(budgets)
     if not args.no_e2e and not host_pool:
+        share = host_mem_available() / max(1, int(os.environ.get("LOCAL_WORLD_SIZE", world)))
+        in_b, out_b = (fam.K + 1) * total * es, total * es
+        if in_b + out_bufs * out_b > 0.85 * share:
+            out_bufs = 1
+        fits = in_b + out_bufs * out_b <= 0.85 * share
+        # every rank must agree: the slowest rank's (largest) need decides
+        need = _max_over_ranks(0.0 if fits else 1.0, world)
+        if need > 0.0:
+            e2e = {"skipped": f"host memory: the inputs and outputs need {(in_b + out_b) / 1e9:.0f} GB pinned per "
+                              f"rank, {share / 1e9:.0f} GB is available per rank"}
+            out_bufs = 0
+    if not args.no_e2e and not host_pool and out_bufs > 0:
         def pinned_copy(t):
             h = torch.empty(t.shape, dtype=t.dtype, pin_memory=True)
             h.copy_(t)
@@ -485,7 +501,8 @@ def native(args, rank, world, local_rank):
 
         base_h = pinned_copy(base)
         experts_h = [pinned_copy(e) for e in experts]
-        outs_h = [torch.empty(outs[0].shape, dtype=outs[0].dtype, pin_memory=True) for _ in budgets]
+        outs_h = [torch.empty(outs[0].shape, dtype=outs[0].dtype, pin_memory=True) for _ in range(out_bufs)]
+        outs_h = [outs_h[min(k, out_bufs - 1)] for k in range(len(budgets))]  # one buffer: reused in order
         # the device-resident inputs of the timed leg are not needed any more: the end-to-end
         # leg brings its own copies in from the pinned host buffers
         shape, dt = base.shape, base.dtype
@@ -578,7 +595,7 @@ def native(args, rank, world, local_rank):
         e2e_ms = _max_over_ranks(e2e_ms, world)
         e2e = {"value": world * len(budgets) * N / (e2e_ms / 1e3), "unit": UNIT,
                "h2d_bytes_per_step": (fam.K + 1) * N * es, "d2h_bytes_per_step": len(budgets) * N * es,
-               "ms_per_step": e2e_ms, "input_sets": n_sets}
+               "ms_per_step": e2e_ms, "input_sets": n_sets, "host_output_buffers": out_bufs}
         del base_h, experts_h, outs_h, sets
 
     elapsed_ms = _max_over_ranks(elapsed_ms, world)
@@ -807,6 +824,18 @@ def measure_h2d(pinned_src) -> float:
         b.synchronize()
         best = max(best, n * pinned_src.element_size() / (a.elapsed_time(b) / 1e3) / 1e9)
     return best
+
+
+def host_mem_available() -> float:
+    """bytes of host memory available now (MemAvailable), or +inf where it cannot be read"""
+    try:
+        with open("/proc/meminfo") as f:
+            for line in f:
+                if line.startswith("MemAvailable:"):
+                    return float(line.split()[1]) * 1024.0
+    except OSError:
+        pass
+    return float("inf")
 
 
 def _max_over_ranks(x: float, world: int) -> float:

@@ -160,3 +160,16 @@ def test_interval_union_and_overlap_of_the_host_timeline():
     assert bench._overlap_ms(2.5, 5.5, iv) == 1.0   # [2.5, 3] and [5, 5.5]
     assert bench._overlap_ms(3.0, 5.0, iv) == 0.0
     assert bench._overlap_ms(-1.0, 10.0, iv) == bench._union_ms(iv)
+
+
+def test_host_memory_reading():
+    """MemAvailable in bytes: positive, and no more than MemTotal"""
+    import bench
+
+    avail = bench.host_mem_available()
+    total = None
+    with open("/proc/meminfo") as f:
+        for line in f:
+            if line.startswith("MemTotal:"):
+                total = float(line.split()[1]) * 1024.0
+    assert 0 < avail <= total

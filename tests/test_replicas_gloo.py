@@ -27,7 +27,9 @@ def _rank(rank, world, port, out):
     try:
         dist.barrier()
         out[rank] = (bench._max_over_ranks(10.0 + 5.0 * rank, world),
-                     bench.replica_value(1000.0, world, bench._max_over_ranks(10.0 + 5.0 * rank, world)))
+                     bench.replica_value(1000.0, world, bench._max_over_ranks(10.0 + 5.0 * rank, world)),
+                     # the end-to-end leg's go / no-go: one rank short of host memory stops both
+                     bench._max_over_ranks(1.0 if rank == 1 else 0.0, world))
         dist.barrier()
     finally:
         dist.destroy_process_group()
@@ -47,6 +49,7 @@ def test_two_gloo_replicas_agree_on_the_slowest_time():
         res = dict(out)
     assert res[0][0] == res[1][0] == 15.0           # max over the ranks' times
     assert res[0][1] == pytest.approx(2 * 1000.0 / 0.015)   # N x units / slowest time
+    assert res[0][2] == res[1][2] == 1.0            # both ranks skip the end-to-end leg together
 
 
 def test_single_rank_is_the_identity():
