@@ -989,18 +989,21 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
     const uint32_t n = ce.n, fast = ce.fast;
     mbar_arrive(&S.empty[e]);  // every read of the chunk's slots and entry is done
     // the elected side's sum and count: the sign of P + N taken exactly as P > -N or P < -N
-    // (then that side holds at least one entry, so c >= 1); otherwise 0 / 1
+    // (then that side holds at least one entry, so c >= 1); otherwise the numerator +0, whose
+    // quotient is +0 whatever count (<= 16, a valid table entry) is paired with it
     auto num_c = [&](int v, float& num, uint32_t& cv) {
       const bool pos = Pp[v] > -Nn[v], any = Pp[v] != -Nn[v];
       num = any ? (pos ? Pp[v] : Nn[v]) : 0.0f;
       const uint32_t cb = __float_as_uint(Cc[v]);
-      cv = any ? ((pos ? cb : cb >> CB) & ((1u << CB) - 1u)) : 0u;
+      cv = (pos ? cb : cb >> CB) & ((1u << CB) - 1u);
     };
     // q = RN(num * y), then Markstein's correction q + RN(num - q c) * y, and the output
     // fma(lambda, q, M_0), two elements per instruction; `checked` also notes the numerators
     // 0 < |num| < 2^-100, which then take the IEEE division under one warp vote
     auto finalise = [&](auto checked) {
-      bool exact = false;
+      // 2 |bits| - 2 wraps the zeros to the top: its minimum over the vector is below
+      // 2 * bits(2^-100) - 2 exactly when some numerator has 0 < |num| < 2^-100
+      uint32_t lowest = 0xFFFFFFFFu;
 #pragma unroll
       for (int v = 0; v < V; v += 2) {
         float a0, a1, q0, q1, r0, r1;
@@ -1008,13 +1011,15 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
         num_c(v, a0, c0);
         num_c(v + 1, a1, c1);
         if constexpr (decltype(checked)::value)
-          exact = exact || div_small_needs_ieee(a0) || div_small_needs_ieee(a1);
+          lowest = min(lowest, min(__float_as_uint(a0) * 2u - 2u, __float_as_uint(a1) * 2u - 2u));
         const float2 t0 = S.ntab[c0], t1 = S.ntab[c1];
         f2_mul(a0, a1, t0.y, t1.y, q0, q1);
         f2_fma(q0, q1, t0.x, t1.x, a0, a1, r0, r1);
         f2_fma(r0, r1, t0.y, t1.y, q0, q1, q0, q1);
         f2_fma(p.lambda, p.lambda, q0, q1, x0[v], x0[v + 1], y[v], y[v + 1]);
       }
+      static_assert(0x0D800000u * 2u - 2u == 0x1AFFFFFEu, "bits of 2^-100");
+      const bool exact = decltype(checked)::value && lowest < 0x1AFFFFFEu;
       if (decltype(checked)::value && __any_sync(0xFFFFFFFFu, exact)) {
 #pragma unroll
         for (int v = 0; v < V; ++v) {
