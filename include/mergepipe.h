@@ -23,7 +23,12 @@
  *    CUDA runtime's cudaStream_t passed as mp_stream (NULL = legacy default).
  *  - Every call enqueues its GPU work on the given stream and returns without
  *    waiting for it, except the accessors (mp_*_info, mp_index_stats), which
- *    wait for the handle's work to finish.  Errors found by a kernel (a
+ *    wait for the handle's work to finish.  mp_index_blocks, mp_plan, mp_merge and
+ *    mp_merge_touched enqueue kernels only (their small tables and results move
+ *    through pinned memory that kernels read and write), so bulk transfers the
+ *    caller runs on other streams do not hold them up; the exceptions use
+ *    cudaMemcpyAsync: a block table above 8 MiB, the thresholds of TIES after
+ *    masking, and the arrays that mp_index_import copies in.  Errors found by a kernel (a
  *    non-finite delta, a timed-out wait) are reported by the next accessor on
  *    that handle or on a handle derived from it.
  *  - On an error return no handle is produced and *out is set to NULL; the

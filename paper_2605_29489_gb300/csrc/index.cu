@@ -293,7 +293,7 @@ template <bool BF16, int KG, int BM>
 __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone, KG>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
   constexpr bool TIES = BM != kBinNone;
-  constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;  // key bins per expert
+  constexpr uint32_t NB = BM == kBinNone ? 1u : (BM == kBinWindow ? kWinBins : 256u);  // key bins per expert
   // The TIES catalog with up to 4 experts per item publishes whole chunks: the base fill and
   // the item's expert fills of one chunk sit in consecutive ring slots under one "full"
   // mbarrier (counting all their bytes) and one "empty" mbarrier, so that a consumer waits
@@ -1012,7 +1012,7 @@ cudaError_t ties_finish_t(const IndexLaunch& p, cudaStream_t st) {
 template <bool BF16, int KG, int BM>
 cudaError_t launch_pass(const IndexLaunch& p, uint32_t G, uint64_t n_items, int sms, cudaStream_t st) {
   constexpr bool ties = BM != kBinNone;
-  constexpr uint32_t NB = BM == kBinWindow ? kWinBins : 256u;
+  constexpr uint32_t NB = BM == kBinNone ? 1u : (BM == kBinWindow ? kWinBins : 256u);
   const size_t smem = sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>);
   static_assert(IxGeo<ties, KG>::kCtasPerSm *
                         (sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>) + 1024) <=
