@@ -1315,7 +1315,8 @@ mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint
   uint32_t err = 0;
   if ((e = cudaMemcpy(&err, index->d_err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
   if (err & kErrNonfinite) return fail(MP_ERR_NONFINITE, "a delta in the family is NaN or infinite");
-  if (err) return fail(MP_ERR_TIMEOUT, "index kernels reported an error");
+  if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the index gave up");
+  if (err) return fail(MP_ERR_CUDA, "an internal check of the index kernels failed");
   return MP_OK;
 }
 
@@ -1336,7 +1337,8 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
     return cuda_fail(e, "copy");
   if (s[6] & kErrNonfinite) return fail(MP_ERR_NONFINITE, "the index saw a NaN or infinite delta");
   if (s[6] & kErrMissing) return fail(MP_ERR_UNSUPPORTED, "a catalog entry without statistics and no tensor map");
-  if (s[6]) return fail(MP_ERR_TIMEOUT, "index kernels reported an error");
+  if (s[6] & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the index gave up");
+  if (s[6]) return fail(MP_ERR_CUDA, "an internal check of the index or plan kernels failed");
   if (s[0] > plan->budget) return fail(MP_ERR_BUDGET, "planned bytes exceed the budget");
   return MP_OK;
 }
