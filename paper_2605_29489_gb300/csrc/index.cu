@@ -302,9 +302,9 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone, KG>::kCtasPe
   // window bins of bf16 deltas: the nonzero count comes from the keys (ties_win2k,
   // nz_halves) and the zeros share the below-window bin
   constexpr bool KNZ = BM == kBinWindow && BF16;
-  constexpr int kIxSlots = IxGeo<TIES>::kSlots;
+  constexpr int kIxSlots = IxGeo<TIES, KG>::kSlots;
   static_assert(!CW || kIxSlots >= 2 * (KG + 1), "two whole chunks fit the ring");
-  constexpr uint32_t kIxSlotBytes = IxGeo<TIES>::kSlotBytes;
+  constexpr uint32_t kIxSlotBytes = IxGeo<TIES, KG>::kSlotBytes;
   constexpr uint32_t ES = BF16 ? 2u : 4u;
   constexpr uint32_t CH = kIxSlotBytes / ES;
   constexpr int V = BF16 ? 8 : 4;
@@ -1013,9 +1013,9 @@ template <bool BF16, int KG, int BM>
 cudaError_t launch_pass(const IndexLaunch& p, uint32_t G, uint64_t n_items, int sms, cudaStream_t st) {
   constexpr bool ties = BM != kBinNone;
   constexpr uint32_t NB = BM == kBinNone ? 1u : (BM == kBinWindow ? kWinBins : 256u);
-  const size_t smem = sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>);
+  const size_t smem = sizeof(IxSmem<KG, IxGeo<ties, KG>::kSlots, IxGeo<ties, KG>::kSlotBytes, NB>);
   static_assert(IxGeo<ties, KG>::kCtasPerSm *
-                        (sizeof(IxSmem<KG, IxGeo<ties>::kSlots, IxGeo<ties>::kSlotBytes, NB>) + 1024) <=
+                        (sizeof(IxSmem<KG, IxGeo<ties, KG>::kSlots, IxGeo<ties, KG>::kSlotBytes, NB>) + 1024) <=
                     228u * 1024u,
                 "the CTAs per SM that the grid assumes fit one SM's shared memory");
   uint64_t grid = (uint64_t)sms * IxGeo<ties, KG>::kCtasPerSm;
