@@ -382,23 +382,24 @@ def native(args, rank, world, local_rank):
             return mp.mp_index_import(fam_c, gop, *catalog, stream=stream)
         return mp.mp_index_blocks(fam_c, gop, stream)
 
-    def step(fam_c, ev=None):
+    def step(fam_c, ev=None, st=None):
+        st = stream if st is None else st
         hs = []
         if ev is not None:
-            ev["i0"].record(stream)
-        idx = make_index(fam_c)
+            ev["i0"].record(st)
+        idx = make_index(fam_c) if st is stream else mp.mp_index_blocks(fam_c, gop, st)
         hs.append(idx)
         if ev is not None:
-            ev["i1"].record(stream)
+            ev["i1"].record(st)
         for k, B in enumerate(Bs):
             if ev is not None:
-                ev["p0"][k].record(stream)
-            plan = mp.mp_plan(idx, gop, B, stream)
+                ev["p0"][k].record(st)
+            plan = mp.mp_plan(idx, gop, B, st)
             if ev is not None:
-                ev["p1"][k].record(stream)
-            man = merge_fn(fam_c, idx, plan, outs[0 if shared_out else k], stream)
+                ev["p1"][k].record(st)
+            man = merge_fn(fam_c, idx, plan, outs[0 if shared_out else k], st)
             if ev is not None:
-                ev["m1"][k].record(stream)
+                ev["m1"][k].record(st)
             hs += [plan, man]
         return hs
 
@@ -459,6 +460,11 @@ def native(args, rank, world, local_rank):
     for hs in handles:
         for h in hs:
             h.free()
+    graph = None
+    # device-resident families whose calls enqueue only kernels (TIES after masking and
+    # imported catalogs copy host arrays in, which a capture cannot hold)
+    if not host_pool and catalog is None and gop.kind != mp.MP_OP_TIES_MASKED:
+        graph = graph_replay(mp, step, mf)
 
     if not touched_mode:   # touched-only outputs hold only the touched blocks
         fidelity_vs_full(fam, budgets, outs, shared_out, per_budget)
@@ -621,6 +627,7 @@ def native(args, rank, world, local_rank):
                                           "budget sweep's launches / their summed CUDA-event time"},
         "gpu_launches": launches,
         "host_timeline": timeline,
+        "graph": graph,
         "host_link": None if link is None else dict(
             h2d_gbs_measured=link, gathered_bytes=[pb["planned_bytes"] for pb in per_budget],
             gathered_gbs=[pb["planned_bytes"] / (pb["merge_ms"] / 1e3) / 1e9 for pb in per_budget],
@@ -653,6 +660,31 @@ def merge_kernel_name(op: str, dtype: int, K: int) -> str:
             "avg_renorm": "AVG_RENORM", "dare_ties": "DARE_TIES"}[op]
     chunk = (inst == "TIES" and K <= 8) or (inst in ("DARE", "DARE_TIES") and K <= 16)
     return f"{'merge_chunk_kernel' if chunk else 'merge_tma_kernel'}<{'bf16' if dtype == 0 else 'f32'}, {inst}>"
+
+
+def graph_replay(mp, step, mf, reps=20):
+    """One step captured into a CUDA graph (catalog, plans and merges, on a capture stream)
+    and replayed: the per-step time without the host's launch work.  Not part of `value`,
+    which times the eager calls."""
+    import torch
+    torch.cuda.synchronize()
+    s = torch.cuda.Stream()
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        hs = step(mf, st=s)
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with torch.cuda.stream(s):
+        g.replay()
+        a.record(s)
+        for _ in range(reps):
+            g.replay()
+        b.record(s)
+    torch.cuda.synchronize()
+    ms = a.elapsed_time(b) / reps
+    for h in hs:  # the handles' memory first, then the graph
+        h.free()
+    del g
+    return {"replay_ms_per_step": ms, "reps": reps}
 
 
 def _union_ms(iv):

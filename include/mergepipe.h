@@ -28,7 +28,15 @@
  *    through pinned memory that kernels read and write), so bulk transfers the
  *    caller runs on other streams do not hold them up; the exceptions use
  *    cudaMemcpyAsync: a block table above 8 MiB, the thresholds of TIES after
- *    masking, and the arrays that mp_index_import copies in.  Errors found by a kernel (a
+ *    masking, and the arrays that mp_index_import copies in.
+ *  - CUDA graphs: for a family whose experts are in device memory, a step made of
+ *    mp_index_blocks, mp_plan and mp_merge / mp_merge_touched calls can be captured
+ *    on a stream (stream capture) and the graph replayed; each replay recomputes the
+ *    catalog, the plans and the merges from the buffers' current contents into the
+ *    handles made during the capture.  The accessors of those handles then wait for
+ *    the whole device (a captured event cannot be waited for from the host).  Free
+ *    such handles before the graph is destroyed.  Host-resident pools, TIES after
+ *    masking and mp_index_import are not capturable.  Errors found by a kernel (a
  *    non-finite delta, a timed-out wait) are reported by the next accessor on
  *    that handle or on a handle derived from it.
  *  - On an error return no handle is produced and *out is set to NULL; the

@@ -64,7 +64,13 @@ void* pin_get(size_t bytes) {
   std::lock_guard<std::mutex> lk(g_pin_mu);
   if (g_pin_free[c].empty()) {
     void* chunk = nullptr;
-    if (cudaHostAlloc(&chunk, kPinChunk[c], cudaHostAllocDefault) != cudaSuccess) {
+    // a new chunk may be needed while a stream of this thread is being captured into a
+    // graph: the allocation is host-side only, so it is made in relaxed capture mode
+    cudaStreamCaptureMode mode = cudaStreamCaptureModeRelaxed;
+    cudaThreadExchangeStreamCaptureMode(&mode);
+    const cudaError_t e = cudaHostAlloc(&chunk, kPinChunk[c], cudaHostAllocDefault);
+    cudaThreadExchangeStreamCaptureMode(&mode);
+    if (e != cudaSuccess) {
       cudaGetLastError();
       return nullptr;
     }
@@ -261,6 +267,30 @@ void set_error(const std::string& msg) {
 void set_static_error(const char* msg) { g_static_error = msg; }
 
 void count_launches(uint64_t n) { g_launches.fetch_add(n, std::memory_order_relaxed); }
+
+bool capturing(cudaStream_t st) {
+  cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+  if (cudaStreamIsCapturing(st, &cs) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return cs == cudaStreamCaptureStatusActive;
+}
+
+// the caller's stream waits for another handle's work: inside one capture state as usual; a
+// call under capture waits for an eager handle through an external event-wait node; an
+// eager call on a handle built under capture relies on the caller to have run the graph
+cudaError_t stream_wait(cudaStream_t cs, cudaEvent_t ev, bool ev_captured, bool now_captured) {
+  if (!ev) return cudaSuccess;
+  if (ev_captured == now_captured) return cudaStreamWaitEvent(cs, ev, 0);
+  if (now_captured) return cudaStreamWaitEvent(cs, ev, cudaEventWaitExternal);
+  return cudaSuccess;
+}
+
+cudaError_t wait_handle(cudaEvent_t done, bool captured) {
+  if (captured) return cudaDeviceSynchronize();
+  return done ? cudaEventSynchronize(done) : cudaSuccess;
+}
 
 mp_status cuda_fail(cudaError_t e, const char* what) {
   cudaGetLastError();
@@ -574,6 +604,8 @@ mp_status new_index(const Geometry& g, const mp_op* op, bool host_pool, size_t w
   ix->n_groups = n_groups;
   ix->has_missing = false;
   ix->done = nullptr;
+  ix->captured = capturing(cs);
+  ix->order_captured = false;
   ix->order_ready = nullptr;
   ix->order_mu = new (std::nothrow) std::mutex();
   if (!ix->order_mu) {
@@ -927,6 +959,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
   pl->budget = budget_bytes;
   pl->n_groups = index->n_groups;
   pl->done = nullptr;
+  pl->captured = capturing(cs);
   pl->h_summary = static_cast<uint64_t*>(pin_get(64));
   if (!pl->h_summary) {
     delete pl;
@@ -957,7 +990,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
     return r;
   };
   cudaError_t e;
-  if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = stream_wait(cs, index->done, index->captured, pl->captured)) != cudaSuccess) return bail(e, "stream wait");
   const uint64_t n_pairs = index->has_missing ? (uint64_t)g.K * g.n_tensors : 0ull;
   if ((e = malloc_async(&scratch.ptr, plan_scratch_bytes(U, n_pairs), cs)) != cudaSuccess) {
     scratch.ptr = nullptr;
@@ -1014,7 +1047,9 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
     std::lock_guard<std::mutex> lk(*ixw->order_mu);
     bool fill = false;
     if (!index->has_missing) {
-      if (ixw->order_mem.ptr && ixw->order_ready && ixw->order_key == order_key) {
+      // a cached order is reused only in the capture state it was written in (an event
+      // recorded in a graph cannot be waited for outside it, nor an eager one inside it)
+      if (ixw->order_mem.ptr && ixw->order_ready && ixw->order_key == order_key && ixw->order_captured == pl->captured) {
         if ((e = cudaStreamWaitEvent(cs, ixw->order_ready, 0)) != cudaSuccess) return bail(e, "stream wait");
         p.cache_order_in = ixw->d_order_cache;
         p.cache_q_in = ixw->d_order_q;
@@ -1034,6 +1069,7 @@ mp_status mp_plan(const mp_index* index, const mp_op* op, uint64_t budget_bytes,
         return bail(e, "event");
       if ((e = cudaEventRecord(ixw->order_ready, cs)) != cudaSuccess) return bail(e, "event record");
       ixw->order_key = order_key;
+      ixw->order_captured = pl->captured;
     }
   }
   if ((e = cudaFreeAsync(scratch.ptr, cs)) != cudaSuccess) return bail(e, "free scratch");
@@ -1098,6 +1134,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   mf->K = g.K;
   mf->n_blocks = g.n_blocks;
   mf->done = nullptr;
+  mf->captured = capturing(cs);
   mf->valid_done = nullptr;
   for (uint32_t i = 0; i <= kMaxK; ++i) mf->lineage[i] = (family->lineage_ids && i <= g.K) ? family->lineage_ids[i] : 0u;
   const size_t counters_bytes = (size_t)kCounterSlots * g.K * 8;
@@ -1136,8 +1173,8 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
     return r;
   };
   cudaError_t e;
-  if ((e = cudaStreamWaitEvent(cs, index->done, 0)) != cudaSuccess) return bail(e, "stream wait");
-  if ((e = cudaStreamWaitEvent(cs, plan->done, 0)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = stream_wait(cs, index->done, index->captured, mf->captured)) != cudaSuccess) return bail(e, "stream wait");
+  if ((e = stream_wait(cs, plan->done, plan->captured, mf->captured)) != cudaSuccess) return bail(e, "stream wait");
   if ((e = launch_fill(mf->mem.ptr, 0, back_bytes, cs)) != cudaSuccess) return bail(e, "fill");
   uint32_t* masked_tau = nullptr;
   if (masked) {
@@ -1260,8 +1297,12 @@ void mp_free(void* handle) {
   uint32_t magic = *static_cast<uint32_t*>(handle);
   if (magic == kMagicIndex) {
     mp_index_s* ix = static_cast<mp_index_s*>(handle);
-    if (ix->done) cudaEventSynchronize(ix->done), cudaEventDestroy(ix->done);
-    if (ix->order_ready) cudaEventSynchronize(ix->order_ready), cudaEventDestroy(ix->order_ready);
+    wait_handle(ix->done, ix->captured);
+    if (ix->done) cudaEventDestroy(ix->done);
+    if (ix->order_ready) {
+      wait_handle(ix->order_ready, ix->order_captured);
+      cudaEventDestroy(ix->order_ready);
+    }
     dev_free(ix->hash_mem);
     dev_free(ix->order_mem);
     dev_free(ix->mem);
@@ -1271,14 +1312,16 @@ void mp_free(void* handle) {
     delete ix;
   } else if (magic == kMagicPlan) {
     mp_plan_s* pl = static_cast<mp_plan_s*>(handle);
-    if (pl->done) cudaEventSynchronize(pl->done), cudaEventDestroy(pl->done);
+    wait_handle(pl->done, pl->captured);
+    if (pl->done) cudaEventDestroy(pl->done);
     dev_free(pl->mem);
     pin_put(pl->h_summary, 64);
     pl->magic = 0;
     delete pl;
   } else if (magic == kMagicManifest) {
     mp_manifest_s* mf = static_cast<mp_manifest_s*>(handle);
-    if (mf->done) cudaEventSynchronize(mf->done), cudaEventDestroy(mf->done);
+    wait_handle(mf->done, mf->captured);
+    if (mf->done) cudaEventDestroy(mf->done);
     if (mf->valid_done) cudaEventSynchronize(mf->valid_done), cudaEventDestroy(mf->valid_done);
     dev_free(mf->valid_mem);
     dev_free(mf->mem);
@@ -1301,7 +1344,7 @@ mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint
   mp_status st;
   if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
   cudaError_t e;
-  if ((e = cudaEventSynchronize(index->done)) != cudaSuccess) return cuda_fail(e, "index work");
+  if ((e = wait_handle(index->done, index->captured)) != cudaSuccess) return cuda_fail(e, "index work");
   const uint64_t U = index->g.n_blocks * index->g.K;
   if (norm && (e = cudaMemcpy(norm, index->d_norm, U * 4, cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail(e, "copy");
@@ -1325,7 +1368,7 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
   mp_status st;
   if ((st = check_handle(plan, kMagicPlan, "plan")) != MP_OK) return st;
   cudaError_t e;
-  if ((e = cudaEventSynchronize(plan->done)) != cudaSuccess) return cuda_fail(e, "plan work");
+  if ((e = wait_handle(plan->done, plan->captured)) != cudaSuccess) return cuda_fail(e, "plan work");
   const uint64_t* s = plan->h_summary;
   if (planned_bytes) *planned_bytes = s[0];
   if (n_selected) *n_selected = s[1];
@@ -1348,7 +1391,7 @@ mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_per_expert
   mp_status st;
   if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
   cudaError_t e;
-  if ((e = cudaEventSynchronize(man->done)) != cudaSuccess) return cuda_fail(e, "merge work");
+  if ((e = wait_handle(man->done, man->captured)) != cudaSuccess) return cuda_fail(e, "merge work");
   const unsigned long long* c = man->h_realized;
   const uint64_t* s = reinterpret_cast<const uint64_t*>(c + (size_t)kCounterSlots * man->K);
   const uint32_t err = *reinterpret_cast<const uint32_t*>(s + 8);
@@ -1403,7 +1446,7 @@ mp_status mp_index_hash_values(const mp_index* index, uint64_t* base_hash, uint6
   if ((st = check_handle(index, kMagicIndex, "index")) != MP_OK) return st;
   if (!index->hash_mem.ptr) return fail(MP_ERR_INVALID_ARG, "the index holds no block hashes (mp_index_hashes)");
   cudaError_t e;
-  if ((e = cudaEventSynchronize(index->done)) != cudaSuccess) return cuda_fail(e, "index work");
+  if ((e = wait_handle(index->done, index->captured)) != cudaSuccess) return cuda_fail(e, "index work");
   const uint64_t nb = index->g.n_blocks;
   if (base_hash && (e = cudaMemcpy(base_hash, index->d_base_hash, nb * 8, cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail(e, "copy");
@@ -1492,7 +1535,7 @@ mp_status mp_manifest_threshold_reads(const mp_manifest* man, uint64_t* bytes) {
   if ((st = check_handle(man, kMagicManifest, "manifest")) != MP_OK) return st;
   if (!bytes) return fail(MP_ERR_INVALID_ARG, "bytes is NULL");
   cudaError_t e;
-  if ((e = cudaEventSynchronize(man->done)) != cudaSuccess) return cuda_fail(e, "merge work");
+  if ((e = wait_handle(man->done, man->captured)) != cudaSuccess) return cuda_fail(e, "merge work");
   *bytes = man->h_realized[(size_t)kCounterSlots * man->K + 10];
   return MP_OK;
 }

@@ -81,6 +81,7 @@ struct mp_index_s {
   uint32_t* d_order_cache;           // [K * n_blocks]
   unsigned long long* d_order_q;     // candidates
   std::vector<uint8_t> order_key;    // the operator's digest header without the budget
+  bool order_captured;               // the cached order was written under stream capture
   cudaEvent_t order_ready;
   std::mutex* order_mu;
   mp::Alloc hash_mem;      // the catalog's block hashes, once computed or imported
@@ -92,6 +93,7 @@ struct mp_index_s {
   uint32_t* d_tau;         // [K][n_groups] (TIES only)
   uint32_t* d_err;         // error word
   cudaEvent_t done;
+  bool captured;           // built under stream capture: waits go through the device
   std::vector<std::pair<void*, size_t>> pinned;  // pinned staging of the uploads (released by mp_free)
   std::vector<uint64_t> h_blk_off;  // host copy of the block table (segments of a host pool)
   std::vector<uint32_t> h_blk_len;
@@ -117,6 +119,7 @@ struct mp_plan_s {
   uint64_t* d_summary;     // [8] chat, n_sel, n_cand, set_hash, digest, touched, err, pad
   uint64_t* h_summary;     // pinned host copy of d_summary
   cudaEvent_t done;
+  bool captured;           // built under stream capture: waits go through the device
 };
 
 struct mp_manifest_s {
@@ -132,6 +135,7 @@ struct mp_manifest_s {
   uint64_t planned, touched, digest;
   uint64_t lineage[mp::kMaxK + 1];  // caller ids of M_0..M_K (zeros when none were given)
   cudaEvent_t done;
+  bool captured;                    // built under stream capture: waits go through the device
   // hash validation (mp_manifest_validate): checked / mismatched / first bad item, and
   // the output's block hashes
   mp::Alloc valid_mem;
@@ -151,6 +155,14 @@ void set_error(const std::string& msg);
 // records a string literal as the last error without allocating
 void set_static_error(const char* msg);
 mp_status cuda_fail(cudaError_t e, const char* what);
+
+// CUDA graphs: a call made while its stream is being captured records its work (and its
+// handle's completion event) into the graph.  Such an event cannot be waited for from the
+// host, so the waits of a handle built under capture go through the whole device, which
+// covers every replay of the graph enqueued so far.
+bool capturing(cudaStream_t st);
+cudaError_t wait_handle(cudaEvent_t done, bool captured);
+cudaError_t stream_wait(cudaStream_t cs, cudaEvent_t ev, bool ev_captured, bool now_captured);
 
 // device-time ranges of the calls (trace.cu): trace_begin records the start of a range on
 // st and returns its ticket, or -1 while no trace is recording (or it is full); trace_end
