@@ -1256,3 +1256,28 @@ def test_ties_masked_thresholds_per_expert_scope(tiny_family):
             allk = np.sort(np.concatenate(parts))[::-1]
             k = int(math.floor(density * allk.size))
             assert got[i, 0] == (oracle.TAU_NONE if k == 0 else int(allk[k - 1])), (density, i)
+
+
+def _dare_seed_keeping_first_dropping_second(p):
+    for seed in range(100000):
+        if oracle.dare_keep(seed, 0, 0, p) and not oracle.dare_keep(seed, 1, 0, p):
+            return seed
+    raise AssertionError("no seed found")
+
+
+def test_dare_omits_a_dropped_entry_even_in_the_sign_of_zero():
+    """R13: a dropped entry is left out of the sum, as an unselected one is.  Expert 1's kept
+    product underflows to -0 (alpha 2^-20 times -2^-132), so the sum is -0; expert 2 is dropped
+    with alpha > 0.  Omitting it keeps -0 and the output is M_0 + (-0) = -0 for M_0 = -0;
+    adding its zero instead would give +0 + (-0) = +0 and the output +0."""
+    p = 0.5
+    seed = _dare_seed_keeping_first_dropping_second(p)
+    base = np.array([0x8000], np.uint16)            # -0
+    e0 = np.array([0x8001], np.uint16)              # -2^-133, the smallest bf16 subnormal
+    e1 = np.array([0x3F80], np.uint16)              # 1.0 (dropped)
+    op = oracle.Op(oracle.DARE, 2, alpha=[2.0 ** -20, 0.5], drop_p=p, seed=seed)
+    out = oracle.merge_block(oracle.BF16, 0, base, [e0, e1], 0b11, op)
+    assert out[0] == 0x8000
+    # with expert 2 kept (p = 0) its contribution is an ordinary nonzero term
+    op0 = oracle.Op(oracle.DARE, 2, alpha=[2.0 ** -20, 0.5], drop_p=0.0, seed=seed)
+    assert oracle.merge_block(oracle.BF16, 0, base, [e0, e1], 0b11, op0)[0] == 0x3F00  # 0.5
