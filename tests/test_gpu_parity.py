@@ -55,16 +55,19 @@ def ordered(bits):
     return np.where(b & 0x8000, -(b & 0x7FFF), b)
 
 
-def assert_merge_close(fam, got, want, what=""):
+def assert_merge_close(fam, got, want, what="", signed_zero=True):
+    """within the tolerance, then identical: bit for bit (signed_zero), or equal in value
+    (+0 == -0) where only the value is defined"""
     if fam.dtype == synth.BF16:
         d = np.abs(ordered(got) - ordered(want))
         assert d.max(initial=0) <= 1, f"{what}: max ulp diff {d.max()}"
-        n_diff = int((d != 0).sum())
+        n_diff = int((got != want).sum()) if signed_zero else int((d != 0).sum())
     else:
         g, w = got.astype(np.float64), want.astype(np.float64)
         rel = np.abs(g - w) / np.maximum(np.abs(w), 1e-30)
         assert np.all((rel <= 1e-6) | (g == w)), f"{what}: max rel {rel.max()}"
-        n_diff = int((got.view(np.uint32) != want.view(np.uint32)).sum())
+        same = (got.view(np.uint32) == want.view(np.uint32)) if signed_zero else ((g == w) | (np.isnan(g) & np.isnan(w)))
+        n_diff = int((~same).sum())
     assert n_diff == 0, f"{what}: {n_diff} elements differ from the oracle (within tolerance, but not identical)"
 
 
@@ -112,6 +115,19 @@ def ops_for(K, kinds=("avg", "ta", "ties", "ties1", "dare")):
         elif k == "ties_masked1":
             out.append(("ties_masked1", mp.make_op(mp.MP_OP_TIES_MASKED, lam=0.7, density=0.35, trim_scope=1),
                         oracle.Op(oracle.TIES_MASKED, K, lam=0.7, density=0.35, trim_scope=1)))
+        elif k == "ta_tiny":   # coefficients small enough that products of subnormals underflow to +-0
+            alpha = [2.0 ** -20, -(2.0 ** -21), 2.0 ** -18][:K] + [2.0 ** -19] * max(0, K - 3)
+            out.append(("ta_tiny", mp.make_op(mp.MP_OP_TA, alpha=alpha), oracle.Op(oracle.TA, K, alpha=alpha)))
+        elif k == "dare_tiny":
+            alpha = [2.0 ** -20, -(2.0 ** -21), 2.0 ** -18][:K] + [2.0 ** -19] * max(0, K - 3)
+            out.append(("dare_tiny", mp.make_op(mp.MP_OP_DARE, alpha=alpha, drop_p=0.5, seed=77),
+                        oracle.Op(oracle.DARE, K, alpha=alpha, drop_p=0.5, seed=77)))
+        elif k == "ties_neg":   # a negative lambda: lambda * +0 = -0 where no sign wins
+            out.append(("ties_neg", mp.make_op(mp.MP_OP_TIES, lam=-0.5, density=0.3),
+                        oracle.Op(oracle.TIES, K, lam=-0.5, density=0.3)))
+        elif k == "dare_ties_neg":
+            out.append(("dare_ties_neg", mp.make_op(mp.MP_OP_DARE_TIES, lam=-0.75, drop_p=0.5, seed=99),
+                        oracle.Op(oracle.DARE_TIES, K, lam=-0.75, drop_p=0.5, seed=99)))
         elif k == "ties_pb":
             out.append(("ties_pb", mp.make_op(mp.MP_OP_TIES, lam=1.0, density=0.2, score_mode=1),
                         oracle.Op(oracle.TIES, K, lam=1.0, density=0.2, score_mode=1)))
@@ -168,8 +184,10 @@ def run_case(fam, base, experts, kinds, fracs, check_merge=True, host_experts=Fa
             if masked:   # the threshold pass re-reads only selected blocks
                 assert 0 <= mp.mp_manifest_threshold_reads(man) <= opl["chat"], what
             if f >= 1.0:   # Eq. 5: full budget reproduces the unmasked operator
+                # in value: the full read also adds the zero deltas of the blocks the plan
+                # leaves out (nnz = 0), and adding a +0 can turn an accumulated -0 into +0
                 phi = oracle.merge(of, oop, tau=o_tau, mask=None)
-                assert_merge_close(fam, got[covered], phi[covered], what + " vs Phi")
+                assert_merge_close(fam, got[covered], phi[covered], what + " vs Phi", signed_zero=False)
             man.free()
             plan.free()
         idx.free()
@@ -258,6 +276,41 @@ def test_parity_tiny_config():
     fam = synth.tiny()
     base, experts = fam.host_arrays()
     run_case(fam, base, experts, ("avg", "ties", "dare"), [1.0, 0.5, 0.25])
+
+
+def signed_zero_family(dtype):
+    """every element drawn from +-0, +-(the smallest subnormal), +-(twice it) and +-1, the
+    experts equal to the base at 40 % of the elements and over whole blocks for some
+    (block, expert) pairs: signed zeros in the base, deltas of +0, -0 results of underflowing
+    products, ties of equal magnitudes in the TIES trim, and zero-delta blocks the plan omits"""
+    fam = synth.custom([3 * 1024 + 77, 2048, 515], dtype=dtype, block_elems=1024, K=3, name=f"signed-zero-{dtype}")
+    _, _, total = fam.layout()
+    rng = np.random.default_rng(2605)
+    if dtype == synth.BF16:
+        pal = np.array([0x0000, 0x8000, 0x0001, 0x8001, 0x0002, 0x8002, 0x3F80, 0xBF80], np.uint16)
+    else:
+        pal = np.array([0x00000000, 0x80000000, 0x00000001, 0x80000001, 0x00000002, 0x80000002, 0x3F800000,
+                        0xBF800000], np.uint32).view(np.float32)
+    base = pal[rng.integers(0, 6, total)]
+    bo, bl, _ = fam.block_table()
+    experts = []
+    for i in range(fam.K):
+        e = np.where(rng.random(total) < 0.4, base, pal[rng.integers(0, len(pal), total)])
+        for b in range(i, fam.n_blocks, 3):   # whole blocks equal to the base: nnz = 0
+            e[int(bo[b]):int(bo[b] + bl[b])] = base[int(bo[b]):int(bo[b] + bl[b])]
+        experts.append(e.astype(base.dtype))
+    return fam, base, experts
+
+
+@pytest.mark.parametrize("dtype", [synth.BF16, synth.F32], ids=["bf16", "f32"])
+def test_signed_zeros_and_subnormals_bit_for_bit(dtype):
+    """the kernels reach the oracle's result bit for bit, the sign of every zero included, on
+    inputs made of signed zeros and subnormals: the merge adds each selected (and, for DARE,
+    kept) term in the oracle's order and omits the rest, and an unselected block is M_0 plus
+    the zero the operator adds"""
+    fam, base, experts = signed_zero_family(dtype)
+    run_case(fam, base, experts, ("avg", "ta", "ta_tiny", "ties", "ties_neg", "dare", "dare_tiny", "avg_renorm",
+                                  "dare_ties", "dare_ties_neg", "ties_masked"), [0.0, 0.3, 1.0])
 
 
 def test_device_fill_matches_host_fill():
