@@ -278,12 +278,13 @@ def test_parity_tiny_config():
     run_case(fam, base, experts, ("avg", "ties", "dare"), [1.0, 0.5, 0.25])
 
 
-def signed_zero_family(dtype):
+def signed_zero_family(dtype, K=3):
     """every element drawn from +-0, +-(the smallest subnormal), +-(twice it) and +-1, the
     experts equal to the base at 40 % of the elements and over whole blocks for some
     (block, expert) pairs: signed zeros in the base, deltas of +0, -0 results of underflowing
     products, ties of equal magnitudes in the TIES trim, and zero-delta blocks the plan omits"""
-    fam = synth.custom([3 * 1024 + 77, 2048, 515], dtype=dtype, block_elems=1024, K=3, name=f"signed-zero-{dtype}")
+    fam = synth.custom([3 * 1024 + 77, 2048, 515], dtype=dtype, block_elems=1024, K=K,
+                        name=f"signed-zero-{dtype}-k{K}")
     _, _, total = fam.layout()
     rng = np.random.default_rng(2605)
     if dtype == synth.BF16:
@@ -296,21 +297,25 @@ def signed_zero_family(dtype):
     experts = []
     for i in range(fam.K):
         e = np.where(rng.random(total) < 0.4, base, pal[rng.integers(0, len(pal), total)])
-        for b in range(i, fam.n_blocks, 3):   # whole blocks equal to the base: nnz = 0
+        for b in range(i % 3, fam.n_blocks, 3):   # whole blocks equal to the base: nnz = 0
             e[int(bo[b]):int(bo[b] + bl[b])] = base[int(bo[b]):int(bo[b] + bl[b])]
         experts.append(e.astype(base.dtype))
     return fam, base, experts
 
 
-@pytest.mark.parametrize("dtype", [synth.BF16, synth.F32], ids=["bf16", "f32"])
-def test_signed_zeros_and_subnormals_bit_for_bit(dtype):
+@pytest.mark.parametrize("dtype,K,host_experts", [(synth.BF16, 3, False), (synth.F32, 3, False), (synth.BF16, 17, False),
+                                                  (synth.BF16, 3, True)],
+                         ids=["bf16", "f32", "bf16-k17", "bf16-host-pool"])
+def test_signed_zeros_and_subnormals_bit_for_bit(dtype, K, host_experts):
     """the kernels reach the oracle's result bit for bit, the sign of every zero included, on
     inputs made of signed zeros and subnormals: the merge adds each selected (and, for DARE,
     kept) term in the oracle's order and omits the rest, and an unselected block is M_0 plus
-    the zero the operator adds"""
-    fam, base, experts = signed_zero_family(dtype)
+    the zero the operator adds.  K = 17 takes the streaming merges for every operator; the
+    host-pool case gathers the experts from pinned host memory"""
+    fam, base, experts = signed_zero_family(dtype, K)
     run_case(fam, base, experts, ("avg", "ta", "ta_tiny", "ties", "ties_neg", "dare", "dare_tiny", "avg_renorm",
-                                  "dare_ties", "dare_ties_neg", "ties_masked"), [0.0, 0.3, 1.0])
+                                  "dare_ties", "dare_ties_neg", "ties_masked"), [0.0, 0.3, 1.0],
+             host_experts=host_experts)
 
 
 def test_device_fill_matches_host_fill():
