@@ -150,6 +150,9 @@ MUTANTS = [
     ("full_read_mask_drops_last_expert", "((1u << f->K) - 1u);", "((1u << f->K) - 1u) >> 1;"),
     ("dare_counter_block_local_in_merge", "} else if (orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) {",
      "} else if (orc_dare_keep(op->seed, i, k, op->drop_p)) {"),
+    ("dare_adds_the_zero_of_a_dropped_entry",
+     "if (!orc_dare_keep(op->seed, i, j0 + k, op->drop_p)) continue; /* dropped: omitted */\n          d = d * sigma;",
+     "d = orc_dare_keep(op->seed, i, j0 + k, op->drop_p) ? d * sigma : 0.0f;"),
     ("merge_known_zero_from_nonzero", "if (nnz[(size_t)i * f->n_blocks + b] == 0) known_zero |= 1u << i;",
      "if (nnz[(size_t)i * f->n_blocks + b] != 0) known_zero |= 1u << i;"),
 ]
