@@ -39,6 +39,14 @@
  *    masking and mp_index_import are not capturable.  Errors found by a kernel (a
  *    non-finite delta, a timed-out wait) are reported by the next accessor on
  *    that handle or on a handle derived from it.
+ *  - Checked build: libmergepipe_checked.so exports the same entry points from the same
+ *    sources compiled with MP_CHECKED.  Before a kernel streams a range of a checkpoint
+ *    (a block of the catalog pass or of the host-pool gather, a chunk of the merge, a
+ *    block of the hash pass) it checks the range against the block table, the call's block
+ *    range, the buffers' extents, the 16-byte alignment of bulk copies and the number of
+ *    experts; a range that fails is not touched, and the accessors of the call's handle
+ *    return MP_ERR_CUDA with "a bounds check of the checked build failed".  mp_version()
+ *    names the build.  Slower; meant for debugging.
  *  - On an error return no handle is produced and *out is set to NULL; the
  *    contents of a merge output buffer are then unspecified.
  *  - mp_last_error() returns a thread-local message for the last failure.
@@ -370,7 +378,7 @@ uint64_t mp_budget_from_fraction(const mp_family* family, double f);
 /* Thread-local text of the last error ("" if none). */
 const char* mp_last_error(void);
 
-/* Library version string. */
+/* Library version string (it ends in ", checked)" in the checked build). */
 const char* mp_version(void);
 
 /* Number of CUDA kernels this library has launched in this process (all devices,

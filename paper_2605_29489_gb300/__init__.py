@@ -75,8 +75,11 @@ _lib = None
 
 
 def library_path() -> str:
+    """the default library, or with MERGEPIPE_CHECKED=1 in the environment the checked build
+    (every range a kernel streams is checked against the block table and the buffers first;
+    a failed check is reported by the accessors as MP_ERR_CUDA)"""
     from . import build as _build
-    return _build.build_mergepipe()
+    return _build.build_mergepipe(checked=os.environ.get("MERGEPIPE_CHECKED", "0") == "1")
 
 
 def lib():

@@ -2,6 +2,10 @@
 
 * ``_build/libmergepipe.so``  — the CUDA path behind ``include/mergepipe.h``
   (every ``csrc/*.cu`` compiled for sm_103a in parallel, then linked);
+* ``_build/libmergepipe_checked.so`` — the same sources with ``-DMP_CHECKED``: every
+  range a kernel streams is checked against the block table and the buffers first
+  (``csrc/checked.cuh``); loaded instead of the default library when the
+  environment sets ``MERGEPIPE_CHECKED=1``;
 * ``_build/libmpsynth_host.so`` — the synthetic-family host fill (gcc);
 * ``_build/libmpsynth_dev.so``  — the synthetic-family device fill (nvcc).
 
@@ -67,19 +71,19 @@ def _run(cmd):
     return r.stdout
 
 
-def build_mergepipe(force: bool = False, verbose: bool = False) -> str:
+def build_mergepipe(force: bool = False, verbose: bool = False, checked: bool = False) -> str:
     os.makedirs(OUT, exist_ok=True)
-    lib = os.path.join(OUT, "libmergepipe.so")
+    lib = os.path.join(OUT, "libmergepipe_checked.so" if checked else "libmergepipe.so")
     srcs = sorted(glob.glob(os.path.join(CSRC, "*.cu")))
     deps = srcs + sorted(glob.glob(os.path.join(CSRC, "*.cuh"))) + sorted(glob.glob(os.path.join(INCLUDE, "*.h")))
-    flags = ARCH + NVCC_FLAGS
+    flags = ARCH + NVCC_FLAGS + (["-DMP_CHECKED"] if checked else [])
     stamp = _stamp(deps, flags)
     if not force and _fresh(lib, stamp):
         return lib
     objs = []
     cmds = []
     for s in srcs:
-        o = os.path.join(OUT, os.path.basename(s)[:-3] + f".{os.getpid()}.o")
+        o = os.path.join(OUT, os.path.basename(s)[:-3] + (".checked" if checked else "") + f".{os.getpid()}.o")
         objs.append(o)
         cmds.append([nvcc(), *flags, "-I", INCLUDE, "-I", CSRC, "-c", s, "-o", o])
     with cf.ThreadPoolExecutor(max_workers=min(len(cmds), os.cpu_count() or 4)) as ex:
@@ -130,9 +134,9 @@ def build_synth_dev(force: bool = False) -> str:
 
 
 def build_all(force: bool = False, verbose: bool = False):
-    with cf.ThreadPoolExecutor(max_workers=3) as ex:
-        fs = [ex.submit(build_mergepipe, force, verbose), ex.submit(build_synth_host, force),
-              ex.submit(build_synth_dev, force)]
+    with cf.ThreadPoolExecutor(max_workers=4) as ex:
+        fs = [ex.submit(build_mergepipe, force, verbose), ex.submit(build_mergepipe, force, verbose, True),
+              ex.submit(build_synth_host, force), ex.submit(build_synth_dev, force)]
         return [f.result() for f in fs]
 
 

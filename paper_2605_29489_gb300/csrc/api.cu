@@ -455,6 +455,8 @@ cudaError_t walk_segments(const IndexLaunch& p, const mp_index_s* ix, cudaStream
     gl.mask = nullptr;
     gl.src = p.experts;
     gl.gate = gate;
+    gl.ext = Extents{p.ext.span, span};
+    gl.err = p.err;
     for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
     if (inject_fault(MP_FAULT_GATHER)) {
       e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
@@ -469,6 +471,7 @@ cudaError_t walk_segments(const IndexLaunch& p, const mp_index_s* ix, cudaStream
     ps.b_begin = g.b0;
     ps.b_end = g.b1;
     ps.expert_origin = g.e0;
+    ps.ext.x_span = span;
     ps.defer_ties_select = 1;
     for (uint32_t i = 0; i < p.K; ++i) ps.experts.p[i] = hp.buf(b, i);
     const int tk = trace_begin(MP_TRACE_SEGMENT, (uint32_t)s, 0, cs);
@@ -533,6 +536,8 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
     gl.blk_len = p.blk_len;
     gl.mask = p.mask;
     gl.src = p.experts;
+    gl.ext = Extents{p.ext.span, span};
+    gl.err = p.err;
     for (uint32_t i = 0; i < p.K; ++i) gl.dst.p[i] = hp.buf(b, i);
     if (inject_fault(MP_FAULT_GATHER)) {
       e = cudaErrorLaunchFailure;  // reported as an injected failure; nothing was launched
@@ -547,6 +552,7 @@ cudaError_t merge_host_pool(MergeLaunch p, const mp_index_s* ix, cudaStream_t cs
     ps.b_begin = g.b0;
     ps.b_end = g.b1;
     ps.expert_origin = g.e0;
+    ps.ext.x_span = span;
     ps.experts = gl.dst;
     const int tk = trace_begin(MP_TRACE_SEGMENT, (uint32_t)s, 0, cs);
     e = launch_merge(ps, cs);
@@ -699,7 +705,9 @@ extern "C" {
 
 const char* mp_last_error(void) { return g_static_error ? g_static_error : g_last_error.c_str(); }
 
-const char* mp_version(void) { return "mergepipe-gb300 0.1 (sm_103a)"; }
+const char* mp_version(void) {
+  return kChecked ? "mergepipe-gb300 0.1 (sm_103a, checked)" : "mergepipe-gb300 0.1 (sm_103a)";
+}
 
 uint64_t mp_kernel_launch_count(void) { return g_launches.load(std::memory_order_relaxed); }
 
@@ -842,6 +850,7 @@ mp_status mp_index_blocks(const mp_family* family, const mp_op* op, mp_stream st
   p.b_begin = 0;
   p.b_end = g.n_blocks;
   p.expert_origin = 0;
+  p.ext = Extents{g.span_elems, g.span_elems};
   if (family->experts_location == 0) {
     if ((e = launch_index(p, cs)) != cudaSuccess) return bail(e, "index kernels");
   } else {
@@ -1217,6 +1226,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
     q.b_begin = 0;
     q.b_end = g.n_blocks;
     q.expert_origin = 0;
+    q.ext = Extents{g.span_elems, g.span_elems};
     q.wait_limit = g_stall_rounds.load(std::memory_order_relaxed);
     q.stall = q.wait_limit ? 1u : 0u;
     if ((e = launch_ties_masked(q, cs)) != cudaSuccess) return bail(e, "masked TIES threshold");
@@ -1258,6 +1268,7 @@ mp_status merge_common(const mp_family* family, const mp_index* index, const mp_
   p.b_begin = 0;
   p.b_end = g.n_blocks;
   p.expert_origin = 0;
+  p.ext = Extents{g.span_elems, g.span_elems};
   p.touched_only = touched_only ? 1u : 0u;
   p.wait_limit = g_stall_rounds.load(std::memory_order_relaxed);
   p.stall = p.wait_limit ? 1u : 0u;
@@ -1359,6 +1370,7 @@ mp_status mp_index_stats(const mp_index* index, float* norm, float* maxabs, uint
   if ((e = cudaMemcpy(&err, index->d_err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
   if (err & kErrNonfinite) return fail(MP_ERR_NONFINITE, "a delta in the family is NaN or infinite");
   if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the index gave up");
+  if (err & kErrBounds) return fail(MP_ERR_CUDA, "a bounds check of the checked build failed in the index kernels");
   if (err) return fail(MP_ERR_CUDA, "an internal check of the index kernels failed");
   return MP_OK;
 }
@@ -1381,6 +1393,7 @@ mp_status mp_plan_info(const mp_plan_t* plan, uint64_t* planned_bytes, uint64_t*
   if (s[6] & kErrNonfinite) return fail(MP_ERR_NONFINITE, "the index saw a NaN or infinite delta");
   if (s[6] & kErrMissing) return fail(MP_ERR_UNSUPPORTED, "a catalog entry without statistics and no tensor map");
   if (s[6] & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the index gave up");
+  if (s[6] & kErrBounds) return fail(MP_ERR_CUDA, "a bounds check of the checked build failed in the index kernels");
   if (s[6]) return fail(MP_ERR_CUDA, "an internal check of the index or plan kernels failed");
   if (s[0] > plan->budget) return fail(MP_ERR_BUDGET, "planned bytes exceed the budget");
   return MP_OK;
@@ -1406,6 +1419,7 @@ mp_status mp_manifest_info(const mp_manifest* man, uint64_t* realized_per_expert
   if (touched_blocks) *touched_blocks = s[5];
   if (digest) *digest = s[4];
   if (err & kErrTimeout) return fail(MP_ERR_TIMEOUT, "a bounded device wait in the merge gave up");
+  if (err & kErrBounds) return fail(MP_ERR_CUDA, "a bounds check of the checked build failed in the merge kernels");
   if (err) return fail(MP_ERR_CUDA, "merge kernels reported an error");
   if (tot > s[0]) return fail(MP_ERR_BUDGET, "realized expert reads exceed the planned bytes");
   return MP_OK;
@@ -1436,6 +1450,8 @@ mp_status mp_index_hashes(const mp_family* family, mp_index* index, mp_stream st
   p.experts = ex;
   p.base_hash = index->d_base_hash;
   p.expert_hash = index->d_expert_hash;
+  p.ext = Extents{g.span_elems, g.span_elems};
+  p.err = index->d_err;
   if ((e = launch_hash(p, cs)) != cudaSuccess) return cuda_fail(e, "hash kernel");
   if ((e = cudaEventRecord(index->done, cs)) != cudaSuccess) return cuda_fail(e, "event record");
   return MP_OK;
@@ -1502,6 +1518,8 @@ mp_status mp_manifest_validate(const mp_family* family, const mp_index* index, c
   p.expert_hash = index->d_expert_hash;
   p.out_hash = man->d_out_hash;
   p.result = man->d_vresult;
+  p.ext = Extents{g.span_elems, g.span_elems};
+  p.err = man->d_err;
   if ((e = launch_hash(p, cs)) != cudaSuccess) return cuda_fail(e, "hash kernel");
   if (!man->valid_done && (e = cudaEventCreateWithFlags(&man->valid_done, cudaEventDisableTiming)) != cudaSuccess)
     return cuda_fail(e, "event");
@@ -1517,6 +1535,9 @@ mp_status mp_manifest_validation(const mp_manifest* man, uint64_t* checked, uint
   if ((e = cudaEventSynchronize(man->valid_done)) != cudaSuccess) return cuda_fail(e, "validation work");
   unsigned long long r[3];
   if ((e = cudaMemcpy(r, man->d_vresult, sizeof(r), cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
+  uint32_t err = 0;
+  if ((e = cudaMemcpy(&err, man->d_err, 4, cudaMemcpyDeviceToHost)) != cudaSuccess) return cuda_fail(e, "copy");
+  if (err & kErrBounds) return fail(MP_ERR_CUDA, "a bounds check of the checked build failed");
   if (out_hash && (e = cudaMemcpy(out_hash, man->d_out_hash, man->n_blocks * 8, cudaMemcpyDeviceToHost)) != cudaSuccess)
     return cuda_fail(e, "copy");
   if (checked) *checked = r[0];

@@ -28,6 +28,11 @@ __global__ void __launch_bounds__(kThreads) gather_kernel(const GatherLaunch g) 
   const uint32_t m = g.mask ? g.mask[b] : all;
   if (m == 0u) return;
   const uint64_t off = g.blk_off[b];
+  if (kChecked && !chunk_in_bounds(b, g.b_begin, g.b_end, off, g.blk_len[b], off, g.blk_len[b], m, g.K, g.elem_size,
+                                   g.origin, g.ext)) {  // uniform over the CTA
+    if (threadIdx.x == 0 && g.err) atomicOr(g.err, kErrBounds);
+    return;
+  }
   const uint64_t bytes = (uint64_t)g.blk_len[b] * g.elem_size;
   const uint64_t nvec = bytes / 16u;
   const uint32_t tail = (uint32_t)(bytes % 16u);

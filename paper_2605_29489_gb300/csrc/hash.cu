@@ -86,6 +86,11 @@ __global__ void __launch_bounds__(kHT) hash_kernel(const HashLaunch p) {
     const uint64_t b = it % nb;
     if (p.validate && k >= 1u && k <= p.K && !((p.mask[b] >> (k - 1u)) & 1u)) continue;  // not read
     const uint64_t off = p.blk_off[b], bytes = (uint64_t)p.blk_len[b] * p.elem_size;
+    if (kChecked && !chunk_in_bounds(b, 0, nb, off, p.blk_len[b], off, p.blk_len[b],
+                                     k >= 1u && k <= p.K ? 1ull << (k - 1u) : 0ull, p.K, p.elem_size, 0, p.ext)) {
+      if (threadIdx.x == 0 && p.err) atomicOr(p.err, kErrBounds);  // uniform over the CTA
+      continue;
+    }
     const uint8_t* src;
     if (k == 0u) src = static_cast<const uint8_t*>(p.base) + off * p.elem_size;
     else if (k <= p.K) src = static_cast<const uint8_t*>(p.experts.p[k - 1u]) + off * p.elem_size;

@@ -289,6 +289,23 @@ __device__ __forceinline__ void ties_fine2(float d0, float d1, uint32_t es, uint
       : "memory");
 }
 
+// Checked build: a work item (block b, experts i0 .. i0 + kc - 1) must lie in the launch's
+// block range before the block table is read for it, and the whole block, read from the
+// base and those experts, must pass chunk_in_bounds (with its TIES trim group below
+// n_groups) before anything is copied or loaded; a failure is recorded in the call's error
+// word and the item is skipped.  Constant true in the default build.
+template <bool TIES>
+__device__ __forceinline__ bool checked_item(const IndexLaunch& p, uint64_t b, uint32_t i0, uint32_t kc,
+                                             uint32_t es) {
+  if constexpr (!kChecked) return true;
+  if (b >= p.b_begin && b < p.b_end && b < p.n_blocks && i0 < p.K && (!TIES || p.blk_group[b] < p.n_groups) &&
+      chunk_in_bounds(b, p.b_begin, p.b_end, p.blk_off[b], p.blk_len[b], p.blk_off[b], p.blk_len[b],
+                      expert_run(i0, kc), p.K, es, p.expert_origin, p.ext))
+    return true;
+  atomicOr(p.err, kErrBounds);
+  return false;
+}
+
 template <bool BF16, int KG, int BM>
 __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone, KG>::kCtasPerSm)
     index_tma_kernel(const IndexLaunch p, uint32_t G, uint64_t n_items, unsigned long long* work) {
@@ -415,6 +432,7 @@ __global__ void __launch_bounds__(kIxThreads, IxGeo<BM != kBinNone, KG>::kCtasPe
         const uint64_t b = p.b_begin + it / G;
         const uint32_t i0 = (uint32_t)(it % G) * KG;
         const uint32_t kc = min((uint32_t)KG, p.K - i0);
+        if (!checked_item<TIES>(p, b, i0, kc, ES)) continue;
         if (BM == kBinCoarse && p.gmiss) {  // windowed fallback: the marked pairs' groups only
           const uint32_t grp = p.blk_group[b];
           bool any = false;
@@ -749,6 +767,7 @@ __global__ void __launch_bounds__(256) ties_fine_kernel(const IndexLaunch p) {
     const uint64_t b = it / G;
     const uint32_t i0 = (uint32_t)(it % G) * KG;
     const uint32_t kc = min((uint32_t)KG, p.K - i0);
+    if (!checked_item<true>(p, b, i0, kc, BF16 ? 2u : 4u)) continue;  // uniform over the CTA
     const uint32_t grp = p.blk_group[b];
 
     uint32_t estar[KG];
@@ -874,6 +893,10 @@ __global__ void __launch_bounds__(256) ties_sample_kernel(const IndexLaunch p) {
   const uint2 span = p.samp_span[blockIdx.x];  // {group, first block}: up to kSampleSpan blocks
   const uint32_t g = span.x, i0 = blockIdx.y * KG;
   const uint32_t kc = min((uint32_t)KG, p.K - i0);
+  if (kChecked && (g >= p.n_groups || i0 >= p.K)) {  // uniform over the CTA
+    if (threadIdx.x == 0) atomicOr(p.err, kErrBounds);
+    return;
+  }
   const uint32_t tid = threadIdx.x, warp = tid >> 5, lane = tid & 31u;
   for (uint32_t x = tid; x < (uint32_t)KG * 256u; x += blockDim.x) (&hist[0][0])[x] = 0u;
   if (tid == 0) s_n = 0;
@@ -882,6 +905,7 @@ __global__ void __launch_bounds__(256) ties_sample_kernel(const IndexLaunch p) {
   const uint64_t b1 = min((uint64_t)span.y + kSampleSpan, gb1);
   unsigned long long my_n = 0;
   for (uint64_t b = span.y + warp; b < b1; b += 8) {
+    if (!checked_item<false>(p, b, i0, kc, BF16 ? 2u : 4u)) continue;  // uniform over the warp
     const uint32_t len = p.blk_len[b];
     const uint64_t off = p.blk_off[b];
     const uint32_t nvec = (len + V - 1) / V;

@@ -290,6 +290,30 @@ __device__ __forceinline__ void store_vec(void* ptr, uint64_t elem, uint32_t nav
   }
 }
 
+// Checked build: a chunk's block must lie in the launch's block range before the block table
+// is read for it, and the chunk (its elements, buffers, alignment, experts and TIES trim
+// group) must pass chunk_in_bounds before anything is copied; a failure is recorded in the
+// call's error word and the chunk is skipped.  Both are constant true in the default build.
+__device__ __forceinline__ bool checked_block(const MergeLaunch& p, uint64_t b) {
+  if constexpr (!kChecked) return true;
+  if (b >= p.b_begin && b < p.b_end && b < p.n_blocks) return true;
+  atomicOr(p.err, kErrBounds);
+  return false;
+}
+
+template <bool TIES>
+__device__ __forceinline__ bool checked_chunk(const MergeLaunch& p, uint64_t b, const ChunkMeta& cm, uint32_t grp,
+                                              uint32_t es) {
+  if constexpr (!kChecked) return true;
+  if (cm.n == 0u) return true;
+  if ((!TIES || grp < p.n_groups) &&
+      chunk_in_bounds(b, p.b_begin, p.b_end, p.blk_off[b], p.blk_len[b], cm.off, cm.n, cm.m, p.K, es,
+                      p.expert_origin, p.ext))
+    return true;
+  atomicOr(p.err, kErrBounds);
+  return false;
+}
+
 // DARE keep words of the vector at flat element j0 for expert i: element j keeps its delta
 // iff 16-bit word j mod 8 of the Philox4x32-10 output for counter j / 8 is >= T.  A bf16
 // vector is exactly the 8 words of one call (chunk and tensor offsets are multiples of 8
@@ -379,7 +403,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
       if (lane < G) {
         const unsigned long long q = q0 + lane;
         ChunkMeta cm{0, 0, 0};
-        if (q < n_chunks) {
+        if (q < n_chunks && checked_block(p, p.b_begin + q / cpb)) {
           const uint64_t b = p.b_begin + q / cpb;
           bq = b;
           const uint32_t start = (uint32_t)(q % cpb) * CH;
@@ -389,6 +413,7 @@ __global__ void __launch_bounds__(Geo<OPC>::kThreads, Geo<OPC>::kCtasPerSm)
           cm.n = start < len ? min(CH, len - start) : 0u;
           if (p.touched_only && cm.m == 0u) cm.n = 0u;  // left as it is: a reference to M_0
           if constexpr (OPC == OP_TIES) grp = p.blk_group[b];
+          if (!checked_chunk<OPC == OP_TIES>(p, b, cm, grp, ES)) cm.n = 0u, grp = 0u;
         }
         S.chunk[lane] = cm;
       }
@@ -743,7 +768,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
       if (lane < G) {
         const unsigned long long q = q0 + lane;
         ChunkMeta cm{0, 0, 0};
-        if (q < n_chunks) {
+        if (q < n_chunks && checked_block(p, p.b_begin + q / cpb)) {
           const uint64_t b = p.b_begin + q / cpb;
           const uint32_t start = (uint32_t)(q % cpb) * CH;
           const uint32_t len = p.blk_len[b];
@@ -752,6 +777,7 @@ __global__ void __launch_bounds__(TcGeo<OPC, KC>::kThreads, TcGeo<OPC, KC>::kCta
           cm.n = start < len ? min(CH, len - start) : 0u;
           if (p.touched_only && cm.m == 0u) cm.n = 0u;  // left as it is: a reference to M_0
           if (OPC == OP_TIES) grp = p.blk_group[b];
+          if (!checked_chunk<OPC == OP_TIES>(p, b, cm, grp, ES)) cm.n = 0u, grp = 0u;
         }
         S.chunk[lane] = cm;
       }

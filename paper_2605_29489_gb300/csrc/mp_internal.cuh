@@ -10,6 +10,7 @@
 #include <utility>
 #include <vector>
 
+#include "checked.cuh"
 #include "mergepipe.h"
 
 namespace mp {
@@ -24,7 +25,8 @@ constexpr int kMaxK = 32;
 constexpr int kCounterSlots = 64;  // realized-byte counters are spread over slots
 
 // device error word bits
-enum : uint32_t { kErrNonfinite = 1u, kErrTimeout = 2u, kErrInternal = 4u, kErrMissing = 8u };
+// (kErrBounds: a range failed a check of the checked build and was skipped)
+enum : uint32_t { kErrNonfinite = 1u, kErrTimeout = 2u, kErrInternal = 4u, kErrMissing = 8u, kErrBounds = 16u };
 // nnz of a catalog entry without block statistics (no block holds 2^32 - 1 elements)
 constexpr uint32_t kNnzMissing = 0xFFFFFFFFu;
 
@@ -229,6 +231,7 @@ struct IndexLaunch {
   // expert_origin of the flat layout (0 for resident experts, a segment start when they
   // point into a staging buffer)
   uint64_t b_begin, b_end, expert_origin;
+  Extents ext;            // buffer extents, for the checks of the checked build
   int defer_ties_select;  // 1: leave the TIES selection to launch_ties_finish
   uint32_t wait_limit;    // try_wait rounds of the pipeline waits (0: the default)
   uint32_t stall;         // test hook: every CTA's first ring fill is never armed
@@ -320,6 +323,7 @@ struct MergeLaunch {
   unsigned long long* work;      // chunk counter of the dynamic scheduler (zeroed per launch)
   uint32_t* err;
   uint64_t b_begin, b_end, expert_origin;  // as in IndexLaunch
+  Extents ext;                             // as in IndexLaunch
   uint32_t touched_only;  // 1: blocks with an empty mask are neither read nor written
   uint32_t wait_limit;    // try_wait rounds of the pipeline waits (0: the default)
   uint32_t stall;         // test hook: every CTA's first ring fill is never armed
@@ -341,6 +345,8 @@ struct GatherLaunch {
   ExpertPtrs dst;         // staging buffers
   unsigned long long* gathered;  // bytes copied, accumulated (may be NULL)
   const uint32_t* gate;          // when set, the launch copies nothing unless *gate != 0
+  Extents ext;                   // span: the host experts; x_span: the staging from origin
+  uint32_t* err;                 // the call's error word (checked build)
 };
 cudaError_t launch_gather(const GatherLaunch& g, cudaStream_t st);
 // copies and fills by kernel on st (no copy engine); host buffers must be pinned memory
@@ -367,6 +373,8 @@ struct HashLaunch {
   unsigned long long* expert_hash;  // [K][n_blocks]
   unsigned long long* out_hash;     // [n_blocks]
   unsigned long long* result;       // [3]
+  Extents ext;                      // every buffer spans the family (x_span = span)
+  uint32_t* err;                    // the call's error word (checked build)
 };
 cudaError_t launch_hash(const HashLaunch& p, cudaStream_t st);
 
