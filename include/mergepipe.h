@@ -44,7 +44,8 @@
  *    (a block of the catalog pass or of the host-pool gather, a chunk of the merge, a
  *    block of the hash pass) it checks the range against the block table, the call's block
  *    range, the buffers' extents, the 16-byte alignment of bulk copies and the number of
- *    experts; a range that fails is not touched, and the accessors of the call's handle
+ *    experts, and the planner checks every compaction slot and unit id it writes; a
+ *    range that fails is not touched, and the accessors of the call's handle
  *    return MP_ERR_CUDA with "a bounds check of the checked build failed".  mp_version()
  *    names the build.  Slower; meant for debugging.
  *  - On an error return no handle is produced and *out is set to NULL; the

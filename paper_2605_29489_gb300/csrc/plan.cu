@@ -346,8 +346,12 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
         uint32_t tot;
         const uint32_t pos = block_scan<uint32_t>(x.cand ? 1u : 0u, tot);
         if (x.cand) {
-          s.keys_a[run + pos] = x.key;
-          p.order[run + pos] = (uint32_t)u;
+          if (kChecked && run + pos >= p.n_blocks * p.K) {  // checked build: a compaction slot past U
+            atomicOr((unsigned long long*)&p.summary[S_ERR], (unsigned long long)kErrBounds);
+          } else {
+            s.keys_a[run + pos] = x.key;
+            p.order[run + pos] = (uint32_t)u;
+          }
         }
         run += tot;
       }
@@ -540,6 +544,10 @@ __global__ void __launch_bounds__(kPT) plan_kernel(const PlanLaunch p, Scratch s
     for (uint64_t j = q0 + tid; j < q1; j += kPT) {
       if ((P == kNoP || j < P) || s.tailsel[j]) {
         const uint32_t u = order[j];
+        if (kChecked && (uint64_t)u >= p.n_blocks * p.K) {  // checked build: a unit id past U
+          atomicOr((unsigned long long*)&p.summary[S_ERR], (unsigned long long)kErrBounds);
+          continue;
+        }
         const uint32_t b = u / p.K, i = u % p.K;
         const uint32_t t = p.fallback ? p.blk_tensor[b] : 0u;
         if (p.fallback && s.pair_flag[i * p.n_tensors + t]) {

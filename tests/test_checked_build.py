@@ -3,8 +3,8 @@
 Its kernels check every range they stream (a block of the catalog pass, a chunk of the
 merge, a block of the host-pool gather or of the hash pass) against the block table, the
 launch's block range, the buffers' extents, the 16-byte alignment of bulk copies and the
-number of experts before touching it; a range that fails is skipped and reported through the
-call's error word.
+number of experts before touching it, and the planner checks every compaction slot and unit
+id it writes; a range that fails is skipped and reported through the call's error word.
 
 CPU: the predicate itself on hand-made ranges, each case written out with the outcome it must
 have; the checked library exports what the header declares.  GPU: the parity cases of the
